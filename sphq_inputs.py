@@ -1,0 +1,147 @@
+"""Seeded synthetic inputs for the SPHQuant decode GEMV.
+
+This module only draws random numbers and lays them out; it holds none of the
+method's arithmetic (no decode, no radius dequantisation, no matvec).  Both the
+CUDA path (tests, bench.py, smoke()) and the oracle consume what it returns.
+
+Recipe (every draw from numpy's PCG64, seed = 20260 + 100*config + shape):
+  draw order  codebook, scale, offset, sign, idx, rcode, x
+  codebook    K rows of |N(0, I_8)|, each scaled to unit length, rounded to fp16
+  scale       Delta_G ~ U(0.5, 2)  -> fp16, one per 128-column group
+  offset      r_min_G ~ U(0, 1)    -> fp16
+  sign        U{0..255} per 8-D vector
+  idx         U{0..K-1}
+  rcode       U{0..15}
+  x           N(0, 1) -> fp16, shape (B, cols)
+Gaussian weight matrices (the encoded configuration) are N(0, 0.02^2) with
+0.1% of the scalars, chosen uniformly, multiplied by 20.
+
+fp16 values are carried as uint16 bit patterns (numpy float16 views).
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass
+
+import numpy as np
+
+VEC = 8
+GROUP_COLS = 128
+RADIUS_BITS = 4
+
+
+def bits_to_K(bits: int) -> int:
+    """Codebook size for the W2 / W3 settings: 2^(7B-8) entries."""
+    return 1 << (7 * bits - 8)
+
+
+@dataclass
+class Codes:
+    """Canonical codes of one quantised rows x cols matrix (host numpy)."""
+    bits: int
+    codebook: np.ndarray  # (K, 8) uint16 fp16 bits
+    scale: np.ndarray     # (rows, cols/128) uint16 fp16 bits
+    offset: np.ndarray    # (rows, cols/128) uint16 fp16 bits
+    sign: np.ndarray      # (rows, cols/8) uint8
+    idx: np.ndarray       # (rows, cols/8) uint16
+    rcode: np.ndarray     # (rows, cols/8) uint8
+
+    @property
+    def rows(self) -> int:
+        return self.sign.shape[0]
+
+    @property
+    def cols(self) -> int:
+        return self.sign.shape[1] * VEC
+
+    @property
+    def K(self) -> int:
+        return self.codebook.shape[0]
+
+    def row_slice(self, r0: int, r1: int) -> "Codes":
+        return Codes(self.bits, self.codebook, self.scale[r0:r1], self.offset[r0:r1],
+                     self.sign[r0:r1], self.idx[r0:r1], self.rcode[r0:r1])
+
+
+def seed_for(config: int, shape: int = 0) -> int:
+    return 20260 + 100 * config + shape
+
+
+def to_f16_bits(a) -> np.ndarray:
+    return np.asarray(a, np.float64).astype(np.float16).view(np.uint16)
+
+
+def make_codebook(rng: np.random.Generator, K: int) -> np.ndarray:
+    c = np.abs(rng.standard_normal((K, VEC)))
+    c /= np.linalg.norm(c, axis=1, keepdims=True)
+    return to_f16_bits(c)
+
+
+def make_params(rng: np.random.Generator, rows: int, cols: int):
+    ng = cols // GROUP_COLS
+    scale = to_f16_bits(rng.uniform(0.5, 2.0, size=(rows, ng)))
+    offset = to_f16_bits(rng.uniform(0.0, 1.0, size=(rows, ng)))
+    return scale, offset
+
+
+def make_x(rng: np.random.Generator, B: int, cols: int) -> np.ndarray:
+    return to_f16_bits(rng.standard_normal((B, cols)))
+
+
+def random_codes(bits: int, rows: int, cols: int, seed: int, B: int = 1,
+                 codebook: np.ndarray | None = None):
+    """Uniformly random codes (configurations 0, 2, 3, 4).  Returns (Codes, x)."""
+    if cols % GROUP_COLS:
+        raise ValueError("cols must be a multiple of 128")
+    rng = np.random.Generator(np.random.PCG64(seed))
+    K = bits_to_K(bits)
+    cb = make_codebook(rng, K)
+    if codebook is not None:
+        cb = codebook
+    scale, offset = make_params(rng, rows, cols)
+    nv = cols // VEC
+    sign = rng.integers(0, 256, size=(rows, nv), dtype=np.uint8)
+    idx = rng.integers(0, K, size=(rows, nv), dtype=np.uint16)
+    rcode = rng.integers(0, 1 << RADIUS_BITS, size=(rows, nv), dtype=np.uint8)
+    x = make_x(rng, B, cols)
+    return Codes(bits, cb, scale, offset, sign, idx, rcode), x
+
+
+def gaussian_weights(rows: int, cols: int, seed: int, std: float = 0.02,
+                     outlier_frac: float = 1e-3, outlier_mult: float = 20.0):
+    """W ~ N(0, std^2) with a uniformly chosen fraction of scalars scaled up."""
+    rng = np.random.Generator(np.random.PCG64(seed + 7))
+    w = rng.standard_normal((rows, cols)) * std
+    n_out = int(round(outlier_frac * rows * cols))
+    pos = rng.choice(rows * cols, size=n_out, replace=False)
+    w.reshape(-1)[pos] *= outlier_mult
+    return w
+
+
+def encoded_inputs_rng(bits: int, cols: int, seed: int, B: int = 1):
+    """Codebook and activations for the encoded configuration (the codes themselves
+    come from an encoder run on gaussian_weights)."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    cb = make_codebook(rng, bits_to_K(bits))
+    x = make_x(rng, B, cols)
+    return cb, x
+
+
+# ---------------------------------------------------------------------------
+# workload shapes
+# ---------------------------------------------------------------------------
+
+# 7B-class decoder projections (hidden 3584, 28 q heads / 4 kv heads of 128, FFN 18944):
+# (name, rows = d_out, cols = d_in)
+DECODER_PROJ = [
+    ("q", 3584, 3584),
+    ("k", 512, 3584),
+    ("v", 512, 3584),
+    ("o", 3584, 3584),
+    ("gate", 18944, 3584),
+    ("up", 18944, 3584),
+    ("down", 3584, 18944),
+]
+DECODER_LAYERS = 28
+
+# square sweep at batch 1: (bits, n)
+SQUARE_SWEEP = [(2, 4096), (2, 8192), (3, 4096), (3, 8192)]
