@@ -1,0 +1,479 @@
+#!/usr/bin/env python3
+"""Benchmark of the SPHQuant decode GEMV on GB300 (one JSON line on stdout).
+
+Workload (one "step" = one pass of the hot path over one batch of input):
+  the batch-1 W2/W3 GEMV sweep at 4096x4096 and 8192x8192.  Each shape has a
+  pool of distinct packed matrices whose total size exceeds twice the L2
+  cache, and a step runs one GEMV on every matrix of every pool (each pool
+  captured once as a CUDA graph of back-to-back launches on one stream), so
+  every GEMV streams its codes from HBM.  Codes are seeded uniformly random
+  codes of the encoded configuration's shapes (the data path and byte count
+  do not depend on the code values; parity on encoder-produced codes is
+  covered by the tests).
+
+value    = algorithmic bytes of all GEMVs / device time of the timed steps (GB/s)
+roofline = the dominant kernel's algorithmic bytes per launch / its average
+           launch time (CUDA events on the launching stream), against the
+           measured HBM copy bandwidth
+e2e      = the same metric through sphq_gemv_host (pinned host x in, y out,
+           copies inside the timed region), one GEMV per shape per step
+stack    = the 28-layer x 7-projection linear stack of a 7B-class decoder at
+           W2 and W3, batch 1, chained on one stream in a CUDA graph: us/token
+
+--impl reference runs the float64 CPU oracle (the reference arm of this
+build) on bounded row samples of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import sphq_inputs as inp  # noqa: E402
+
+METRIC = "batch-1 W2/W3 GEMV effective GB/s and % of GB300 HBM peak; µs/token for linear stack"
+UNIT = "GB/s"
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+# ---------------------------------------------------------------------------
+# clocks sampled during the timed region
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except (FileNotFoundError, OSError):
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.t.join(timeout=2)
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            p = [t.strip() for t in ln.split(",")]
+            if len(p) < 8:
+                continue
+            try:
+                sm.append(float(p[0]))
+                mx.append(float(p[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, p[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# distributed (replicas only: every rank runs its own pools)
+# ---------------------------------------------------------------------------
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        dist.init_process_group(backend)
+    return world, rank, local
+
+
+def dist_barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def dist_max(world, v: float) -> float:
+    if world == 1:
+        return v
+    import torch
+    import torch.distributed as dist
+    dev = torch.device("cuda", torch.cuda.current_device()) if torch.cuda.is_available() else "cpu"
+    t = torch.tensor([v], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+
+def l2_bytes() -> int:
+    import torch
+    p = torch.cuda.get_device_properties(torch.cuda.current_device())
+    return int(getattr(p, "L2_cache_size", 0) or getattr(p, "l2_cache_size", 0) or 128 << 20)
+
+
+def make_pool(bits: int, rows: int, cols: int, n: int, seed: int, dev):
+    """n distinct device copies of one seeded matrix (distinct buffers, so no
+    L2 reuse between consecutive GEMVs)."""
+    import torch
+
+    from paper_2609_24875_gb300 import SphqMatrix
+    codes, x = inp.random_codes(bits, rows, cols, seed=seed)
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int16) if a.dtype == np.uint16 else a)).to(dev)
+    cb, sc, of = t(codes.codebook), t(codes.scale), t(codes.offset)
+    sg, ix, rc = t(codes.sign), t(codes.idx), t(codes.rcode)
+    mats = []
+    for _ in range(n):
+        m = SphqMatrix(rows, cols, bits, cb, sc, of)
+        m.pack(sg, ix, rc)
+        mats.append(m)
+    del sg, ix, rc
+    xd = t(x).view(torch.float16)
+    return mats, xd, codes, x
+
+
+def capture(mats, xd, ys, stream):
+    import torch
+    with torch.cuda.stream(stream):
+        for m, y in zip(mats, ys):
+            m.gemv_ptr(xd.data_ptr(), y.data_ptr(), 1, stream.cuda_stream)
+    stream.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for m, y in zip(mats, ys):
+            m.gemv_ptr(xd.data_ptr(), y.data_ptr(), 1, stream.cuda_stream)
+    return g
+
+
+def run_gpu(args, world, rank, local):
+    import torch
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2609_24875_gb300 import load
+    load()
+    hbm_peak, peak_kind = measured_peaks()
+    L2 = l2_bytes()
+    stream = torch.cuda.Stream(device=dev)
+
+    # --- pools for the square sweep ---
+    shapes = []
+    for sid, (bits, n) in enumerate(inp.SQUARE_SWEEP):
+        probe_bytes = n * n * (8 + 7 * bits - 8 + 4) // 64 + (n * n // 128) * 4
+        P = max(2, int(np.ceil(2 * L2 / probe_bytes)) + 1)
+        if args.quick:
+            P = 2
+        mats, xd, codes, x = make_pool(bits, n, n, P, inp.seed_for(1, sid), dev)
+        ys = [torch.empty((1, n), dtype=torch.float16, device=dev) for _ in mats]
+        g = capture(mats, xd, ys, stream)
+        shapes.append(dict(name=f"W{bits} {n}x{n}", bits=bits, n=n, mats=mats, xd=xd, ys=ys,
+                           graph=g, bytes=mats[0].bytes(1), P=P))
+    torch.cuda.synchronize()
+
+    def step(evs=None):
+        for i, s in enumerate(shapes):
+            if evs is not None:
+                evs[i][0].record(stream)
+            s["graph"].replay()
+            if evs is not None:
+                evs[i][1].record(stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            step()
+    torch.cuda.synchronize()
+
+    K = args.steps
+    ev = [[[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in shapes]
+          for _ in range(K)]
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    dist_barrier(world)
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        with torch.cuda.stream(stream):
+            t0.record(stream)
+            for k in range(K):
+                step(ev[k])
+            t1.record(stream)
+        torch.cuda.synchronize()
+    dist_barrier(world)
+    total_ms = t0.elapsed_time(t1)
+    total_ms = dist_max(world, total_ms)
+    per_shape_ms = [sum(ev[k][i][0].elapsed_time(ev[k][i][1]) for k in range(K))
+                    for i in range(len(shapes))]
+    launches = sum(s["P"] for s in shapes) * K
+    step_bytes = sum(s["P"] * s["bytes"] for s in shapes)
+    value = step_bytes * K * world / (total_ms * 1e-3) / 1e9
+
+    sweep = {}
+    for s, ms in zip(shapes, per_shape_ms):
+        us = ms * 1e3 / (K * s["P"])
+        gbs = s["bytes"] / (us * 1e-6) / 1e9
+        sweep[s["name"]] = {"us_per_gemv": round(us, 3), "GB/s": round(gbs, 1),
+                            "hbm_frac": round(gbs / hbm_peak, 4), "bytes": s["bytes"],
+                            "pool": s["P"]}
+    dom = max(range(len(shapes)), key=lambda i: per_shape_ms[i])
+    ds = shapes[dom]
+    d_us = per_shape_ms[dom] * 1e3 / (K * ds["P"])
+    achieved = ds["bytes"] / (d_us * 1e-6) / 1e9
+    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm_peak,
+                "unit": "GB/s", "frac": round(achieved / hbm_peak, 4),
+                "traffic": None, "kernel": f"gemv_kernel ({ds['name']}, batch 1)",
+                "peak_kind": peak_kind}
+
+    # --- end to end through the host-buffer entry point ---
+    e2e = run_e2e(args, shapes, stream)
+
+    # --- 28-layer linear stack ---
+    stack = None if args.no_stack else run_stack(args, dev, stream, hbm_peak)
+
+    for s in shapes:
+        for m in s["mats"]:
+            m.close()
+    out = {
+        "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
+        "steps": K, "warmup": args.warmup, "ms_per_step": round(total_ms / K, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "fp16 in, fp32 accumulate (2.25/3.125-bit codes)", "data": "synthetic",
+        "config": {"workload": "W2+W3 GEMV sweep 4096^2 and 8192^2, batch 1",
+                   "pools": {s["name"]: s["P"] for s in shapes},
+                   "l2_policy": "each pool > 2x L2, distinct buffers per GEMV",
+                   "parallelism": f"replicas x{world}"},
+        "hbm_frac": round(value / hbm_peak, 4),
+        "sweep": sweep, "roofline": roofline, "e2e": e2e, "stack": stack,
+        "gpu_launches": launches,
+    }
+    return out, clk.summary()
+
+
+def run_e2e(args, shapes, stream):
+    import torch
+    K = max(1, min(args.steps, 50))
+    xs = [torch.empty((1, s["n"]), dtype=torch.float16).pin_memory() for s in shapes]
+    ys = [torch.empty((1, s["n"]), dtype=torch.float16).pin_memory() for s in shapes]
+    for xh, s in zip(xs, shapes):
+        xh.copy_(s["xd"].cpu())
+    for _ in range(3):
+        for i, s in enumerate(shapes):
+            s["mats"][0].gemv_host(xs[i], ys[i], stream=stream)
+    stream.synchronize()
+    t0 = time.perf_counter()
+    for k in range(K):
+        for i, s in enumerate(shapes):
+            s["mats"][k % s["P"]].gemv_host(xs[i], ys[i], stream=stream)
+        stream.synchronize()
+    dt = time.perf_counter() - t0
+    b = sum(s["bytes"] for s in shapes)
+    return {"value": round(b * K / dt / 1e9, 1), "unit": UNIT,
+            "h2d_bytes_per_step": sum(2 * s["n"] for s in shapes),
+            "d2h_bytes_per_step": sum(2 * s["n"] for s in shapes),
+            "us_per_step": round(dt / K * 1e6, 2)}
+
+
+def run_stack(args, dev, stream, hbm_peak):
+    import torch
+
+    from paper_2609_24875_gb300 import SphqMatrix
+    res = {}
+    layers = 2 if args.quick else inp.DECODER_LAYERS
+    for bits in (2, 3):
+        mats, ys, xs = [], [], []
+        # one seeded code set per projection shape, packed into a distinct
+        # buffer per layer (28 x 7 distinct matrices, 6.5e9 weights)
+        for i, (name, rows, cols) in enumerate(inp.DECODER_PROJ):
+            codes, x = inp.random_codes(bits, rows, cols, seed=inp.seed_for(4, 10 * bits + i))
+            t = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int16) if a.dtype == np.uint16 else a)).to(dev)
+            cb, sc, of = t(codes.codebook), t(codes.scale), t(codes.offset)
+            sg, ix, rc = t(codes.sign), t(codes.idx), t(codes.rcode)
+            xd = t(x).view(torch.float16)
+            for l in range(layers):
+                m = SphqMatrix(rows, cols, bits, cb, sc, of)
+                m.pack(sg, ix, rc)
+                mats.append((l, i, m))
+                xs.append(xd)
+                ys.append(torch.empty((1, rows), dtype=torch.float16, device=dev))
+            del sg, ix, rc
+        order = sorted(range(len(mats)), key=lambda j: (mats[j][0], mats[j][1]))
+        seq = [(mats[j][2], xs[j], ys[j]) for j in order]
+        with torch.cuda.stream(stream):
+            for m, xd, yd in seq:
+                m.gemv_ptr(xd.data_ptr(), yd.data_ptr(), 1, stream.cuda_stream)
+        stream.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for m, xd, yd in seq:
+                m.gemv_ptr(xd.data_ptr(), yd.data_ptr(), 1, stream.cuda_stream)
+        for _ in range(3):
+            g.replay()
+        torch.cuda.synchronize()
+        reps = max(3, min(args.steps, 20))
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(reps):
+                g.replay()
+            e1.record(stream)
+        torch.cuda.synchronize()
+        us = e0.elapsed_time(e1) * 1e3 / reps
+        byts = sum(m.bytes(1) for m, _, _ in seq)
+        gbs = byts / (us * 1e-6) / 1e9
+        res[f"W{bits}"] = {"us_per_token": round(us * inp.DECODER_LAYERS / layers, 2),
+                           "layers_timed": layers, "gemvs": len(seq),
+                           "GB/s": round(gbs, 1), "hbm_frac": round(gbs / hbm_peak, 4)}
+        del g
+        for m, _, _ in seq:
+            m.close()
+        torch.cuda.empty_cache()
+    return res
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle (cpu_baseline leg and --impl reference)
+# ---------------------------------------------------------------------------
+
+def oracle_sample(seconds: float, threads: int):
+    """Times the float64 oracle (decode + matvec, row by row) on row samples of
+    the sweep's four shapes until about `seconds` have elapsed.  Returns
+    (GB/s over the sampled rows' share of the algorithmic bytes, description)."""
+    import oracle
+    oracle.set_threads(threads)
+    per_shape = []
+    for sid, (bits, n) in enumerate(inp.SQUARE_SWEEP):
+        rows = 64
+        codes, x = inp.random_codes(bits, rows, n, seed=inp.seed_for(1, sid))
+        per_shape.append((bits, n, codes, x))
+    done_bytes, t_total, rows_done = 0.0, 0.0, 0
+    budget = seconds / len(per_shape)
+    for bits, n, codes, x in per_shape:
+        full_bytes = n * n * (7 * bits + 4) / 64 + n * n / 128 * 4 + (1 << (7 * bits - 8)) * 16 + 4 * n
+        t0 = time.perf_counter()
+        while True:
+            oracle.decode_gemv(codes.codebook, codes.scale, codes.offset, codes.sign,
+                               codes.idx, codes.rcode, x)
+            rows_done += codes.rows
+            done_bytes += full_bytes * codes.rows / n
+            if time.perf_counter() - t0 > budget:
+                break
+        t_total += time.perf_counter() - t0
+    gbs = done_bytes / t_total / 1e9
+    desc = (f"float64 oracle decode+matvec on 64-row samples of the W2/W3 4096^2 and 8192^2 "
+            f"matrices, {rows_done} rows in {t_total:.1f} s, bytes scaled to the rows' share")
+    return gbs, desc, t_total
+
+
+def run_reference(args, world, rank):
+    if rank != 0:
+        return None
+    import oracle
+    threads = oracle.max_threads()
+    vals = []
+    for _ in range(args.warmup):
+        oracle_sample(0.2, threads)
+    t0 = time.perf_counter()
+    per = max(0.5, min(10.0, 60.0 / max(1, args.steps)))
+    for _ in range(args.steps):
+        v, desc, _ = oracle_sample(per, threads)
+        vals.append(v)
+    dt = time.perf_counter() - t0
+    value = statistics.median(vals)
+    hbm_peak, _ = measured_peaks()
+    return {
+        "impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": UNIT,
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(dt / args.steps * 1e3, 2), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": "W2+W3 GEMV sweep 4096^2 and 8192^2, batch 1",
+                   "parallelism": "cpu oracle"},
+        "hbm_frac": round(value / hbm_peak, 6),
+        "cpu_baseline": {"value": round(value, 4), "unit": UNIT, "cores": threads,
+                         "kind": "oracle", "sample": desc},
+        "e2e": {"value": round(value, 4), "unit": UNIT, "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--quick", action="store_true", help="small pools / 2 stack layers")
+    ap.add_argument("--no-stack", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    world, rank, local = dist_setup()
+
+    if args.impl == "reference":
+        out = run_reference(args, world, rank)
+        if rank == 0:
+            print(json.dumps(out), flush=True)
+        return
+
+    out, clocks = run_gpu(args, world, rank, local)
+    if rank == 0:
+        out["clocks"] = clocks
+        if world == 1 and not args.no_cpu_baseline:
+            import oracle
+            threads = oracle.max_threads()
+            v, desc, _ = oracle_sample(args.cpu_seconds, threads)
+            out["cpu_baseline"] = {"value": round(v, 4), "unit": UNIT, "cores": threads,
+                                   "kind": "oracle", "sample": desc}
+        print(json.dumps(out), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,169 @@
+/*
+ * sphq.h -- C ABI of the GB300 (sm_103a) SPHQuant decode library.
+ *
+ * The library runs one operation: the fused dequantize-GEMV that decodes
+ * spherically quantised weights and multiplies them with fp16 activations
+ * during autoregressive decode (SPHQuant, §3.4 "Efficient Kernel
+ * Implementation" and App. D).  Each 8-D weight vector w_i of a row is stored
+ * as 8 coordinate sign bits s_i, a direction index z_i into a codebook of
+ * non-negative unit vectors c_k, and a 4-bit radius code q_i; every group of
+ * 16 consecutive vectors (128 scalars) along the input dimension shares an
+ * fp16 scale Delta_G and offset r_min_G (§3.1, Eq. (7)).  The library
+ * reconstructs (Eq. (7) then Eq. (4))
+ *
+ *     r_hat_i = RN16(q_i * Delta_G + r_min_G)          one fp16 fused multiply-add
+ *     w_hat_i = RN16(r_hat_i * c_{z_i})  with coordinate j negated when bit j of s_i is set
+ *
+ * and computes y[b][r] = sum_j w_hat[r][j] * x[b][j] with fp32 accumulation,
+ * rounding y to fp16 (round to nearest even).
+ *
+ * Supported settings (§3.1 bit budget, App. B): bits = 2 (W2: K = 64 entries,
+ * 8 sign + 6 index + 4 radius bits = 2.25 bits/weight) and bits = 3
+ * (W3: K = 8192 entries, 8 + 13 + 4 = 3.125 bits/weight); batch 1..8.
+ *
+ * Conventions
+ *   - All fp16 data are IEEE binary16 bit patterns (uint16_t storage).
+ *   - Row-major everywhere.  rows = d_out, cols = d_in; cols % 128 == 0.
+ *   - "device pointer": memory the current CUDA device can access
+ *     (cudaMalloc, managed, or mapped pinned host memory).
+ *   - Every call acts on the CUDA device that was current when the handle
+ *     was created; the caller keeps that device current.
+ *   - Errors: every call returns a status and launches nothing on error.
+ *     sphq_last_error() gives a message for the calling thread.
+ *   - No call traps, asserts or spins on the device.
+ */
+#ifndef SPHQ_H_
+#define SPHQ_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Opaque handle to one quantised weight matrix resident in device memory. */
+typedef struct sphq_handle_s* sphq_handle;
+
+/* A cudaStream_t (the runtime's stream type is `struct CUstream_st*`).
+ * NULL means the legacy default stream. */
+typedef struct CUstream_st* sphq_stream;
+
+typedef enum sphq_status {
+  SPHQ_OK = 0,
+  SPHQ_ERR_INVALID_ARG = 1,   /* bad size, pointer, alignment or code value */
+  SPHQ_ERR_UNSUPPORTED = 2,   /* bits/K/batch outside the supported set      */
+  SPHQ_ERR_NOT_PACKED = 3,    /* gemv/decode before a successful sphq_pack   */
+  SPHQ_ERR_CUDA = 4,          /* a CUDA runtime call failed                  */
+  SPHQ_ERR_OOM = 5,           /* device allocation failed                    */
+  SPHQ_ERR_DEVICE = 6         /* no usable sm_103 device                     */
+} sphq_status;
+
+#define SPHQ_MAX_BATCH 8
+#define SPHQ_GROUP_COLS 128   /* scalars per radius group (§3.1)   */
+#define SPHQ_VECTOR_DIM 8     /* 8-D vectors (§3.1)                */
+
+/*
+ * sphq_create -- describe one quantised matrix and allocate its device storage.
+ *
+ *   rows, cols   d_out and d_in; rows >= 1, cols >= 128, cols % 128 == 0.
+ *   bits         2 (W2) or 3 (W3), the target bit-width B of §3.1.
+ *   K            codebook entries; must equal 2^(7*bits - 8) (§3.1): 64 or 8192.
+ *   codebook     K x 8 fp16, entry k = direction c_k (§3.1, Eq. (5)); values are
+ *                used as given (the paper's entries are non-negative unit vectors).
+ *   scale        rows x (cols/128) fp16, Delta_G of Eq. (7) for group G = (row, col/128).
+ *   offset       rows x (cols/128) fp16, r_min_G of Eq. (7).
+ *   out          receives the handle.
+ *
+ * codebook, scale and offset may be host or device pointers (they are read
+ * with cudaMemcpyDefault); the call is synchronous and copies them, so the
+ * caller may free them on return.  The handle owns all device memory it
+ * allocates (packed codes, parameters, codebook, split-K workspace).
+ * Returns SPHQ_ERR_INVALID_ARG / SPHQ_ERR_UNSUPPORTED / SPHQ_ERR_OOM /
+ * SPHQ_ERR_DEVICE / SPHQ_ERR_CUDA; *out is NULL on error.
+ */
+sphq_status sphq_create(int rows, int cols, int bits, int K, const void* codebook,
+                        const void* scale, const void* offset, sphq_handle* out);
+
+/*
+ * sphq_pack -- convert canonical codes into the library's device layout
+ * (the finalise-and-pack step, App. A step 10).
+ *
+ *   sign   rows x (cols/8) uint8, bit j set <=> coordinate j of the vector is
+ *          negative (§3.1, Eq. (3)); vector t of a row covers columns 8t..8t+7.
+ *   idx    rows x (cols/8) uint16, direction index z < K (Eq. (5)).
+ *   rcode  rows x (cols/8) uint8, radius code q < 16 (Eq. (7), V = 4).
+ *   stream stream the pack kernel runs on.
+ *
+ * All three are device pointers.  The call validates every code on the
+ * device and synchronises `stream` before returning; out-of-range codes give
+ * SPHQ_ERR_INVALID_ARG and leave the handle unpacked.  May be called again
+ * to replace the codes.  Not for use inside CUDA graph capture.
+ */
+sphq_status sphq_pack(sphq_handle h, const uint8_t* sign, const uint16_t* idx,
+                      const uint8_t* rcode, sphq_stream stream);
+
+/*
+ * sphq_gemv -- y = W_hat x for a batch of activation rows (§3.4, App. D).
+ *
+ *   x      batch x cols fp16, device pointer, 16-byte aligned.
+ *   y      batch x rows fp16, device pointer, 4-byte aligned; written in full.
+ *   batch  1..SPHQ_MAX_BATCH.
+ *
+ * Asynchronous on `stream`: no host synchronisation and no allocation, so it
+ * may be captured in a CUDA graph.  The handle owns a split-K workspace, so
+ * one handle must not run two gemv calls concurrently (different streams);
+ * calls on one stream, or on different handles, are independent.  Numerics:
+ * fp32 accumulation; |y - W_hat x| <= 1e-3 * sum_j |w_hat_j||x_j| + 2^-24 per
+ * output (fp16 output rounding included), where W_hat is the exact decode
+ * that sphq_decode returns.
+ */
+sphq_status sphq_gemv(sphq_handle h, const void* x, void* y, int batch, sphq_stream stream);
+
+/*
+ * sphq_gemv_host -- the same GEMV for host-resident activations and outputs.
+ *
+ *   x_host  batch x cols fp16 in host memory; y_host  batch x rows fp16.
+ *
+ * Enqueues on `stream`: a copy of x into a device staging buffer owned by the
+ * handle, the GEMV, and a copy of y back to y_host.  With page-locked
+ * (pinned) host buffers the call returns without waiting and y_host is valid
+ * once `stream` has been synchronised; with pageable buffers the CUDA runtime
+ * makes the copies synchronous.  Same numerics, alignment-free host pointers;
+ * the staging buffer makes concurrent calls on one handle invalid, as for
+ * sphq_gemv.
+ */
+sphq_status sphq_gemv_host(sphq_handle h, const void* x_host, void* y_host, int batch,
+                           sphq_stream stream);
+
+/*
+ * sphq_decode -- write the decoded weights W_hat (rows x cols fp16, device
+ * pointer, 16-byte aligned) on `stream`.  Bit-exact with Eq. (7) + Eq. (4) as
+ * stated at the top of this header.  For verification; the GEMV never
+ * materialises W_hat.  Asynchronous; no allocation.
+ */
+sphq_status sphq_decode(sphq_handle h, void* w, sphq_stream stream);
+
+/*
+ * sphq_bytes -- algorithmic bytes one gemv of this batch moves: packed codes
+ * (2.25 or 3.125 bits per weight) + group parameters (4 bytes per 128 weights)
+ * + codebook (K*16 bytes, once) + activations (2*batch*cols) + outputs
+ * (2*batch*rows).  Returns 0 for a NULL handle or a batch outside 1..8.
+ */
+size_t sphq_bytes(sphq_handle h, int batch);
+
+/* Release the handle and its device memory.  NULL is accepted.  The caller
+ * ensures no kernel using the handle is still running. */
+sphq_status sphq_destroy(sphq_handle h);
+
+/* Message describing the last error returned on the calling thread ("" if none). */
+const char* sphq_last_error(void);
+
+/* Library ABI version (major*10000 + minor*100 + patch). */
+int sphq_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SPHQ_H_ */

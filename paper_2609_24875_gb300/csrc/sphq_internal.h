@@ -1,0 +1,54 @@
+// Host-side internals of the sphq library (not part of the C ABI).
+#pragma once
+#include <cuda_runtime.h>
+
+#include <cstddef>
+#include <cstdint>
+#include <string>
+
+#include "../../include/sphq.h"
+
+namespace sphq {
+
+// Launch plan of the GEMV kernel for one batch size.
+struct GemvPlan {
+  int warps_per_cta = 0;   // threads / 32
+  int grid = 0;            // CTAs (persistent: at most SMs x resident CTAs)
+  int units_per_warp = 0;  // contiguous (row block, group) units per warp
+  int max_slots = 0;       // most warps that share one row block
+  size_t smem = 0;         // dynamic shared memory per CTA
+};
+
+}  // namespace sphq
+
+struct sphq_handle_s {
+  int rows = 0, cols = 0, bits = 0, K = 0;
+  int nrb = 0;             // row blocks of 32 rows
+  int ng = 0;              // radius groups per row (cols / 128)
+  int device = 0;
+  int sm_count = 0;
+  size_t tile_bytes = 0;
+  void* tiles = nullptr;       // packed group tiles, nrb * ng * tile_bytes
+  void* codebook = nullptr;    // K * 8 fp16
+  uint32_t* params = nullptr;  // rows * ng words: Delta | r_min << 16
+  float* ws = nullptr;         // split-K partial sums
+  size_t ws_floats = 0;
+  unsigned* tickets = nullptr; // one arrival counter per row block
+  int* flag = nullptr;         // pack validation flag
+  void* xstage = nullptr;      // SPHQ_MAX_BATCH x cols fp16 (sphq_gemv_host)
+  void* ystage = nullptr;      // SPHQ_MAX_BATCH x rows fp16
+  bool packed = false;
+  sphq::GemvPlan plan[SPHQ_MAX_BATCH + 1];
+};
+
+namespace sphq {
+
+sphq_status set_error(sphq_status s, const std::string& msg);
+sphq_status cuda_error(cudaError_t e, const char* what);
+
+// Builds the GEMV launch plans of a handle (sizes its workspace needs).
+sphq_status make_gemv_plans(sphq_handle h);
+// Enqueues the GEMV (validated arguments).
+sphq_status launch_gemv(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s);
+
+}  // namespace sphq

@@ -1,0 +1,177 @@
+"""Thin Python binding of libsphq.so (include/sphq.h): argument marshalling only.
+
+Every step of the decode-GEMV runs in the library's CUDA kernels; PyTorch is
+used here only to own device memory and to name the current CUDA stream.
+If the library has not been built this module raises on import of the
+library -- there is no CPU fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libsphq.so")
+HEADER = os.path.join(os.path.dirname(HERE), "include", "sphq.h")
+
+SPHQ_OK = 0
+STATUS = {0: "SPHQ_OK", 1: "SPHQ_ERR_INVALID_ARG", 2: "SPHQ_ERR_UNSUPPORTED",
+          3: "SPHQ_ERR_NOT_PACKED", 4: "SPHQ_ERR_CUDA", 5: "SPHQ_ERR_OOM",
+          6: "SPHQ_ERR_DEVICE"}
+MAX_BATCH = 8
+
+_lib = None
+
+
+class SphqError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"{STATUS.get(status, status)}: {msg}")
+        self.status = status
+
+
+def load() -> ctypes.CDLL:
+    """Load libsphq.so (built by __graft_entry__.build()); raises if missing."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(
+                f"{LIB_PATH} is missing: build the CUDA library first "
+                "(python -c 'import __graft_entry__ as g; g.build()')")
+        L = ctypes.CDLL(LIB_PATH)
+        vp, i32, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
+        L.sphq_create.argtypes = [i32, i32, i32, i32, vp, vp, vp, ctypes.POINTER(vp)]
+        L.sphq_create.restype = i32
+        L.sphq_pack.argtypes = [vp, vp, vp, vp, vp]
+        L.sphq_pack.restype = i32
+        L.sphq_gemv.argtypes = [vp, vp, vp, i32, vp]
+        L.sphq_gemv.restype = i32
+        L.sphq_gemv_host.argtypes = [vp, vp, vp, i32, vp]
+        L.sphq_gemv_host.restype = i32
+        L.sphq_decode.argtypes = [vp, vp, vp]
+        L.sphq_decode.restype = i32
+        L.sphq_bytes.argtypes = [vp, i32]
+        L.sphq_bytes.restype = sz
+        L.sphq_destroy.argtypes = [vp]
+        L.sphq_destroy.restype = i32
+        L.sphq_last_error.argtypes = []
+        L.sphq_last_error.restype = ctypes.c_char_p
+        L.sphq_version.argtypes = []
+        L.sphq_version.restype = i32
+        _lib = L
+    return _lib
+
+
+def header_functions() -> list[str]:
+    """Names of the functions include/sphq.h declares."""
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(sphq_[a-z_0-9]+)\s*\(", text)))
+
+
+def _check(status: int) -> None:
+    if status != SPHQ_OK:
+        raise SphqError(status, load().sphq_last_error().decode())
+
+
+def _stream_ptr(stream) -> int:
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return int(stream.cuda_stream)
+
+
+class SphqMatrix:
+    """One quantised weight matrix resident on the current CUDA device.
+
+    codebook: (K, 8) float16/uint16 tensor; scale, offset: (rows, cols/128).
+    Host or device tensors are accepted for these three (they are copied).
+    """
+
+    def __init__(self, rows: int, cols: int, bits: int, codebook, scale, offset):
+        import torch
+        L = load()
+        K = 1 << (7 * bits - 8)
+        cb = codebook.contiguous()
+        sc = scale.contiguous()
+        of = offset.contiguous()
+        for t, shape in ((cb, (K, 8)), (sc, (rows, cols // 128)), (of, (rows, cols // 128))):
+            if tuple(t.shape) != shape or t.element_size() != 2:
+                raise ValueError(f"expected a 2-byte tensor of shape {shape}, got "
+                                 f"{tuple(t.shape)} {t.dtype}")
+        h = ctypes.c_void_p()
+        _check(L.sphq_create(rows, cols, bits, K, cb.data_ptr(), sc.data_ptr(), of.data_ptr(),
+                             ctypes.byref(h)))
+        self._h = h
+        self.rows, self.cols, self.bits, self.K = rows, cols, bits, K
+        self.device = torch.device("cuda", torch.cuda.current_device())
+
+    @property
+    def handle(self) -> int:
+        return self._h.value
+
+    def pack(self, sign, idx, rcode, stream=None) -> None:
+        """sign/idx/rcode: (rows, cols/8) uint8 / uint16(int16) / uint8 device tensors."""
+        nv = self.cols // 8
+        for t in (sign, idx, rcode):
+            if tuple(t.shape) != (self.rows, nv) or not t.is_cuda or not t.is_contiguous():
+                raise ValueError("codes must be contiguous CUDA tensors of shape (rows, cols/8)")
+        if sign.element_size() != 1 or rcode.element_size() != 1 or idx.element_size() != 2:
+            raise ValueError("sign/rcode must be 1-byte and idx 2-byte tensors")
+        _check(load().sphq_pack(self._h, sign.data_ptr(), idx.data_ptr(), rcode.data_ptr(),
+                                _stream_ptr(stream)))
+
+    def gemv(self, x, y=None, stream=None):
+        """y = W_hat x.  x: (batch, cols) fp16 on the device; returns (batch, rows) fp16."""
+        import torch
+        if x.dim() == 1:
+            x = x.unsqueeze(0)
+        B = x.shape[0]
+        if x.shape[1] != self.cols or x.element_size() != 2 or not x.is_cuda:
+            raise ValueError("x must be a (batch, cols) 2-byte CUDA tensor")
+        x = x.contiguous()
+        if y is None:
+            y = torch.empty((B, self.rows), dtype=torch.float16, device=x.device)
+        _check(load().sphq_gemv(self._h, x.data_ptr(), y.data_ptr(), B, _stream_ptr(stream)))
+        return y
+
+    def gemv_ptr(self, x_ptr: int, y_ptr: int, batch: int, stream_ptr: int) -> None:
+        """Raw-pointer call (no tensor checks), for graph capture and benchmarks."""
+        _check(load().sphq_gemv(self._h, x_ptr, y_ptr, batch, stream_ptr))
+
+    def gemv_host(self, x_host, y_host, stream=None) -> None:
+        """Host-buffer GEMV: x_host (batch, cols) and y_host (batch, rows) are
+        2-byte CPU tensors (pinned for asynchrony); the copies and the GEMV are
+        enqueued on the stream, so synchronise it before reading y_host."""
+        if x_host.is_cuda or y_host.is_cuda:
+            raise ValueError("gemv_host takes host tensors")
+        if x_host.dim() == 1:
+            x_host = x_host.unsqueeze(0)
+        B = x_host.shape[0]
+        if (x_host.shape[1] != self.cols or tuple(y_host.shape[-1:]) != (self.rows,)
+                or not x_host.is_contiguous() or not y_host.is_contiguous()
+                or y_host.numel() != B * self.rows):
+            raise ValueError("x_host must be (batch, cols) and y_host (batch, rows), contiguous")
+        _check(load().sphq_gemv_host(self._h, x_host.data_ptr(), y_host.data_ptr(), B,
+                                     _stream_ptr(stream)))
+
+    def decode(self, stream=None):
+        """W_hat as a (rows, cols) fp16 tensor (verification path)."""
+        import torch
+        w = torch.empty((self.rows, self.cols), dtype=torch.float16, device=self.device)
+        _check(load().sphq_decode(self._h, w.data_ptr(), _stream_ptr(stream)))
+        return w
+
+    def bytes(self, batch: int = 1) -> int:
+        return int(load().sphq_bytes(self._h, batch))
+
+    def close(self) -> None:
+        if getattr(self, "_h", None) is not None and self._h.value:
+            load().sphq_destroy(self._h)
+            self._h = ctypes.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
