@@ -13,6 +13,8 @@
 namespace sphq {
 
 static thread_local std::string g_last_error;
+// zero block read by GEMV lanes that supply no activations (4 words x 4 lanes x 16 B)
+constexpr size_t kZeroBytes = 256;
 
 sphq_status set_error(sphq_status s, const std::string& msg) {
   g_last_error = msg;
@@ -32,79 +34,93 @@ sphq_status cuda_error(cudaError_t e, const char* what) {
   } while (0)
 
 // ---------------------------------------------------------------------------
-// pack: canonical codes -> group tiles (the finalise-and-pack step, App. A step 10)
+// pack: canonical codes -> units (the finalise-and-pack step, App. A step 10)
 // ---------------------------------------------------------------------------
 
-// One thread per (row block, group, lane): composes the lane's part of a tile.
+// One thread per (unit, lane): composes the lane's four words and its share of
+// the quad records.  The unit buffer is zeroed before the launch, so padded
+// rows keep zero codes and byte-wise record writes need no read-modify-write.
 template <int BITS>
 __global__ void pack_kernel(const uint8_t* __restrict__ sign, const uint16_t* __restrict__ idx,
                             const uint8_t* __restrict__ rcode,
                             const uint16_t* __restrict__ scale,
-                            const uint16_t* __restrict__ offset, uint8_t* __restrict__ tiles,
-                            int rows, int ng, int nrb, int* __restrict__ flag) {
+                            const uint16_t* __restrict__ offset, uint8_t* __restrict__ units,
+                            int rows, int ng, int nrt, int* __restrict__ flag) {
   const long long tid = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-  const long long total = (long long)nrb * ng * kRowsPerBlock;
+  const long long total = (long long)nrt * ng * 32;
   if (tid >= total) return;
-  const int lane = (int)(tid % kRowsPerBlock);
-  const long long unit = tid / kRowsPerBlock;  // rb * ng + g
+  const int lane = (int)(tid & 31);
+  const long long unit = tid >> 5;  // rt * ng + g
   const int g = (int)(unit % ng);
-  const int rb = (int)(unit / ng);
-  const int row = rb * kRowsPerBlock + lane;
+  const int rt = (int)(unit / ng);
+  const int gid = lane >> 2, q = lane & 3;
   const int nv = ng * kGroupVecs;
-  uint8_t* tile = tiles + (size_t)unit * Layout<BITS>::kTileBytes;
+  uint8_t* base = units + (size_t)unit * Layout<BITS>::kUnitBytes;
 
-  uint32_t words[kGroupVecs];
-  uint32_t aux0 = 0, aux1 = 0, aux2 = 0, aux3 = 0, top = 0, params = 0;
+  uint32_t words[4] = {0, 0, 0, 0};
+  uint32_t e_lo = 0, e_hi = 0;       // W2: pair-3 sign bytes of the lane
+  uint32_t mid = 0, qn = 0, top = 0; // W3
   bool bad = false;
-  for (int j = 0; j < kGroupVecs; ++j) {
-    uint32_t s = 0, k = 0, q = 0;
-    if (row < rows) {
-      const size_t v = (size_t)row * nv + (size_t)g * kGroupVecs + j;
-      s = sign[v];
-      k = idx[v];
-      q = rcode[v];
-      if (k >= (uint32_t)Layout<BITS>::K || q > 15u) {
-        bad = true;
-        k = 0;
-        q = 0;
+  for (int m = 0; m < 4; ++m) {
+    for (int half = 0; half < 2; ++half) {  // 0: A (row gid), 1: B (row gid + 8)
+      const int row = rt * kRowsPerTile + gid + 8 * half;
+      uint32_t s = 0, k = 0, rq = 0;
+      if (row < rows) {
+        const size_t v = (size_t)row * nv + (size_t)g * kGroupVecs + 4 * m + q;
+        s = sign[v];
+        k = idx[v];
+        rq = rcode[v];
+        if (k >= (uint32_t)Layout<BITS>::K || rq > 15u) {
+          bad = true;
+          k = 0;
+          rq = 0;
+        }
       }
-    }
-    if (BITS == 2) {
-      words[j] = s | (k << 8) | ((q & 3u) << 14);
-      aux0 |= ((q >> 2) & 3u) << (2 * j);
-    } else {
-      words[j] = s | ((k & 0xFFu) << 8);
-      const int n = 4 * (j & 7);
-      if (j < 8) {
-        aux0 |= q << n;
-        aux2 |= ((k >> 8) & 0xFu) << n;
+      const int v8 = 2 * m + half;   // vector number within the lane, 0..7
+      const int hs = 16 * half;      // B's index/radius fields sit 16 bits higher
+      // sign bits 2p / 2p+1 go to bits (top - p) / (top - p + 16), where top is
+      // 15 for A and, below A's bits, 12 (W2) or 11 (W3) for B
+      const int top_bit = half == 0 ? 15 : (BITS == 2 ? 12 : 11);
+      const int npairs = BITS == 2 ? 3 : 4;
+      uint32_t w = 0;
+      for (int p = 0; p < npairs; ++p) {
+        w |= ((s >> (2 * p)) & 1u) << (top_bit - p);
+        w |= ((s >> (2 * p + 1)) & 1u) << (top_bit - p + 16);
+      }
+      if (BITS == 2) {
+        w |= (rq | (k << 4)) << hs;
+        e_lo |= ((s >> 6) & 1u) << (7 - v8);
+        e_hi |= ((s >> 7) & 1u) << (7 - v8);
       } else {
-        aux1 |= q << n;
-        aux3 |= ((k >> 8) & 0xFu) << n;
+        w |= (k & 0xFFu) << hs;
+        qn |= rq << (4 * m + hs);
+        mid |= ((k >> 8) & 0xFu) << (((8 + 4 * m) & 15) + hs);
+        top |= ((k >> 12) & 1u) << (4 * q + m + hs);
       }
-      top |= ((k >> 12) & 1u) << j;
+      words[m] |= w;
     }
-  }
-  if (row < rows) {
-    const size_t gi = (size_t)row * ng + g;
-    params = (uint32_t)scale[gi] | ((uint32_t)offset[gi] << 16);
   }
   if (bad) atomicOr(flag, 1);
-  for (int c = 0; c < 2; ++c) {
-    uint4 v;
-    v.x = words[8 * c + 0] | (words[8 * c + 1] << 16);
-    v.y = words[8 * c + 2] | (words[8 * c + 3] << 16);
-    v.z = words[8 * c + 4] | (words[8 * c + 5] << 16);
-    v.w = words[8 * c + 6] | (words[8 * c + 7] << 16);
-    *reinterpret_cast<uint4*>(tile + c * 512 + lane * 16) = v;
-  }
+  *reinterpret_cast<uint4*>(base + lane * 16) = make_uint4(words[0], words[1], words[2], words[3]);
+  uint32_t pa = 0, pb = 0;
+  const int ra = rt * kRowsPerTile + gid, rb = ra + 8;
+  if (ra < rows) pa = (uint32_t)scale[(size_t)ra * ng + g] | ((uint32_t)offset[(size_t)ra * ng + g] << 16);
+  if (rb < rows) pb = (uint32_t)scale[(size_t)rb * ng + g] | ((uint32_t)offset[(size_t)rb * ng + g] << 16);
   if (BITS == 2) {
-    *reinterpret_cast<uint2*>(tile + Layout<2>::kAuxOff + lane * 8) = make_uint2(aux0, params);
+    uint8_t* rec = base + Layout<2>::kRecOff + gid * 16;
+    uint8_t* sw = rec + 4 * (q >> 1);          // S01 or S23
+    const int b0 = (q & 1) ? 0 : 1;            // even lane: bytes 1, 3; odd lane: bytes 0, 2
+    sw[b0] = (uint8_t)e_lo;
+    sw[b0 + 2] = (uint8_t)e_hi;
+    if (q == 0) {
+      *reinterpret_cast<uint32_t*>(rec + 8) = pa;
+      *reinterpret_cast<uint32_t*>(rec + 12) = pb;
+    }
   } else {
-    *reinterpret_cast<uint4*>(tile + Layout<3>::kAuxOff + lane * 16) =
-        make_uint4(aux0, aux1, aux2, aux3);
-    *reinterpret_cast<uint32_t*>(tile + Layout<3>::kParamOff + lane * 4) = params;
-    *reinterpret_cast<uint16_t*>(tile + Layout<3>::kTopOff + lane * 2) = (uint16_t)top;
+    *reinterpret_cast<uint2*>(base + Layout<3>::kMidOff + lane * 8) = make_uint2(mid, qn);
+    if (q == 0)
+      *reinterpret_cast<uint2*>(base + Layout<3>::kParamOff + gid * 8) = make_uint2(pa, pb);
+    atomicOr(reinterpret_cast<unsigned*>(base + Layout<3>::kTopOff + gid * 4), top);
   }
 }
 
@@ -113,21 +129,36 @@ __global__ void pack_kernel(const uint8_t* __restrict__ sign, const uint16_t* __
 // ---------------------------------------------------------------------------
 
 template <int BITS>
-__global__ void decode_kernel(const uint8_t* __restrict__ tiles, const uint4* __restrict__ codebook,
+__global__ void decode_kernel(const uint8_t* __restrict__ units, const uint8_t* __restrict__ codebook,
                               uint16_t* __restrict__ w, int rows, int cols, int ng) {
   const long long tid = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   const int nv = cols / kVec;
   if (tid >= (long long)rows * nv) return;
   const int row = (int)(tid / nv);
   const int t = (int)(tid % nv);
-  const int rb = row / kRowsPerBlock, lane = row % kRowsPerBlock;
-  const int g = t / kGroupVecs, j = t % kGroupVecs;
-  const uint8_t* tile = tiles + ((size_t)rb * ng + g) * Layout<BITS>::kTileBytes;
-  const GroupData<BITS> d = load_group<BITS>(tile, lane);
-  const Fields f = unpack(d, j);
-  const uint16_t r = radius16(f.q, d.params);
-  const uint4 c = codebook[f.k];
-  *reinterpret_cast<uint4*>(w + (size_t)row * cols + (size_t)t * kVec) = reconstruct(f.sign, r, c);
+  const int rt = row / kRowsPerTile, r16 = row % kRowsPerTile;
+  const int gid = r16 & 7, half = r16 >> 3;
+  const int g = t / kGroupVecs, s = t % kGroupVecs;
+  const int m = s >> 2, q = s & 3;
+  const int lane = 4 * gid + q;
+  const uint8_t* unit = units + ((size_t)rt * ng + g) * Layout<BITS>::kUnitBytes;
+  const Unit<BITS> u = load_unit<BITS>(unit, lane);
+  GlobalCodebook cb{codebook};
+  uint4 sa, sb;
+  uint32_t r;
+  if constexpr (BITS == 2) {
+    const uint32_t W = word_of(u.w, m);
+    directions_w2(W, w2_sign3(u, q), m, cb, 0u, false, sa, sb);
+    r = radius_pair(qpair_w2(W), params_delta(u.rec.z, u.rec.w), params_rmin(u.rec.z, u.rec.w));
+  } else {
+    directions_w3(u, m, q, cb, sa, sb);
+    r = radius_pair(qpair_w3(u, m), params_delta(u.par.x, u.par.y),
+                    params_rmin(u.par.x, u.par.y));
+  }
+  // Eq. (4): w_hat = RN16(r_hat * (s (.) c))
+  const uint4 wa = scale_block(sa, bcast_lo(r));
+  const uint4 wb = scale_block(sb, bcast_hi(r));
+  *reinterpret_cast<uint4*>(w + (size_t)row * cols + (size_t)t * kVec) = half ? wb : wa;
 }
 
 }  // namespace sphq
@@ -142,7 +173,7 @@ const char* sphq_last_error(void) { return g_last_error.c_str(); }
 
 static void free_handle(sphq_handle h) {
   if (!h) return;
-  cudaFree(h->tiles);
+  cudaFree(h->units);
   cudaFree(h->codebook);
   cudaFree(h->params);
   cudaFree(h->ws);
@@ -150,6 +181,7 @@ static void free_handle(sphq_handle h) {
   cudaFree(h->flag);
   cudaFree(h->xstage);
   cudaFree(h->ystage);
+  cudaFree(h->zeros);
   delete h;
 }
 
@@ -167,7 +199,7 @@ sphq_status sphq_create(int rows, int cols, int bits, int K, const void* codeboo
     return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_create: K must be 2^(7*bits-8)");
   if (!codebook || !scale || !offset)
     return set_error(SPHQ_ERR_INVALID_ARG, "sphq_create: NULL codebook/scale/offset");
-  const long long nrb = (rows + kRowsPerBlock - 1) / kRowsPerBlock;
+  const long long nrt = (rows + kRowsPerTile - 1) / kRowsPerTile;
   const long long ng = cols / kGroupCols;
   if ((long long)rows * cols > (1LL << 40))
     return set_error(SPHQ_ERR_INVALID_ARG, "sphq_create: matrix too large");
@@ -184,24 +216,26 @@ sphq_status sphq_create(int rows, int cols, int bits, int K, const void* codeboo
   h->cols = cols;
   h->bits = bits;
   h->K = K;
-  h->nrb = (int)nrb;
+  h->nrt = (int)nrt;
   h->ng = (int)ng;
   h->device = dev;
   h->sm_count = prop.multiProcessorCount;
-  h->tile_bytes = bits == 2 ? Layout<2>::kTileBytes : Layout<3>::kTileBytes;
+  h->unit_bytes = bits == 2 ? Layout<2>::kUnitBytes : Layout<3>::kUnitBytes;
 
   auto fail = [&](sphq_status s) {
     free_handle(h);
     return s;
   };
   cudaError_t e;
-  if ((e = cudaMalloc(&h->tiles, (size_t)nrb * ng * h->tile_bytes)) != cudaSuccess)
-    return fail(cuda_error(e, "cudaMalloc(tiles)"));
+  // two guard units after the last one: the GEMV prefetches up to two units
+  // past a warp's span without bounds checks
+  if ((e = cudaMalloc(&h->units, ((size_t)nrt * ng + 2) * h->unit_bytes)) != cudaSuccess)
+    return fail(cuda_error(e, "cudaMalloc(units)"));
   if ((e = cudaMalloc(&h->codebook, (size_t)K * 16)) != cudaSuccess)
     return fail(cuda_error(e, "cudaMalloc(codebook)"));
   if ((e = cudaMalloc(&h->params, (size_t)rows * ng * 4)) != cudaSuccess)
     return fail(cuda_error(e, "cudaMalloc(params)"));
-  if ((e = cudaMalloc(&h->tickets, (size_t)nrb * sizeof(unsigned))) != cudaSuccess)
+  if ((e = cudaMalloc(&h->tickets, (size_t)nrt * sizeof(unsigned))) != cudaSuccess)
     return fail(cuda_error(e, "cudaMalloc(tickets)"));
   if ((e = cudaMalloc(&h->flag, sizeof(int))) != cudaSuccess)
     return fail(cuda_error(e, "cudaMalloc(flag)"));
@@ -209,6 +243,10 @@ sphq_status sphq_create(int rows, int cols, int bits, int K, const void* codeboo
     return fail(cuda_error(e, "cudaMalloc(x staging)"));
   if ((e = cudaMalloc(&h->ystage, (size_t)SPHQ_MAX_BATCH * rows * 2)) != cudaSuccess)
     return fail(cuda_error(e, "cudaMalloc(y staging)"));
+  if ((e = cudaMalloc(&h->zeros, kZeroBytes)) != cudaSuccess)
+    return fail(cuda_error(e, "cudaMalloc(zeros)"));
+  if ((e = cudaMemset(h->zeros, 0, kZeroBytes)) != cudaSuccess)
+    return fail(cuda_error(e, "memset zeros"));
   if ((e = cudaMemcpy(h->codebook, codebook, (size_t)K * 16, cudaMemcpyDefault)) != cudaSuccess)
     return fail(cuda_error(e, "copy codebook"));
   // params are kept as two planes (scale, offset) until pack interleaves them
@@ -218,7 +256,7 @@ sphq_status sphq_create(int rows, int cols, int bits, int K, const void* codeboo
     return fail(cuda_error(e, "copy scale"));
   if ((e = cudaMemcpy(p16 + np, offset, np * 2, cudaMemcpyDefault)) != cudaSuccess)
     return fail(cuda_error(e, "copy offset"));
-  if ((e = cudaMemset(h->tickets, 0, (size_t)nrb * sizeof(unsigned))) != cudaSuccess)
+  if ((e = cudaMemset(h->tickets, 0, (size_t)nrt * sizeof(unsigned))) != cudaSuccess)
     return fail(cuda_error(e, "memset tickets"));
   sphq_status st = make_gemv_plans(h);
   if (st != SPHQ_OK) return fail(st);
@@ -241,16 +279,18 @@ sphq_status sphq_pack(sphq_handle h, const uint8_t* sign, const uint16_t* idx,
   const uint16_t* scale = reinterpret_cast<const uint16_t*>(h->params);
   const uint16_t* offset = scale + (size_t)h->rows * h->ng;
   SPHQ_CUDA(cudaMemsetAsync(h->flag, 0, sizeof(int), s), "memset flag");
-  SPHQ_CUDA(cudaMemsetAsync(h->tickets, 0, (size_t)h->nrb * sizeof(unsigned), s), "memset tickets");
-  const long long threads = (long long)h->nrb * h->ng * kRowsPerBlock;
+  SPHQ_CUDA(cudaMemsetAsync(h->tickets, 0, (size_t)h->nrt * sizeof(unsigned), s), "memset tickets");
+  SPHQ_CUDA(cudaMemsetAsync(h->units, 0, ((size_t)h->nrt * h->ng + 2) * h->unit_bytes, s),
+            "memset units");
+  const long long threads = (long long)h->nrt * h->ng * 32;
   const int block = 256;
   const unsigned grid = (unsigned)((threads + block - 1) / block);
   if (h->bits == 2)
     pack_kernel<2><<<grid, block, 0, s>>>(sign, idx, rcode, scale, offset,
-                                          (uint8_t*)h->tiles, h->rows, h->ng, h->nrb, h->flag);
+                                          (uint8_t*)h->units, h->rows, h->ng, h->nrt, h->flag);
   else
     pack_kernel<3><<<grid, block, 0, s>>>(sign, idx, rcode, scale, offset,
-                                          (uint8_t*)h->tiles, h->rows, h->ng, h->nrb, h->flag);
+                                          (uint8_t*)h->units, h->rows, h->ng, h->nrt, h->flag);
   SPHQ_CUDA(cudaGetLastError(), "pack kernel launch");
   int flag = 0;
   SPHQ_CUDA(cudaMemcpyAsync(&flag, h->flag, sizeof(int), cudaMemcpyDeviceToHost, s), "read flag");
@@ -273,10 +313,10 @@ sphq_status sphq_decode(sphq_handle h, void* w, sphq_stream stream) {
   const int block = 256;
   const unsigned grid = (unsigned)((n + block - 1) / block);
   if (h->bits == 2)
-    decode_kernel<2><<<grid, block, 0, s>>>((const uint8_t*)h->tiles, (const uint4*)h->codebook,
+    decode_kernel<2><<<grid, block, 0, s>>>((const uint8_t*)h->units, (const uint8_t*)h->codebook,
                                             (uint16_t*)w, h->rows, h->cols, h->ng);
   else
-    decode_kernel<3><<<grid, block, 0, s>>>((const uint8_t*)h->tiles, (const uint4*)h->codebook,
+    decode_kernel<3><<<grid, block, 0, s>>>((const uint8_t*)h->units, (const uint8_t*)h->codebook,
                                             (uint16_t*)w, h->rows, h->cols, h->ng);
   SPHQ_CUDA(cudaGetLastError(), "decode kernel launch");
   return SPHQ_OK;

@@ -17,26 +17,28 @@ struct GemvPlan {
   int units_per_warp = 0;  // contiguous (row block, group) units per warp
   int max_slots = 0;       // most warps that share one row block
   size_t smem = 0;         // dynamic shared memory per CTA
+  int mode = 0;            // radius application: 1, 2 (factored) or 8 (full)
 };
 
 }  // namespace sphq
 
 struct sphq_handle_s {
   int rows = 0, cols = 0, bits = 0, K = 0;
-  int nrb = 0;             // row blocks of 32 rows
+  int nrt = 0;             // row tiles of 16 rows
   int ng = 0;              // radius groups per row (cols / 128)
   int device = 0;
   int sm_count = 0;
-  size_t tile_bytes = 0;
-  void* tiles = nullptr;       // packed group tiles, nrb * ng * tile_bytes
+  size_t unit_bytes = 0;
+  void* units = nullptr;       // packed units, nrt * ng * unit_bytes
   void* codebook = nullptr;    // K * 8 fp16
   uint32_t* params = nullptr;  // rows * ng words: Delta | r_min << 16
   float* ws = nullptr;         // split-K partial sums
   size_t ws_floats = 0;
-  unsigned* tickets = nullptr; // one arrival counter per row block
+  unsigned* tickets = nullptr; // one arrival counter per row tile
   int* flag = nullptr;         // pack validation flag
   void* xstage = nullptr;      // SPHQ_MAX_BATCH x cols fp16 (sphq_gemv_host)
   void* ystage = nullptr;      // SPHQ_MAX_BATCH x rows fp16
+  void* zeros = nullptr;       // 256 B of zeros (activations of non-supplying lanes)
   bool packed = false;
   sphq::GemvPlan plan[SPHQ_MAX_BATCH + 1];
 };

@@ -1,32 +1,49 @@
 // Device layout of packed SPHQuant codes and the per-vector decode shared by
 // the GEMV and decode kernels.  sm_103a only.
 //
-// Device layout ("group tiles").  Rows are padded to a multiple of 32 and cut
-// into row blocks of 32 rows (one row per lane of a warp).  For row block rb
-// and radius group g (16 consecutive 8-D vectors = 128 columns, §3.1) one
-// contiguous tile holds, for each of the 32 rows, the group's 16 vectors:
+// Tiles.  Rows are padded to a multiple of 16 and cut into row tiles of 16
+// rows (the M extent of one m16n8k16 MMA).  For row tile rt and radius group g
+// (16 consecutive 8-D vectors = 128 columns, §3.1) one contiguous "unit" holds
+// the 256 vectors (16 rows x 16 slots) in the order the GEMV's threads consume
+// them: lane l = 4*gid + q (gid = l/4, q = l%4) owns rows gid and gid+8 at the
+// group's slots q, 4+q, 8+q, 12+q.  Its 16-byte block holds four 32-bit words
+// w_m (m = 0..3); word w_m holds vector A = (row gid, slot 4m+q) and vector
+// B = (row gid+8, slot 4m+q).  Units are stored in (rt, g) order, so a warp
+// that walks the groups of one row tile streams contiguous memory and every
+// warp-wide 16-byte load is a 512-byte burst.
 //
-//   W2 (1280 B = 32 rows x 40 B: 2.25 bits/weight + 4 B of group parameters)
-//     [0, 1024)     codes: chunk c in {0,1} (vectors 8c..8c+7), lane l:
-//                   16 B at c*512 + l*16 = eight 16-bit words in the paper's
-//                   W2 format (§3.4): bits [0,8) signs, [8,14) direction
-//                   index, [14,16) the low 2 bits of the radius code
-//     [1024, 1280)  lane l: 8 B at 1024 + l*8 = { the paper's per-group 32-bit
-//                   word of high radius bits (vector j at bits [2j, 2j+2)),
-//                   params = Delta_G (low 16 bits) | r_min_G (high 16 bits) }
+// W2 unit (640 B = 256 x 2.25 bits + 16 x 4 B of group parameters, §3.1, §3.4):
+//   [0, 512)    lane l: words w_0..w_3 at 16*l, bits of w_m:
+//                 0-3 radius code of A   4-9 direction index of A
+//                 16-19 radius code of B 20-25 direction index of B
+//                 15,31 / 14,30 / 13,29  sign bits (2p, 2p+1) of A, pairs p = 0,1,2
+//                 12,28 / 11,27 / 10,26  sign bits of B, pairs p = 0,1,2
+//   [512, 640)  quad gid (lanes 4gid..4gid+3): 16 B at 512 + 16*gid =
+//                 { S01, S23, P_gid, P_gid+8 }
+//                 S01: the sign bits 6, 7 of lane q=0's eight vectors in bits
+//                      8-15 / 24-31 and of lane q=1's in bits 0-7 / 16-23
+//                      (vector v = 2m + {0: A, 1: B}: bit 15-v = s6, bit 31-v = s7)
+//                 S23: the same for lanes q = 2, 3
+//                 P_r: Delta_G (low 16 bits) | r_min_G (high 16 bits) of row r
+//   The bit positions make each sign mask one shift of a loaded word away
+//   from bits 15/31 (the fp16 sign bits of a half2 register) and the two
+//   radius codes of a word one AND away from two fp16 integers.
 //
-//   W3 (1728 B = 32 rows x 54 B: 3.125 bits/weight + 4 B of group parameters)
-//     [0, 1024)     codes: as W2 but each 16-bit word = signs (bits 0-7) |
-//                   index bits 0-7 (bits 8-15)
-//     [1024, 1536)  lane l: 16 B = { radius codes of vectors 0-7 (nibble j),
-//                   radius codes 8-15, index bits 8-11 of vectors 0-7
-//                   (nibble j), index bits 8-11 of vectors 8-15 }
-//     [1536, 1664)  lane l: 4 B params, as W2
-//     [1664, 1728)  lane l: 2 B, bit j = index bit 12 of vector j
+// W3 unit (864 B = 256 x 3.125 bits + 64 B of group parameters):
+//   [0, 512)    lane l: words w_0..w_3, bits of w_m:
+//                 0-7 direction index bits 0-7 of A, 16-23 of B
+//                 15,31 / 14,30 / 13,29 / 12,28  sign bits of A, pairs 0..3
+//                 11,27 / 10,26 /  9,25 /  8,24  sign bits of B, pairs 0..3
+//   [512, 768)  lane l: 8 B at 512 + 8*l = { MID, QN }
+//                 QN:  radius codes, word m: A at bits 4m..4m+3, B at 16+4m..
+//                 MID: index bits 8-11, word m: A at bits 8-11 rotated right by
+//                      4m (m=0: 8-11, 1: 12-15, 2: 0-3, 3: 4-7), B 16 bits higher
+//   [768, 832)  quad gid: 8 B = { P_gid, P_gid+8 }
+//   [832, 864)  quad gid: 4 B, bit (4q + m) = index bit 12 of A of lane q's
+//                 word m, bit (16 + 4q + m) = that of B
 //
-// Tiles are stored in (rb, g) order, so a warp that walks the groups of one
-// row block streams contiguous memory, and each warp-wide 16-byte load is
-// 512 contiguous bytes.  No byte beyond the algorithmic payload is stored.
+// No byte beyond the algorithmic payload is stored; padded rows hold zero
+// codes and parameters.
 #pragma once
 #include <cstdint>
 
@@ -35,123 +52,79 @@ namespace sphq {
 constexpr int kVec = 8;                 // 8-D vectors (§3.1)
 constexpr int kGroupVecs = 16;          // vectors per radius group
 constexpr int kGroupCols = kVec * kGroupVecs;
-constexpr int kRowsPerBlock = 32;       // rows per tile (one per lane)
+constexpr int kRowsPerTile = 16;        // rows per unit (MMA M)
 constexpr int kMaxBatch = 8;
+constexpr uint32_t kSignMask = 0x80008000u;
 
 template <int BITS> struct Layout;
 template <> struct Layout<2> {
   static constexpr int K = 64;
-  static constexpr int kTileBytes = 1280;
-  static constexpr int kAuxOff = 1024;
+  static constexpr int kUnitBytes = 640;
+  static constexpr int kRecOff = 512;
 };
 template <> struct Layout<3> {
   static constexpr int K = 8192;
-  static constexpr int kTileBytes = 1728;
-  static constexpr int kAuxOff = 1024;
-  static constexpr int kParamOff = 1536;
-  static constexpr int kTopOff = 1664;
+  static constexpr int kUnitBytes = 864;
+  static constexpr int kMidOff = 512;
+  static constexpr int kParamOff = 768;
+  static constexpr int kTopOff = 832;
 };
 
-// Per-lane data of one group tile.
-template <int BITS> struct GroupData;
-template <> struct GroupData<2> {
-  uint4 code[2];      // 16 x 16-bit words
-  uint32_t extra;     // high radius bits
-  uint32_t params;    // Delta | r_min << 16 (fp16 bits)
+// Per-lane data of one unit.
+template <int BITS> struct Unit;
+template <> struct Unit<2> {
+  uint4 w;      // words w_0..w_3
+  uint4 rec;    // quad record {S01, S23, P_gid, P_gid+8}
 };
-template <> struct GroupData<3> {
-  uint4 code[2];      // 16 x (signs | index bits 0-7)
-  uint4 aux;          // radius nibbles (x: 0-7, y: 8-15), index-hi nibbles (z: 0-7, w: 8-15)
-  uint32_t params;
-  uint32_t top;       // 16 bits: index bit 12
+template <> struct Unit<3> {
+  uint4 w;
+  uint2 mq;     // {MID, QN}
+  uint2 par;    // {P_gid, P_gid+8}
+  uint32_t top; // index bit 12 of the quad
 };
 
+// Code streams are read once: cache them in L2 only, never in L1.
 __device__ __forceinline__ uint4 ldg_stream16(const void* p) {
   uint4 v;
-  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+  asm volatile("ld.global.cg.v4.u32 {%0,%1,%2,%3}, [%4];"
                : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
   return v;
 }
 __device__ __forceinline__ uint2 ldg_stream8(const void* p) {
   uint2 v;
-  asm volatile("ld.global.nc.L1::no_allocate.v2.u32 {%0,%1}, [%2];"
+  asm volatile("ld.global.cg.v2.u32 {%0,%1}, [%2];"
                : "=r"(v.x), "=r"(v.y) : "l"(p));
   return v;
 }
 __device__ __forceinline__ uint32_t ldg_stream4(const void* p) {
   uint32_t v;
-  asm volatile("ld.global.nc.L1::no_allocate.u32 %0, [%1];" : "=r"(v) : "l"(p));
-  return v;
-}
-__device__ __forceinline__ uint32_t ldg_stream2(const void* p) {
-  unsigned short v;
-  asm volatile("ld.global.nc.L1::no_allocate.u16 %0, [%1];" : "=h"(v) : "l"(p));
+  asm volatile("ld.global.cg.u32 %0, [%1];" : "=r"(v) : "l"(p));
   return v;
 }
 
 template <int BITS>
-__device__ __forceinline__ GroupData<BITS> load_group(const uint8_t* tile, int lane);
+__device__ __forceinline__ Unit<BITS> load_unit(const uint8_t* unit, int lane);
 
 template <>
-__device__ __forceinline__ GroupData<2> load_group<2>(const uint8_t* tile, int lane) {
-  GroupData<2> d;
-  d.code[0] = ldg_stream16(tile + lane * 16);
-  d.code[1] = ldg_stream16(tile + 512 + lane * 16);
-  uint2 a = ldg_stream8(tile + Layout<2>::kAuxOff + lane * 8);
-  d.extra = a.x;
-  d.params = a.y;
-  return d;
+__device__ __forceinline__ Unit<2> load_unit<2>(const uint8_t* unit, int lane) {
+  Unit<2> u;
+  u.w = ldg_stream16(unit + lane * 16);
+  u.rec = ldg_stream16(unit + Layout<2>::kRecOff + (lane >> 2) * 16);
+  return u;
 }
 
 template <>
-__device__ __forceinline__ GroupData<3> load_group<3>(const uint8_t* tile, int lane) {
-  GroupData<3> d;
-  d.code[0] = ldg_stream16(tile + lane * 16);
-  d.code[1] = ldg_stream16(tile + 512 + lane * 16);
-  d.aux = ldg_stream16(tile + Layout<3>::kAuxOff + lane * 16);
-  d.params = ldg_stream4(tile + Layout<3>::kParamOff + lane * 4);
-  d.top = ldg_stream2(tile + Layout<3>::kTopOff + lane * 2);
-  return d;
+__device__ __forceinline__ Unit<3> load_unit<3>(const uint8_t* unit, int lane) {
+  Unit<3> u;
+  u.w = ldg_stream16(unit + lane * 16);
+  u.mq = ldg_stream8(unit + Layout<3>::kMidOff + lane * 8);
+  u.par = ldg_stream8(unit + Layout<3>::kParamOff + (lane >> 2) * 8);
+  u.top = ldg_stream4(unit + Layout<3>::kTopOff + (lane >> 2) * 4);
+  return u;
 }
 
-__device__ __forceinline__ uint32_t word16(const GroupData<2>& d, int j) {
-  const uint4& c = d.code[j >> 3];
-  const int w = (j >> 1) & 3;
-  uint32_t v = (w == 0) ? c.x : (w == 1) ? c.y : (w == 2) ? c.z : c.w;
-  return (j & 1) ? (v >> 16) : (v & 0xFFFFu);
-}
-__device__ __forceinline__ uint32_t word16(const GroupData<3>& d, int j) {
-  const uint4& c = d.code[j >> 3];
-  const int w = (j >> 1) & 3;
-  uint32_t v = (w == 0) ? c.x : (w == 1) ? c.y : (w == 2) ? c.z : c.w;
-  return (j & 1) ? (v >> 16) : (v & 0xFFFFu);
-}
-
-// Unpacked fields of vector j (0..15) of a group: sign byte, direction index,
-// radius code.  j must be a compile-time constant after unrolling.
-struct Fields {
-  uint32_t sign, k, q;
-};
-
-__device__ __forceinline__ Fields unpack(const GroupData<2>& d, int j) {
-  const uint32_t w = word16(d, j);
-  Fields f;
-  f.sign = w & 0xFFu;
-  f.k = (w >> 8) & 0x3Fu;
-  f.q = (w >> 14) | (((d.extra >> (2 * j)) & 3u) << 2);
-  return f;
-}
-
-__device__ __forceinline__ Fields unpack(const GroupData<3>& d, int j) {
-  const uint32_t w = word16(d, j);
-  const uint32_t qw = (j < 8) ? d.aux.x : d.aux.y;
-  const uint32_t hw = (j < 8) ? d.aux.z : d.aux.w;
-  const int n = 4 * (j & 7);
-  Fields f;
-  f.sign = w & 0xFFu;
-  f.k = (w >> 8) | (((hw >> n) & 0xFu) << 8) | (((d.top >> j) & 1u) << 12);
-  f.q = (qw >> n) & 0xFu;
-  return f;
+__device__ __forceinline__ uint32_t word_of(const uint4& w, int m) {
+  return m == 0 ? w.x : m == 1 ? w.y : m == 2 ? w.z : w.w;
 }
 
 // ---------------------------------------------------------------------------
@@ -163,65 +136,166 @@ __device__ __forceinline__ uint32_t hmul2_rn(uint32_t a, uint32_t b) {
   asm("mul.rn.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
   return d;
 }
-
-__device__ __forceinline__ uint16_t hfma_rn(uint16_t a, uint16_t b, uint16_t c) {
-  uint16_t d;
-  asm("fma.rn.f16 %0, %1, %2, %3;" : "=h"(d) : "h"(a), "h"(b), "h"(c));
-  return d;
-}
-
-__device__ __forceinline__ uint16_t hsub_rn(uint16_t a, uint16_t b) {
-  uint16_t d;
-  asm("sub.rn.f16 %0, %1, %2;" : "=h"(d) : "h"(a), "h"(b));
-  return d;
-}
-
-// r_hat = RN16(q * Delta + r_min): Eq. (7), one fp16 fused multiply-add.
-// q (0..15) becomes an exact fp16 value through 1024 + q (bits 0x6400 | q) - 1024.
-__device__ __forceinline__ uint16_t radius16(uint32_t q, uint32_t params) {
-  const uint16_t qh = hsub_rn((uint16_t)(0x6400u | q), (uint16_t)0x6400u);
-  return hfma_rn(qh, (uint16_t)(params & 0xFFFFu), (uint16_t)(params >> 16));
-}
-
-// Sign mask for coordinate pair p (coordinates 2p, 2p+1) of a half2 register.
-__device__ __forceinline__ uint32_t sign_mask(uint32_t s, int p) {
-  const uint32_t t = s >> (2 * p);
-  return ((t << 15) & 0x8000u) | ((t << 30) & 0x80000000u);
-}
-
-// w_hat = s (.) RN16(r_hat * c): Eq. (4) on one block, as four half2 pairs.
-__device__ __forceinline__ uint4 reconstruct(uint32_t sign, uint16_t r_hat, uint4 c) {
-  const uint32_t r2 = (uint32_t)r_hat | ((uint32_t)r_hat << 16);
-  uint4 w;
-  w.x = hmul2_rn(r2, c.x) ^ sign_mask(sign, 0);
-  w.y = hmul2_rn(r2, c.y) ^ sign_mask(sign, 1);
-  w.z = hmul2_rn(r2, c.z) ^ sign_mask(sign, 2);
-  w.w = hmul2_rn(r2, c.w) ^ sign_mask(sign, 3);
-  return w;
-}
-
-// acc += w.lo * x.lo + w.hi * x.hi with fp16 inputs and fp32 accumulation:
-// each product is exact in fp32 and added with one rounding.
-__device__ __forceinline__ float fma_h2_f32(uint32_t w2, uint32_t x2, float acc) {
-  asm("{\n\t.reg .f16 wl, wh, xl, xh;\n\t"
-      "mov.b32 {wl, wh}, %1;\n\t"
-      "mov.b32 {xl, xh}, %2;\n\t"
-      "fma.rn.f32.f16 %0, wl, xl, %0;\n\t"
-      "fma.rn.f32.f16 %0, wh, xh, %0;\n\t}"
-      : "+f"(acc) : "r"(w2), "r"(x2));
-  return acc;
-}
-
-__device__ __forceinline__ uint32_t f32x2_to_h2_rn(float lo, float hi) {
+__device__ __forceinline__ uint32_t hfma2_rn(uint32_t a, uint32_t b, uint32_t c) {
   uint32_t d;
-  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+  asm("fma.rn.f16x2 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
   return d;
 }
-
+__device__ __forceinline__ uint32_t hsub2_rn(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
+}
+template <uint32_t SEL>
+__device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "n"(SEL));
+  return d;
+}
+// a << S as an integer multiply-add: it issues to the FMA pipe instead of the
+// (half-rate, busier) integer ALU pipe that the masks and XORs use.
+template <int S>
+__device__ __forceinline__ uint32_t shl_fma(uint32_t a) {
+  if constexpr (S == 0) {
+    return a;
+  } else {
+    uint32_t d;
+    asm("mad.lo.u32 %0, %1, %2, 0;" : "=r"(d) : "r"(a), "n"(1u << S));
+    return d;
+  }
+}
+__device__ __forceinline__ uint32_t shl_fma_rt(uint32_t a, int s) {
+  uint32_t d;
+  asm("mad.lo.u32 %0, %1, %2, 0;" : "=r"(d) : "r"(a), "r"(1u << s));
+  return d;
+}
+__device__ __forceinline__ uint32_t rotl(uint32_t a, uint32_t n) {
+  uint32_t d;
+  asm("shf.l.wrap.b32 %0, %1, %1, %2;" : "=r"(d) : "r"(a), "r"(n));
+  return d;
+}
 __device__ __forceinline__ uint16_t f32_to_h_rn(float v) {
   uint16_t d;
   asm("cvt.rn.f16.f32 %0, %1;" : "=h"(d) : "f"(v));
   return d;
 }
+
+// Radius pair of one word, Eq. (7): r_hat = RN16(q * Delta + r_min) with one
+// fp16 fused multiply-add per vector.  qpair holds the codes of A (bits 0-3)
+// and B (bits 16-19); 1024 + q is an exact fp16 value (bits 0x6400 | q), so
+// subtracting 1024 gives q exactly.  d2 / m2: (Delta, r_min) of rows (A, B).
+__device__ __forceinline__ uint32_t radius_pair(uint32_t qpair, uint32_t d2, uint32_t m2) {
+  const uint32_t qh = (qpair & 0x000F000Fu) | 0x64006400u;
+  return hfma2_rn(hsub2_rn(qh, 0x64006400u), d2, m2);
+}
+
+// Sign flip of one block: the signed unit direction s (.) c as four half2
+// pairs.  masks m_p carry sign bits (2p, 2p+1) at bits 15 and 31 (the fp16
+// sign bits of a half2 register); other bits are ignored.
+__device__ __forceinline__ uint4 apply_signs(uint4 c, uint32_t m0, uint32_t m1, uint32_t m2,
+                                             uint32_t m3) {
+  return make_uint4(c.x ^ (m0 & kSignMask), c.y ^ (m1 & kSignMask), c.z ^ (m2 & kSignMask),
+                    c.w ^ (m3 & kSignMask));
+}
+
+// Eq. (4) for one block: w_hat = RN16(r_hat * (s (.) c)).  Flipping the sign of
+// c before the product equals flipping the rounded product (round-to-nearest
+// is symmetric, and the sign of a product of zeros is the XOR of the signs).
+__device__ __forceinline__ uint4 scale_block(uint4 a, uint32_t r2) {
+  return make_uint4(hmul2_rn(r2, a.x), hmul2_rn(r2, a.y), hmul2_rn(r2, a.z), hmul2_rn(r2, a.w));
+}
+
+__device__ __forceinline__ uint32_t bcast_lo(uint32_t r) { return prmt<0x1010u>(r, 0u); }
+__device__ __forceinline__ uint32_t bcast_hi(uint32_t r) { return prmt<0x3232u>(r, 0u); }
+
+__device__ __forceinline__ uint4 lds16(uint32_t saddr) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(saddr));
+  return v;
+}
+
+// Codebook access.  W2: eight interleaved copies in shared memory, entry k of
+// copy c at byte 128*k + 16*c; lane l uses copy l % 8 (the eight lanes of a
+// quarter-warp then touch eight distinct 16-byte bank groups).  W3: a single
+// copy, entry k at byte 16*k.  `base` is a shared-memory address, or for the
+// global-memory variant used by the decode kernel a generic pointer.
+struct SmemCodebook {
+  const uint8_t* base;  // the shared-memory table (a __shared__ array)
+  uint32_t copyoff;     // W2: 16 * (lane % 8), W3: 0
+  __device__ __forceinline__ uint4 at(uint32_t off) const {
+    return *reinterpret_cast<const uint4*>(base + off);
+  }
+};
+struct GlobalCodebook {
+  const uint8_t* base;  // K x 16 B
+  __device__ __forceinline__ uint4 at(uint32_t off) const {
+    return *reinterpret_cast<const uint4*>(base + off);
+  }
+};
+
+// Signed directions of the two vectors of word m of a W2 unit (A = row gid,
+// B = row gid+8).  `e` is the lane's pair-3 sign word aligned to bits 8-15 /
+// 24-31.  Codebook offsets: 128*k + copy offset (interleaved smem copies) or
+// 16*k (a plain table).
+template <class CB>
+__device__ __forceinline__ void directions_w2(uint32_t W, uint32_t e, int m, const CB& cb,
+                                              uint32_t copyoff, bool interleaved, uint4& sa,
+                                              uint4& sb) {
+  const uint32_t w3 = shl_fma<3>(W);
+  uint32_t offA, offB;
+  if (interleaved) {
+    offA = (w3 & 0x1F80u) | copyoff;
+    offB = ((W >> 13) & 0x1F80u) | copyoff;
+  } else {
+    offA = (W & 0x3F0u);
+    offB = (W >> 16) & 0x3F0u;
+  }
+  const uint4 ca = cb.at(offA);
+  const uint4 cbv = cb.at(offB);
+  const uint32_t ea = shl_fma_rt(e, 2 * m);
+  const uint32_t eb = shl_fma_rt(e, 2 * m + 1);
+  sa = apply_signs(ca, W, shl_fma<1>(W), shl_fma<2>(W), ea);
+  sb = apply_signs(cbv, w3, shl_fma<4>(W), shl_fma<5>(W), eb);
+}
+
+// The lane's pair-3 sign word of a W2 unit, aligned to bits 8-15 / 24-31.
+__device__ __forceinline__ uint32_t w2_sign3(const Unit<2>& u, int q) {
+  const uint32_t s = (q & 2) ? u.rec.y : u.rec.x;
+  return (q & 1) ? (s << 8) : s;
+}
+__device__ __forceinline__ uint32_t params_delta(uint32_t pa, uint32_t pb) {
+  return prmt<0x5410u>(pa, pb);
+}
+__device__ __forceinline__ uint32_t params_rmin(uint32_t pa, uint32_t pb) {
+  return prmt<0x7632u>(pa, pb);
+}
+
+// Signed directions of word m of a W3 unit.  The index-bit-12 word is
+// rotated by (12 - 4q - m) mod 32 to bring the lane's pair to bits 12 / 28.
+template <class CB>
+__device__ __forceinline__ void directions_w3(const Unit<3>& u, int m, int q, const CB& cb,
+                                              uint4& sa, uint4& sb) {
+  const uint32_t W = word_of(u.w, m);
+  uint32_t mid;
+  if (m == 0) mid = u.mq.x;
+  else if (m == 1) mid = u.mq.x >> 4;
+  else if (m == 2) mid = shl_fma<8>(u.mq.x);
+  else mid = shl_fma<4>(u.mq.x);
+  const uint32_t top = rotl(u.top, (uint32_t)(12 - 4 * q - m) & 31u);
+  // bits 8-11 from mid, bit 12 from top (bits above 12 / 28 are don't-care)
+  const uint32_t hi = (mid & 0x0F000F00u) | (top & ~0x0F000F00u);
+  const uint32_t k2 = (W & 0x00FF00FFu) | (hi & ~0x00FF00FFu);
+  const uint32_t offA = shl_fma<4>(k2) & 0x1FFF0u;
+  const uint32_t offB = (k2 >> 12) & 0x1FFF0u;
+  const uint4 ca = cb.at(offA);
+  const uint4 cbv = cb.at(offB);
+  sa = apply_signs(ca, W, shl_fma<1>(W), shl_fma<2>(W), shl_fma<3>(W));
+  sb = apply_signs(cbv, shl_fma<4>(W), shl_fma<5>(W), shl_fma<6>(W), shl_fma<7>(W));
+}
+
+// Radius codes of word m as a pair (A at bits 0-3, B at bits 16-19).
+__device__ __forceinline__ uint32_t qpair_w2(uint32_t W) { return W; }
+__device__ __forceinline__ uint32_t qpair_w3(const Unit<3>& u, int m) { return u.mq.y >> (4 * m); }
 
 }  // namespace sphq
