@@ -137,6 +137,41 @@ sphq_status sphq_gemv_host(sphq_handle h, const void* x_host, void* y_host, int 
                            sphq_stream stream);
 
 /*
+ * sphq_gemv_noalloc -- sphq_gemv for callers that must not allocate GPU memory
+ * at run time.  (This entry point has no counterpart in the paper; it is an
+ * interface choice of this library.)
+ *
+ * Who needs it: code that may not call cudaMalloc/cudaFree (or any allocator)
+ * on its serving path -- a real-time decode loop, because cudaMalloc and
+ * cudaFree synchronise the device and their latency is unbounded; programs
+ * that reserve all device memory up front or run under a fixed memory budget;
+ * and callers that hold their own allocator's lock or run inside a region
+ * where allocation is not allowed.  sphq_gemv itself does not allocate either
+ * (sphq_create allocated the handle's workspace), but this variant also works
+ * for handles whose workspace memory the caller would rather not keep per
+ * matrix: its split-K scratch is a single fixed 4 MiB device array compiled
+ * into the library, which every GPU that loads the library holds until the
+ * process exits.
+ *
+ * Arguments, numerics and asynchrony are those of sphq_gemv.  It calls no
+ * cudaMalloc, cudaFree or other allocating routine.  Limits: the matrix may
+ * have at most 16384 row tiles (rows <= 262144) and may need at most
+ * 4128768 bytes of partial sums; larger shapes return SPHQ_ERR_UNSUPPORTED
+ * with a message naming the limit.  The current device must be the handle's
+ * device (else SPHQ_ERR_DEVICE).
+ *
+ * The first call on each device looks up the array's device address (one
+ * cudaGetSymbolAddress with that device current) and caches it; make that
+ * first call before any stream capture.  All calls share the one array and it
+ * keeps the last call's contents: each call clears the counters it uses (an
+ * asynchronous memset on `stream`), and calls that overlap on the GPU -- on
+ * different streams or from different host threads -- race on the array and
+ * give wrong results.  Serialise them, e.g. on one stream.
+ */
+sphq_status sphq_gemv_noalloc(sphq_handle h, const void* x, void* y, int batch,
+                              sphq_stream stream);
+
+/*
  * sphq_decode -- write the decoded weights W_hat (rows x cols fp16, device
  * pointer, 16-byte aligned) on `stream`.  Bit-exact with Eq. (7) + Eq. (4) as
  * stated at the top of this header.  For verification; the GEMV never

@@ -547,4 +547,41 @@ sphq_status launch_gemv(sphq_handle h, const void* x, void* y, int batch, cudaSt
   return SPHQ_OK;
 }
 
+// Same launch as launch_gemv, with caller-provided split-K scratch (partials
+// and per-row-tile tickets) instead of the handle's own workspace.
+sphq_status launch_gemv_scratch(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s,
+                                float* ws, unsigned* tickets) {
+  const GemvPlan& p = h->plan[batch];
+  GemvArgs a;
+  a.units = (const uint8_t*)h->units;
+  a.codebook = (const uint4*)h->codebook;
+  a.x = (const uint16_t*)x;
+  a.y = (uint16_t*)y;
+  a.ws = ws;
+  a.tickets = tickets;
+  a.rows = h->rows;
+  a.cols = h->cols;
+  a.ng = h->ng;
+  a.nrt = h->nrt;
+  a.batch = batch;
+  a.units_per_warp = p.units_per_warp;
+  a.max_slots = p.max_slots;
+  a.total_units = (long long)h->nrt * h->ng;
+  a.zeros = (const uint16_t*)h->zeros;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.grid);
+  cfg.blockDim = dim3(p.warps_per_cta * 32);
+  cfg.dynamicSmemBytes = p.smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  void* args[] = {&a};
+  cudaError_t e = cudaLaunchKernelExC(&cfg, select_kernel(h->bits, p.mode), args);
+  if (e != cudaSuccess) return cuda_error(e, "gemv launch");
+  return SPHQ_OK;
+}
+
 }  // namespace sphq

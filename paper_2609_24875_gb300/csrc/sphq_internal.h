@@ -52,5 +52,9 @@ sphq_status cuda_error(cudaError_t e, const char* what);
 sphq_status make_gemv_plans(sphq_handle h);
 // Enqueues the GEMV (validated arguments).
 sphq_status launch_gemv(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s);
+// Enqueues the GEMV with caller-provided split-K scratch: `ws` holds at least
+// h->ws_floats floats and `tickets` h->nrt zeroed counters.
+sphq_status launch_gemv_scratch(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s,
+                                float* ws, unsigned* tickets);
 
 }  // namespace sphq

@@ -139,6 +139,23 @@ class SphqMatrix:
         """Raw-pointer call (no tensor checks), for graph capture and benchmarks."""
         _check(load().sphq_gemv(self._h, x_ptr, y_ptr, batch, stream_ptr))
 
+    def gemv_noalloc(self, x, y, stream=None):
+        """sphq_gemv_noalloc: the GEMV with the library's fixed device scratch
+        instead of the handle's workspace (no allocation on any call).
+        x: (batch, cols) and y: (batch, rows) fp16 CUDA tensors."""
+        L = load()
+        L.sphq_gemv_noalloc.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
+                                        ctypes.c_int, ctypes.c_void_p]
+        L.sphq_gemv_noalloc.restype = ctypes.c_int
+        if x.dim() == 1:
+            x = x.unsqueeze(0)
+        B = x.shape[0]
+        if (x.shape[1] != self.cols or not x.is_cuda or not y.is_cuda
+                or not x.is_contiguous() or not y.is_contiguous() or y.numel() != B * self.rows):
+            raise ValueError("x must be (batch, cols) and y (batch, rows), contiguous CUDA tensors")
+        _check(L.sphq_gemv_noalloc(self._h, x.data_ptr(), y.data_ptr(), B, _stream_ptr(stream)))
+        return y
+
     def gemv_host(self, x_host, y_host, stream=None) -> None:
         """Host-buffer GEMV: x_host (batch, cols) and y_host (batch, rows) are
         2-byte CPU tensors (pinned for asynchrony); the copies and the GEMV are
