@@ -2,23 +2,28 @@
 """Benchmark of the SPHQuant decode GEMV on GB300 (one JSON line on stdout).
 
 Workload (one "step" = one pass of the hot path over one batch of input):
-  the batch-1 W2/W3 GEMV sweep at 4096x4096 and 8192x8192.  Each shape has a
-  pool of distinct packed matrices whose total size exceeds twice the L2
-  cache, and a step runs one GEMV on every matrix of every pool (each pool
-  captured once as a CUDA graph of back-to-back launches on one stream), so
-  every GEMV streams its codes from HBM.  Codes are seeded uniformly random
-  codes of the encoded configuration's shapes (the data path and byte count
-  do not depend on the code values; parity on encoder-produced codes is
-  covered by the tests).
+  1. the batch-1 W2/W3 GEMV sweep at 4096x4096 and 8192x8192.  Each shape has
+     a pool of distinct packed matrices whose total size exceeds twice the L2
+     cache, and a step runs one GEMV on every matrix of every pool, so every
+     GEMV streams its codes from HBM;
+  2. one token through the 28-layer x 7-projection linear stack of a
+     7B-class decoder at W2 and at W3 (196 distinct matrices each, batch 1).
+  Each pool and each stack is captured once as a CUDA graph of back-to-back
+  launches on one stream.  Codes are seeded uniformly random codes of the
+  encoded configuration's shapes (the data path and byte count do not depend
+  on the code values; parity on encoder-produced codes is covered by the
+  tests).
 
-value    = algorithmic bytes of all GEMVs / device time of the timed steps (GB/s)
+value    = algorithmic bytes of all GEMVs of a step / device time per step (GB/s)
+sweep    = per shape: us per GEMV, GB/s and fraction of HBM (CUDA events
+           around each pool's graph)
+stack    = us per token for the W2 and W3 stacks (CUDA events around each)
 roofline = the dominant kernel's algorithmic bytes per launch / its average
            launch time (CUDA events on the launching stream), against the
            measured HBM copy bandwidth
 e2e      = the same metric through sphq_gemv_host (pinned host x in, y out,
-           copies inside the timed region), one GEMV per shape per step
-stack    = the 28-layer x 7-projection linear stack of a 7B-class decoder at
-           W2 and W3, batch 1, chained on one stream in a CUDA graph: us/token
+           copies inside the timed region), one GEMV per sweep shape per step
+clocks   = nvidia-smi samples taken while the timed steps run
 
 --impl reference runs the float64 CPU oracle (the reference arm of this
 build) on bounded row samples of the same workload.
@@ -67,23 +72,29 @@ class ClockSampler:
     def __init__(self, index: int):
         self.index = index
         self.proc = None
-        self.lines = []
+        self.lines = []  # (host time, csv line)
+        self.window = None
 
     def __enter__(self):
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "100"],
+                 "--format=csv,noheader,nounits", "-lms", "50"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.t = threading.Thread(target=self._read, daemon=True)
             self.t.start()
         except (FileNotFoundError, OSError):
             self.proc = None
+        time.sleep(1.0)  # nvidia-smi start-up; samples before the window are dropped
         return self
 
     def _read(self):
         for line in self.proc.stdout:
-            self.lines.append(line.strip())
+            self.lines.append((time.perf_counter(), line.strip()))
+
+    def mark(self, t0: float, t1: float):
+        """Host times bracketing the timed region (enqueue .. synchronize)."""
+        self.window = (t0, t1)
 
     def __exit__(self, *exc):
         if self.proc is not None:
@@ -97,7 +108,9 @@ class ClockSampler:
     def summary(self):
         sm, mx, reasons = [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for ln in self.lines:
+        for ts, ln in self.lines:
+            if self.window is not None and not (self.window[0] <= ts <= self.window[1]):
+                continue
             p = [t.strip() for t in ln.split(",")]
             if len(p) < 8:
                 continue
@@ -212,11 +225,14 @@ def run_gpu(args, world, rank, local):
         ys = [torch.empty((1, n), dtype=torch.float16, device=dev) for _ in mats]
         g = capture(mats, xd, ys, stream)
         shapes.append(dict(name=f"W{bits} {n}x{n}", bits=bits, n=n, mats=mats, xd=xd, ys=ys,
-                           graph=g, bytes=mats[0].bytes(1), P=P))
+                           graph=g, bytes=mats[0].bytes(1), P=P, launches=P))
+    # --- the W2 and W3 decoder stacks ---
+    stacks = [] if args.no_stack else [make_stack(args, bits, dev, stream) for bits in (2, 3)]
+    parts = shapes + stacks
     torch.cuda.synchronize()
 
     def step(evs=None):
-        for i, s in enumerate(shapes):
+        for i, s in enumerate(parts):
             if evs is not None:
                 evs[i][0].record(stream)
             s["graph"].replay()
@@ -229,51 +245,68 @@ def run_gpu(args, world, rank, local):
     torch.cuda.synchronize()
 
     K = args.steps
-    ev = [[[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in shapes]
+    ev = [[[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in parts]
           for _ in range(K)]
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     dist_barrier(world)
     torch.cuda.synchronize()
     with ClockSampler(local) as clk:
+        h0 = time.perf_counter()
         with torch.cuda.stream(stream):
             t0.record(stream)
             for k in range(K):
                 step(ev[k])
             t1.record(stream)
         torch.cuda.synchronize()
+        clk.mark(h0, time.perf_counter())
     dist_barrier(world)
     total_ms = t0.elapsed_time(t1)
     total_ms = dist_max(world, total_ms)
-    per_shape_ms = [sum(ev[k][i][0].elapsed_time(ev[k][i][1]) for k in range(K))
-                    for i in range(len(shapes))]
-    launches = sum(s["P"] for s in shapes) * K
-    step_bytes = sum(s["P"] * s["bytes"] for s in shapes)
+    part_ms = [sum(ev[k][i][0].elapsed_time(ev[k][i][1]) for k in range(K))
+               for i in range(len(parts))]
+    launches = sum(s["launches"] for s in parts) * K
+    step_bytes = sum(s["P"] * s["bytes"] for s in parts)
     value = step_bytes * K * world / (total_ms * 1e-3) / 1e9
 
     sweep = {}
-    for s, ms in zip(shapes, per_shape_ms):
+    for s, ms in zip(shapes, part_ms):
         us = ms * 1e3 / (K * s["P"])
         gbs = s["bytes"] / (us * 1e-6) / 1e9
         sweep[s["name"]] = {"us_per_gemv": round(us, 3), "GB/s": round(gbs, 1),
                             "hbm_frac": round(gbs / hbm_peak, 4), "bytes": s["bytes"],
                             "pool": s["P"]}
-    dom = max(range(len(shapes)), key=lambda i: per_shape_ms[i])
-    ds = shapes[dom]
-    d_us = per_shape_ms[dom] * 1e3 / (K * ds["P"])
-    achieved = ds["bytes"] / (d_us * 1e-6) / 1e9
+    stack = {}
+    for s, ms in zip(stacks, part_ms[len(shapes):]):
+        us = ms * 1e3 / K
+        gbs = s["bytes"] / (us * 1e-6) / 1e9
+        stack[s["name"]] = {"us_per_token": round(us, 2), "layers": s["layers"], "gemvs": s["launches"],
+                            "bytes_per_token": s["bytes"], "GB/s": round(gbs, 1),
+                            "hbm_frac": round(gbs / hbm_peak, 4)}
+    # dominant kernel: the instantiation (W2 or W3, batch 1) with the most
+    # device time per step, over all its launches in the step
+    per_bits = {}
+    for s, ms in zip(parts, part_ms):
+        b = per_bits.setdefault(s["bits"], [0.0, 0, 0])
+        b[0] += ms
+        b[1] += s["P"] * s["bytes"]
+        b[2] += s["launches"]
+    dom_bits = max(per_bits, key=lambda b: per_bits[b][0])
+    d_ms, d_bytes, d_launches = per_bits[dom_bits]
+    achieved = d_bytes * K / (d_ms * 1e-3) / 1e9
     roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm_peak,
                 "unit": "GB/s", "frac": round(achieved / hbm_peak, 4),
-                "traffic": None, "kernel": f"gemv_kernel ({ds['name']}, batch 1)",
+                "traffic": None,
+                "kernel": f"gemv_kernel W{dom_bits} batch 1 ({d_launches} launches/step, "
+                          f"{round(100 * d_ms / sum(part_ms), 1)}% of step device time)",
+                "bytes_per_launch": round(d_bytes / d_launches),
+                "us_per_launch": round(d_ms * 1e3 / (K * d_launches), 3),
                 "peak_kind": peak_kind}
 
     # --- end to end through the host-buffer entry point ---
     e2e = run_e2e(args, shapes, stream)
 
-    # --- 28-layer linear stack ---
-    stack = None if args.no_stack else run_stack(args, dev, stream, hbm_peak)
-
-    for s in shapes:
+    for s in parts:
         for m in s["mats"]:
             m.close()
     out = {
@@ -281,12 +314,14 @@ def run_gpu(args, world, rank, local):
         "steps": K, "warmup": args.warmup, "ms_per_step": round(total_ms / K, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "fp16 in, fp32 accumulate (2.25/3.125-bit codes)", "data": "synthetic",
-        "config": {"workload": "W2+W3 GEMV sweep 4096^2 and 8192^2, batch 1",
+        "config": {"workload": "W2+W3 GEMV sweep 4096^2 and 8192^2 + 28-layer W2/W3 "
+                               "decoder linear stack, batch 1",
                    "pools": {s["name"]: s["P"] for s in shapes},
-                   "l2_policy": "each pool > 2x L2, distinct buffers per GEMV",
+                   "l2_policy": "inputs larger than L2: each pool > 2x L2 and each stack "
+                                "> 10x L2, distinct buffers per GEMV",
                    "parallelism": f"replicas x{world}"},
         "hbm_frac": round(value / hbm_peak, 4),
-        "sweep": sweep, "roofline": roofline, "e2e": e2e, "stack": stack,
+        "sweep": sweep, "stack": stack or None, "roofline": roofline, "e2e": e2e,
         "gpu_launches": launches,
     }
     return out, clk.summary()
@@ -316,62 +351,40 @@ def run_e2e(args, shapes, stream):
             "us_per_step": round(dt / K * 1e6, 2)}
 
 
-def run_stack(args, dev, stream, hbm_peak):
+def make_stack(args, bits, dev, stream):
+    """The 28-layer x 7-projection linear stack at `bits`, as one CUDA graph
+    of its 196 GEMVs in layer order (one distinct packed matrix each)."""
     import torch
 
     from paper_2609_24875_gb300 import SphqMatrix
-    res = {}
     layers = 2 if args.quick else inp.DECODER_LAYERS
-    for bits in (2, 3):
-        mats, ys, xs = [], [], []
-        # one seeded code set per projection shape, packed into a distinct
-        # buffer per layer (28 x 7 distinct matrices, 6.5e9 weights)
-        for i, (name, rows, cols) in enumerate(inp.DECODER_PROJ):
-            codes, x = inp.random_codes(bits, rows, cols, seed=inp.seed_for(4, 10 * bits + i))
-            t = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int16) if a.dtype == np.uint16 else a)).to(dev)
-            cb, sc, of = t(codes.codebook), t(codes.scale), t(codes.offset)
-            sg, ix, rc = t(codes.sign), t(codes.idx), t(codes.rcode)
-            xd = t(x).view(torch.float16)
-            for l in range(layers):
-                m = SphqMatrix(rows, cols, bits, cb, sc, of)
-                m.pack(sg, ix, rc)
-                mats.append((l, i, m))
-                xs.append(xd)
-                ys.append(torch.empty((1, rows), dtype=torch.float16, device=dev))
-            del sg, ix, rc
-        order = sorted(range(len(mats)), key=lambda j: (mats[j][0], mats[j][1]))
-        seq = [(mats[j][2], xs[j], ys[j]) for j in order]
-        with torch.cuda.stream(stream):
-            for m, xd, yd in seq:
-                m.gemv_ptr(xd.data_ptr(), yd.data_ptr(), 1, stream.cuda_stream)
-        stream.synchronize()
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g, stream=stream):
-            for m, xd, yd in seq:
-                m.gemv_ptr(xd.data_ptr(), yd.data_ptr(), 1, stream.cuda_stream)
-        for _ in range(3):
-            g.replay()
-        torch.cuda.synchronize()
-        reps = max(3, min(args.steps, 20))
-        e0 = torch.cuda.Event(enable_timing=True)
-        e1 = torch.cuda.Event(enable_timing=True)
-        with torch.cuda.stream(stream):
-            e0.record(stream)
-            for _ in range(reps):
-                g.replay()
-            e1.record(stream)
-        torch.cuda.synchronize()
-        us = e0.elapsed_time(e1) * 1e3 / reps
-        byts = sum(m.bytes(1) for m, _, _ in seq)
-        gbs = byts / (us * 1e-6) / 1e9
-        res[f"W{bits}"] = {"us_per_token": round(us * inp.DECODER_LAYERS / layers, 2),
-                           "layers_timed": layers, "gemvs": len(seq),
-                           "GB/s": round(gbs, 1), "hbm_frac": round(gbs / hbm_peak, 4)}
-        del g
-        for m, _, _ in seq:
-            m.close()
-        torch.cuda.empty_cache()
-    return res
+    mats, ys, xs = [], [], []
+    for i, (name, rows, cols) in enumerate(inp.DECODER_PROJ):
+        codes, x = inp.random_codes(bits, rows, cols, seed=inp.seed_for(4, 10 * bits + i))
+        t = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int16) if a.dtype == np.uint16 else a)).to(dev)
+        cb, sc, of = t(codes.codebook), t(codes.scale), t(codes.offset)
+        sg, ix, rc = t(codes.sign), t(codes.idx), t(codes.rcode)
+        xd = t(x).view(torch.float16)
+        for l in range(layers):
+            m = SphqMatrix(rows, cols, bits, cb, sc, of)
+            m.pack(sg, ix, rc)
+            mats.append((l, i, m))
+            xs.append(xd)
+            ys.append(torch.empty((1, rows), dtype=torch.float16, device=dev))
+        del sg, ix, rc
+    order = sorted(range(len(mats)), key=lambda j: (mats[j][0], mats[j][1]))
+    seq = [(mats[j][2], xs[j], ys[j]) for j in order]
+    with torch.cuda.stream(stream):
+        for m, xd, yd in seq:
+            m.gemv_ptr(xd.data_ptr(), yd.data_ptr(), 1, stream.cuda_stream)
+    stream.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for m, xd, yd in seq:
+            m.gemv_ptr(xd.data_ptr(), yd.data_ptr(), 1, stream.cuda_stream)
+    return dict(name=f"W{bits}", bits=bits, graph=g, mats=[m for m, _, _ in seq], keep=(xs, ys),
+                layers=layers,
+                bytes=sum(m.bytes(1) for m, _, _ in seq), P=1, launches=len(seq))
 
 
 # ---------------------------------------------------------------------------
@@ -442,10 +455,10 @@ def run_reference(args, world, rank):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--quick", action="store_true", help="small pools / 2 stack layers")
+    ap.add_argument("--quick", action="store_true", help="pools of 2 / 2 stack layers (smoke runs)")
     ap.add_argument("--no-stack", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
