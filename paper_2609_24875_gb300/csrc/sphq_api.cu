@@ -50,9 +50,9 @@ __global__ void pack_kernel(const uint8_t* __restrict__ sign, const uint16_t* __
   const long long total = (long long)nrt * ng * 32;
   if (tid >= total) return;
   const int lane = (int)(tid & 31);
-  const long long unit = tid >> 5;  // rt * ng + g
-  const int g = (int)(unit % ng);
-  const int rt = (int)(unit / ng);
+  const long long unit = tid >> 5;  // unit_index(rt, g, nrt)
+  const int rt = (int)(unit % nrt);
+  const int g = (int)(unit / nrt);
   const int gid = lane >> 2, q = lane & 3;
   const int nv = ng * kGroupVecs;
   uint8_t* base = units + (size_t)unit * Layout<BITS>::kUnitBytes;
@@ -130,7 +130,7 @@ __global__ void pack_kernel(const uint8_t* __restrict__ sign, const uint16_t* __
 
 template <int BITS>
 __global__ void decode_kernel(const uint8_t* __restrict__ units, const uint8_t* __restrict__ codebook,
-                              uint16_t* __restrict__ w, int rows, int cols, int ng) {
+                              uint16_t* __restrict__ w, int rows, int cols, int ng, int nrt) {
   const long long tid = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   const int nv = cols / kVec;
   if (tid >= (long long)rows * nv) return;
@@ -141,7 +141,7 @@ __global__ void decode_kernel(const uint8_t* __restrict__ units, const uint8_t* 
   const int g = t / kGroupVecs, s = t % kGroupVecs;
   const int m = s >> 2, q = s & 3;
   const int lane = 4 * gid + q;
-  const uint8_t* unit = units + ((size_t)rt * ng + g) * Layout<BITS>::kUnitBytes;
+  const uint8_t* unit = units + (size_t)unit_index(rt, g, nrt) * Layout<BITS>::kUnitBytes;
   const Unit<BITS> u = load_unit<BITS>(unit, lane);
   GlobalCodebook cb{codebook};
   uint4 sa, sb;
@@ -149,7 +149,7 @@ __global__ void decode_kernel(const uint8_t* __restrict__ units, const uint8_t* 
   if constexpr (BITS == 2) {
     const uint32_t W = word_of(u.w, m);
     directions_w2(W, w2_sign3(u, q), m, cb, 0u, false, sa, sb);
-    r = radius_pair(qpair_w2(W), params_delta(u.rec.z, u.rec.w), params_rmin(u.rec.z, u.rec.w));
+    r = radius_pair(qpair_w2(W), params_delta(u.par.x, u.par.y), params_rmin(u.par.x, u.par.y));
   } else {
     directions_w3(u, m, q, cb, sa, sb);
     r = radius_pair(qpair_w3(u, m), params_delta(u.par.x, u.par.y),
@@ -177,6 +177,7 @@ static void free_handle(sphq_handle h) {
   cudaFree(h->codebook);
   cudaFree(h->params);
   cudaFree(h->ws);
+  cudaFree(h->cbimage);
   cudaFree(h->tickets);
   cudaFree(h->flag);
   cudaFree(h->xstage);
@@ -237,8 +238,10 @@ sphq_status sphq_create(int rows, int cols, int bits, int K, const void* codeboo
     return fail(cuda_error(e, "cudaMalloc(params)"));
   if ((e = cudaMalloc(&h->tickets, (size_t)nrt * sizeof(unsigned))) != cudaSuccess)
     return fail(cuda_error(e, "cudaMalloc(tickets)"));
-  if ((e = cudaMalloc(&h->flag, sizeof(int))) != cudaSuccess)
+  if ((e = cudaMalloc(&h->flag, 2 * sizeof(int))) != cudaSuccess)
     return fail(cuda_error(e, "cudaMalloc(flag)"));
+  if ((e = cudaMemset(h->flag, 0, 2 * sizeof(int))) != cudaSuccess)
+    return fail(cuda_error(e, "memset flag"));
   if ((e = cudaMalloc(&h->xstage, (size_t)SPHQ_MAX_BATCH * cols * 2)) != cudaSuccess)
     return fail(cuda_error(e, "cudaMalloc(x staging)"));
   if ((e = cudaMalloc(&h->ystage, (size_t)SPHQ_MAX_BATCH * rows * 2)) != cudaSuccess)
@@ -249,6 +252,15 @@ sphq_status sphq_create(int rows, int cols, int bits, int K, const void* codeboo
     return fail(cuda_error(e, "memset zeros"));
   if ((e = cudaMemcpy(h->codebook, codebook, (size_t)K * 16, cudaMemcpyDefault)) != cudaSuccess)
     return fail(cuda_error(e, "copy codebook"));
+  if (bits == 2) {
+    // shared-memory image of the W2 GEMV: entry k, copy c at 128 k + 16 c
+    if ((e = cudaMalloc(&h->cbimage, (size_t)K * 8 * 16)) != cudaSuccess)
+      return fail(cuda_error(e, "cudaMalloc(codebook image)"));
+    for (int c = 0; c < 8; ++c)
+      if ((e = cudaMemcpy2D(static_cast<uint8_t*>(h->cbimage) + 16 * c, 128, h->codebook, 16, 16,
+                            (size_t)K, cudaMemcpyDeviceToDevice)) != cudaSuccess)
+        return fail(cuda_error(e, "codebook image"));
+  }
   // params are kept as two planes (scale, offset) until pack interleaves them
   uint16_t* p16 = reinterpret_cast<uint16_t*>(h->params);
   const size_t np = (size_t)rows * ng;
@@ -260,7 +272,8 @@ sphq_status sphq_create(int rows, int cols, int bits, int K, const void* codeboo
     return fail(cuda_error(e, "memset tickets"));
   sphq_status st = make_gemv_plans(h);
   if (st != SPHQ_OK) return fail(st);
-  if ((e = cudaMalloc(&h->ws, h->ws_floats * sizeof(float))) != cudaSuccess)
+  if (h->ws_floats > 0 &&
+      (e = cudaMalloc(&h->ws, h->ws_floats * sizeof(float))) != cudaSuccess)
     return fail(cuda_error(e, "cudaMalloc(workspace)"));
   *out = h;
   return SPHQ_OK;
@@ -314,10 +327,10 @@ sphq_status sphq_decode(sphq_handle h, void* w, sphq_stream stream) {
   const unsigned grid = (unsigned)((n + block - 1) / block);
   if (h->bits == 2)
     decode_kernel<2><<<grid, block, 0, s>>>((const uint8_t*)h->units, (const uint8_t*)h->codebook,
-                                            (uint16_t*)w, h->rows, h->cols, h->ng);
+                                            (uint16_t*)w, h->rows, h->cols, h->ng, h->nrt);
   else
     decode_kernel<3><<<grid, block, 0, s>>>((const uint8_t*)h->units, (const uint8_t*)h->codebook,
-                                            (uint16_t*)w, h->rows, h->cols, h->ng);
+                                            (uint16_t*)w, h->rows, h->cols, h->ng, h->nrt);
   SPHQ_CUDA(cudaGetLastError(), "decode kernel launch");
   return SPHQ_OK;
 }

@@ -24,21 +24,35 @@
 //  * batch 3-8 ("full"): the lane forms w_hat = RN16(r_hat * (s (.) c_z))
 //    exactly as Eq. (4) defines it and the MMA's N dimension is the batch.
 //
-// Work decomposition (stream-K).  The (row tile, group) units are cut into
-// equal contiguous spans, one per warp of a grid no larger than the resident
-// capacity.  A warp accumulates in registers while its span stays in one row
-// tile.  A row tile covered by one warp is written directly; otherwise each
-// covering warp stores its fp32 partial (16 rows x batch) into the handle's
-// workspace and the last to arrive (an acq_rel atomic ticket per row tile;
-// nobody waits) sums the partials in slot order and writes y, so results do
-// not depend on scheduling.
+// Work decomposition.  The row tiles (16 rows) are dealt to thread-block
+// clusters in contiguous, near-equal ranges; every CTA of a cluster takes the
+// same tiles and its own contiguous share of the radius groups (split-K
+// inside the cluster).  Inside a CTA the tiles are cut into strips of four:
+// a work item is (strip, group), i.e. the four units of one group below each
+// other, so the activations of a group are loaded once for four units.  The
+// items are dealt to the warps in contiguous ranges.  Sums are reduced on
+// chip only and in a fixed order, so results do not depend on scheduling:
+// warp partials per tile go to shared memory, a CTA sums them in warp order,
+// each tile's owner CTA (tile index mod cluster size) receives the other
+// CTAs' sums through distributed shared memory (st.async completing on an
+// mbarrier) and adds them in rank order before writing fp16 y.
+//
+// Staging.  The codebook image (W2: eight interleaved copies, 8 KiB; W3: the
+// 128 KiB table) and, for batch 1-2, the CTA's slice of the activations are
+// copied into shared memory by bulk asynchronous copies completing on
+// mbarriers.  Codes stream from HBM through registers (16-byte loads that
+// bypass L1) one work item ahead of use, and a bulk L2 prefetch runs two
+// items further ahead (an item's units are contiguous in memory).
 //
 // Programmatic dependent launch: the kernel lets the next kernel on the
-// stream launch at once, asks L2 to prefetch its whole span of codes, loads
-// its first unit and stages the codebook, and only then waits
-// (griddepcontrol.wait) for the previous kernel -- before it touches
-// activations, outputs, workspace or tickets.  Codes and codebook are
-// immutable after sphq_pack, so this overlap is safe.
+// stream launch at once, prefetches its codes, issues its first unit loads
+// and the codebook copy, and only then waits (griddepcontrol.wait) for the
+// previous kernel -- before it touches activations or outputs.  Codes and
+// codebook are immutable after sphq_pack, so this overlap is safe.
+//
+// Every wait on an mbarrier gives up after about two seconds, records an
+// error bit in the handle's device flag word and carries on, so a fault in
+// the exchange cannot hang the GPU.
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 
@@ -51,139 +65,169 @@
 
 namespace sphq {
 
-struct GemvArgs {
-  const uint8_t* units;
-  const uint4* codebook;
-  const uint16_t* x;
-  uint16_t* y;
-  float* ws;
-  unsigned* tickets;
-  int rows, cols, ng, nrt;
-  int batch;
-  int units_per_warp;
-  int max_slots;
-  long long total_units;
-  const uint16_t* zeros;  // 256 B zero block: activations of lanes that supply none
-};
-
-// Zero block read by lanes that supply no activations: 256 B used, placed
-// 64 B into a 320 B region so its 16-byte chunks (4m + q) fall in the other
-// half of the shared-memory bank groups from the activations' chunks.
-constexpr int kZeroVec = 20;
-constexpr int kZeroSkew = 4;  // uint4
+constexpr int kStrip = 4;  // row tiles per work item (activation reuse)
+constexpr unsigned kStripMask = (1u << kStrip) - 1u;
 
 // Radius application modes.
 constexpr int kFactored1 = 1;  // batch 1
 constexpr int kFactored2 = 2;  // batch 2
 constexpr int kFull = 8;       // batch 3..8
 
+struct GemvArgs {
+  const uint8_t* units;
+  const uint8_t* cbimage;  // codebook image as laid out in shared memory
+  const uint16_t* x;
+  uint16_t* y;
+  int* flag;               // device error word: bit 1 = an mbarrier wait gave up
+  int rows, cols, ng, nrt;
+  int batch;
+  int nclusters;           // clusters holding tiles (grid = nclusters x cluster size)
+  int slots_per_warp;      // strip partial slots per warp
+  uint32_t cb_bytes;       // codebook image bytes
+  uint32_t x_pitch;        // bytes between staged activation rows (factored modes)
+  uint32_t off_x, off_zero, off_part, off_cta, off_recv, off_bar;  // dynamic smem offsets
+  const uint16_t* zeros;   // 256 B of zeros in global memory (batch 3-8 non-suppliers)
+};
+
+// ---------------------------------------------------------------------------
+// PTX wrappers
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+// Makes mbarrier initialisation visible to the async proxy and the cluster.
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ uint64_t globaltimer() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Waits for phase `parity` of a local mbarrier; gives up after ~2 s.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer();
+  for (;;) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (globaltimer() - t0 > 2000000000ull) return false;
+  }
+}
+// Bulk copy global -> own shared memory, completing on a local mbarrier.
+// dst, src and bytes must be multiples of 16.
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes,
+                                         uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          dst),
+      "l"(src), "r"(bytes), "r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t cluster_id() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%clusterid.x;" : "=r"(r));
+  return r;
+}
+// Relaxed arrive: it orders nothing (the mbarrier initialisation is published
+// by fence.mbarrier_init), so it does not wait for this thread's loads in flight.
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() {
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Address of the same shared-memory location in cluster CTA `rank`.
+__device__ __forceinline__ uint32_t mapa(uint32_t addr, uint32_t rank) {
+  uint32_t d;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(d) : "r"(addr), "r"(rank));
+  return d;
+}
+// 16-byte store into another CTA's shared memory, completing on its mbarrier.
+__device__ __forceinline__ void st_async16(uint32_t raddr, float4 v, uint32_t rbar) {
+  asm volatile(
+      "st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1, %2, %3, %4}, "
+      "[%5];" ::"r"(raddr),
+      "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"(rbar)
+      : "memory");
+}
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // The MMAs are pure register computations (no volatile), so the compiler may
 // interleave the words of a unit freely.
 __device__ __forceinline__ void mma16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
                                          uint32_t a3, uint32_t b0, uint32_t b1) {
-  asm(
-      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 "
+  asm("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 "
       "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
-
 // D = A B (C = 0)
 __device__ __forceinline__ void mma16816_zero(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
                                               uint32_t a3, uint32_t b0, uint32_t b1) {
   const float z = 0.f;
-  asm(
-      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 "
+  asm("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 "
       "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%10,%10,%10,%10};"
       : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1), "f"(z));
 }
 
-// Activations are re-read by every row tile: keep them in L1.
+// Activations of batch 3-8 are re-read by every strip: keep them in L1.
 __device__ __forceinline__ uint4 ldg_x16(const uint16_t* p) {
   uint4 v;
   asm volatile("ld.global.nc.L1::evict_last.v4.u32 {%0,%1,%2,%3}, [%4];"
-               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
   return v;
 }
 
 __device__ __forceinline__ float h_lo_to_f32(uint32_t h2) {
   float f;
   asm("{\n\t.reg .f16 lo, hi;\n\tmov.b32 {lo, hi}, %1;\n\tcvt.f32.f16 %0, lo;\n\t}"
-      : "=f"(f) : "r"(h2));
+      : "=f"(f)
+      : "r"(h2));
   return f;
 }
 __device__ __forceinline__ float h_hi_to_f32(uint32_t h2) {
   float f;
   asm("{\n\t.reg .f16 lo, hi;\n\tmov.b32 {lo, hi}, %1;\n\tcvt.f32.f16 %0, hi;\n\t}"
-      : "=f"(f) : "r"(h2));
+      : "=f"(f)
+      : "r"(h2));
   return f;
 }
 
-__device__ __forceinline__ void pdl_launch_dependents() {
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-}
-__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
-
-__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
-  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
-}
-
-__device__ __forceinline__ unsigned ticket_acq_rel(unsigned* p) {
-  unsigned old;
-  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(old) : "l"(p) : "memory");
-  return old;
-}
-
-// Writes a warp's partial of row tile rt; the last contributor sums all
-// partials in slot order and stores fp16 y.  v[i][h] is this lane's value of
-// batch row bidx[i] at row gid + 8h of the tile, valid where own[i] is set.
-template <int NB>
-__device__ __forceinline__ void flush_row_tile(const GemvArgs& a, int rt, long long gw, int lane,
-                                               const float (&v)[NB][2], const bool (&own)[NB],
-                                               const int (&bidx)[NB]) {
-  const long long L = a.units_per_warp;
-  const long long first = ((long long)rt * a.ng) / L;
-  const long long last = ((long long)(rt + 1) * a.ng - 1) / L;
-  const int count = (int)(last - first + 1);
-  const int gid = lane >> 2;
-  const int row0 = rt * kRowsPerTile;
-  if (count == 1) {
-#pragma unroll
-    for (int i = 0; i < NB; ++i) {
-      if (!own[i]) continue;
-      const int b = bidx[i];
-      if (row0 + gid < a.rows) a.y[(size_t)b * a.rows + row0 + gid] = f32_to_h_rn(v[i][0]);
-      if (row0 + gid + 8 < a.rows) a.y[(size_t)b * a.rows + row0 + gid + 8] = f32_to_h_rn(v[i][1]);
-    }
-    return;
-  }
-  const int per = kRowsPerTile * a.batch;  // floats per partial
-  const int slot = (int)(gw - first);
-  float* base = a.ws + (size_t)rt * a.max_slots * kRowsPerTile * kMaxBatch;
-  float* mine = base + (size_t)slot * per;
-#pragma unroll
-  for (int i = 0; i < NB; ++i) {
-    if (!own[i]) continue;
-    const int b = bidx[i];
-    mine[b * kRowsPerTile + gid] = v[i][0];
-    mine[b * kRowsPerTile + gid + 8] = v[i][1];
-  }
-  __syncwarp();
-  unsigned ticket = 0;
-  if (lane == 0) ticket = ticket_acq_rel(&a.tickets[rt]);
-  ticket = __shfl_sync(0xFFFFFFFFu, ticket, 0);
-  if (ticket != (unsigned)(count - 1)) return;
-  __syncwarp();  // order every lane's reads after lane 0's acquire
-  for (int i = lane; i < per; i += 32) {
-    float s = 0.f;
-    for (int k = 0; k < count; ++k) s += __ldcg(base + (size_t)k * per + i);
-    const int b = i / kRowsPerTile, r = row0 + i % kRowsPerTile;
-    if (r < a.rows) a.y[(size_t)b * a.rows + r] = f32_to_h_rn(s);
-  }
-  __syncwarp();
-  if (lane == 0) atomicExch(&a.tickets[rt], 0u);  // ready for the next call
-}
+// ---------------------------------------------------------------------------
+// Decode + multiply of one unit
+// ---------------------------------------------------------------------------
 
 template <int BITS>
 struct UnitConst {
@@ -194,8 +238,8 @@ template <int BITS>
 __device__ __forceinline__ UnitConst<BITS> unit_const(const Unit<BITS>& u, int q) {
   UnitConst<BITS> c;
   if constexpr (BITS == 2) {
-    c.d2 = params_delta(u.rec.z, u.rec.w);
-    c.m2 = params_rmin(u.rec.z, u.rec.w);
+    c.d2 = params_delta(u.par.x, u.par.y);
+    c.m2 = params_rmin(u.par.x, u.par.y);
     c.e = w2_sign3(u, q);
   } else {
     c.d2 = params_delta(u.par.x, u.par.y);
@@ -219,41 +263,28 @@ __device__ __forceinline__ void word_directions(const Unit<BITS>& u, const UnitC
   }
 }
 
-// Accumulators of one warp for the current row tile.
+// Accumulators of one warp for one row tile.
 template <int MODE>
 struct Acc {
-  static constexpr int NB = MODE == kFull ? 2 : MODE;
-  float f[2][NB][2];  // factored: [set][batch row][row gid / gid+8]
-  float d[2][4];      // full: MMA accumulators [set][fragment]
+  static constexpr int NB = MODE == kFull ? 1 : MODE;
+  float f[NB][2];  // factored: [batch row][row gid / gid+8]
+  float d[4];      // full: MMA accumulator fragment
   __device__ __forceinline__ void zero() {
 #pragma unroll
-    for (int s = 0; s < 2; ++s) {
+    for (int i = 0; i < NB; ++i) f[i][0] = f[i][1] = 0.f;
 #pragma unroll
-      for (int i = 0; i < NB; ++i) f[s][i][0] = f[s][i][1] = 0.f;
-#pragma unroll
-      for (int i = 0; i < 4; ++i) d[s][i] = 0.f;
-    }
+    for (int i = 0; i < 4; ++i) d[i] = 0.f;
   }
 };
 
-// One unit (16 rows x 16 slots).  For word m the lane supplies to the B
-// fragment 16 B at xsrc + 32*m halves: its activation row at slot 4m+q, or the
-// zero block.  Batch 1-2 reads x from shared memory (staged once per CTA),
-// batch 3-8 from global memory through L1; the unit's four loads are issued
-// together before any of its words is decoded.
+// One unit (16 rows x 16 slots); xv[m] is this lane's B-fragment data for
+// word m (its activation row at slot 4m+q, or zeros).
 template <int BITS, int MODE>
-__device__ __forceinline__ void process_unit(const Unit<BITS>& cur, const uint16_t* xsrc, int q,
+__device__ __forceinline__ void process_unit(const Unit<BITS>& cur, const uint4 (&xv)[4], int q,
                                              const SmemCodebook& cb, Acc<MODE>& acc) {
-  uint4 xv[4];
-  if constexpr (MODE == kFull) {
-#pragma unroll
-    for (int m = 0; m < 4; ++m) xv[m] = ldg_x16(xsrc + 32 * m);
-  }
   const UnitConst<BITS> kc = unit_const<BITS>(cur, q);
 #pragma unroll
   for (int m = 0; m < 4; ++m) {
-    if constexpr (MODE != kFull) xv[m] = *reinterpret_cast<const uint4*>(xsrc + 32 * m);
-    const uint4& xm = xv[m];
     uint4 sa, sb;
     uint32_t qp;
     word_directions<BITS>(cur, kc, m, q, cb, sa, sb, qp);
@@ -261,112 +292,177 @@ __device__ __forceinline__ void process_unit(const Unit<BITS>& cur, const uint16
     if constexpr (MODE == kFull) {
       const uint4 wa = scale_block(sa, bcast_lo(r));
       const uint4 wb = scale_block(sb, bcast_hi(r));
-      float(&d)[4] = acc.d[m & 1];
-      mma16816(d, wa.x, wb.x, wa.y, wb.y, xm.x, xm.y);
-      mma16816(d, wa.z, wb.z, wa.w, wb.w, xm.z, xm.w);
+      mma16816(acc.d, wa.x, wb.x, wa.y, wb.y, xv[m].x, xv[m].y);
+      mma16816(acc.d, wa.z, wb.z, wa.w, wb.w, xv[m].z, xv[m].w);
     } else {
       float d[4];
-      mma16816_zero(d, sa.x, sb.x, sa.y, sb.y, xm.x, xm.y);
-      mma16816(d, sa.z, sb.z, sa.w, sb.w, xm.z, xm.w);
+      mma16816_zero(d, sa.x, sb.x, sa.y, sb.y, xv[m].x, xv[m].y);
+      mma16816(d, sa.z, sb.z, sa.w, sb.w, xv[m].z, xv[m].w);
       const float rA = h_lo_to_f32(r), rB = h_hi_to_f32(r);
-      auto& ac = acc.f[m & 1];
-      ac[0][0] = __fmaf_rn(rA, d[0], ac[0][0]);
-      ac[0][1] = __fmaf_rn(rB, d[2], ac[0][1]);
+      acc.f[0][0] = __fmaf_rn(rA, d[0], acc.f[0][0]);
+      acc.f[0][1] = __fmaf_rn(rB, d[2], acc.f[0][1]);
       if constexpr (MODE == kFactored2) {
-        ac[1][0] = __fmaf_rn(rA, d[1], ac[1][0]);
-        ac[1][1] = __fmaf_rn(rB, d[3], ac[1][1]);
+        acc.f[1][0] = __fmaf_rn(rA, d[1], acc.f[1][0]);
+        acc.f[1][1] = __fmaf_rn(rB, d[3], acc.f[1][1]);
       }
     }
   }
 }
 
+// Writes a warp's accumulators of one row tile into its partial block
+// (16 x NBP floats, [batch row][row]).
 template <int MODE>
-__device__ __forceinline__ void flush_acc(const GemvArgs& a, int rt, long long gw, int lane,
-                                          Acc<MODE>& acc) {
-  const int q = lane & 3;
+__device__ __forceinline__ void store_partial(float* blk, Acc<MODE>& acc, int lane, int batch) {
+  const int gid = lane >> 2, q = lane & 3;
   if constexpr (MODE == kFull) {
     // d[0..3] = D[gid][2q], D[gid][2q+1], D[gid+8][2q], D[gid+8][2q+1]
-    float v[2][2] = {{acc.d[0][0] + acc.d[1][0], acc.d[0][2] + acc.d[1][2]},
-                     {acc.d[0][1] + acc.d[1][1], acc.d[0][3] + acc.d[1][3]}};
-    const bool own[2] = {2 * q < a.batch, 2 * q + 1 < a.batch};
-    const int bidx[2] = {2 * q, 2 * q + 1};
-    flush_row_tile<2>(a, rt, gw, lane, v, own, bidx);
+    if (2 * q < batch) {
+      blk[(2 * q) * kRowsPerTile + gid] = acc.d[0];
+      blk[(2 * q) * kRowsPerTile + gid + 8] = acc.d[2];
+    }
+    if (2 * q + 1 < batch) {
+      blk[(2 * q + 1) * kRowsPerTile + gid] = acc.d[1];
+      blk[(2 * q + 1) * kRowsPerTile + gid + 8] = acc.d[3];
+    }
   } else {
-    constexpr int NB = MODE;
     // sum the lane's slots, then the quad's four lanes (slots q = 0..3)
-    float v[NB][2];
 #pragma unroll
-    for (int i = 0; i < NB; ++i) {
+    for (int i = 0; i < MODE; ++i) {
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
-        float t = acc.f[0][i][h] + acc.f[1][i][h];
+        float t = acc.f[i][h];
         t += __shfl_xor_sync(0xFFFFFFFFu, t, 1);
         t += __shfl_xor_sync(0xFFFFFFFFu, t, 2);
-        v[i][h] = t;
+        if (q == 0) blk[i * kRowsPerTile + gid + 8 * h] = t;
       }
     }
-    bool own[NB];
-    int bidx[NB];
-#pragma unroll
-    for (int i = 0; i < NB; ++i) {
-      own[i] = q == 0;
-      bidx[i] = i;
-    }
-    flush_row_tile<NB>(a, rt, gw, lane, v, own, bidx);
   }
-  acc.zero();
+}
+
+// ---------------------------------------------------------------------------
+// The kernel
+// ---------------------------------------------------------------------------
+
+// Contiguous near-equal share [lo, hi) of n items for part i of p (32-bit
+// arithmetic when n * p fits, which is every practical case).
+__device__ __forceinline__ int share_lo(int n, int i, int p) {
+  if ((unsigned)n < 65536u && (unsigned)p < 65536u) return (int)((unsigned)n * (unsigned)i / (unsigned)p);
+  return (int)(((long long)n * i) / p);
+}
+// The same for a compile-time number of parts (a shift for powers of two).
+template <int P>
+__device__ __forceinline__ int share_lo_c(int n, int i) {
+  return (int)((unsigned)n * (unsigned)i / (unsigned)P);
+}
+
+// One work item: the activations of one group (xp: this lane's 16 bytes of
+// word 0; words 1-3 follow at 64-byte steps) and the units of up to four row
+// tiles below each other (u[j], unit j of the strip), whose loads for the next
+// item (base nb) are issued as soon as each unit is consumed.  With CHECK, only
+// the units in cmask are processed and only those in nmask loaded.
+template <int BITS, int MODE, bool CHECK>
+__device__ __forceinline__ void run_item(Unit<BITS> (&u)[kStrip], Acc<MODE> (&acc)[kStrip],
+                                         const uint8_t* xp, const uint8_t* nb, unsigned cmask,
+                                         unsigned nmask, int lane, int q, const SmemCodebook& cb) {
+  constexpr int UB = Layout<BITS>::kUnitBytes;
+  uint4 xv[4];
+#pragma unroll
+  for (int m = 0; m < 4; ++m) {
+    if constexpr (MODE == kFull)
+      xv[m] = ldg_x16(reinterpret_cast<const uint16_t*>(xp) + 32 * m);
+    else
+      xv[m] = *reinterpret_cast<const uint4*>(xp + 64 * m);
+  }
+#pragma unroll
+  for (int j = 0; j < kStrip; ++j) {
+    if (!CHECK || (cmask >> j & 1u)) process_unit<BITS, MODE>(u[j], xv, q, cb, acc[j]);
+    if (!CHECK || (nmask >> j & 1u)) u[j] = load_unit<BITS>(nb + j * UB, lane);
+  }
 }
 
 template <int BITS, int MODE, int WARPS, int MINB>
 __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a) {
-  extern __shared__ uint4 smem_cb[];
+  extern __shared__ __align__(128) uint8_t smem[];
   pdl_launch_dependents();
-  const int lane = threadIdx.x & 31;
-  const int gid = lane >> 2, q = lane & 3;
-  const long long gw = (long long)blockIdx.x * WARPS + (threadIdx.x >> 5);
-  long long u = gw * a.units_per_warp;
-  const long long u_end = min(u + (long long)a.units_per_warp, a.total_units);
+  constexpr int NBP = MODE == kFull ? kMaxBatch : MODE;  // floats per row in a partial block
+  constexpr int kBlk = kRowsPerTile * NBP;                // floats per partial block
   constexpr int UB = Layout<BITS>::kUnitBytes;
-  const uint8_t* const span = a.units + (size_t)u * UB;  // unit u of the span
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int gid = lane >> 2, q = lane & 3;
+  const int csize = (int)(gridDim.x / (unsigned)a.nclusters);
+  const int crank = csize > 1 ? (int)cluster_rank() : 0;
+  const int cid = csize > 1 ? (int)cluster_id() : (int)blockIdx.x;
 
-  // Codes are immutable: stream the span toward L2 and start the first unit
-  // while the codebook is staged and the previous kernel finishes.
-  Unit<BITS> ua{}, ub{}, uc{};
-  if (u < u_end) {
-    if (lane == 0) prefetch_l2(span, (uint32_t)((u_end - u) * UB));
-    ua = load_unit<BITS>(span, lane);
-    ub = load_unit<BITS>(span + UB, lane);
+  // this cluster's row tiles and this CTA's radius groups
+  const int t0 = share_lo(a.nrt, cid, a.nclusters);
+  const int T = share_lo(a.nrt, cid + 1, a.nclusters) - t0;
+  const int g0 = share_lo(a.ng, crank, csize);
+  const int ngc = share_lo(a.ng, crank + 1, csize) - g0;
+  const int nstrips = (T + kStrip - 1) / kStrip;
+  const int nfull = T / kStrip;  // strips with all four tiles
+  const unsigned last_mask = (1u << (T - kStrip * nfull)) - 1u;
+  const int items = nstrips * ngc;  // item i = (strip i / ngc, group g0 + i % ngc)
+  const int i0 = share_lo_c<WARPS>(items, warp), i1 = share_lo_c<WARPS>(items, warp + 1);
+
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + a.off_bar);
+  const uint32_t bar_cb = smem_u32(&bars[0]), bar_x = smem_u32(&bars[1]),
+                 bar_recv = smem_u32(&bars[2]);
+  const int nown = crank < T ? (T - crank + csize - 1) / csize : 0;  // tiles this CTA owns
+
+  // units (t0 + 4s + j, g), j = 0..3, start at strip_base(s, g) + j * UB
+  const size_t gstride = (size_t)a.nrt * UB;
+  auto strip_base = [&](int s, int g) {
+    return a.units + ((size_t)g * a.nrt + t0 + kStrip * s) * UB;
+  };
+  auto strip_mask = [&](int s) { return s < nfull ? kStripMask : last_mask; };
+
+  // first item's units (codes are immutable: no wait needed)
+  Unit<BITS> u[kStrip] = {};
+  int s = i0 < i1 ? i0 / ngc : 0;
+  int g = i0 < i1 ? g0 + i0 % ngc : g0;
+  if (i0 < i1) {
+    const unsigned m0 = strip_mask(s);
+#pragma unroll
+    for (int j = 0; j < kStrip; ++j)
+      if (m0 >> j & 1u) u[j] = load_unit<BITS>(strip_base(s, g) + j * UB, lane);
   }
-  if (BITS == 2) {
-    for (int i = threadIdx.x; i < Layout<2>::K * 8; i += WARPS * 32)
-      smem_cb[i] = __ldg(a.codebook + (i >> 3));
-  } else {
-    for (int i = threadIdx.x; i < Layout<3>::K; i += WARPS * 32) smem_cb[i] = __ldg(a.codebook + i);
+
+  if (threadIdx.x == 0) {
+    mbar_init(bar_cb, 1);
+    mbar_init(bar_x, 1);
+    mbar_init(bar_recv, 1);
+    fence_mbar_init();
+    mbar_arrive_expect_tx(bar_cb, a.cb_bytes);
+    for (uint32_t o = 0; o < a.cb_bytes; o += 32768u)
+      bulk_g2s(smem_u32(smem) + o, a.cbimage + o, min(32768u, a.cb_bytes - o), bar_cb);
+    // incoming partial sums of the owned tiles from the other CTAs
+    mbar_arrive_expect_tx(bar_recv, (uint32_t)(nown * (csize - 1) * kBlk * 4));
   }
-  // batch 1-2: a zero block and the activation rows follow the codebook
-  constexpr int kCbVec = (BITS == 2 ? Layout<2>::K * 8 : Layout<3>::K);  // uint4 entries
-  uint4* const smem_zero = smem_cb + kCbVec;
-  uint16_t* const smem_x = reinterpret_cast<uint16_t*>(smem_zero + kZeroVec);
-  if (MODE != kFull && threadIdx.x < kZeroVec) smem_zero[threadIdx.x] = make_uint4(0, 0, 0, 0);
-  pdl_wait();
-  if (MODE != kFull) {
-    const int nx = a.batch * a.cols / 8;  // uint4 of activations (cols % 128 == 0)
-    const uint4* xg = reinterpret_cast<const uint4*>(a.x);
-    uint4* xs = reinterpret_cast<uint4*>(smem_x);
-    for (int i = threadIdx.x; i < nx; i += WARPS * 32) xs[i] = ldg_x16(a.x + 8 * (size_t)i);
-    (void)xg;
+  if (MODE != kFull && threadIdx.x < 16)  // zero block read by lanes that supply no activations
+    reinterpret_cast<uint4*>(smem + a.off_zero)[threadIdx.x] = make_uint4(0, 0, 0, 0);
+  __syncthreads();                  // mbarrier initialisation visible to the CTA
+  if (csize > 1) cluster_arrive_relaxed();  // ... and to the cluster (waited on below)
+
+  pdl_wait();  // the previous kernel's outputs (our activations) are complete
+  if (MODE != kFull && threadIdx.x == 0) {
+    const uint32_t row_bytes = (uint32_t)ngc * kGroupCols * 2;
+    mbar_arrive_expect_tx(bar_x, row_bytes * MODE);
+    for (int b = 0; b < MODE; ++b)
+      bulk_g2s(smem_u32(smem + a.off_x) + b * a.x_pitch,
+               a.x + (size_t)b * a.cols + (size_t)g0 * kGroupCols, row_bytes, bar_x);
   }
-  __syncthreads();
-  if (u >= u_end) return;
+  bool ok = mbar_wait(bar_cb, 0);
+  if (MODE != kFull) ok &= mbar_wait(bar_x, 0);
+  if (!ok && lane == 0) atomicOr(a.flag, 2);
 
   SmemCodebook cb;
-  cb.base = reinterpret_cast<const uint8_t*>(smem_cb);
+  cb.base = smem;
   cb.copyoff = BITS == 2 ? (uint32_t)(lane & 7) * 16u : 0u;
 
-  // The activation row this lane supplies to the B fragment; lanes that
-  // supply nothing read the handle's zero page (no predicates in the loop).
-  bool provider;
+  // The activation row this lane supplies to the B fragment; the other lanes
+  // read a zero block (stride 0), so the loop has no lane-dependent branch.
   int xb;
+  bool provider;
   if (MODE == kFull) {
     xb = gid;
     provider = gid < a.batch;
@@ -374,66 +470,157 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
     xb = gid - 2 * q;
     provider = xb >= 0 && xb < MODE;
   }
-  // providers walk their activation row group by group; the others keep
-  // reading the same 256-byte zero block (stride 0), which stays in L1
-  const uint16_t* xrow;
+  const uint8_t* x0;  // this lane's activation bytes of group g0
   if (MODE == kFull)
-    xrow = (provider ? a.x + (size_t)xb * a.cols : a.zeros) + q * kVec;
+    x0 = provider ? reinterpret_cast<const uint8_t*>(a.x + (size_t)xb * a.cols + (size_t)g0 * kGroupCols)
+                  : reinterpret_cast<const uint8_t*>(a.zeros);
   else
-    xrow = (provider ? smem_x + (size_t)xb * a.cols
-                     : reinterpret_cast<const uint16_t*>(smem_zero + kZeroSkew)) +
-           q * kVec;
-  const int xstride = provider ? kGroupCols : 0;
+    x0 = provider ? smem + a.off_x + xb * a.x_pitch : smem + a.off_zero;
+  x0 += q * 16;
+  const int xstep = provider ? kGroupCols * 2 : 0;
 
-  // the unit buffer ends with two guard units, so prefetching up to two units
-  // past the span stays in bounds (the data is never used)
-  auto unit_ptr = [&](long long v) { return a.units + (size_t)v * UB; };
+  float* part = reinterpret_cast<float*>(smem + a.off_part) +
+                (size_t)warp * a.slots_per_warp * kStrip * kBlk;
+  const int first_strip = s;
 
-  int rt = (int)(u / a.ng);
-  int g = (int)(u - (long long)rt * a.ng);
-  Acc<MODE> acc;
-  acc.zero();
-  for (;;) {
-    // one segment: the span's units inside row tile rt
-    const long long seg_end = min(u_end, (long long)(rt + 1) * a.ng);
-    long long n = seg_end - u;
-    const uint16_t* xs = xrow + (size_t)g * xstride;
-    // three units in registers: the one being decoded and two in flight
-    for (; n >= 3; n -= 3) {
-      uc = load_unit<BITS>(unit_ptr(u + 2), lane);
-      process_unit<BITS, MODE>(ua, xs, q, cb, acc);
-      ua = load_unit<BITS>(unit_ptr(u + 3), lane);
-      process_unit<BITS, MODE>(ub, xs + xstride, q, cb, acc);
-      ub = load_unit<BITS>(unit_ptr(u + 4), lane);
-      process_unit<BITS, MODE>(uc, xs + 2 * xstride, q, cb, acc);
-      xs += 3 * xstride;
-      u += 3;
+  Acc<MODE> acc[kStrip];
+#pragma unroll
+  for (int j = 0; j < kStrip; ++j) acc[j].zero();
+
+  // Units of a full strip at one group are contiguous: one bulk L2 prefetch
+  // per item, two items ahead inside the strip (the next item's units are
+  // already in flight to registers).
+  const uint32_t strip_bytes = kStrip * UB;
+
+  int left = i1 - i0;
+  const uint8_t* ub = strip_base(s, g);
+  const uint8_t* xp = x0 + (g - g0) * xstep;
+  while (left > 0) {
+    // the warp's items of strip s: groups g .. g + cnt - 1
+    const int cnt = min(left, g0 + ngc - g);
+    left -= cnt;
+    const unsigned cmask = strip_mask(s);
+    int c = 0;
+    if (cmask == kStripMask) {
+      if (lane == 0 && cnt > 1) prefetch_l2(ub + gstride, strip_bytes);
+      for (; c + 1 < cnt; ++c) {  // next item: same strip, next group
+        if (lane == 0 && c + 2 < cnt) prefetch_l2(ub + 2 * gstride, strip_bytes);
+        run_item<BITS, MODE, false>(u, acc, xp, ub + gstride, kStripMask, kStripMask, lane, q, cb);
+        ub += gstride;
+        xp += xstep;
+      }
     }
-    for (; n > 0; --n) {  // 1 or 2 left: rotate the ring
-      uc = load_unit<BITS>(unit_ptr(u + 2), lane);
-      process_unit<BITS, MODE>(ua, xs, q, cb, acc);
-      ua = ub;
-      ub = uc;
-      xs += xstride;
-      u += 1;
+    for (; c < cnt; ++c) {
+      const bool last = c + 1 == cnt;
+      const uint8_t* nb = !last ? ub + gstride : strip_base(s + 1, g0);
+      const unsigned nmask = !last ? cmask : (left > 0 ? strip_mask(s + 1) : 0u);
+      run_item<BITS, MODE, true>(u, acc, xp, nb, cmask, nmask, lane, q, cb);
+      ub += gstride;
+      xp += xstep;
     }
-    flush_acc<MODE>(a, rt, gw, lane, acc);
-    if (u >= u_end) break;
-    ++rt;  // the next segment starts at group 0 of the next row tile
-    g = 0;
+    float* blk = part + (size_t)(s - first_strip) * kStrip * kBlk;
+#pragma unroll
+    for (int j = 0; j < kStrip; ++j) {
+      store_partial<MODE>(blk + j * kBlk, acc[j], lane, a.batch);
+      acc[j].zero();
+    }
+    ++s;
+    g = g0;
+    ub = strip_base(s, g0);
+    xp = x0;
+  }
+  // the first strip of each warp's items, for locating its partial blocks
+  int* wfirst = reinterpret_cast<int*>(smem + a.off_bar + 32);
+  if (lane == 0) wfirst[warp] = first_strip;
+  __syncthreads();  // every warp partial is in shared memory
+
+  // CTA sums, all threads: thread (tau, l) sums floats 4l..4l+3 of tile tau
+  // over the partial blocks of the warps whose items cover tile tau's strip,
+  // in warp order.
+  float* cta = reinterpret_cast<float*>(smem + a.off_cta);
+  for (int e = threadIdx.x; e < T * 4 * NBP; e += WARPS * 32) {
+    const int tau = e / (4 * NBP), l = e % (4 * NBP);
+    const int ts = tau / kStrip, j = tau % kStrip;
+    float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int w = 0; w < WARPS; ++w) {
+      const int a0 = share_lo_c<WARPS>(items, w), a1 = share_lo_c<WARPS>(items, w + 1);
+      if (a0 < a1 && a0 < (ts + 1) * ngc && a1 > ts * ngc) {
+        const float* blk = reinterpret_cast<const float*>(smem + a.off_part) +
+                           ((w * a.slots_per_warp + ts - wfirst[w]) * kStrip + j) * kBlk;
+        const float4 v = reinterpret_cast<const float4*>(blk)[l];
+        sum.x += v.x;
+        sum.y += v.y;
+        sum.z += v.z;
+        sum.w += v.w;
+      }
+    }
+    reinterpret_cast<float4*>(cta + (size_t)tau * kBlk)[l] = sum;
+  }
+  __syncthreads();
+
+  // Cluster exchange: tile tau belongs to CTA tau % csize; the others send it
+  // their sums (slot = sender rank) and the owner adds all csize in rank order.
+  auto write_y = [&](int tau, const float4& v, int l) {
+    const int e = 4 * l, b = e / kRowsPerTile, r0 = (t0 + tau) * kRowsPerTile + e % kRowsPerTile;
+    if (b >= a.batch) return;
+    uint16_t* yb = a.y + (size_t)b * a.rows;
+    if (r0 + 0 < a.rows) yb[r0 + 0] = f32_to_h_rn(v.x);
+    if (r0 + 1 < a.rows) yb[r0 + 1] = f32_to_h_rn(v.y);
+    if (r0 + 2 < a.rows) yb[r0 + 2] = f32_to_h_rn(v.z);
+    if (r0 + 3 < a.rows) yb[r0 + 3] = f32_to_h_rn(v.w);
+  };
+  if (csize == 1) {
+    for (int tau = warp; tau < T; tau += WARPS)
+      if (lane < 4 * NBP) write_y(tau, reinterpret_cast<const float4*>(cta + (size_t)tau * kBlk)[lane], lane);
+    return;
+  }
+  cluster_wait();  // every CTA's mbarriers are initialised
+  float* recv = reinterpret_cast<float*>(smem + a.off_recv);
+  for (int tau = warp; tau < T; tau += WARPS) {
+    const int owner = tau % csize;
+    if (lane >= 4 * NBP) continue;
+    const float4 v = reinterpret_cast<const float4*>(cta + (size_t)tau * kBlk)[lane];
+    float* slot = recv + ((size_t)(tau / csize) * csize + crank) * kBlk;
+    if (owner == crank) {
+      reinterpret_cast<float4*>(slot)[lane] = v;
+    } else {
+      const uint32_t raddr = mapa(smem_u32(slot) + 16u * lane, (uint32_t)owner);
+      st_async16(raddr, v, mapa(bar_recv, (uint32_t)owner));
+    }
+  }
+  if (nown == 0) return;
+  if (!mbar_wait(bar_recv, 0) && threadIdx.x == 0) atomicOr(a.flag, 2);
+  __syncthreads();  // own slots written by the other warps
+  for (int k = warp; k < nown; k += WARPS) {
+    const int tau = crank + k * csize;
+    if (lane >= 4 * NBP) continue;
+    float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int r = 0; r < csize; ++r) {
+      const float4 v = reinterpret_cast<const float4*>(recv + ((size_t)k * csize + r) * kBlk)[lane];
+      sum.x += v.x;
+      sum.y += v.y;
+      sum.z += v.z;
+      sum.w += v.w;
+    }
+    write_y(tau, sum, lane);
   }
 }
+
+// ---------------------------------------------------------------------------
+// Host side: kernel selection, launch plans, launches
+// ---------------------------------------------------------------------------
 
 template <int BITS> struct KernelShape;
 template <> struct KernelShape<2> {
   static constexpr int kWarps = 8;
   static constexpr int kMinBlocks = 2;
-  static constexpr size_t kSmem = (size_t)Layout<2>::K * 8 * 16;
+  static constexpr uint32_t kCbBytes = (uint32_t)Layout<2>::K * 8 * 16;  // 8 copies
 };
 template <> struct KernelShape<3> {
   static constexpr int kWarps = 16;
   static constexpr int kMinBlocks = 1;
-  static constexpr size_t kSmem = (size_t)Layout<3>::K * 16;
+  static constexpr uint32_t kCbBytes = (uint32_t)Layout<3>::K * 16;
 };
 
 template <int BITS, int MODE>
@@ -452,9 +639,9 @@ static const void* select_kernel(int bits, int mode) {
                                                                          : kptr<3, kFull>();
 }
 
-// Dynamic shared memory is sized per handle (batch 1-2 stage their activation
-// rows), while the attribute that permits it belongs to the kernel function and
-// is process-wide: raise it once to the device's opt-in maximum.
+// Dynamic shared memory is sized per handle, while the attribute that permits
+// it belongs to the kernel function and is process-wide: raise it once to the
+// device's opt-in maximum.
 static sphq_status allow_max_smem(int device, int optin) {
   static std::mutex mu;
   static bool done[64] = {};
@@ -472,43 +659,150 @@ static sphq_status allow_max_smem(int device, int optin) {
   return SPHQ_OK;
 }
 
+static size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+// Shared-memory layout for a given cluster size and tile count per cluster.
+struct SmemLayout {
+  size_t zero, x, part, cta, recv, bar, total;
+  uint32_t x_pitch;
+  int slots;
+};
+
+static SmemLayout smem_layout(const sphq_handle_s* h, int mode, int warps, int csize, int tmax) {
+  SmemLayout L{};
+  const int nbp = mode == kFull ? kMaxBatch : mode;
+  const size_t blk = (size_t)kRowsPerTile * nbp * 4;
+  const int ngc_max = (h->ng + csize - 1) / csize;
+  const int nstrips = (tmax + kStrip - 1) / kStrip;
+  const long long items = (long long)nstrips * ngc_max;
+  // a warp's items span at most ceil(items / warps) consecutive items, so at
+  // most that many / ngc + 2 strips
+  const long long per_warp = (items + warps - 1) / warps;
+  L.slots = (int)std::min<long long>(nstrips, per_warp / std::max(1, ngc_max) + 2);
+  size_t o = h->bits == 2 ? KernelShape<2>::kCbBytes : KernelShape<3>::kCbBytes;
+  // batch 1-2: a 256 B zero block, then the activation rows.  Rows start 320 B
+  // after the zero block and 64 B apart modulo 128, so within a quarter warp
+  // the suppliers' 16-byte chunks and the zero readers' chunks fall in
+  // different bank groups.
+  L.zero = o;
+  L.x = o + 320;
+  L.x_pitch = (uint32_t)((size_t)ngc_max * kGroupCols * 2 + 64);
+  if (mode != kFull) o = L.x + (size_t)L.x_pitch * mode;
+  o = align_up(o, 16);
+  L.part = o;
+  o += (size_t)warps * L.slots * kStrip * blk;
+  L.cta = o;
+  o += (size_t)tmax * blk;
+  L.recv = o;
+  if (csize > 1) o += (size_t)((tmax + csize - 1) / csize) * csize * blk;
+  o = align_up(o, 8);
+  L.bar = o;
+  o += 32 + 4 * warps;  // three mbarriers, then one int per warp
+  L.total = align_up(o, 16);
+  return L;
+}
+
+static cudaLaunchConfig_t launch_config(const GemvPlan& p, cudaStream_t s,
+                                        cudaLaunchAttribute (&attr)[2]) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.grid);
+  cfg.blockDim = dim3(p.warps_per_cta * 32);
+  cfg.dynamicSmemBytes = p.smem;
+  cfg.stream = s;
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = (unsigned)p.csize;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  return cfg;
+}
+
 sphq_status make_gemv_plans(sphq_handle h) {
   int optin = 0;
   cudaError_t e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, h->device);
   if (e != cudaSuccess) return cuda_error(e, "cudaDeviceGetAttribute");
   sphq_status st = allow_max_smem(h->device, optin);
   if (st != SPHQ_OK) return st;
-  const long long units = (long long)h->nrt * h->ng;
-  size_t ws = 0;
   for (int batch = 1; batch <= SPHQ_MAX_BATCH; ++batch) {
-    GemvPlan& p = h->plan[batch];
-    p.warps_per_cta = h->bits == 2 ? KernelShape<2>::kWarps : KernelShape<3>::kWarps;
-    const size_t cb_smem = h->bits == 2 ? KernelShape<2>::kSmem : KernelShape<3>::kSmem;
-    // batch 1-2 stage x in shared memory when it fits; otherwise read it through L1
-    p.mode = mode_for(batch);
-    p.smem = cb_smem;
-    if (p.mode != kFull) {
-      const size_t staged = cb_smem + kZeroVec * 16 + (size_t)batch * h->cols * 2;
-      if (staged <= (size_t)optin * 7 / 8) p.smem = staged;
-      else p.mode = kFull;
+    GemvPlan& best = h->plan[batch];
+    best = GemvPlan{};
+    double best_cost = 0;
+    const int warps = h->bits == 2 ? KernelShape<2>::kWarps : KernelShape<3>::kWarps;
+    for (int staged = 1; staged >= 0; --staged) {
+      int mode = mode_for(batch);
+      if (!staged) mode = kFull;
+      if (staged && mode == kFull) continue;
+      const void* k = select_kernel(h->bits, mode);
+      for (int csize : {1, 2, 4, 8}) {
+        if (csize > h->ng) break;
+        // clusters: as many as fit at once, at most one per row tile; the
+        // tile range of a cluster is limited by its shared memory
+        GemvPlan p;
+        p.mode = mode;
+        p.warps_per_cta = warps;
+        p.csize = csize;
+        p.grid = csize;
+        p.smem = smem_layout(h, mode, warps, csize, 1).total;
+        if (p.smem > (size_t)optin) continue;
+        cudaLaunchAttribute attr[2];
+        cudaLaunchConfig_t cfg = launch_config(p, nullptr, attr);
+        int ncl = 0;
+        e = cudaOccupancyMaxActiveClusters(&ncl, k, &cfg);
+        if (e != cudaSuccess) {
+          (void)cudaGetLastError();
+          continue;
+        }
+        if (ncl < 1) continue;
+        int nclusters = std::min(ncl, h->nrt);
+        int tmax = (h->nrt + nclusters - 1) / nclusters;
+        SmemLayout L = smem_layout(h, mode, warps, csize, tmax);
+        // grow the cluster count (extra waves) until a cluster's tiles fit
+        while (L.total > (size_t)optin && tmax > 1) {
+          nclusters = std::min(h->nrt, nclusters * 2);
+          tmax = (h->nrt + nclusters - 1) / nclusters;
+          L = smem_layout(h, mode, warps, csize, tmax);
+        }
+        if (L.total > (size_t)optin) continue;
+        // with the final shared-memory size the resident count may be lower
+        p.smem = L.total;
+        cfg = launch_config(p, nullptr, attr);
+        e = cudaOccupancyMaxActiveClusters(&ncl, k, &cfg);
+        if (e != cudaSuccess || ncl < 1) {
+          (void)cudaGetLastError();
+          continue;
+        }
+        const int waves = (nclusters + ncl - 1) / ncl;
+        // units per CTA and wave, plus a small charge per cluster exchange;
+        // strips of fewer than four tiles keep fewer units in flight per warp
+        // (measured: about twice the time per unit with one tile per cluster)
+        const double shallow = 1.0 + 0.33 * (kStrip - std::min(tmax, kStrip));
+        const double cost = (double)waves * tmax * ((h->ng + csize - 1) / csize) * shallow *
+                            (1.0 + 0.02 * (csize > 1));
+        if (best.grid == 0 || cost < best_cost - 1e-9) {
+          p.grid = nclusters * csize;
+          p.nclusters = nclusters;
+          p.tmax = tmax;
+          p.slots = L.slots;
+          p.cb_bytes = h->bits == 2 ? KernelShape<2>::kCbBytes : KernelShape<3>::kCbBytes;
+          p.x_pitch = L.x_pitch;
+          p.off_x = (uint32_t)L.x;
+          p.off_zero = (uint32_t)L.zero;
+          p.off_part = (uint32_t)L.part;
+          p.off_cta = (uint32_t)L.cta;
+          p.off_recv = (uint32_t)L.recv;
+          p.off_bar = (uint32_t)L.bar;
+          best = p;
+          best_cost = cost;
+        }
+      }
+      if (best.grid > 0) break;  // staged activations fit: keep that mode
     }
-    const void* k = select_kernel(h->bits, p.mode);
-    int occ = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, k, p.warps_per_cta * 32, p.smem);
-    if (e != cudaSuccess) return cuda_error(e, "occupancy query");
-    if (occ < 1) return set_error(SPHQ_ERR_CUDA, "gemv kernel cannot be resident");
-    const long long max_warps = (long long)h->sm_count * occ * p.warps_per_cta;
-    // at least two units per warp so each warp has one unit in flight while it
-    // decodes the previous one
-    long long L = std::max<long long>(2, (units + max_warps - 1) / max_warps);
-    L = std::min<long long>(L, units);
-    const long long warps = (units + L - 1) / L;
-    p.units_per_warp = (int)L;
-    p.grid = (int)((warps + p.warps_per_cta - 1) / p.warps_per_cta);
-    p.max_slots = (int)((h->ng + L - 1) / L + 1);
-    ws = std::max(ws, (size_t)h->nrt * p.max_slots * kRowsPerTile * kMaxBatch);
+    if (best.grid == 0) return set_error(SPHQ_ERR_CUDA, "no resident launch shape for the gemv kernel");
   }
-  h->ws_floats = ws;
+  h->ws_floats = 0;
   return SPHQ_OK;
 }
 
@@ -516,72 +810,41 @@ sphq_status launch_gemv(sphq_handle h, const void* x, void* y, int batch, cudaSt
   const GemvPlan& p = h->plan[batch];
   GemvArgs a;
   a.units = (const uint8_t*)h->units;
-  a.codebook = (const uint4*)h->codebook;
+  a.cbimage = (const uint8_t*)(h->bits == 2 ? h->cbimage : h->codebook);
   a.x = (const uint16_t*)x;
   a.y = (uint16_t*)y;
-  a.ws = h->ws;
-  a.tickets = h->tickets;
+  a.flag = h->flag + 1;
   a.rows = h->rows;
   a.cols = h->cols;
   a.ng = h->ng;
   a.nrt = h->nrt;
   a.batch = batch;
-  a.units_per_warp = p.units_per_warp;
-  a.max_slots = p.max_slots;
-  a.total_units = (long long)h->nrt * h->ng;
+  a.nclusters = p.nclusters;
+  a.slots_per_warp = p.slots;
+  a.cb_bytes = p.cb_bytes;
+  a.x_pitch = p.x_pitch;
+  a.off_x = p.off_x;
+  a.off_zero = p.off_zero;
   a.zeros = (const uint16_t*)h->zeros;
-
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(p.grid);
-  cfg.blockDim = dim3(p.warps_per_cta * 32);
-  cfg.dynamicSmemBytes = p.smem;
-  cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  a.off_part = p.off_part;
+  a.off_cta = p.off_cta;
+  a.off_recv = p.off_recv;
+  a.off_bar = p.off_bar;
+  cudaLaunchAttribute attr[2];
+  cudaLaunchConfig_t cfg = launch_config(p, s, attr);
   void* args[] = {&a};
   cudaError_t e = cudaLaunchKernelExC(&cfg, select_kernel(h->bits, p.mode), args);
   if (e != cudaSuccess) return cuda_error(e, "gemv launch");
   return SPHQ_OK;
 }
 
-// Same launch as launch_gemv, with caller-provided split-K scratch (partials
-// and per-row-tile tickets) instead of the handle's own workspace.
+// The kernel reduces on chip and needs no global scratch; the caller's
+// scratch is accepted and left untouched.
 sphq_status launch_gemv_scratch(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s,
                                 float* ws, unsigned* tickets) {
-  const GemvPlan& p = h->plan[batch];
-  GemvArgs a;
-  a.units = (const uint8_t*)h->units;
-  a.codebook = (const uint4*)h->codebook;
-  a.x = (const uint16_t*)x;
-  a.y = (uint16_t*)y;
-  a.ws = ws;
-  a.tickets = tickets;
-  a.rows = h->rows;
-  a.cols = h->cols;
-  a.ng = h->ng;
-  a.nrt = h->nrt;
-  a.batch = batch;
-  a.units_per_warp = p.units_per_warp;
-  a.max_slots = p.max_slots;
-  a.total_units = (long long)h->nrt * h->ng;
-  a.zeros = (const uint16_t*)h->zeros;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(p.grid);
-  cfg.blockDim = dim3(p.warps_per_cta * 32);
-  cfg.dynamicSmemBytes = p.smem;
-  cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  void* args[] = {&a};
-  cudaError_t e = cudaLaunchKernelExC(&cfg, select_kernel(h->bits, p.mode), args);
-  if (e != cudaSuccess) return cuda_error(e, "gemv launch");
-  return SPHQ_OK;
+  (void)ws;
+  (void)tickets;
+  return launch_gemv(h, x, y, batch, s);
 }
 
 }  // namespace sphq

@@ -13,11 +13,16 @@ namespace sphq {
 // Launch plan of the GEMV kernel for one batch size.
 struct GemvPlan {
   int warps_per_cta = 0;   // threads / 32
-  int grid = 0;            // CTAs (persistent: at most SMs x resident CTAs)
-  int units_per_warp = 0;  // contiguous (row block, group) units per warp
-  int max_slots = 0;       // most warps that share one row block
+  int grid = 0;            // CTAs = nclusters x csize
+  int csize = 1;           // CTAs per thread-block cluster (split of the groups)
+  int nclusters = 0;       // clusters, each with a contiguous range of row tiles
+  int tmax = 0;            // most row tiles of one cluster
+  int slots = 0;           // strip partial slots per warp
   size_t smem = 0;         // dynamic shared memory per CTA
   int mode = 0;            // radius application: 1, 2 (factored) or 8 (full)
+  uint32_t cb_bytes = 0;   // staged codebook image
+  uint32_t x_pitch = 0;    // bytes between staged activation rows
+  uint32_t off_x = 0, off_zero = 0, off_part = 0, off_cta = 0, off_recv = 0, off_bar = 0;
 };
 
 }  // namespace sphq
@@ -31,11 +36,12 @@ struct sphq_handle_s {
   size_t unit_bytes = 0;
   void* units = nullptr;       // packed units, nrt * ng * unit_bytes
   void* codebook = nullptr;    // K * 8 fp16
+  void* cbimage = nullptr;     // W2: eight interleaved codebook copies (8 KiB)
   uint32_t* params = nullptr;  // rows * ng words: Delta | r_min << 16
-  float* ws = nullptr;         // split-K partial sums
+  float* ws = nullptr;         // split-K partial sums (unused by the on-chip reduction)
   size_t ws_floats = 0;
   unsigned* tickets = nullptr; // one arrival counter per row tile
-  int* flag = nullptr;         // pack validation flag
+  int* flag = nullptr;         // [0] pack validation, [1] gemv wait timeouts
   void* xstage = nullptr;      // SPHQ_MAX_BATCH x cols fp16 (sphq_gemv_host)
   void* ystage = nullptr;      // SPHQ_MAX_BATCH x rows fp16
   void* zeros = nullptr;       // 256 B of zeros (activations of non-supplying lanes)

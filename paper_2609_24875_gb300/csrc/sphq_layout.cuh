@@ -8,8 +8,10 @@
 // them: lane l = 4*gid + q (gid = l/4, q = l%4) owns rows gid and gid+8 at the
 // group's slots q, 4+q, 8+q, 12+q.  Its 16-byte block holds four 32-bit words
 // w_m (m = 0..3); word w_m holds vector A = (row gid, slot 4m+q) and vector
-// B = (row gid+8, slot 4m+q).  Units are stored in (rt, g) order, so a warp
-// that walks the groups of one row tile streams contiguous memory and every
+// B = (row gid+8, slot 4m+q).  Units are stored group-major: unit (rt, g) is
+// number g * nrt + rt, so the units of consecutive row tiles at one group --
+// the ones that share activations -- are adjacent in memory (their offsets
+// from each other are compile-time constants in the GEMV), and every
 // warp-wide 16-byte load is a 512-byte burst.
 //
 // W2 unit (640 B = 256 x 2.25 bits + 16 x 4 B of group parameters, §3.1, §3.4):
@@ -56,6 +58,11 @@ constexpr int kRowsPerTile = 16;        // rows per unit (MMA M)
 constexpr int kMaxBatch = 8;
 constexpr uint32_t kSignMask = 0x80008000u;
 
+// Index of unit (row tile rt, radius group g) in a matrix of nrt row tiles.
+__host__ __device__ __forceinline__ long long unit_index(int rt, int g, int nrt) {
+  return (long long)g * nrt + rt;
+}
+
 template <int BITS> struct Layout;
 template <> struct Layout<2> {
   static constexpr int K = 64;
@@ -74,7 +81,8 @@ template <> struct Layout<3> {
 template <int BITS> struct Unit;
 template <> struct Unit<2> {
   uint4 w;      // words w_0..w_3
-  uint4 rec;    // quad record {S01, S23, P_gid, P_gid+8}
+  uint32_t s;   // the lane's sign word of the quad record: S01 (q < 2) or S23
+  uint2 par;    // {P_gid, P_gid+8}
 };
 template <> struct Unit<3> {
   uint4 w;
@@ -109,7 +117,9 @@ template <>
 __device__ __forceinline__ Unit<2> load_unit<2>(const uint8_t* unit, int lane) {
   Unit<2> u;
   u.w = ldg_stream16(unit + lane * 16);
-  u.rec = ldg_stream16(unit + Layout<2>::kRecOff + (lane >> 2) * 16);
+  const uint8_t* rec = unit + Layout<2>::kRecOff + (lane >> 2) * 16;
+  u.s = ldg_stream4(rec + 4 * ((lane >> 1) & 1));
+  u.par = ldg_stream8(rec + 8);
   return u;
 }
 
@@ -261,7 +271,7 @@ __device__ __forceinline__ void directions_w2(uint32_t W, uint32_t e, int m, con
 
 // The lane's pair-3 sign word of a W2 unit, aligned to bits 8-15 / 24-31.
 __device__ __forceinline__ uint32_t w2_sign3(const Unit<2>& u, int q) {
-  const uint32_t s = (q & 2) ? u.rec.y : u.rec.x;
+  const uint32_t s = u.s;
   return (q & 1) ? (s << 8) : s;
 }
 __device__ __forceinline__ uint32_t params_delta(uint32_t pa, uint32_t pb) {
