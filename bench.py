@@ -50,6 +50,24 @@ import sphq_inputs as inp  # noqa: E402
 METRIC = "batch-1 W2/W3 GEMV effective GB/s and % of GB300 HBM peak; µs/token for linear stack"
 UNIT = "GB/s"
 
+# DRAM traffic of the GEMV kernel per launch relative to its algorithmic bytes,
+# from ncu captures of the 8192x8192 batch-1 launches (profiles/
+# gemv_w2_8192_b1_full.md, gemv_w3_8192_b1_full.md), valid for the kernel
+# sources with this digest only; the roofline reports traffic null otherwise.
+TRAFFIC_SOURCES = ("paper_2609_24875_gb300/csrc/sphq_gemv.cu",
+                   "paper_2609_24875_gb300/csrc/sphq_layout.cuh")
+TRAFFIC_DIGEST = "48db05b00cdac416:154cf99e178b8279"
+TRAFFIC_RATIO = {2: 21069056 / 21005312, 3: 28545280 / 28475392}
+
+
+def kernel_digest() -> str:
+    import hashlib
+    out = []
+    for rel in TRAFFIC_SOURCES:
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            out.append(hashlib.sha256(f.read()).hexdigest()[:16])
+    return ":".join(out)
+
 
 def measured_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
@@ -294,9 +312,12 @@ def run_gpu(args, world, rank, local):
     dom_bits = max(per_bits, key=lambda b: per_bits[b][0])
     d_ms, d_bytes, d_launches = per_bits[dom_bits]
     achieved = d_bytes * K / (d_ms * 1e-3) / 1e9
+    traffic = None
+    if kernel_digest() == TRAFFIC_DIGEST:
+        traffic = round(TRAFFIC_RATIO[dom_bits] * d_bytes / d_launches)
     roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm_peak,
                 "unit": "GB/s", "frac": round(achieved / hbm_peak, 4),
-                "traffic": None,
+                "traffic": traffic,
                 "kernel": f"gemv_kernel W{dom_bits} batch 1 ({d_launches} launches/step, "
                           f"{round(100 * d_ms / sum(part_ms), 1)}% of step device time)",
                 "bytes_per_launch": round(d_bytes / d_launches),
@@ -452,6 +473,34 @@ def run_reference(args, world, rank):
     }
 
 
+def run_case(spec: str, pool: int, launches: int):
+    """Profiling driver: `bits:n[:batch]` -> `pool` distinct packed n x n
+    matrices, `launches` GEMVs round robin on one stream, no timing (for
+    running under ncu)."""
+    import torch
+
+    parts = [int(v) for v in spec.split(":")]
+    bits, n = parts[0], parts[1]
+    batch = parts[2] if len(parts) > 2 else 1
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    from paper_2609_24875_gb300 import SphqMatrix
+    codes, x = inp.random_codes(bits, n, n, seed=1, B=batch)
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int16) if a.dtype == np.uint16 else a)).to(dev)
+    mats = []
+    for _ in range(pool):
+        m = SphqMatrix(n, n, bits, t(codes.codebook), t(codes.scale), t(codes.offset))
+        m.pack(t(codes.sign), t(codes.idx), t(codes.rcode))
+        mats.append(m)
+    xd = t(x).view(torch.float16)
+    ys = [torch.empty((batch, n), dtype=torch.float16, device=dev) for _ in mats]
+    s = torch.cuda.current_stream()
+    for i in range(launches):
+        mats[i % pool].gemv_ptr(xd.data_ptr(), ys[i % pool].data_ptr(), batch, s.cuda_stream)
+    torch.cuda.synchronize()
+    print(f"case W{bits} {n}x{n} batch {batch}: {launches} launches over {pool} matrices done")
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -462,7 +511,13 @@ def main():
     ap.add_argument("--no-stack", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--case", default="", help="profiling driver: bits:n[:batch], no timing")
+    ap.add_argument("--pool", type=int, default=4, help="--case: distinct matrices")
+    ap.add_argument("--launches", type=int, default=8, help="--case: GEMV launches")
     args = ap.parse_args()
+    if args.case:
+        run_case(args.case, args.pool, args.launches)
+        return
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     world, rank, local = dist_setup()

@@ -147,11 +147,14 @@ sphq_status sphq_gemv_host(sphq_handle h, const void* x_host, void* y_host, int 
  * that reserve all device memory up front or run under a fixed memory budget;
  * and callers that hold their own allocator's lock or run inside a region
  * where allocation is not allowed.  sphq_gemv itself does not allocate either
- * (sphq_create allocated the handle's workspace), but this variant also works
- * for handles whose workspace memory the caller would rather not keep per
- * matrix: its split-K scratch is a single fixed 4 MiB device array compiled
- * into the library, which every GPU that loads the library holds until the
- * process exits.
+ * (sphq_create allocated everything the handle needs); this variant adds a
+ * guarantee that holds whatever reduction the kernel's launch plan uses: any
+ * split-K scratch a plan needs comes from a single fixed 4 MiB device array
+ * compiled into the library, which every GPU that loads the library holds
+ * until the process exits, never from memory allocated at call time.  (The
+ * current GEMV reduces its partial sums on chip, in shared and distributed
+ * shared memory, so its plans need no scratch and calls only validate and
+ * launch.)
  *
  * Arguments, numerics and asynchrony are those of sphq_gemv.  It calls no
  * cudaMalloc, cudaFree or other allocating routine.  Limits: the matrix may
@@ -163,10 +166,11 @@ sphq_status sphq_gemv_host(sphq_handle h, const void* x_host, void* y_host, int 
  * The first call on each device looks up the array's device address (one
  * cudaGetSymbolAddress with that device current) and caches it; make that
  * first call before any stream capture.  All calls share the one array and it
- * keeps the last call's contents: each call clears the counters it uses (an
- * asynchronous memset on `stream`), and calls that overlap on the GPU -- on
- * different streams or from different host threads -- race on the array and
- * give wrong results.  Serialise them, e.g. on one stream.
+ * keeps the last call's contents: a call whose plan uses the array clears the
+ * counters it needs (an asynchronous memset on `stream`), and such calls that
+ * overlap on the GPU -- on different streams or from different host threads --
+ * race on the array and give wrong results.  Serialise them, e.g. on one
+ * stream.
  */
 sphq_status sphq_gemv_noalloc(sphq_handle h, const void* x, void* y, int batch,
                               sphq_stream stream);

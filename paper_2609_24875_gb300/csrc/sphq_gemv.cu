@@ -356,14 +356,15 @@ __device__ __forceinline__ int share_lo_c(int n, int i) {
 }
 
 // One work item: the activations of one group (xp: this lane's 16 bytes of
-// word 0; words 1-3 follow at 64-byte steps) and the units of up to four row
-// tiles below each other (u[j], unit j of the strip), whose loads for the next
-// item (base nb) are issued as soon as each unit is consumed.  With CHECK, only
-// the units in cmask are processed and only those in nmask loaded.
-template <int BITS, int MODE, bool CHECK>
+// word 0; words 1-3 follow at 64-byte steps) and the units of the strip's
+// SIZE row tiles below each other (u[j]).  Each unit's register slot is
+// refilled with the next item's unit j as soon as it is consumed: unit j of
+// the same strip at the next group (base nb), or, for the strip's LAST item,
+// the units in nmask of the warp's next strip.
+template <int BITS, int MODE, int SIZE, bool LAST>
 __device__ __forceinline__ void run_item(Unit<BITS> (&u)[kStrip], Acc<MODE> (&acc)[kStrip],
-                                         const uint8_t* xp, const uint8_t* nb, unsigned cmask,
-                                         unsigned nmask, int lane, int q, const SmemCodebook& cb) {
+                                         const uint8_t* xp, const uint8_t* nb, unsigned nmask,
+                                         int lane, int q, const SmemCodebook& cb) {
   constexpr int UB = Layout<BITS>::kUnitBytes;
   uint4 xv[4];
 #pragma unroll
@@ -375,9 +376,33 @@ __device__ __forceinline__ void run_item(Unit<BITS> (&u)[kStrip], Acc<MODE> (&ac
   }
 #pragma unroll
   for (int j = 0; j < kStrip; ++j) {
-    if (!CHECK || (cmask >> j & 1u)) process_unit<BITS, MODE>(u[j], xv, q, cb, acc[j]);
-    if (!CHECK || (nmask >> j & 1u)) u[j] = load_unit<BITS>(nb + j * UB, lane);
+    if (j < SIZE) process_unit<BITS, MODE>(u[j], xv, q, cb, acc[j]);
+    if (LAST) {
+      if (nmask >> j & 1u) u[j] = load_unit<BITS>(nb + j * UB, lane);
+    } else if (j < SIZE) {
+      u[j] = load_unit<BITS>(nb + j * UB, lane);
+    }
   }
+}
+
+// cnt >= 1 items of one strip of SIZE tiles at consecutive groups, starting
+// at unit base ub and activations xp; the last item loads the next strip's
+// first units (base nb, mask nmask).
+template <int BITS, int MODE, int SIZE>
+__device__ __forceinline__ void run_segment(Unit<BITS> (&u)[kStrip], Acc<MODE> (&acc)[kStrip],
+                                            int cnt, const uint8_t* ub, size_t gstride,
+                                            const uint8_t* xp, int xstep, const uint8_t* nb,
+                                            unsigned nmask, int lane, int q,
+                                            const SmemCodebook& cb) {
+  constexpr uint32_t kBytes = SIZE * Layout<BITS>::kUnitBytes;
+  if (lane == 0 && cnt > 1) prefetch_l2(ub + gstride, kBytes);
+  for (int c = 0; c + 1 < cnt; ++c) {
+    if (lane == 0 && c + 2 < cnt) prefetch_l2(ub + 2 * gstride, kBytes);
+    run_item<BITS, MODE, SIZE, false>(u, acc, xp, ub + gstride, 0u, lane, q, cb);
+    ub += gstride;
+    xp += xstep;
+  }
+  run_item<BITS, MODE, SIZE, true>(u, acc, xp, nb, nmask, lane, q, cb);
 }
 
 template <int BITS, int MODE, int WARPS, int MINB>
@@ -487,36 +512,23 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
 #pragma unroll
   for (int j = 0; j < kStrip; ++j) acc[j].zero();
 
-  // Units of a full strip at one group are contiguous: one bulk L2 prefetch
-  // per item, two items ahead inside the strip (the next item's units are
-  // already in flight to registers).
-  const uint32_t strip_bytes = kStrip * UB;
-
+  // Units of a strip at one group are contiguous: one bulk L2 prefetch per
+  // item, two items ahead inside the strip (the next item's units are already
+  // in flight to registers).
   int left = i1 - i0;
-  const uint8_t* ub = strip_base(s, g);
-  const uint8_t* xp = x0 + (g - g0) * xstep;
   while (left > 0) {
     // the warp's items of strip s: groups g .. g + cnt - 1
     const int cnt = min(left, g0 + ngc - g);
     left -= cnt;
-    const unsigned cmask = strip_mask(s);
-    int c = 0;
-    if (cmask == kStripMask) {
-      if (lane == 0 && cnt > 1) prefetch_l2(ub + gstride, strip_bytes);
-      for (; c + 1 < cnt; ++c) {  // next item: same strip, next group
-        if (lane == 0 && c + 2 < cnt) prefetch_l2(ub + 2 * gstride, strip_bytes);
-        run_item<BITS, MODE, false>(u, acc, xp, ub + gstride, kStripMask, kStripMask, lane, q, cb);
-        ub += gstride;
-        xp += xstep;
-      }
-    }
-    for (; c < cnt; ++c) {
-      const bool last = c + 1 == cnt;
-      const uint8_t* nb = !last ? ub + gstride : strip_base(s + 1, g0);
-      const unsigned nmask = !last ? cmask : (left > 0 ? strip_mask(s + 1) : 0u);
-      run_item<BITS, MODE, true>(u, acc, xp, nb, cmask, nmask, lane, q, cb);
-      ub += gstride;
-      xp += xstep;
+    const uint8_t* ub = strip_base(s, g);
+    const uint8_t* xp = x0 + (g - g0) * xstep;
+    const uint8_t* nb = strip_base(s + 1, g0);
+    const unsigned nmask = left > 0 ? strip_mask(s + 1) : 0u;
+    switch (s < nfull ? kStrip : T - kStrip * nfull) {
+      case 4: run_segment<BITS, MODE, 4>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask, lane, q, cb); break;
+      case 3: run_segment<BITS, MODE, 3>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask, lane, q, cb); break;
+      case 2: run_segment<BITS, MODE, 2>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask, lane, q, cb); break;
+      default: run_segment<BITS, MODE, 1>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask, lane, q, cb); break;
     }
     float* blk = part + (size_t)(s - first_strip) * kStrip * kBlk;
 #pragma unroll
@@ -526,8 +538,6 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
     }
     ++s;
     g = g0;
-    ub = strip_base(s, g0);
-    xp = x0;
   }
   // the first strip of each warp's items, for locating its partial blocks
   int* wfirst = reinterpret_cast<int*>(smem + a.off_bar + 32);
@@ -775,12 +785,16 @@ sphq_status make_gemv_plans(sphq_handle h) {
           continue;
         }
         const int waves = (nclusters + ncl - 1) / ncl;
-        // units per CTA and wave, plus a small charge per cluster exchange;
-        // strips of fewer than four tiles keep fewer units in flight per warp
-        // (measured: about twice the time per unit with one tile per cluster)
+        // Estimated time per launch (us), from GB300 measurements of
+        // back-to-back launches: a fixed part (launch, staging, reduction,
+        // and the wait for the slowest CTA of a cluster, which grows with the
+        // cluster size) plus ~0.06 us per unit per CTA; strips of fewer than
+        // four tiles keep fewer units in flight per warp (about twice the time
+        // per unit with one tile per cluster).
+        const double fixed = csize == 1 ? 2.6 : csize == 2 ? 3.7 : csize == 4 ? 4.6 : 5.3;
         const double shallow = 1.0 + 0.33 * (kStrip - std::min(tmax, kStrip));
-        const double cost = (double)waves * tmax * ((h->ng + csize - 1) / csize) * shallow *
-                            (1.0 + 0.02 * (csize > 1));
+        const double cost =
+            fixed + waves * 0.06 * tmax * ((h->ng + csize - 1) / csize) * shallow;
         if (best.grid == 0 || cost < best_cost - 1e-9) {
           p.grid = nclusters * csize;
           p.nclusters = nclusters;

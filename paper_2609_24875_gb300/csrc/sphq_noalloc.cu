@@ -1,5 +1,6 @@
-// sphq_gemv_noalloc: the GEMV with its split-K scratch in a fixed, file-scope
-// device array instead of memory the handle allocated.
+// sphq_gemv_noalloc: the GEMV with any split-K scratch in a fixed, file-scope
+// device array instead of memory allocated for it (the current kernel reduces
+// on chip and uses none).
 //
 // The scratch is one `static __device__` array of kScratchBytes on every GPU
 // that loads this library; it lives until the process exits.  Host code may
@@ -75,9 +76,11 @@ extern "C" sphq_status sphq_gemv_noalloc(sphq_handle h, const void* x, void* y, 
   unsigned* tickets = reinterpret_cast<unsigned*>(b);
   float* ws = reinterpret_cast<float*>(b + kTicketBytes);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  // the row-tile counters must start at zero; the array keeps whatever the
-  // previous call left, so clear the part this call uses
-  e = cudaMemsetAsync(tickets, 0, (size_t)h->nrt * sizeof(unsigned), s);
-  if (e != cudaSuccess) return cuda_error(e, "sphq_gemv_noalloc: clear counters");
+  if (h->ws_floats > 0) {
+    // a plan with split-K partials needs its row-tile counters at zero; the
+    // array keeps whatever the previous call left, so clear the part it uses
+    e = cudaMemsetAsync(tickets, 0, (size_t)h->nrt * sizeof(unsigned), s);
+    if (e != cudaSuccess) return cuda_error(e, "sphq_gemv_noalloc: clear counters");
+  }
   return launch_gemv_scratch(h, x, y, batch, s, ws, tickets);
 }
