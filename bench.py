@@ -18,6 +18,8 @@ value    = algorithmic bytes of all GEMVs of a step / device time per step (GB/s
 sweep    = per shape: us per GEMV, GB/s and fraction of HBM (CUDA events
            around each pool's graph)
 stack    = us per token for the W2 and W3 stacks (CUDA events around each)
+stack_fused = the same stacks with q|k|v and gate|up fused by row
+           concatenation (4 GEMVs per layer), timed after the steps
 roofline = the dominant kernel's algorithmic bytes per launch / its average
            launch time (CUDA events on the launching stream), against the
            measured HBM copy bandwidth
@@ -327,6 +329,9 @@ def run_gpu(args, world, rank, local):
     # --- end to end through the host-buffer entry point ---
     e2e = run_e2e(args, shapes, stream)
 
+    # --- the stacks with q|k|v and gate|up fused (4 GEMVs per layer) ---
+    stack_fused = None if args.no_stack else run_fused_stacks(args, dev, stream, hbm_peak)
+
     for s in parts:
         for m in s["mats"]:
             m.close()
@@ -342,7 +347,8 @@ def run_gpu(args, world, rank, local):
                                 "> 10x L2, distinct buffers per GEMV",
                    "parallelism": f"replicas x{world}"},
         "hbm_frac": round(value / hbm_peak, 4),
-        "sweep": sweep, "stack": stack or None, "roofline": roofline, "e2e": e2e,
+        "sweep": sweep, "stack": stack or None, "stack_fused": stack_fused,
+        "roofline": roofline, "e2e": e2e,
         "gpu_launches": launches,
     }
     return out, clk.summary()
@@ -372,15 +378,49 @@ def run_e2e(args, shapes, stream):
             "us_per_step": round(dt / K * 1e6, 2)}
 
 
-def make_stack(args, bits, dev, stream):
-    """The 28-layer x 7-projection linear stack at `bits`, as one CUDA graph
-    of its 196 GEMVs in layer order (one distinct packed matrix each)."""
+def run_fused_stacks(args, dev, stream, hbm_peak):
+    """us/token of the W2 and W3 stacks with fused projections (CUDA events
+    around each graph replay, after 3 warm-up replays)."""
+    import torch
+    res = {}
+    for bits in (2, 3):
+        st = make_stack(args, bits, dev, stream, fused=True)
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                st["graph"].replay()
+        torch.cuda.synchronize()
+        reps = max(3, min(args.steps, 50))
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(reps):
+                st["graph"].replay()
+            e1.record(stream)
+        torch.cuda.synchronize()
+        us = e0.elapsed_time(e1) * 1e3 / reps
+        gbs = st["bytes"] / (us * 1e-6) / 1e9
+        res[st["name"]] = {"us_per_token": round(us, 2), "layers": st["layers"],
+                           "gemvs": st["launches"], "bytes_per_token": st["bytes"],
+                           "GB/s": round(gbs, 1), "hbm_frac": round(gbs / hbm_peak, 4)}
+        for m in st["mats"]:
+            m.close()
+        del st
+        torch.cuda.empty_cache()
+    return res
+
+
+def make_stack(args, bits, dev, stream, fused=False):
+    """The 28-layer linear stack at `bits`, as one CUDA graph of its GEMVs in
+    layer order (one distinct packed matrix each): 7 per layer, or 4 with
+    q|k|v and gate|up fused by row concatenation."""
     import torch
 
     from paper_2609_24875_gb300 import SphqMatrix
     layers = 2 if args.quick else inp.DECODER_LAYERS
+    proj = inp.DECODER_PROJ_FUSED if fused else inp.DECODER_PROJ
     mats, ys, xs = [], [], []
-    for i, (name, rows, cols) in enumerate(inp.DECODER_PROJ):
+    for i, (name, rows, cols) in enumerate(proj):
         codes, x = inp.random_codes(bits, rows, cols, seed=inp.seed_for(4, 10 * bits + i))
         t = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int16) if a.dtype == np.uint16 else a)).to(dev)
         cb, sc, of = t(codes.codebook), t(codes.scale), t(codes.offset)
@@ -403,8 +443,8 @@ def make_stack(args, bits, dev, stream):
     with torch.cuda.graph(g, stream=stream):
         for m, xd, yd in seq:
             m.gemv_ptr(xd.data_ptr(), yd.data_ptr(), 1, stream.cuda_stream)
-    return dict(name=f"W{bits}", bits=bits, graph=g, mats=[m for m, _, _ in seq], keep=(xs, ys),
-                layers=layers,
+    return dict(name=f"W{bits}" + (" fused" if fused else ""), bits=bits, graph=g,
+                mats=[m for m, _, _ in seq], keep=(xs, ys), layers=layers,
                 bytes=sum(m.bytes(1) for m, _, _ in seq), P=1, launches=len(seq))
 
 

@@ -627,8 +627,11 @@ template <> struct KernelShape<2> {
   static constexpr int kMinBlocks = 2;
   static constexpr uint32_t kCbBytes = (uint32_t)Layout<2>::K * 8 * 16;  // 8 copies
 };
+// W3: the 128 KiB codebook allows one CTA per SM; 8 warps with the whole
+// register file (up to 255 registers each) hide the codebook's bank-conflict
+// latency better than 16 warps at 128 (measured 9-15% faster).
 template <> struct KernelShape<3> {
-  static constexpr int kWarps = 16;
+  static constexpr int kWarps = 8;
   static constexpr int kMinBlocks = 1;
   static constexpr uint32_t kCbBytes = (uint32_t)Layout<3>::K * 16;
 };

@@ -142,6 +142,10 @@ DECODER_PROJ = [
     ("down", 3584, 18944),
 ]
 DECODER_LAYERS = 28
+# The same linears with the projections that read the same activations fused
+# by row concatenation (q|k|v and gate|up), as serving engines store them.
+DECODER_PROJ_FUSED = [("qkv", 3584 + 512 + 512, 3584), ("o", 3584, 3584),
+                      ("gate_up", 2 * 18944, 3584), ("down", 3584, 18944)]
 
 # square sweep at batch 1: (bits, n)
 SQUARE_SWEEP = [(2, 4096), (2, 8192), (3, 4096), (3, 8192)]
