@@ -27,15 +27,16 @@
 // Work decomposition.  The row tiles (16 rows) are dealt to thread-block
 // clusters in contiguous, near-equal ranges; every CTA of a cluster takes the
 // same tiles and its own contiguous share of the radius groups (split-K
-// inside the cluster).  Inside a CTA the tiles are cut into strips of four:
-// a work item is (strip, group), i.e. the four units of one group below each
-// other, so the activations of a group are loaded once for four units.  The
+// inside the cluster).  Inside a CTA the tiles are cut into strips of two: a
+// work item is (strip, group), i.e. the two units of one group below each
+// other, so the activations of a group are loaded once for two units.  The
 // items are dealt to the warps in contiguous ranges.  Sums are reduced on
 // chip only and in a fixed order, so results do not depend on scheduling:
-// warp partials per tile go to shared memory, a CTA sums them in warp order,
-// each tile's owner CTA (tile index mod cluster size) receives the other
-// CTAs' sums through distributed shared memory (st.async completing on an
-// mbarrier) and adds them in rank order before writing fp16 y.
+// when a warp leaves a strip it sends its quad-reduced sums of each of the
+// strip's tiles to the tile's owner CTA (tile index mod cluster size) with
+// st.async into the owner's shared memory, completing on the owner's
+// mbarrier; the owner adds the blocks of all covering warps in (rank, warp)
+// order and writes fp16 y.
 //
 // Staging.  The codebook image (W2: eight interleaved copies, 8 KiB; W3: the
 // 128 KiB table) and, for batch 1-2, the CTA's slice of the activations are
@@ -65,7 +66,7 @@
 
 namespace sphq {
 
-constexpr int kStrip = 4;  // row tiles per work item (activation reuse)
+constexpr int kStrip = 2;  // row tiles per work item (activation reuse)
 constexpr unsigned kStripMask = (1u << kStrip) - 1u;
 
 // Radius application modes.
@@ -82,10 +83,9 @@ struct GemvArgs {
   int rows, cols, ng, nrt;
   int batch;
   int nclusters;           // clusters holding tiles (grid = nclusters x cluster size)
-  int slots_per_warp;      // strip partial slots per warp
   uint32_t cb_bytes;       // codebook image bytes
   uint32_t x_pitch;        // bytes between staged activation rows (factored modes)
-  uint32_t off_x, off_zero, off_part, off_cta, off_recv, off_bar;  // dynamic smem offsets
+  uint32_t off_x, off_zero, off_recv, off_bar;  // dynamic smem offsets
   const uint16_t* zeros;   // 256 B of zeros in global memory (batch 3-8 non-suppliers)
 };
 
@@ -107,14 +107,17 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t byt
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
                : "memory");
 }
+// Tests phase `parity` of a local mbarrier; while it is incomplete the thread
+// may sleep up to ~20 us (it wakes as soon as the phase completes), so a
+// waiting warp does not spin on the issue slots.
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
-      : "r"(bar), "r"(parity)
+      : "r"(bar), "r"(parity), "r"(20000u)
       : "memory");
   return ok != 0;
 }
@@ -175,6 +178,12 @@ __device__ __forceinline__ void st_async16(uint32_t raddr, float4 v, uint32_t rb
       "st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1, %2, %3, %4}, "
       "[%5];" ::"r"(raddr),
       "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"(rbar)
+      : "memory");
+}
+__device__ __forceinline__ void st_async4(uint32_t raddr, float v, uint32_t rbar) {
+  asm volatile(
+      "st.async.shared::cluster.mbarrier::complete_tx::bytes.b32 [%0], %1, [%2];" ::"r"(raddr),
+      "r"(__float_as_uint(v)), "r"(rbar)
       : "memory");
 }
 __device__ __forceinline__ void pdl_launch_dependents() {
@@ -309,20 +318,23 @@ __device__ __forceinline__ void process_unit(const Unit<BITS>& cur, const uint4 
   }
 }
 
-// Writes a warp's accumulators of one row tile into its partial block
-// (16 x NBP floats, [batch row][row]).
+// Sends a warp's accumulators of one row tile to the tile's owner CTA:
+// 4-byte st.async stores into the owner's receive slot ([batch row][row]),
+// completing on the owner's receive mbarrier (raddr / rbar are addresses in
+// the owner's shared memory).
 template <int MODE>
-__device__ __forceinline__ void store_partial(float* blk, Acc<MODE>& acc, int lane, int batch) {
+__device__ __forceinline__ void send_partial(uint32_t raddr, uint32_t rbar, Acc<MODE>& acc,
+                                             int lane, int batch) {
   const int gid = lane >> 2, q = lane & 3;
   if constexpr (MODE == kFull) {
     // d[0..3] = D[gid][2q], D[gid][2q+1], D[gid+8][2q], D[gid+8][2q+1]
     if (2 * q < batch) {
-      blk[(2 * q) * kRowsPerTile + gid] = acc.d[0];
-      blk[(2 * q) * kRowsPerTile + gid + 8] = acc.d[2];
+      st_async4(raddr + 4u * ((2 * q) * kRowsPerTile + gid), acc.d[0], rbar);
+      st_async4(raddr + 4u * ((2 * q) * kRowsPerTile + gid + 8), acc.d[2], rbar);
     }
     if (2 * q + 1 < batch) {
-      blk[(2 * q + 1) * kRowsPerTile + gid] = acc.d[1];
-      blk[(2 * q + 1) * kRowsPerTile + gid + 8] = acc.d[3];
+      st_async4(raddr + 4u * ((2 * q + 1) * kRowsPerTile + gid), acc.d[1], rbar);
+      st_async4(raddr + 4u * ((2 * q + 1) * kRowsPerTile + gid + 8), acc.d[3], rbar);
     }
   } else {
     // sum the lane's slots, then the quad's four lanes (slots q = 0..3)
@@ -333,10 +345,23 @@ __device__ __forceinline__ void store_partial(float* blk, Acc<MODE>& acc, int la
         float t = acc.f[i][h];
         t += __shfl_xor_sync(0xFFFFFFFFu, t, 1);
         t += __shfl_xor_sync(0xFFFFFFFFu, t, 2);
-        if (q == 0) blk[i * kRowsPerTile + gid + 8 * h] = t;
+        if (q == 0) st_async4(raddr + 4u * (i * kRowsPerTile + gid + 8 * h), t, rbar);
       }
     }
   }
+}
+
+// Warps of CTA `rank` (of csize) whose items cover strip ts, as a bit mask.
+template <int WARPS>
+__device__ __forceinline__ uint32_t cover_mask(int ng, int nstrips, int rank, int csize, int ts) {
+  const int lo = (int)((unsigned)ng * rank / csize), hi = (int)((unsigned)ng * (rank + 1) / csize);
+  const int ngc = hi - lo, items = nstrips * ngc;
+  uint32_t m = 0;
+  for (int w = 0; w < WARPS; ++w) {
+    const int a0 = (int)((unsigned)items * w / WARPS), a1 = (int)((unsigned)items * (w + 1) / WARPS);
+    if (a0 < a1 && a0 < (ts + 1) * ngc && a1 > ts * ngc) m |= 1u << w;
+  }
+  return m;
 }
 
 // ---------------------------------------------------------------------------
@@ -430,6 +455,7 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
   const int i0 = share_lo_c<WARPS>(items, warp), i1 = share_lo_c<WARPS>(items, warp + 1);
 
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + a.off_bar);
+  uint32_t* masks = reinterpret_cast<uint32_t*>(smem + a.off_bar + 32);  // [owned tile][rank]
   const uint32_t bar_cb = smem_u32(&bars[0]), bar_x = smem_u32(&bars[1]),
                  bar_recv = smem_u32(&bars[2]);
   const int nown = crank < T ? (T - crank + csize - 1) / csize : 0;  // tiles this CTA owns
@@ -460,8 +486,16 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
     mbar_arrive_expect_tx(bar_cb, a.cb_bytes);
     for (uint32_t o = 0; o < a.cb_bytes; o += 32768u)
       bulk_g2s(smem_u32(smem) + o, a.cbimage + o, min(32768u, a.cb_bytes - o), bar_cb);
-    // incoming partial sums of the owned tiles from the other CTAs
-    mbar_arrive_expect_tx(bar_recv, (uint32_t)(nown * (csize - 1) * kBlk * 4));
+    // every warp of the cluster that covers an owned tile sends 64 * batch
+    // bytes for it; remember who, for the final sum
+    uint32_t bytes = 0;
+    for (int k = 0; k < nown; ++k)
+      for (int r = 0; r < csize; ++r) {
+        const uint32_t m = cover_mask<WARPS>(a.ng, nstrips, r, csize, (crank + k * csize) / kStrip);
+        masks[k * csize + r] = m;
+        bytes += (uint32_t)__popc(m) * 64u * (uint32_t)a.batch;
+      }
+    mbar_arrive_expect_tx(bar_recv, bytes);
   }
   if (MODE != kFull && threadIdx.x < 16)  // zero block read by lanes that supply no activations
     reinterpret_cast<uint4*>(smem + a.off_zero)[threadIdx.x] = make_uint4(0, 0, 0, 0);
@@ -476,6 +510,7 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
       bulk_g2s(smem_u32(smem + a.off_x) + b * a.x_pitch,
                a.x + (size_t)b * a.cols + (size_t)g0 * kGroupCols, row_bytes, bar_x);
   }
+  if (csize > 1) cluster_wait();  // every CTA's receive mbarrier is initialised
   bool ok = mbar_wait(bar_cb, 0);
   if (MODE != kFull) ok &= mbar_wait(bar_x, 0);
   if (!ok && lane == 0) atomicOr(a.flag, 2);
@@ -504,9 +539,8 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
   x0 += q * 16;
   const int xstep = provider ? kGroupCols * 2 : 0;
 
-  float* part = reinterpret_cast<float*>(smem + a.off_part) +
-                (size_t)warp * a.slots_per_warp * kStrip * kBlk;
-  const int first_strip = s;
+  // receive slot of (owned tile k, rank r, warp w): ((k * csize + r) * WARPS + w) * kBlk floats
+  const uint32_t recv_base = smem_u32(smem + a.off_recv);
 
   Acc<MODE> acc[kStrip];
 #pragma unroll
@@ -524,96 +558,43 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
     const uint8_t* xp = x0 + (g - g0) * xstep;
     const uint8_t* nb = strip_base(s + 1, g0);
     const unsigned nmask = left > 0 ? strip_mask(s + 1) : 0u;
-    switch (s < nfull ? kStrip : T - kStrip * nfull) {
-      case 4: run_segment<BITS, MODE, 4>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask, lane, q, cb); break;
-      case 3: run_segment<BITS, MODE, 3>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask, lane, q, cb); break;
-      case 2: run_segment<BITS, MODE, 2>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask, lane, q, cb); break;
-      default: run_segment<BITS, MODE, 1>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask, lane, q, cb); break;
-    }
-    float* blk = part + (size_t)(s - first_strip) * kStrip * kBlk;
+    static_assert(kStrip == 2, "strip sizes dispatched below");
+    if (s < nfull)
+      run_segment<BITS, MODE, 2>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask, lane, q, cb);
+    else
+      run_segment<BITS, MODE, 1>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask, lane, q, cb);
 #pragma unroll
     for (int j = 0; j < kStrip; ++j) {
-      store_partial<MODE>(blk + j * kBlk, acc[j], lane, a.batch);
+      const int tau = s * kStrip + j;
+      if (tau < T) {
+        const int owner = tau % csize;
+        const uint32_t slot =
+            recv_base + 4u * (uint32_t)((((tau / csize) * csize + crank) * WARPS + warp) * kBlk);
+        send_partial<MODE>(mapa(slot, (uint32_t)owner), mapa(bar_recv, (uint32_t)owner), acc[j],
+                           lane, a.batch);
+      }
       acc[j].zero();
     }
     ++s;
     g = g0;
   }
-  // the first strip of each warp's items, for locating its partial blocks
-  int* wfirst = reinterpret_cast<int*>(smem + a.off_bar + 32);
-  if (lane == 0) wfirst[warp] = first_strip;
-  __syncthreads();  // every warp partial is in shared memory
-
-  // CTA sums, all threads: thread (tau, l) sums floats 4l..4l+3 of tile tau
-  // over the partial blocks of the warps whose items cover tile tau's strip,
-  // in warp order.
-  float* cta = reinterpret_cast<float*>(smem + a.off_cta);
-  for (int e = threadIdx.x; e < T * 4 * NBP; e += WARPS * 32) {
-    const int tau = e / (4 * NBP), l = e % (4 * NBP);
-    const int ts = tau / kStrip, j = tau % kStrip;
-    float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-    for (int w = 0; w < WARPS; ++w) {
-      const int a0 = share_lo_c<WARPS>(items, w), a1 = share_lo_c<WARPS>(items, w + 1);
-      if (a0 < a1 && a0 < (ts + 1) * ngc && a1 > ts * ngc) {
-        const float* blk = reinterpret_cast<const float*>(smem + a.off_part) +
-                           ((w * a.slots_per_warp + ts - wfirst[w]) * kStrip + j) * kBlk;
-        const float4 v = reinterpret_cast<const float4*>(blk)[l];
-        sum.x += v.x;
-        sum.y += v.y;
-        sum.z += v.z;
-        sum.w += v.w;
-      }
-    }
-    reinterpret_cast<float4*>(cta + (size_t)tau * kBlk)[l] = sum;
-  }
-  __syncthreads();
-
-  // Cluster exchange: tile tau belongs to CTA tau % csize; the others send it
-  // their sums (slot = sender rank) and the owner adds all csize in rank order.
-  auto write_y = [&](int tau, const float4& v, int l) {
-    const int e = 4 * l, b = e / kRowsPerTile, r0 = (t0 + tau) * kRowsPerTile + e % kRowsPerTile;
-    if (b >= a.batch) return;
-    uint16_t* yb = a.y + (size_t)b * a.rows;
-    if (r0 + 0 < a.rows) yb[r0 + 0] = f32_to_h_rn(v.x);
-    if (r0 + 1 < a.rows) yb[r0 + 1] = f32_to_h_rn(v.y);
-    if (r0 + 2 < a.rows) yb[r0 + 2] = f32_to_h_rn(v.z);
-    if (r0 + 3 < a.rows) yb[r0 + 3] = f32_to_h_rn(v.w);
-  };
-  if (csize == 1) {
-    for (int tau = warp; tau < T; tau += WARPS)
-      if (lane < 4 * NBP) write_y(tau, reinterpret_cast<const float4*>(cta + (size_t)tau * kBlk)[lane], lane);
-    return;
-  }
-  cluster_wait();  // every CTA's mbarriers are initialised
-  float* recv = reinterpret_cast<float*>(smem + a.off_recv);
-  for (int tau = warp; tau < T; tau += WARPS) {
-    const int owner = tau % csize;
-    if (lane >= 4 * NBP) continue;
-    const float4 v = reinterpret_cast<const float4*>(cta + (size_t)tau * kBlk)[lane];
-    float* slot = recv + ((size_t)(tau / csize) * csize + crank) * kBlk;
-    if (owner == crank) {
-      reinterpret_cast<float4*>(slot)[lane] = v;
-    } else {
-      const uint32_t raddr = mapa(smem_u32(slot) + 16u * lane, (uint32_t)owner);
-      st_async16(raddr, v, mapa(bar_recv, (uint32_t)owner));
-    }
-  }
+  // Owned tiles (tau = crank + k * csize): wait for every covering warp of
+  // the cluster, then sum their blocks in (rank, warp) order and write y.
   if (nown == 0) return;
   if (!mbar_wait(bar_recv, 0) && threadIdx.x == 0) atomicOr(a.flag, 2);
-  __syncthreads();  // own slots written by the other warps
-  for (int k = warp; k < nown; k += WARPS) {
-    const int tau = crank + k * csize;
-    if (lane >= 4 * NBP) continue;
-    float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int r = 0; r < csize; ++r) {
-      const float4 v = reinterpret_cast<const float4*>(recv + ((size_t)k * csize + r) * kBlk)[lane];
-      sum.x += v.x;
-      sum.y += v.y;
-      sum.z += v.z;
-      sum.w += v.w;
+  const float* recv = reinterpret_cast<const float*>(smem + a.off_recv);
+  for (int e = threadIdx.x; e < nown * kBlk; e += WARPS * 32) {
+    const int k = e / kBlk, i = e % kBlk;
+    const int b = i / kRowsPerTile, r = (t0 + crank + k * csize) * kRowsPerTile + i % kRowsPerTile;
+    if (b >= a.batch || r >= a.rows) continue;
+    float sum = 0.f;
+    for (int rk = 0; rk < csize; ++rk) {
+      const uint32_t m = masks[k * csize + rk];
+#pragma unroll
+      for (int w = 0; w < WARPS; ++w)
+        if (m >> w & 1u) sum += recv[(((size_t)k * csize + rk) * WARPS + w) * kBlk + i];
     }
-    write_y(tau, sum, lane);
+    a.y[(size_t)b * a.rows + r] = f32_to_h_rn(sum);
   }
 }
 
@@ -676,9 +657,8 @@ static size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
 // Shared-memory layout for a given cluster size and tile count per cluster.
 struct SmemLayout {
-  size_t zero, x, part, cta, recv, bar, total;
+  size_t zero, x, recv, bar, total;
   uint32_t x_pitch;
-  int slots;
 };
 
 static SmemLayout smem_layout(const sphq_handle_s* h, int mode, int warps, int csize, int tmax) {
@@ -686,12 +666,7 @@ static SmemLayout smem_layout(const sphq_handle_s* h, int mode, int warps, int c
   const int nbp = mode == kFull ? kMaxBatch : mode;
   const size_t blk = (size_t)kRowsPerTile * nbp * 4;
   const int ngc_max = (h->ng + csize - 1) / csize;
-  const int nstrips = (tmax + kStrip - 1) / kStrip;
-  const long long items = (long long)nstrips * ngc_max;
-  // a warp's items span at most ceil(items / warps) consecutive items, so at
-  // most that many / ngc + 2 strips
-  const long long per_warp = (items + warps - 1) / warps;
-  L.slots = (int)std::min<long long>(nstrips, per_warp / std::max(1, ngc_max) + 2);
+  const int nown_max = (tmax + csize - 1) / csize;  // tiles one CTA owns
   size_t o = h->bits == 2 ? KernelShape<2>::kCbBytes : KernelShape<3>::kCbBytes;
   // batch 1-2: a 256 B zero block, then the activation rows.  Rows start 320 B
   // after the zero block and 64 B apart modulo 128, so within a quarter warp
@@ -701,16 +676,13 @@ static SmemLayout smem_layout(const sphq_handle_s* h, int mode, int warps, int c
   L.x = o + 320;
   L.x_pitch = (uint32_t)((size_t)ngc_max * kGroupCols * 2 + 64);
   if (mode != kFull) o = L.x + (size_t)L.x_pitch * mode;
+  // receive slots: one block per (owned tile, rank, warp)
   o = align_up(o, 16);
-  L.part = o;
-  o += (size_t)warps * L.slots * kStrip * blk;
-  L.cta = o;
-  o += (size_t)tmax * blk;
   L.recv = o;
-  if (csize > 1) o += (size_t)((tmax + csize - 1) / csize) * csize * blk;
+  o += (size_t)nown_max * csize * warps * blk;
   o = align_up(o, 8);
   L.bar = o;
-  o += 32 + 4 * warps;  // three mbarriers, then one int per warp
+  o += 32 + 4 * (size_t)nown_max * csize;  // three mbarriers, then the cover masks
   L.total = align_up(o, 16);
   return L;
 }
@@ -802,13 +774,10 @@ sphq_status make_gemv_plans(sphq_handle h) {
           p.grid = nclusters * csize;
           p.nclusters = nclusters;
           p.tmax = tmax;
-          p.slots = L.slots;
           p.cb_bytes = h->bits == 2 ? KernelShape<2>::kCbBytes : KernelShape<3>::kCbBytes;
           p.x_pitch = L.x_pitch;
           p.off_x = (uint32_t)L.x;
           p.off_zero = (uint32_t)L.zero;
-          p.off_part = (uint32_t)L.part;
-          p.off_cta = (uint32_t)L.cta;
           p.off_recv = (uint32_t)L.recv;
           p.off_bar = (uint32_t)L.bar;
           best = p;
@@ -837,14 +806,11 @@ sphq_status launch_gemv(sphq_handle h, const void* x, void* y, int batch, cudaSt
   a.nrt = h->nrt;
   a.batch = batch;
   a.nclusters = p.nclusters;
-  a.slots_per_warp = p.slots;
   a.cb_bytes = p.cb_bytes;
   a.x_pitch = p.x_pitch;
   a.off_x = p.off_x;
   a.off_zero = p.off_zero;
   a.zeros = (const uint16_t*)h->zeros;
-  a.off_part = p.off_part;
-  a.off_cta = p.off_cta;
   a.off_recv = p.off_recv;
   a.off_bar = p.off_bar;
   cudaLaunchAttribute attr[2];

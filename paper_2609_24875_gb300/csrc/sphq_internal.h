@@ -17,12 +17,11 @@ struct GemvPlan {
   int csize = 1;           // CTAs per thread-block cluster (split of the groups)
   int nclusters = 0;       // clusters, each with a contiguous range of row tiles
   int tmax = 0;            // most row tiles of one cluster
-  int slots = 0;           // strip partial slots per warp
   size_t smem = 0;         // dynamic shared memory per CTA
   int mode = 0;            // radius application: 1, 2 (factored) or 8 (full)
   uint32_t cb_bytes = 0;   // staged codebook image
   uint32_t x_pitch = 0;    // bytes between staged activation rows
-  uint32_t off_x = 0, off_zero = 0, off_part = 0, off_cta = 0, off_recv = 0, off_bar = 0;
+  uint32_t off_x = 0, off_zero = 0, off_recv = 0, off_bar = 0;
 };
 
 }  // namespace sphq
