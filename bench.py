@@ -541,6 +541,124 @@ def run_case(spec: str, pool: int, launches: int):
     print(f"case W{bits} {n}x{n} batch {batch}: {launches} launches over {pool} matrices done")
 
 
+def steady_us(mats, xd, ys, batch, stream, reps=20):
+    """Median over `reps` graph replays of the mean time per GEMV of a CUDA
+    graph of back-to-back launches over the pool."""
+    import torch
+    with torch.cuda.stream(stream):
+        for m, y in zip(mats, ys):
+            m.gemv_ptr(xd.data_ptr(), y.data_ptr(), batch, stream.cuda_stream)
+    stream.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for m, y in zip(mats, ys):
+            m.gemv_ptr(xd.data_ptr(), y.data_ptr(), batch, stream.cuda_stream)
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    times = []
+    for _ in range(reps):
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            g.replay()
+            e1.record(stream)
+        torch.cuda.synchronize()
+        times.append(e0.elapsed_time(e1) * 1e3 / len(mats))
+    del g
+    return statistics.median(times)
+
+
+def cold_us(m, xd, y, batch, stream, flush, reps=10):
+    """Isolated call: L2 flushed by writing a buffer of twice its size, then
+    one GEMV timed alone with events (median of `reps`)."""
+    import torch
+    times = []
+    for _ in range(reps):
+        with torch.cuda.stream(stream):
+            flush.fill_(1.0)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            m.gemv_ptr(xd.data_ptr(), y.data_ptr(), batch, stream.cuda_stream)
+            e1.record(stream)
+        torch.cuda.synchronize()
+        times.append(e0.elapsed_time(e1) * 1e3)
+    return statistics.median(times)
+
+
+def run_report(args):
+    """Per-configuration table (steady state, isolated cold calls, small
+    batch, 7B-class projections, CPU oracle) printed as one JSON object.
+    Supplementary to the contract line; not part of the timed step."""
+    import torch
+
+    from paper_2609_24875_gb300 import SphqMatrix
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.Stream(device=dev)
+    hbm_peak, _ = measured_peaks()
+    L2 = l2_bytes()
+    flush = torch.empty(2 * L2 // 4, dtype=torch.float32, device=dev)
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int16) if a.dtype == np.uint16 else a)).to(dev)
+
+    def pool_for(bits, rows, cols, seed, batch):
+        codes, x = inp.random_codes(bits, rows, cols, seed=seed, B=batch)
+        one = (7 * bits + 4) * rows * cols // 64
+        P = min(512, max(2, int(np.ceil(2 * L2 / one)) + 1))
+        cb, sc, of = t(codes.codebook), t(codes.scale), t(codes.offset)
+        sg, ix, rc = t(codes.sign), t(codes.idx), t(codes.rcode)
+        mats = []
+        for _ in range(P):
+            m = SphqMatrix(rows, cols, bits, cb, sc, of)
+            m.pack(sg, ix, rc)
+            mats.append(m)
+        xd = t(x).view(torch.float16)
+        ys = [torch.empty((batch, rows), dtype=torch.float16, device=dev) for _ in mats]
+        return mats, xd, ys
+
+    def entry(bits, rows, cols, seed, batch, cold=False):
+        mats, xd, ys = pool_for(bits, rows, cols, seed, batch)
+        b = mats[0].bytes(batch)
+        us = steady_us(mats, xd, ys, batch, stream)
+        e = {"us": round(us, 3), "GB/s": round(b / us / 1e3, 1),
+             "hbm_frac": round(b / us / 1e3 / hbm_peak, 4), "bytes": b, "pool": len(mats)}
+        if cold:
+            cu = cold_us(mats[0], xd, ys[0], batch, stream, flush)
+            e["cold_us"] = round(cu, 3)
+        for m in mats:
+            m.close()
+        torch.cuda.empty_cache()
+        return e
+
+    rep = {"steady": "median of 20 graph replays over a pool > 2x L2, back-to-back with PDL",
+           "cold": "one call after writing a 2x L2 buffer, events around the call"}
+    rep["cfg0_w2_1024"] = entry(2, 1024, 1024, inp.seed_for(0, 0), 1, cold=True)
+    rep["cfg1_sweep"] = {f"W{b} {n}x{n}": entry(b, n, n, inp.seed_for(1, i), 1, cold=True)
+                         for i, (b, n) in enumerate(inp.SQUARE_SWEEP)}
+    rep["cfg2_w2_proj"] = {f"{nm} {r}x{c}": entry(2, r, c, inp.seed_for(2, i), 1)
+                           for i, (nm, r, c) in enumerate(inp.DECODER_PROJ) if nm not in ("v", "up")}
+    rep["cfg3_w3_proj_batch"] = {f"{nm} {r}x{c} B{bt}": entry(3, r, c, inp.seed_for(3, i), bt)
+                                 for i, (nm, r, c) in enumerate(inp.DECODER_PROJ)
+                                 if nm in ("q", "k", "gate", "down") for bt in (1, 2, 4, 8)}
+    # CPU oracle on the 1024^2 matrix: single thread and all cores
+    import oracle
+    codes, x = inp.random_codes(2, 1024, 1024, seed=inp.seed_for(0, 0))
+    ocpu = {}
+    for th in (1, oracle.max_threads()):
+        oracle.set_threads(th)
+        t0 = time.perf_counter()
+        n = 0
+        while time.perf_counter() - t0 < 3.0:
+            oracle.decode_gemv(codes.codebook, codes.scale, codes.offset, codes.sign, codes.idx,
+                               codes.rcode, x)
+            n += 1
+        ocpu[f"threads_{th}"] = round((time.perf_counter() - t0) / n * 1e6, 1)
+    rep["oracle_cfg0_us_per_gemv"] = ocpu
+    print(json.dumps(rep), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -554,9 +672,14 @@ def main():
     ap.add_argument("--case", default="", help="profiling driver: bits:n[:batch], no timing")
     ap.add_argument("--pool", type=int, default=4, help="--case: distinct matrices")
     ap.add_argument("--launches", type=int, default=8, help="--case: GEMV launches")
+    ap.add_argument("--report", action="store_true",
+                    help="supplementary per-configuration table (one JSON object)")
     args = ap.parse_args()
     if args.case:
         run_case(args.case, args.pool, args.launches)
+        return
+    if args.report:
+        run_report(args)
         return
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

@@ -351,14 +351,27 @@ __device__ __forceinline__ void send_partial(uint32_t raddr, uint32_t rbar, Acc<
   }
 }
 
+// First item of warp w when the items of a CTA are dealt to WARPS warps in
+// contiguous ranges of near-equal unit counts: items are (strip, group) in
+// strip-major order, ngc per strip, two units each except in the last strip
+// when the tile count T is odd (one unit).  The unit share of warp w starts
+// at unit U*w/WARPS, rounded to an item boundary.
+template <int WARPS>
+__device__ __forceinline__ int warp_item(int T, int ngc, int w) {
+  const int full = (T / kStrip) * ngc;    // items of two units
+  const int units = T * ngc;
+  const int u = (int)((unsigned)units * (unsigned)w / (unsigned)WARPS);
+  return u < 2 * full ? (u + 1) / 2 : full + (u - 2 * full);
+}
+
 // Warps of CTA `rank` (of csize) whose items cover strip ts, as a bit mask.
 template <int WARPS>
-__device__ __forceinline__ uint32_t cover_mask(int ng, int nstrips, int rank, int csize, int ts) {
+__device__ __forceinline__ uint32_t cover_mask(int ng, int T, int rank, int csize, int ts) {
   const int lo = (int)((unsigned)ng * rank / csize), hi = (int)((unsigned)ng * (rank + 1) / csize);
-  const int ngc = hi - lo, items = nstrips * ngc;
+  const int ngc = hi - lo;
   uint32_t m = 0;
   for (int w = 0; w < WARPS; ++w) {
-    const int a0 = (int)((unsigned)items * w / WARPS), a1 = (int)((unsigned)items * (w + 1) / WARPS);
+    const int a0 = warp_item<WARPS>(T, ngc, w), a1 = warp_item<WARPS>(T, ngc, w + 1);
     if (a0 < a1 && a0 < (ts + 1) * ngc && a1 > ts * ngc) m |= 1u << w;
   }
   return m;
@@ -452,7 +465,7 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
   const int nfull = T / kStrip;  // strips with all four tiles
   const unsigned last_mask = (1u << (T - kStrip * nfull)) - 1u;
   const int items = nstrips * ngc;  // item i = (strip i / ngc, group g0 + i % ngc)
-  const int i0 = share_lo_c<WARPS>(items, warp), i1 = share_lo_c<WARPS>(items, warp + 1);
+  const int i0 = warp_item<WARPS>(T, ngc, warp), i1 = warp_item<WARPS>(T, ngc, warp + 1);
 
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + a.off_bar);
   uint32_t* masks = reinterpret_cast<uint32_t*>(smem + a.off_bar + 32);  // [owned tile][rank]
@@ -491,7 +504,7 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
     uint32_t bytes = 0;
     for (int k = 0; k < nown; ++k)
       for (int r = 0; r < csize; ++r) {
-        const uint32_t m = cover_mask<WARPS>(a.ng, nstrips, r, csize, (crank + k * csize) / kStrip);
+        const uint32_t m = cover_mask<WARPS>(a.ng, T, r, csize, (crank + k * csize) / kStrip);
         masks[k * csize + r] = m;
         bytes += (uint32_t)__popc(m) * 64u * (uint32_t)a.batch;
       }
