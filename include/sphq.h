@@ -191,6 +191,38 @@ sphq_status sphq_decode(sphq_handle h, void* w, sphq_stream stream);
  */
 size_t sphq_bytes(sphq_handle h, int batch);
 
+/*
+ * sphq_plan_info / sphq_get_plan -- the launch shape sphq_gemv uses for one
+ * batch size.  (No counterpart in the paper: introspection of this library's
+ * work split.)  Row tiles of 16 rows go to thread-block clusters in contiguous
+ * ranges; the CTAs of a cluster split the 128-column groups and reduce their
+ * partial sums through distributed shared memory.  Fills *out; returns
+ * SPHQ_ERR_INVALID_ARG for a NULL handle or out, or a batch outside 1..8.
+ */
+typedef struct sphq_plan_info {
+  int grid;              /* CTAs launched */
+  int cluster_size;      /* CTAs per thread-block cluster: 1, 2, 4 or 8 */
+  int clusters;          /* clusters, each with a contiguous range of row tiles */
+  int tiles_per_cluster; /* most row tiles of one cluster */
+  int warps_per_cta;
+  int smem_bytes;        /* dynamic shared memory per CTA */
+  int staged_x;          /* 1: activations copied to shared memory (batch 1-2), 0: read via L1 */
+} sphq_plan_info;
+sphq_status sphq_get_plan(sphq_handle h, int batch, sphq_plan_info* out);
+
+/*
+ * sphq_set_cluster_size -- fix the cluster size of the launch shape used for
+ * one batch size (1, 2, 4 or 8), or restore the automatic choice (0).  (No
+ * counterpart in the paper: a tuning and testing knob.)  The library then
+ * uses the cheapest shape at that size by its cost model.  Results do not
+ * change beyond fp32 summation order.  Returns SPHQ_ERR_UNSUPPORTED when the
+ * matrix has fewer 128-column groups than the size or no launch at that size
+ * fits the device (the previous shape stays), SPHQ_ERR_INVALID_ARG for bad
+ * arguments.  Not safe while a GEMV on the handle is being enqueued from
+ * another thread; kernels already enqueued keep their shape.
+ */
+sphq_status sphq_set_cluster_size(sphq_handle h, int batch, int cluster_size);
+
 /* Release the handle and its device memory.  NULL is accepted.  The caller
  * ensures no kernel using the handle is still running. */
 sphq_status sphq_destroy(sphq_handle h);

@@ -167,7 +167,41 @@ using namespace sphq;
 
 extern "C" {
 
-int sphq_version(void) { return 10000; }
+int sphq_version(void) { return 10100; }
+
+sphq_status sphq_get_plan(sphq_handle h, int batch, sphq_plan_info* out) {
+  g_last_error.clear();
+  if (!h || !out) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_get_plan: NULL handle or out");
+  if (batch < 1 || batch > SPHQ_MAX_BATCH)
+    return set_error(SPHQ_ERR_INVALID_ARG, "sphq_get_plan: batch must be 1..8");
+  const GemvPlan& p = h->plan[batch];
+  out->grid = p.grid;
+  out->cluster_size = p.csize;
+  out->clusters = p.nclusters;
+  out->tiles_per_cluster = p.tmax;
+  out->warps_per_cta = p.warps_per_cta;
+  out->smem_bytes = (int)p.smem;
+  out->staged_x = p.mode != 8;
+  return SPHQ_OK;
+}
+
+sphq_status sphq_set_cluster_size(sphq_handle h, int batch, int cluster_size) {
+  g_last_error.clear();
+  if (!h) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_set_cluster_size: NULL handle");
+  if (batch < 1 || batch > SPHQ_MAX_BATCH)
+    return set_error(SPHQ_ERR_INVALID_ARG, "sphq_set_cluster_size: batch must be 1..8");
+  if (cluster_size != 0 && cluster_size != 1 && cluster_size != 2 && cluster_size != 4 &&
+      cluster_size != 8)
+    return set_error(SPHQ_ERR_INVALID_ARG, "sphq_set_cluster_size: size must be 0, 1, 2, 4 or 8");
+  if (cluster_size > h->ng)
+    return set_error(SPHQ_ERR_UNSUPPORTED,
+                     "sphq_set_cluster_size: more CTAs per cluster than 128-column groups");
+  int dev = -1;
+  SPHQ_CUDA(cudaGetDevice(&dev), "cudaGetDevice");
+  if (dev != h->device)
+    return set_error(SPHQ_ERR_DEVICE, "sphq_set_cluster_size: current device is not the handle's");
+  return set_gemv_cluster_size(h, batch, cluster_size);
+}
 
 const char* sphq_last_error(void) { return g_last_error.c_str(); }
 

@@ -461,10 +461,8 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
   const int T = share_lo(a.nrt, cid + 1, a.nclusters) - t0;
   const int g0 = share_lo(a.ng, crank, csize);
   const int ngc = share_lo(a.ng, crank + 1, csize) - g0;
-  const int nstrips = (T + kStrip - 1) / kStrip;
   const int nfull = T / kStrip;  // strips with all four tiles
   const unsigned last_mask = (1u << (T - kStrip * nfull)) - 1u;
-  const int items = nstrips * ngc;  // item i = (strip i / ngc, group g0 + i % ngc)
   const int i0 = warp_item<WARPS>(T, ngc, warp), i1 = warp_item<WARPS>(T, ngc, warp + 1);
 
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + a.off_bar);
@@ -718,15 +716,12 @@ static cudaLaunchConfig_t launch_config(const GemvPlan& p, cudaStream_t s,
   return cfg;
 }
 
-sphq_status make_gemv_plans(sphq_handle h) {
-  int optin = 0;
-  cudaError_t e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, h->device);
-  if (e != cudaSuccess) return cuda_error(e, "cudaDeviceGetAttribute");
-  sphq_status st = allow_max_smem(h->device, optin);
-  if (st != SPHQ_OK) return st;
-  for (int batch = 1; batch <= SPHQ_MAX_BATCH; ++batch) {
-    GemvPlan& best = h->plan[batch];
-    best = GemvPlan{};
+// Launch plan for one batch size: the cheapest shape by the cost model, or
+// the cheapest at cluster size `forced` (1, 2, 4, 8) when it is nonzero.
+static sphq_status make_plan(sphq_handle h, int batch, int forced, int optin, GemvPlan& out) {
+  cudaError_t e;
+  {
+    GemvPlan best{};
     double best_cost = 0;
     const int warps = h->bits == 2 ? KernelShape<2>::kWarps : KernelShape<3>::kWarps;
     for (int staged = 1; staged >= 0; --staged) {
@@ -736,6 +731,7 @@ sphq_status make_gemv_plans(sphq_handle h) {
       const void* k = select_kernel(h->bits, mode);
       for (int csize : {1, 2, 4, 8}) {
         if (csize > h->ng) break;
+        if (forced && csize != forced) continue;
         // clusters: as many as fit at once, at most one per row tile; the
         // tile range of a cluster is limited by its shared memory
         GemvPlan p;
@@ -799,9 +795,41 @@ sphq_status make_gemv_plans(sphq_handle h) {
       }
       if (best.grid > 0) break;  // staged activations fit: keep that mode
     }
-    if (best.grid == 0) return set_error(SPHQ_ERR_CUDA, "no resident launch shape for the gemv kernel");
+    if (best.grid == 0)
+      return set_error(forced ? SPHQ_ERR_UNSUPPORTED : SPHQ_ERR_CUDA,
+                       forced ? "no resident launch shape at this cluster size"
+                              : "no resident launch shape for the gemv kernel");
+    out = best;
+  }
+  return SPHQ_OK;
+}
+
+static sphq_status device_optin(sphq_handle h, int* optin) {
+  cudaError_t e = cudaDeviceGetAttribute(optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, h->device);
+  if (e != cudaSuccess) return cuda_error(e, "cudaDeviceGetAttribute");
+  return allow_max_smem(h->device, *optin);
+}
+
+sphq_status make_gemv_plans(sphq_handle h) {
+  int optin = 0;
+  sphq_status st = device_optin(h, &optin);
+  if (st != SPHQ_OK) return st;
+  for (int batch = 1; batch <= SPHQ_MAX_BATCH; ++batch) {
+    st = make_plan(h, batch, 0, optin, h->plan[batch]);
+    if (st != SPHQ_OK) return st;
   }
   h->ws_floats = 0;
+  return SPHQ_OK;
+}
+
+sphq_status set_gemv_cluster_size(sphq_handle h, int batch, int csize) {
+  int optin = 0;
+  sphq_status st = device_optin(h, &optin);
+  if (st != SPHQ_OK) return st;
+  GemvPlan p;
+  st = make_plan(h, batch, csize, optin, p);
+  if (st != SPHQ_OK) return st;
+  h->plan[batch] = p;
   return SPHQ_OK;
 }
 

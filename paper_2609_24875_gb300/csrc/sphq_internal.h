@@ -55,6 +55,8 @@ sphq_status cuda_error(cudaError_t e, const char* what);
 
 // Builds the GEMV launch plans of a handle (sizes its workspace needs).
 sphq_status make_gemv_plans(sphq_handle h);
+// Re-plans one batch size at a fixed cluster size (0: automatic choice).
+sphq_status set_gemv_cluster_size(sphq_handle h, int batch, int csize);
 // Enqueues the GEMV (validated arguments).
 sphq_status launch_gemv(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s);
 // Enqueues the GEMV with caller-provided split-K scratch: `ws` holds at least

@@ -30,6 +30,14 @@ class SphqError(RuntimeError):
         self.status = status
 
 
+class PlanInfo(ctypes.Structure):
+    """sphq_plan_info: the GEMV launch shape for one batch size."""
+    _fields_ = [("grid", ctypes.c_int), ("cluster_size", ctypes.c_int),
+                ("clusters", ctypes.c_int), ("tiles_per_cluster", ctypes.c_int),
+                ("warps_per_cta", ctypes.c_int), ("smem_bytes", ctypes.c_int),
+                ("staged_x", ctypes.c_int)]
+
+
 def load() -> ctypes.CDLL:
     """Load libsphq.so (built by __graft_entry__.build()); raises if missing."""
     global _lib
@@ -58,6 +66,10 @@ def load() -> ctypes.CDLL:
         L.sphq_last_error.restype = ctypes.c_char_p
         L.sphq_version.argtypes = []
         L.sphq_version.restype = i32
+        L.sphq_get_plan.argtypes = [vp, i32, ctypes.POINTER(PlanInfo)]
+        L.sphq_get_plan.restype = i32
+        L.sphq_set_cluster_size.argtypes = [vp, i32, i32]
+        L.sphq_set_cluster_size.restype = i32
         _lib = L
     return _lib
 
@@ -181,6 +193,16 @@ class SphqMatrix:
 
     def bytes(self, batch: int = 1) -> int:
         return int(load().sphq_bytes(self._h, batch))
+
+    def plan(self, batch: int = 1) -> dict:
+        """The launch shape sphq_gemv uses for `batch` (sphq_get_plan)."""
+        info = PlanInfo()
+        _check(load().sphq_get_plan(self._h, batch, ctypes.byref(info)))
+        return {name: getattr(info, name) for name, _ in PlanInfo._fields_}
+
+    def set_cluster_size(self, batch: int, cluster_size: int) -> None:
+        """Fix the cluster size of the launch shape for `batch` (0: automatic)."""
+        _check(load().sphq_set_cluster_size(self._h, batch, cluster_size))
 
     def close(self) -> None:
         if getattr(self, "_h", None) is not None and self._h.value:

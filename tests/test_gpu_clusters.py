@@ -1,0 +1,65 @@
+"""The GEMV at every thread-block cluster size (sphq_set_cluster_size), on
+shapes whose row-tile counts leave partial strips and uneven clusters, checked
+against the oracle through the C ABI.  Every cluster size exercises another
+reduction path: CTAs of a cluster split the radius groups and send their
+partial sums to each tile's owner CTA through distributed shared memory."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import sphq_inputs as inp
+
+pytestmark = pytest.mark.gpu
+
+import _gpu as G  # noqa: E402
+
+# (bits, rows, cols): 5 and 63 row tiles (a ragged last tile), 8 and 16 groups
+SHAPES = [(2, 80, 1024), (2, 1000, 2048), (3, 112, 2048), (3, 1000, 1024)]
+
+
+def _check(m, codes, x, batch):
+    y = m.gemv(G.x_dev(x))
+    torch.cuda.synchronize()
+    got = y.float().cpu().numpy().astype(np.float64)
+    w = G.oracle_decode(codes)
+    ref, absdot = oracle.gemv(w, x)
+    tol = oracle.gemv_tolerance(absdot)
+    assert got.shape == (batch, codes.rows)
+    assert np.all(np.isfinite(got))
+    assert np.all(np.abs(got - ref) <= tol), float(np.max(np.abs(got - ref) / tol))
+    return y
+
+
+@pytest.mark.parametrize("bits,rows,cols", SHAPES)
+@pytest.mark.parametrize("batch", [1, 2, 5])
+def test_every_cluster_size_matches_oracle(bits, rows, cols, batch):
+    codes, x = inp.random_codes(bits, rows, cols, seed=900 + rows + bits + batch, B=batch)
+    m = G.make_matrix(codes)
+    auto = m.plan(batch)
+    assert auto["cluster_size"] in (1, 2, 4, 8)
+    assert auto["grid"] == auto["clusters"] * auto["cluster_size"]
+    for cs in (1, 2, 4, 8):
+        m.set_cluster_size(batch, cs)
+        p = m.plan(batch)
+        assert p["cluster_size"] == cs
+        assert p["clusters"] * p["tiles_per_cluster"] >= (rows + 15) // 16
+        y1 = _check(m, codes, x, batch)
+        y2 = m.gemv(G.x_dev(x))
+        torch.cuda.synchronize()
+        assert torch.equal(y1, y2)  # fixed summation order
+    m.set_cluster_size(batch, 0)
+    assert m.plan(batch) == auto
+    m.close()
+
+
+def test_cluster_size_larger_than_groups_is_rejected():
+    codes, x = inp.random_codes(2, 64, 256, seed=77)  # 2 groups
+    m = G.make_matrix(codes)
+    before = m.plan(1)
+    from paper_2609_24875_gb300.sphq import SphqError
+    with pytest.raises(SphqError):
+        m.set_cluster_size(1, 4)
+    assert m.plan(1) == before
+    _check(m, codes, x, 1)
+    m.close()

@@ -28,7 +28,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_version(lib):
-    assert lib.sphq_version() >= 10000
+    assert lib.sphq_version() >= 10100
 
 
 def test_invalid_arguments_rejected_on_host(lib):
@@ -50,5 +50,8 @@ def test_invalid_arguments_rejected_on_host(lib):
     assert lib.sphq_decode(None, p, None) == 1
     assert lib.sphq_pack(None, p, p, p, None) == 1
     assert lib.sphq_bytes(None, 1) == 0
+    info = sphq.PlanInfo()
+    assert lib.sphq_get_plan(None, 1, ctypes.byref(info)) == 1
+    assert lib.sphq_set_cluster_size(None, 1, 2) == 1
     assert lib.sphq_destroy(None) == 0
     assert lib.sphq_last_error() == b""
