@@ -433,6 +433,43 @@ __device__ __forceinline__ void run_segment(Unit<BITS> (&u)[kStrip], Acc<MODE> (
                                             unsigned nmask, int lane, int q,
                                             const SmemCodebook& cb) {
   constexpr uint32_t kBytes = SIZE * Layout<BITS>::kUnitBytes;
+  if constexpr (SIZE == 1) {
+    // One-tile strips use the two register slots as a two-item ring (slot
+    // c % 2 holds item c), so two units stay in flight.  The strip is the
+    // warp's last, so nothing is loaded past it (nmask is 0).
+    (void)nb;
+    (void)nmask;
+    if (cnt > 1) u[1] = load_unit<BITS>(ub + gstride, lane);
+    int c = 0;
+    for (; c + 1 < cnt; c += 2) {
+      // items c+2, c+3 go to registers below; c+4, c+5 toward L2
+      if (lane == 0 && c + 4 < cnt) prefetch_l2(ub + 4 * gstride, kBytes);
+      if (lane == 0 && c + 5 < cnt) prefetch_l2(ub + 5 * gstride, kBytes);
+      uint4 xv[4];
+#pragma unroll
+      for (int m = 0; m < 4; ++m) {
+        if constexpr (MODE == kFull)
+          xv[m] = ldg_x16(reinterpret_cast<const uint16_t*>(xp) + 32 * m);
+        else
+          xv[m] = *reinterpret_cast<const uint4*>(xp + 64 * m);
+      }
+      process_unit<BITS, MODE>(u[0], xv, q, cb, acc[0]);
+      if (c + 2 < cnt) u[0] = load_unit<BITS>(ub + 2 * gstride, lane);
+#pragma unroll
+      for (int m = 0; m < 4; ++m) {
+        if constexpr (MODE == kFull)
+          xv[m] = ldg_x16(reinterpret_cast<const uint16_t*>(xp + xstep) + 32 * m);
+        else
+          xv[m] = *reinterpret_cast<const uint4*>(xp + xstep + 64 * m);
+      }
+      process_unit<BITS, MODE>(u[1], xv, q, cb, acc[0]);
+      if (c + 3 < cnt) u[1] = load_unit<BITS>(ub + 3 * gstride, lane);
+      ub += 2 * gstride;
+      xp += 2 * xstep;
+    }
+    if (c < cnt) run_item<BITS, MODE, 1, true>(u, acc, xp, nb, 0u, lane, q, cb);
+    return;
+  }
   if (lane == 0 && cnt > 1) prefetch_l2(ub + gstride, kBytes);
   for (int c = 0; c + 1 < cnt; ++c) {
     if (lane == 0 && c + 2 < cnt) prefetch_l2(ub + 2 * gstride, kBytes);
