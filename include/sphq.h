@@ -125,13 +125,17 @@ sphq_status sphq_gemv(sphq_handle h, const void* x, void* y, int batch, sphq_str
  *
  *   x_host  batch x cols fp16 in host memory; y_host  batch x rows fp16.
  *
- * Enqueues on `stream`: a copy of x into a device staging buffer owned by the
- * handle, the GEMV, and a copy of y back to y_host.  With page-locked
- * (pinned) host buffers the call returns without waiting and y_host is valid
- * once `stream` has been synchronised; with pageable buffers the CUDA runtime
- * makes the copies synchronous.  Same numerics, alignment-free host pointers;
- * the staging buffer makes concurrent calls on one handle invalid, as for
- * sphq_gemv.
+ * With page-locked (pinned) host buffers that are mapped into the device
+ * address space (cudaHostAlloc / cudaHostRegister with mapping, the default
+ * on this platform) and aligned like sphq_gemv's (x 16 bytes, y 4 bytes), the
+ * GEMV kernel reads x and writes y in host memory directly over the
+ * CPU-GPU link: one launch on `stream`, no copy operations.  Otherwise it
+ * enqueues a copy of x into a device staging buffer owned by the handle, the
+ * GEMV, and a copy of y back to y_host; with pageable buffers the CUDA runtime
+ * makes those copies synchronous.  Either way the call returns without
+ * waiting for the GPU (pageable copies aside) and y_host is valid once
+ * `stream` has been synchronised.  Same numerics; the staging buffer makes
+ * concurrent calls on one handle invalid, as for sphq_gemv.
  */
 sphq_status sphq_gemv_host(sphq_handle h, const void* x_host, void* y_host, int batch,
                            sphq_stream stream);

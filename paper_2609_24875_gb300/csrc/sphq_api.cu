@@ -382,6 +382,20 @@ sphq_status sphq_gemv(sphq_handle h, const void* x, void* y, int batch, sphq_str
   return launch_gemv(h, x, y, batch, reinterpret_cast<cudaStream_t>(stream));
 }
 
+// Device address of a page-locked, mapped host buffer, or null for any other
+// pointer (pageable memory, device memory, or an error from the query).
+static const void* mapped_device_pointer(const void* p) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return nullptr;
+  }
+  if (a.type != cudaMemoryTypeHost || !a.devicePointer || !a.hostPointer) return nullptr;
+  // the attributes describe the allocation's base; keep p's offset into it
+  const ptrdiff_t off = static_cast<const char*>(p) - static_cast<const char*>(a.hostPointer);
+  return static_cast<const char*>(a.devicePointer) + off;
+}
+
 sphq_status sphq_gemv_host(sphq_handle h, const void* x_host, void* y_host, int batch,
                            sphq_stream stream) {
   g_last_error.clear();
@@ -391,6 +405,14 @@ sphq_status sphq_gemv_host(sphq_handle h, const void* x_host, void* y_host, int 
   if (!x_host || !y_host) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemv_host: NULL buffer");
   if (!h->packed) return set_error(SPHQ_ERR_NOT_PACKED, "sphq_gemv_host: handle not packed");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  // Page-locked host buffers mapped into the device address space: the
+  // kernel reads x and writes y over the CPU-GPU link directly (coherent on
+  // Grace-Blackwell), with no separate copy operations on the stream.
+  const void* xd = mapped_device_pointer(x_host);
+  void* yd = const_cast<void*>(mapped_device_pointer(y_host));
+  if (xd && yd && reinterpret_cast<uintptr_t>(xd) % 16 == 0 &&
+      reinterpret_cast<uintptr_t>(yd) % 4 == 0)
+    return launch_gemv(h, xd, yd, batch, s);
   SPHQ_CUDA(cudaMemcpyAsync(h->xstage, x_host, (size_t)batch * h->cols * 2,
                             cudaMemcpyHostToDevice, s), "copy x to device");
   sphq_status st = launch_gemv(h, h->xstage, h->ystage, batch, s);
