@@ -63,3 +63,28 @@ def test_cluster_size_larger_than_groups_is_rejected():
     assert m.plan(1) == before
     _check(m, codes, x, 1)
     m.close()
+
+
+# Extreme aspect ratios: one row tile split over a whole cluster of CTAs
+# (long rows), and 16384 row tiles of one group each (tall and thin), plus a
+# W3 row so wide that its staged activations do not fit in shared memory at
+# batch 2 (the plan falls back to reading them through L1).
+@pytest.mark.parametrize("bits,rows,cols,batch", [(2, 16, 262144, 1), (2, 262144, 128, 1),
+                                                  (3, 32, 196608, 2)])
+def test_extreme_shapes(bits, rows, cols, batch):
+    codes, x = inp.random_codes(bits, rows, cols, seed=4100 + bits + batch, B=batch)
+    m = G.make_matrix(codes)
+    p = m.plan(batch)
+    if cols >= 196608 and bits == 3:
+        assert p["staged_x"] == 0
+    rows_chk = G.sample_rows(rows, 512, seed=5) if rows > 4096 else None
+    y = m.gemv(G.x_dev(x))
+    torch.cuda.synchronize()
+    got = y.float().cpu().numpy().astype(np.float64)
+    sel = np.arange(rows) if rows_chk is None else rows_chk
+    w = G.oracle_decode(codes, sel)
+    ref, absdot = oracle.gemv(w, x)
+    err = np.abs(got[:, sel] - ref)
+    assert np.all(np.isfinite(got[:, sel]))
+    assert np.all(err <= oracle.gemv_tolerance(absdot)), float(np.max(err / oracle.gemv_tolerance(absdot)))
+    m.close()
