@@ -212,7 +212,6 @@ static void free_handle(sphq_handle h) {
   cudaFree(h->params);
   cudaFree(h->ws);
   cudaFree(h->cbimage);
-  cudaFree(h->tickets);
   cudaFree(h->flag);
   cudaFree(h->xstage);
   cudaFree(h->ystage);
@@ -270,8 +269,6 @@ sphq_status sphq_create(int rows, int cols, int bits, int K, const void* codeboo
     return fail(cuda_error(e, "cudaMalloc(codebook)"));
   if ((e = cudaMalloc(&h->params, (size_t)rows * ng * 4)) != cudaSuccess)
     return fail(cuda_error(e, "cudaMalloc(params)"));
-  if ((e = cudaMalloc(&h->tickets, (size_t)nrt * sizeof(unsigned))) != cudaSuccess)
-    return fail(cuda_error(e, "cudaMalloc(tickets)"));
   if ((e = cudaMalloc(&h->flag, 2 * sizeof(int))) != cudaSuccess)
     return fail(cuda_error(e, "cudaMalloc(flag)"));
   if ((e = cudaMemset(h->flag, 0, 2 * sizeof(int))) != cudaSuccess)
@@ -302,8 +299,6 @@ sphq_status sphq_create(int rows, int cols, int bits, int K, const void* codeboo
     return fail(cuda_error(e, "copy scale"));
   if ((e = cudaMemcpy(p16 + np, offset, np * 2, cudaMemcpyDefault)) != cudaSuccess)
     return fail(cuda_error(e, "copy offset"));
-  if ((e = cudaMemset(h->tickets, 0, (size_t)nrt * sizeof(unsigned))) != cudaSuccess)
-    return fail(cuda_error(e, "memset tickets"));
   sphq_status st = make_gemv_plans(h);
   if (st != SPHQ_OK) return fail(st);
   if (h->ws_floats > 0 &&
@@ -326,7 +321,6 @@ sphq_status sphq_pack(sphq_handle h, const uint8_t* sign, const uint16_t* idx,
   const uint16_t* scale = reinterpret_cast<const uint16_t*>(h->params);
   const uint16_t* offset = scale + (size_t)h->rows * h->ng;
   SPHQ_CUDA(cudaMemsetAsync(h->flag, 0, sizeof(int), s), "memset flag");
-  SPHQ_CUDA(cudaMemsetAsync(h->tickets, 0, (size_t)h->nrt * sizeof(unsigned), s), "memset tickets");
   SPHQ_CUDA(cudaMemsetAsync(h->units, 0, ((size_t)h->nrt * h->ng + 2) * h->unit_bytes, s),
             "memset units");
   const long long threads = (long long)h->nrt * h->ng * 32;

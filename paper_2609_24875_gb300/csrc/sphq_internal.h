@@ -37,9 +37,8 @@ struct sphq_handle_s {
   void* codebook = nullptr;    // K * 8 fp16
   void* cbimage = nullptr;     // W2: eight interleaved codebook copies (8 KiB)
   uint32_t* params = nullptr;  // rows * ng words: Delta | r_min << 16
-  float* ws = nullptr;         // split-K partial sums (unused by the on-chip reduction)
+  float* ws = nullptr;         // split-K partial sums of plans that need them (none today)
   size_t ws_floats = 0;
-  unsigned* tickets = nullptr; // one arrival counter per row tile
   int* flag = nullptr;         // [0] pack validation, [1] gemv wait timeouts
   void* xstage = nullptr;      // SPHQ_MAX_BATCH x cols fp16 (sphq_gemv_host)
   void* ystage = nullptr;      // SPHQ_MAX_BATCH x rows fp16
