@@ -321,3 +321,73 @@ def encode(w, codebook, V: int = 4, chunk: int = 1 << 14):
     q = np.clip(qf, 0, levels).astype(np.uint8).reshape(rows, cols // VEC)
     return dict(sign=sign, idx=z.astype(np.uint16), rcode=q, scale=scale16,
                 offset=offset16, r_tilde=r_tilde)
+
+
+# ---------------------------------------------------------------------------
+# Quantize side of the path: codebook construction (§3.1, §3.3)
+# ---------------------------------------------------------------------------
+
+def angle_codebook(phi, eps: float = 1e-4) -> np.ndarray:
+    """Positive unit directions from angle logits (§3.3).
+
+    Eq. (sph-angle-logits): theta_j = eps + (pi/2 - 2 eps) * sigmoid(phi_j),
+    so every angle lies in (0, pi/2).  Eq. (sph-angle-codebook): hyperspherical
+    coordinates c_1 = cos th_1, c_i = (prod_{j<i} sin th_j) cos th_i for
+    2 <= i <= 7, c_8 = prod_{j<=7} sin th_j.  phi has shape (..., 7); the result
+    (..., 8) float64 is non-negative with unit norm by construction."""
+    phi = np.asarray(phi, np.float64)
+    assert phi.shape[-1] == VEC - 1
+    theta = eps + (np.pi / 2 - 2 * eps) / (1.0 + np.exp(-phi))
+    c = np.empty(phi.shape[:-1] + (VEC,), np.float64)
+    run = np.ones(phi.shape[:-1], np.float64)  # prod of sines so far
+    for i in range(VEC - 1):
+        c[..., i] = run * np.cos(theta[..., i])
+        run = run * np.sin(theta[..., i])
+    c[..., VEC - 1] = run
+    return c
+
+
+def codebook_angles(c) -> np.ndarray:
+    """Inverse of the coordinates map of Eq. (sph-angle-codebook) for unit
+    vectors with non-negative coordinates: theta_i = atan2(||c_{i+1..8}||, c_i)."""
+    c = np.asarray(c, np.float64)
+    theta = np.empty(c.shape[:-1] + (VEC - 1,), np.float64)
+    for i in range(VEC - 1):
+        tail = np.sqrt(np.sum(c[..., i + 1:] ** 2, axis=-1))
+        theta[..., i] = np.arctan2(tail, c[..., i])
+    return theta
+
+
+def kmeans_codebook(w, K: int, samples: int = 65536, iters: int = 20, seed: int = 0):
+    """Radius-weighted spherical k-means initialisation of the positive
+    direction codebook (§3.1, App. A step 6; 65,536 samples and 20 iterations
+    in the paper's runs).
+
+    The 8-D vectors of w (rows, cols) are decomposed by Eq. (3); `samples`
+    directions d_i are drawn with probability proportional to r_i^2; K of them
+    seed the centres; each iteration assigns every sample to the centre of
+    largest cosine (Eq. (5), ties to the lowest index) and replaces each centre
+    by the normalised mean of its members (an empty cluster keeps its centre).
+    Directions are non-negative, so the centres stay in the positive orthant.
+    Returns (centres (K, 8) float64, objective per iteration: the mean of
+    max_k d_i . c_k over the samples, taken before each update)."""
+    rng = np.random.default_rng(seed)
+    w = np.asarray(w, np.float64)
+    _, _, r, d = decompose(w.reshape(-1, VEC))
+    p = r * r
+    if p.sum() <= 0:
+        raise ValueError("all vectors are zero")
+    pick = rng.choice(d.shape[0], size=samples, replace=True, p=p / p.sum())
+    D = d[pick]
+    centres = D[rng.choice(samples, size=K, replace=False)].copy()
+    history = []
+    for _ in range(iters):
+        scores = D @ centres.T
+        z = np.argmax(scores, axis=1)
+        history.append(float(np.mean(scores[np.arange(samples), z])))
+        sums = np.zeros_like(centres)
+        np.add.at(sums, z, D)
+        norms = np.sqrt(np.sum(sums * sums, axis=1))
+        keep = norms > 0
+        centres[keep] = sums[keep] / norms[keep, None]
+    return centres, history
