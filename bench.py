@@ -516,20 +516,23 @@ def run_reference(args, world, rank):
 def run_case(spec: str, pool: int, launches: int):
     """Profiling driver: `bits:n[:batch]` -> `pool` distinct packed n x n
     matrices, `launches` GEMVs round robin on one stream, no timing (for
-    running under ncu)."""
+    running under ncu).  bits `3v3` selects W3 with 3-bit radius codes."""
     import torch
 
-    parts = [int(v) for v in spec.split(":")]
-    bits, n = parts[0], parts[1]
-    batch = parts[2] if len(parts) > 2 else 1
+    head, *rest = spec.split(":")
+    bits, vbits = (3, 3) if head == "3v3" else (int(head), 4)
+    parts = [int(v) for v in rest]
+    n = parts[0]
+    batch = parts[1] if len(parts) > 1 else 1
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     from paper_2609_24875_gb300 import SphqMatrix
-    codes, x = inp.random_codes(bits, n, n, seed=1, B=batch)
+    codes, x = inp.random_codes(bits, n, n, seed=1, B=batch, radius_bits=vbits)
     t = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int16) if a.dtype == np.uint16 else a)).to(dev)
     mats = []
     for _ in range(pool):
-        m = SphqMatrix(n, n, bits, t(codes.codebook), t(codes.scale), t(codes.offset))
+        m = SphqMatrix(n, n, bits, t(codes.codebook), t(codes.scale), t(codes.offset),
+                       radius_bits=vbits)
         m.pack(t(codes.sign), t(codes.idx), t(codes.rcode))
         mats.append(m)
     xd = t(x).view(torch.float16)
@@ -538,7 +541,8 @@ def run_case(spec: str, pool: int, launches: int):
     for i in range(launches):
         mats[i % pool].gemv_ptr(xd.data_ptr(), ys[i % pool].data_ptr(), batch, s.cuda_stream)
     torch.cuda.synchronize()
-    print(f"case W{bits} {n}x{n} batch {batch}: {launches} launches over {pool} matrices done")
+    print(f"case W{bits} V={vbits} {n}x{n} batch {batch}: {launches} launches over {pool} "
+          "matrices done")
 
 
 def steady_us(mats, xd, ys, batch, stream, reps=20):
@@ -603,23 +607,23 @@ def run_report(args):
     flush = torch.empty(2 * L2 // 4, dtype=torch.float32, device=dev)
     t = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int16) if a.dtype == np.uint16 else a)).to(dev)
 
-    def pool_for(bits, rows, cols, seed, batch):
-        codes, x = inp.random_codes(bits, rows, cols, seed=seed, B=batch)
-        one = (7 * bits + 4) * rows * cols // 64
+    def pool_for(bits, rows, cols, seed, batch, vbits=4):
+        codes, x = inp.random_codes(bits, rows, cols, seed=seed, B=batch, radius_bits=vbits)
+        one = (7 * bits + vbits) * rows * cols // 64
         P = min(512, max(2, int(np.ceil(2 * L2 / one)) + 1))
         cb, sc, of = t(codes.codebook), t(codes.scale), t(codes.offset)
         sg, ix, rc = t(codes.sign), t(codes.idx), t(codes.rcode)
         mats = []
         for _ in range(P):
-            m = SphqMatrix(rows, cols, bits, cb, sc, of)
+            m = SphqMatrix(rows, cols, bits, cb, sc, of, radius_bits=vbits)
             m.pack(sg, ix, rc)
             mats.append(m)
         xd = t(x).view(torch.float16)
         ys = [torch.empty((batch, rows), dtype=torch.float16, device=dev) for _ in mats]
         return mats, xd, ys
 
-    def entry(bits, rows, cols, seed, batch, cold=False):
-        mats, xd, ys = pool_for(bits, rows, cols, seed, batch)
+    def entry(bits, rows, cols, seed, batch, cold=False, vbits=4):
+        mats, xd, ys = pool_for(bits, rows, cols, seed, batch, vbits)
         b = mats[0].bytes(batch)
         us = steady_us(mats, xd, ys, batch, stream)
         e = {"us": round(us, 3), "GB/s": round(b / us / 1e3, 1),
@@ -642,6 +646,10 @@ def run_report(args):
     rep["cfg3_w3_proj_batch"] = {f"{nm} {r}x{c} B{bt}": entry(3, r, c, inp.seed_for(3, i), bt)
                                  for i, (nm, r, c) in enumerate(inp.DECODER_PROJ)
                                  if nm in ("q", "k", "gate", "down") for bt in (1, 2, 4, 8)}
+    # general bit split: W3 with 3-bit radius codes (3.00 bits per weight)
+    rep["w3v3_square"] = {f"W3V3 {n}x{n} B{bt}": entry(3, n, n, inp.seed_for(1, 10 + i), bt,
+                                                       cold=bt == 1, vbits=3)
+                          for i, n in enumerate((4096, 8192)) for bt in (1, 4)}
     # CPU oracle on the 1024^2 matrix: single thread and all cores
     import oracle
     codes, x = inp.random_codes(2, 1024, 1024, seed=inp.seed_for(0, 0))

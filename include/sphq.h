@@ -78,12 +78,30 @@ typedef enum sphq_status {
  * codebook, scale and offset may be host or device pointers (they are read
  * with cudaMemcpyDefault); the call is synchronous and copies them, so the
  * caller may free them on return.  The handle owns all device memory it
- * allocates (packed codes, parameters, codebook, split-K workspace).
+ * allocates (packed codes and parameters, codebook images, an error word and
+ * the staging buffer of sphq_gemv_host).
  * Returns SPHQ_ERR_INVALID_ARG / SPHQ_ERR_UNSUPPORTED / SPHQ_ERR_OOM /
  * SPHQ_ERR_DEVICE / SPHQ_ERR_CUDA; *out is NULL on error.
  */
 sphq_status sphq_create(int rows, int cols, int bits, int K, const void* codebook,
                         const void* scale, const void* offset, sphq_handle* out);
+
+/*
+ * sphq_create_v -- sphq_create with an explicit radius-code width V
+ * (radius_bits), the general bit split of §3.1 and Eq. (7): a vector costs
+ * 8 sign bits + log2(K) index bits + V radius bits.
+ *
+ *   radius_bits  4 (any bits; identical to sphq_create), or 3 with bits = 3:
+ *                W3 at 8 + 13 + 3 = 24 bits per vector (3.00 bits per weight,
+ *                radius codes q < 8).  Other combinations give
+ *                SPHQ_ERR_UNSUPPORTED.
+ *
+ * The other arguments, ownership and errors are those of sphq_create.  With
+ * V = 3 sphq_pack rejects radius codes above 7.
+ */
+sphq_status sphq_create_v(int rows, int cols, int bits, int radius_bits, int K,
+                          const void* codebook, const void* scale, const void* offset,
+                          sphq_handle* out);
 
 /*
  * sphq_pack -- convert canonical codes into the library's device layout
@@ -92,7 +110,8 @@ sphq_status sphq_create(int rows, int cols, int bits, int K, const void* codeboo
  *   sign   rows x (cols/8) uint8, bit j set <=> coordinate j of the vector is
  *          negative (§3.1, Eq. (3)); vector t of a row covers columns 8t..8t+7.
  *   idx    rows x (cols/8) uint16, direction index z < K (Eq. (5)).
- *   rcode  rows x (cols/8) uint8, radius code q < 16 (Eq. (7), V = 4).
+ *   rcode  rows x (cols/8) uint8, radius code q < 2^V (Eq. (7); V = 4, or
+ *          the handle's radius_bits).
  *   stream stream the pack kernel runs on.
  *
  * All three are device pointers.  The call validates every code on the
@@ -111,9 +130,10 @@ sphq_status sphq_pack(sphq_handle h, const uint8_t* sign, const uint16_t* idx,
  *   batch  1..SPHQ_MAX_BATCH.
  *
  * Asynchronous on `stream`: no host synchronisation and no allocation, so it
- * may be captured in a CUDA graph.  The handle owns a split-K workspace, so
- * one handle must not run two gemv calls concurrently (different streams);
- * calls on one stream, or on different handles, are independent.  Numerics:
+ * may be captured in a CUDA graph.  One handle should not run two gemv calls
+ * concurrently (different streams): they share the handle's error word, so a
+ * timeout reported by one could be charged to the other; calls on one stream,
+ * or on different handles, are independent.  Numerics:
  * fp32 accumulation; |y - W_hat x| <= 1e-3 * sum_j |w_hat_j||x_j| + 2^-24 per
  * output (fp16 output rounding included), where W_hat is the exact decode
  * that sphq_decode returns.
@@ -189,7 +209,8 @@ sphq_status sphq_decode(sphq_handle h, void* w, sphq_stream stream);
 
 /*
  * sphq_bytes -- algorithmic bytes one gemv of this batch moves: packed codes
- * (2.25 or 3.125 bits per weight) + group parameters (4 bytes per 128 weights)
+ * ((8 + log2 K + V) / 8 bits per weight: 2.25, 3.125, or 3.00 with V = 3) +
+ * group parameters (4 bytes per 128 weights)
  * + codebook (K*16 bytes, once) + activations (2*batch*cols) + outputs
  * (2*batch*rows).  Returns 0 for a NULL handle or a batch outside 1..8.
  */

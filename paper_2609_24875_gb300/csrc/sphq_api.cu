@@ -60,6 +60,7 @@ __global__ void pack_kernel(const uint8_t* __restrict__ sign, const uint16_t* __
   uint32_t words[4] = {0, 0, 0, 0};
   uint32_t e_lo = 0, e_hi = 0;       // W2: pair-3 sign bytes of the lane
   uint32_t mid = 0, qn = 0, top = 0; // W3
+  uint32_t hw[2] = {0, 0};            // W3, 3-bit radius: H0, H1
   bool bad = false;
   for (int m = 0; m < 4; ++m) {
     for (int half = 0; half < 2; ++half) {  // 0: A (row gid), 1: B (row gid + 8)
@@ -70,7 +71,7 @@ __global__ void pack_kernel(const uint8_t* __restrict__ sign, const uint16_t* __
         s = sign[v];
         k = idx[v];
         rq = rcode[v];
-        if (k >= (uint32_t)Layout<BITS>::K || rq > 15u) {
+        if (k >= (uint32_t)Layout<BITS>::K || rq > (BITS == kFmtW3V3 ? 7u : 15u)) {
           bad = true;
           k = 0;
           rq = 0;
@@ -91,6 +92,9 @@ __global__ void pack_kernel(const uint8_t* __restrict__ sign, const uint16_t* __
         w |= (rq | (k << 4)) << hs;
         e_lo |= ((s >> 6) & 1u) << (7 - v8);
         e_hi |= ((s >> 7) & 1u) << (7 - v8);
+      } else if (BITS == kFmtW3V3) {
+        w |= (k & 0xFFu) << hs;
+        hw[m >> 1] |= (((k >> 8) & 0x1Fu) | (rq << 5)) << (8 * (2 * (m & 1) + half));
       } else {
         w |= (k & 0xFFu) << hs;
         qn |= rq << (4 * m + hs);
@@ -116,6 +120,10 @@ __global__ void pack_kernel(const uint8_t* __restrict__ sign, const uint16_t* __
       *reinterpret_cast<uint32_t*>(rec + 8) = pa;
       *reinterpret_cast<uint32_t*>(rec + 12) = pb;
     }
+  } else if (BITS == kFmtW3V3) {
+    *reinterpret_cast<uint2*>(base + Layout<kFmtW3V3>::kHiOff + lane * 8) = make_uint2(hw[0], hw[1]);
+    if (q == 0)
+      *reinterpret_cast<uint2*>(base + Layout<kFmtW3V3>::kParamOff + gid * 8) = make_uint2(pa, pb);
   } else {
     *reinterpret_cast<uint2*>(base + Layout<3>::kMidOff + lane * 8) = make_uint2(mid, qn);
     if (q == 0)
@@ -150,6 +158,10 @@ __global__ void decode_kernel(const uint8_t* __restrict__ units, const uint8_t* 
     const uint32_t W = word_of(u.w, m);
     directions_w2(W, w2_sign3(u, q), m, cb, 0u, false, sa, sb);
     r = radius_pair(qpair_w2(W), params_delta(u.par.x, u.par.y), params_rmin(u.par.x, u.par.y));
+  } else if constexpr (BITS == kFmtW3V3) {
+    directions_w3v3(u, m, cb, sa, sb);
+    r = radius_pair(qpair_w3v3(u, m), params_delta(u.par.x, u.par.y),
+                    params_rmin(u.par.x, u.par.y));
   } else {
     directions_w3(u, m, q, cb, sa, sb);
     r = radius_pair(qpair_w3(u, m), params_delta(u.par.x, u.par.y),
@@ -221,6 +233,12 @@ static void free_handle(sphq_handle h) {
 
 sphq_status sphq_create(int rows, int cols, int bits, int K, const void* codebook,
                         const void* scale, const void* offset, sphq_handle* out) {
+  return sphq_create_v(rows, cols, bits, 4, K, codebook, scale, offset, out);
+}
+
+sphq_status sphq_create_v(int rows, int cols, int bits, int radius_bits, int K,
+                          const void* codebook, const void* scale, const void* offset,
+                          sphq_handle* out) {
   g_last_error.clear();
   if (!out) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_create: out is NULL");
   *out = nullptr;
@@ -231,6 +249,9 @@ sphq_status sphq_create(int rows, int cols, int bits, int K, const void* codeboo
     return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_create: bits must be 2 or 3");
   if (K != (1 << (7 * bits - 8)))
     return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_create: K must be 2^(7*bits-8)");
+  if (radius_bits != 4 && !(radius_bits == 3 && bits == 3))
+    return set_error(SPHQ_ERR_UNSUPPORTED,
+                     "sphq_create: radius_bits must be 4, or 3 with bits = 3");
   if (!codebook || !scale || !offset)
     return set_error(SPHQ_ERR_INVALID_ARG, "sphq_create: NULL codebook/scale/offset");
   const long long nrt = (rows + kRowsPerTile - 1) / kRowsPerTile;
@@ -254,7 +275,11 @@ sphq_status sphq_create(int rows, int cols, int bits, int K, const void* codeboo
   h->ng = (int)ng;
   h->device = dev;
   h->sm_count = prop.multiProcessorCount;
-  h->unit_bytes = bits == 2 ? Layout<2>::kUnitBytes : Layout<3>::kUnitBytes;
+  h->vbits = radius_bits;
+  h->fmt = bits == 2 ? 2 : radius_bits == 3 ? kFmtW3V3 : 3;
+  h->unit_bytes = h->fmt == 2   ? Layout<2>::kUnitBytes
+                  : h->fmt == 3 ? Layout<3>::kUnitBytes
+                                : Layout<kFmtW3V3>::kUnitBytes;
 
   auto fail = [&](sphq_status s) {
     free_handle(h);
@@ -326,19 +351,24 @@ sphq_status sphq_pack(sphq_handle h, const uint8_t* sign, const uint16_t* idx,
   const long long threads = (long long)h->nrt * h->ng * 32;
   const int block = 256;
   const unsigned grid = (unsigned)((threads + block - 1) / block);
-  if (h->bits == 2)
+  if (h->fmt == 2)
     pack_kernel<2><<<grid, block, 0, s>>>(sign, idx, rcode, scale, offset,
                                           (uint8_t*)h->units, h->rows, h->ng, h->nrt, h->flag);
-  else
+  else if (h->fmt == 3)
     pack_kernel<3><<<grid, block, 0, s>>>(sign, idx, rcode, scale, offset,
                                           (uint8_t*)h->units, h->rows, h->ng, h->nrt, h->flag);
+  else
+    pack_kernel<kFmtW3V3><<<grid, block, 0, s>>>(sign, idx, rcode, scale, offset,
+                                                 (uint8_t*)h->units, h->rows, h->ng, h->nrt,
+                                                 h->flag);
   SPHQ_CUDA(cudaGetLastError(), "pack kernel launch");
   int flag = 0;
   SPHQ_CUDA(cudaMemcpyAsync(&flag, h->flag, sizeof(int), cudaMemcpyDeviceToHost, s), "read flag");
   SPHQ_CUDA(cudaStreamSynchronize(s), "pack");
   if (flag)
     return set_error(SPHQ_ERR_INVALID_ARG,
-                     "sphq_pack: a direction index >= K or a radius code > 15");
+                     h->vbits == 3 ? "sphq_pack: a direction index >= K or a radius code > 7"
+                                   : "sphq_pack: a direction index >= K or a radius code > 15");
   h->packed = true;
   return SPHQ_OK;
 }
@@ -353,12 +383,16 @@ sphq_status sphq_decode(sphq_handle h, void* w, sphq_stream stream) {
   const long long n = (long long)h->rows * (h->cols / kVec);
   const int block = 256;
   const unsigned grid = (unsigned)((n + block - 1) / block);
-  if (h->bits == 2)
+  if (h->fmt == 2)
     decode_kernel<2><<<grid, block, 0, s>>>((const uint8_t*)h->units, (const uint8_t*)h->codebook,
                                             (uint16_t*)w, h->rows, h->cols, h->ng, h->nrt);
-  else
+  else if (h->fmt == 3)
     decode_kernel<3><<<grid, block, 0, s>>>((const uint8_t*)h->units, (const uint8_t*)h->codebook,
                                             (uint16_t*)w, h->rows, h->cols, h->ng, h->nrt);
+  else
+    decode_kernel<kFmtW3V3><<<grid, block, 0, s>>>((const uint8_t*)h->units,
+                                                   (const uint8_t*)h->codebook, (uint16_t*)w,
+                                                   h->rows, h->cols, h->ng, h->nrt);
   SPHQ_CUDA(cudaGetLastError(), "decode kernel launch");
   return SPHQ_OK;
 }
@@ -419,8 +453,8 @@ sphq_status sphq_gemv_host(sphq_handle h, const void* x_host, void* y_host, int 
 size_t sphq_bytes(sphq_handle h, int batch) {
   if (!h || batch < 1 || batch > SPHQ_MAX_BATCH) return 0;
   const size_t weights = (size_t)h->rows * h->cols;
-  // payload bits per 8-D vector: 8 signs + (7B-8) index bits + 4 radius bits
-  const size_t vec_bits = 8 + (7 * h->bits - 8) + 4;
+  // payload bits per 8-D vector: 8 signs + (7B-8) index bits + V radius bits
+  const size_t vec_bits = 8 + (7 * h->bits - 8) + h->vbits;
   const size_t payload = weights / kVec * vec_bits / 8;
   const size_t params = (size_t)h->rows * h->ng * 4;
   const size_t codebook = (size_t)h->K * 16;

@@ -266,6 +266,9 @@ __device__ __forceinline__ void word_directions(const Unit<BITS>& u, const UnitC
     const uint32_t W = word_of(u.w, m);
     directions_w2(W, k.e, m, cb, cb.copyoff, true, sa, sb);
     qp = qpair_w2(W);
+  } else if constexpr (BITS == kFmtW3V3) {
+    directions_w3v3(u, m, cb, sa, sb);
+    qp = qpair_w3v3(u, m);
   } else {
     directions_w3(u, m, q, cb, sa, sb);
     qp = qpair_w3(u, m);
@@ -664,6 +667,16 @@ template <> struct KernelShape<3> {
   static constexpr int kMinBlocks = 1;
   static constexpr uint32_t kCbBytes = (uint32_t)Layout<3>::K * 16;
 };
+template <> struct KernelShape<kFmtW3V3> : KernelShape<3> {};
+
+static int warps_for(int fmt) {
+  return fmt == 2 ? KernelShape<2>::kWarps : fmt == 3 ? KernelShape<3>::kWarps
+                                                      : KernelShape<kFmtW3V3>::kWarps;
+}
+static uint32_t cb_bytes_for(int fmt) {
+  return fmt == 2 ? KernelShape<2>::kCbBytes : fmt == 3 ? KernelShape<3>::kCbBytes
+                                                        : KernelShape<kFmtW3V3>::kCbBytes;
+}
 
 template <int BITS, int MODE>
 static const void* kptr() {
@@ -673,12 +686,14 @@ static const void* kptr() {
 
 static int mode_for(int batch) { return batch == 1 ? kFactored1 : batch == 2 ? kFactored2 : kFull; }
 
-static const void* select_kernel(int bits, int mode) {
-  if (bits == 2)
-    return mode == kFactored1 ? kptr<2, kFactored1>() : mode == kFactored2 ? kptr<2, kFactored2>()
-                                                                           : kptr<2, kFull>();
-  return mode == kFactored1 ? kptr<3, kFactored1>() : mode == kFactored2 ? kptr<3, kFactored2>()
-                                                                         : kptr<3, kFull>();
+template <int FMT>
+static const void* kptr_mode(int mode) {
+  return mode == kFactored1 ? kptr<FMT, kFactored1>() : mode == kFactored2 ? kptr<FMT, kFactored2>()
+                                                                           : kptr<FMT, kFull>();
+}
+
+static const void* select_kernel(int fmt, int mode) {
+  return fmt == 2 ? kptr_mode<2>(mode) : fmt == 3 ? kptr_mode<3>(mode) : kptr_mode<kFmtW3V3>(mode);
 }
 
 // Dynamic shared memory is sized per handle, while the attribute that permits
@@ -691,9 +706,9 @@ static sphq_status allow_max_smem(int device, int optin) {
   if (device < 0 || device >= 64) return set_error(SPHQ_ERR_DEVICE, "device index out of range");
   if (done[device]) return SPHQ_OK;
   const int modes[3] = {kFactored1, kFactored2, kFull};
-  for (int bits = 2; bits <= 3; ++bits)
+  for (int fmt : {2, 3, kFmtW3V3})
     for (int mode : modes) {
-      cudaError_t e = cudaFuncSetAttribute(select_kernel(bits, mode),
+      cudaError_t e = cudaFuncSetAttribute(select_kernel(fmt, mode),
                                            cudaFuncAttributeMaxDynamicSharedMemorySize, optin);
       if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute");
     }
@@ -715,7 +730,7 @@ static SmemLayout smem_layout(const sphq_handle_s* h, int mode, int warps, int c
   const size_t blk = (size_t)kRowsPerTile * nbp * 4;
   const int ngc_max = (h->ng + csize - 1) / csize;
   const int nown_max = (tmax + csize - 1) / csize;  // tiles one CTA owns
-  size_t o = h->bits == 2 ? KernelShape<2>::kCbBytes : KernelShape<3>::kCbBytes;
+  size_t o = cb_bytes_for(h->fmt);
   // batch 1-2: a 256 B zero block, then the activation rows.  Rows start 320 B
   // after the zero block and 64 B apart modulo 128, so within a quarter warp
   // the suppliers' 16-byte chunks and the zero readers' chunks fall in
@@ -760,12 +775,12 @@ static sphq_status make_plan(sphq_handle h, int batch, int forced, int optin, Ge
   {
     GemvPlan best{};
     double best_cost = 0;
-    const int warps = h->bits == 2 ? KernelShape<2>::kWarps : KernelShape<3>::kWarps;
+    const int warps = warps_for(h->fmt);
     for (int staged = 1; staged >= 0; --staged) {
       int mode = mode_for(batch);
       if (!staged) mode = kFull;
       if (staged && mode == kFull) continue;
-      const void* k = select_kernel(h->bits, mode);
+      const void* k = select_kernel(h->fmt, mode);
       for (int csize : {1, 2, 4, 8}) {
         if (csize > h->ng) break;
         if (forced && csize != forced) continue;
@@ -820,7 +835,7 @@ static sphq_status make_plan(sphq_handle h, int batch, int forced, int optin, Ge
           p.grid = nclusters * csize;
           p.nclusters = nclusters;
           p.tmax = tmax;
-          p.cb_bytes = h->bits == 2 ? KernelShape<2>::kCbBytes : KernelShape<3>::kCbBytes;
+          p.cb_bytes = cb_bytes_for(h->fmt);
           p.x_pitch = L.x_pitch;
           p.off_x = (uint32_t)L.x;
           p.off_zero = (uint32_t)L.zero;
@@ -894,7 +909,7 @@ sphq_status launch_gemv(sphq_handle h, const void* x, void* y, int batch, cudaSt
   cudaLaunchAttribute attr[2];
   cudaLaunchConfig_t cfg = launch_config(p, s, attr);
   void* args[] = {&a};
-  cudaError_t e = cudaLaunchKernelExC(&cfg, select_kernel(h->bits, p.mode), args);
+  cudaError_t e = cudaLaunchKernelExC(&cfg, select_kernel(h->fmt, p.mode), args);
   if (e != cudaSuccess) return cuda_error(e, "gemv launch");
   return SPHQ_OK;
 }

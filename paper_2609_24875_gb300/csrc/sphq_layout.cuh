@@ -44,6 +44,14 @@
 //   [832, 864)  quad gid: 4 B, bit (4q + m) = index bit 12 of A of lane q's
 //                 word m, bit (16 + 4q + m) = that of B
 //
+// W3 unit with 3-bit radius codes (the 3.00-bit split of App. B,
+// (7B + V)/8 with V = 3; format id 4 below), 832 B = 256 x 3 bits x 8 + 64 B:
+//   [0, 512)    lane l: words w_0..w_3 exactly as in the W3 unit
+//   [512, 768)  lane l: 8 B = { H0, H1 }; word m owns byte 2*(m%2) (A) and
+//                 byte 2*(m%2)+1 (B) of H_{m/2}: index bits 8-12 in bits 0-4,
+//                 radius code (0..7) in bits 5-7
+//   [768, 832)  quad gid: 8 B = { P_gid, P_gid+8 }
+//
 // No byte beyond the algorithmic payload is stored; padded rows hold zero
 // codes and parameters.
 #pragma once
@@ -63,11 +71,22 @@ __host__ __device__ __forceinline__ long long unit_index(int rt, int g, int nrt)
   return (long long)g * nrt + rt;
 }
 
+// Format ids used as template arguments: 2 = W2, 3 = W3, 4 = W3 with 3-bit
+// radius codes.  The codebook size follows the weight bit-width B.
+constexpr int kFmtW3V3 = 4;
+__host__ __device__ constexpr int fmt_bits(int fmt) { return fmt == kFmtW3V3 ? 3 : fmt; }
+
 template <int BITS> struct Layout;
 template <> struct Layout<2> {
   static constexpr int K = 64;
   static constexpr int kUnitBytes = 640;
   static constexpr int kRecOff = 512;
+};
+template <> struct Layout<kFmtW3V3> {
+  static constexpr int K = 8192;
+  static constexpr int kUnitBytes = 832;
+  static constexpr int kHiOff = 512;
+  static constexpr int kParamOff = 768;
 };
 template <> struct Layout<3> {
   static constexpr int K = 8192;
@@ -82,6 +101,11 @@ template <int BITS> struct Unit;
 template <> struct Unit<2> {
   uint4 w;      // words w_0..w_3
   uint32_t s;   // the lane's sign word of the quad record: S01 (q < 2) or S23
+  uint2 par;    // {P_gid, P_gid+8}
+};
+template <> struct Unit<kFmtW3V3> {
+  uint4 w;
+  uint2 hi;     // {H0, H1}
   uint2 par;    // {P_gid, P_gid+8}
 };
 template <> struct Unit<3> {
@@ -130,6 +154,15 @@ __device__ __forceinline__ Unit<3> load_unit<3>(const uint8_t* unit, int lane) {
   u.mq = ldg_stream8(unit + Layout<3>::kMidOff + lane * 8);
   u.par = ldg_stream8(unit + Layout<3>::kParamOff + (lane >> 2) * 8);
   u.top = ldg_stream4(unit + Layout<3>::kTopOff + (lane >> 2) * 4);
+  return u;
+}
+
+template <>
+__device__ __forceinline__ Unit<kFmtW3V3> load_unit<kFmtW3V3>(const uint8_t* unit, int lane) {
+  Unit<kFmtW3V3> u;
+  u.w = ldg_stream16(unit + lane * 16);
+  u.hi = ldg_stream8(unit + Layout<kFmtW3V3>::kHiOff + lane * 8);
+  u.par = ldg_stream8(unit + Layout<kFmtW3V3>::kParamOff + (lane >> 2) * 8);
   return u;
 }
 
@@ -302,6 +335,32 @@ __device__ __forceinline__ void directions_w3(const Unit<3>& u, int m, int q, co
   const uint4 cbv = cb.at(offB);
   sa = apply_signs(ca, W, shl_fma<1>(W), shl_fma<2>(W), shl_fma<3>(W));
   sb = apply_signs(cbv, shl_fma<4>(W), shl_fma<5>(W), shl_fma<6>(W), shl_fma<7>(W));
+}
+
+// The two bytes of word m of a 3-bit-radius W3 unit moved to bits 8-15 (A)
+// and 24-31 (B) of a zeroed word: index bits 8-12 at 8-12 / 24-28, radius
+// code at 13-15 / 29-31.
+__device__ __forceinline__ uint32_t w3v3_hi(const Unit<kFmtW3V3>& u, int m) {
+  const uint32_t h = (m < 2) ? u.hi.x : u.hi.y;
+  return (m & 1) ? prmt<0x3424u>(h, 0u) : prmt<0x1404u>(h, 0u);
+}
+
+// Signed directions of word m of a 3-bit-radius W3 unit.
+template <class CB>
+__device__ __forceinline__ void directions_w3v3(const Unit<kFmtW3V3>& u, int m, const CB& cb,
+                                                uint4& sa, uint4& sb) {
+  const uint32_t W = word_of(u.w, m);
+  const uint32_t k2 = (W & 0x00FF00FFu) | (w3v3_hi(u, m) & 0x1F001F00u);
+  const uint32_t offA = shl_fma<4>(k2) & 0x1FFF0u;
+  const uint32_t offB = (k2 >> 12) & 0x1FFF0u;
+  const uint4 ca = cb.at(offA);
+  const uint4 cbv = cb.at(offB);
+  sa = apply_signs(ca, W, shl_fma<1>(W), shl_fma<2>(W), shl_fma<3>(W));
+  sb = apply_signs(cbv, shl_fma<4>(W), shl_fma<5>(W), shl_fma<6>(W), shl_fma<7>(W));
+}
+// Radius codes of word m (A at bits 0-2, B at bits 16-18; bit 3 / 19 zero).
+__device__ __forceinline__ uint32_t qpair_w3v3(const Unit<kFmtW3V3>& u, int m) {
+  return w3v3_hi(u, m) >> 13;
 }
 
 // Radius codes of word m as a pair (A at bits 0-3, B at bits 16-19).

@@ -50,6 +50,8 @@ def load() -> ctypes.CDLL:
         vp, i32, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
         L.sphq_create.argtypes = [i32, i32, i32, i32, vp, vp, vp, ctypes.POINTER(vp)]
         L.sphq_create.restype = i32
+        L.sphq_create_v.argtypes = [i32, i32, i32, i32, i32, vp, vp, vp, ctypes.POINTER(vp)]
+        L.sphq_create_v.restype = i32
         L.sphq_pack.argtypes = [vp, vp, vp, vp, vp]
         L.sphq_pack.restype = i32
         L.sphq_gemv.argtypes = [vp, vp, vp, i32, vp]
@@ -100,7 +102,8 @@ class SphqMatrix:
     Host or device tensors are accepted for these three (they are copied).
     """
 
-    def __init__(self, rows: int, cols: int, bits: int, codebook, scale, offset):
+    def __init__(self, rows: int, cols: int, bits: int, codebook, scale, offset,
+                 radius_bits: int = 4):
         import torch
         L = load()
         K = 1 << (7 * bits - 8)
@@ -112,10 +115,11 @@ class SphqMatrix:
                 raise ValueError(f"expected a 2-byte tensor of shape {shape}, got "
                                  f"{tuple(t.shape)} {t.dtype}")
         h = ctypes.c_void_p()
-        _check(L.sphq_create(rows, cols, bits, K, cb.data_ptr(), sc.data_ptr(), of.data_ptr(),
-                             ctypes.byref(h)))
+        _check(L.sphq_create_v(rows, cols, bits, radius_bits, K, cb.data_ptr(), sc.data_ptr(),
+                               of.data_ptr(), ctypes.byref(h)))
         self._h = h
         self.rows, self.cols, self.bits, self.K = rows, cols, bits, K
+        self.radius_bits = radius_bits
         self.device = torch.device("cuda", torch.cuda.current_device())
 
     @property
@@ -152,8 +156,8 @@ class SphqMatrix:
         _check(load().sphq_gemv(self._h, x_ptr, y_ptr, batch, stream_ptr))
 
     def gemv_noalloc(self, x, y, stream=None):
-        """sphq_gemv_noalloc: the GEMV with the library's fixed device scratch
-        instead of the handle's workspace (no allocation on any call).
+        """sphq_gemv_noalloc: the GEMV through the entry point that guarantees
+        no allocation on any call, the first included.
         x: (batch, cols) and y: (batch, rows) fp16 CUDA tensors."""
         L = load()
         L.sphq_gemv_noalloc.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,

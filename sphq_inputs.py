@@ -11,7 +11,7 @@ Recipe (every draw from numpy's PCG64, seed = 20260 + 100*config + shape):
   offset      r_min_G ~ U(0, 1)    -> fp16
   sign        U{0..255} per 8-D vector
   idx         U{0..K-1}
-  rcode       U{0..15}
+  rcode       U{0..2^V - 1}, V = 4 (or 3 for the 3-bit-radius W3 split)
   x           N(0, 1) -> fp16, shape (B, cols)
 Gaussian weight matrices (the encoded configuration) are N(0, 0.02^2) with
 0.1% of the scalars, chosen uniformly, multiplied by 20.
@@ -44,6 +44,7 @@ class Codes:
     sign: np.ndarray      # (rows, cols/8) uint8
     idx: np.ndarray       # (rows, cols/8) uint16
     rcode: np.ndarray     # (rows, cols/8) uint8
+    vbits: int = RADIUS_BITS  # radius code width V (codes < 2^V)
 
     @property
     def rows(self) -> int:
@@ -59,7 +60,7 @@ class Codes:
 
     def row_slice(self, r0: int, r1: int) -> "Codes":
         return Codes(self.bits, self.codebook, self.scale[r0:r1], self.offset[r0:r1],
-                     self.sign[r0:r1], self.idx[r0:r1], self.rcode[r0:r1])
+                     self.sign[r0:r1], self.idx[r0:r1], self.rcode[r0:r1], self.vbits)
 
 
 def seed_for(config: int, shape: int = 0) -> int:
@@ -88,8 +89,9 @@ def make_x(rng: np.random.Generator, B: int, cols: int) -> np.ndarray:
 
 
 def random_codes(bits: int, rows: int, cols: int, seed: int, B: int = 1,
-                 codebook: np.ndarray | None = None):
-    """Uniformly random codes (configurations 0, 2, 3, 4).  Returns (Codes, x)."""
+                 codebook: np.ndarray | None = None, radius_bits: int = RADIUS_BITS):
+    """Uniformly random codes (configurations 0, 2, 3, 4), radius codes drawn
+    from U{0..2^radius_bits - 1}.  Returns (Codes, x)."""
     if cols % GROUP_COLS:
         raise ValueError("cols must be a multiple of 128")
     rng = np.random.Generator(np.random.PCG64(seed))
@@ -101,9 +103,9 @@ def random_codes(bits: int, rows: int, cols: int, seed: int, B: int = 1,
     nv = cols // VEC
     sign = rng.integers(0, 256, size=(rows, nv), dtype=np.uint8)
     idx = rng.integers(0, K, size=(rows, nv), dtype=np.uint16)
-    rcode = rng.integers(0, 1 << RADIUS_BITS, size=(rows, nv), dtype=np.uint8)
+    rcode = rng.integers(0, 1 << radius_bits, size=(rows, nv), dtype=np.uint8)
     x = make_x(rng, B, cols)
-    return Codes(bits, cb, scale, offset, sign, idx, rcode), x
+    return Codes(bits, cb, scale, offset, sign, idx, rcode, radius_bits), x
 
 
 def gaussian_weights(rows: int, cols: int, seed: int, std: float = 0.02,

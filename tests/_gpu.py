@@ -18,7 +18,7 @@ def to_dev(a):
 
 def make_matrix(codes: inp.Codes) -> SphqMatrix:
     m = SphqMatrix(codes.rows, codes.cols, codes.bits, to_dev(codes.codebook),
-                   to_dev(codes.scale), to_dev(codes.offset))
+                   to_dev(codes.scale), to_dev(codes.offset), radius_bits=codes.vbits)
     m.pack(to_dev(codes.sign), to_dev(codes.idx), to_dev(codes.rcode))
     return m
 
@@ -38,7 +38,7 @@ def decoded_bits(m: SphqMatrix, rows=None) -> np.ndarray:
 def oracle_decode(codes: inp.Codes, rows=None) -> np.ndarray:
     c = codes if rows is None else inp.Codes(codes.bits, codes.codebook, codes.scale[rows],
                                              codes.offset[rows], codes.sign[rows],
-                                             codes.idx[rows], codes.rcode[rows])
+                                             codes.idx[rows], codes.rcode[rows], codes.vbits)
     return oracle.decode(c.codebook, c.scale, c.offset, c.sign, c.idx, c.rcode)
 
 
