@@ -87,17 +87,20 @@ sphq_status sphq_create(int rows, int cols, int bits, int K, const void* codeboo
                         const void* scale, const void* offset, sphq_handle* out);
 
 /*
- * sphq_create_v -- sphq_create with an explicit radius-code width V
- * (radius_bits), the general bit split of §3.1 and Eq. (7): a vector costs
- * 8 sign bits + log2(K) index bits + V radius bits.
+ * sphq_create_v -- sphq_create for a general bit split (§3.1, Eq. (7),
+ * Tab. 4, App. B): a vector costs 8 sign bits + D = log2(K) direction-index
+ * bits + V = radius_bits radius bits, i.e. (8 + D + V) / 8 bits per weight.
  *
- *   radius_bits  4 (any bits; identical to sphq_create), or 3 with bits = 3:
- *                W3 at 8 + 13 + 3 = 24 bits per vector (3.00 bits per weight,
- *                radius codes q < 8).  Other combinations give
- *                SPHQ_ERR_UNSUPPORTED.
+ *   bits = 3     K = 8192 (D = 13) with radius_bits 4 (W3, 3.125 b/w; the
+ *                same as sphq_create) or 3 (3.00 b/w, radius codes q < 8).
+ *   bits = 2     K = 64, 128 or 256 (D = 6, 7, 8) with D + V <= 10:
+ *                8/6/4 (W2, 2.25 b/w; the same as sphq_create), 8/6/3,
+ *                8/6/2 (2.00 b/w), 8/7/3, 8/7/2, 8/8/2 -- the splits of the
+ *                bit-allocation ablation (Tab. 4).
  *
- * The other arguments, ownership and errors are those of sphq_create.  With
- * V = 3 sphq_pack rejects radius codes above 7.
+ * codebook is K x 8 fp16.  Other combinations give SPHQ_ERR_UNSUPPORTED.  The
+ * other arguments, ownership and errors are those of sphq_create; sphq_pack
+ * then rejects direction indices >= K and radius codes >= 2^V.
  */
 sphq_status sphq_create_v(int rows, int cols, int bits, int radius_bits, int K,
                           const void* codebook, const void* scale, const void* offset,
@@ -209,7 +212,8 @@ sphq_status sphq_decode(sphq_handle h, void* w, sphq_stream stream);
 
 /*
  * sphq_bytes -- algorithmic bytes one gemv of this batch moves: packed codes
- * ((8 + log2 K + V) / 8 bits per weight: 2.25, 3.125, or 3.00 with V = 3) +
+ * ((8 + log2 K + V) / 8 bits per weight: 2.25 (W2), 3.125 (W3), or the split
+ * chosen with sphq_create_v) +
  * group parameters (4 bytes per 128 weights)
  * + codebook (K*16 bytes, once) + activations (2*batch*cols) + outputs
  * (2*batch*rows).  Returns 0 for a NULL handle or a batch outside 1..8.

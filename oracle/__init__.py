@@ -257,6 +257,12 @@ def codebook_bytes(bits: int, dim: int = VEC, signed: bool = False) -> int:
     return n * dim * 2
 
 
+def split_bits_per_weight(dir_bits: int, V: int, dim: int = VEC) -> float:
+    """Encoded payload per weight of a sign / direction-index / radius split
+    (Tab. 4): (dim sign bits + dir_bits + V) / dim."""
+    return (dim + dir_bits + V) / dim
+
+
 def payload_bits_per_weight(bits: int, V: int, dim: int = VEC) -> float:
     """Encoded payload (7B + V)/8 per weight for 8-D vectors (App. B): sign bits,
     direction index and radius code, excluding group parameters and codebook."""

@@ -12,6 +12,9 @@
 
 namespace sphq {
 
+// every format id (sphq_layout.cuh)
+#define SPHQ_FOR_EACH_FMT(X) X(2) X(3) X(4) X(5) X(6) X(7) X(8) X(9)
+
 static thread_local std::string g_last_error;
 // zero block read by GEMV lanes that supply no activations (4 words x 4 lanes x 16 B)
 constexpr size_t kZeroBytes = 256;
@@ -57,8 +60,12 @@ __global__ void pack_kernel(const uint8_t* __restrict__ sign, const uint16_t* __
   const int nv = ng * kGroupVecs;
   uint8_t* base = units + (size_t)unit * Layout<BITS>::kUnitBytes;
 
+  constexpr bool kSmall = fmt_small(BITS);
+  constexpr int kV = fmt_radius_bits(BITS);
+  constexpr int kExtra = kSmall ? fmt_dir_bits(BITS) + kV - 8 : 0;
   uint32_t words[4] = {0, 0, 0, 0};
-  uint32_t e_lo = 0, e_hi = 0;       // W2: pair-3 sign bytes of the lane
+  uint32_t e_lo = 0, e_hi = 0;       // W2 record: pair-3 sign bytes of the lane
+  uint32_t rword = 0;                // one extra bit per vector: the lane's bits of R
   uint32_t mid = 0, qn = 0, top = 0; // W3
   uint32_t hw[2] = {0, 0};            // W3, 3-bit radius: H0, H1
   bool bad = false;
@@ -71,7 +78,7 @@ __global__ void pack_kernel(const uint8_t* __restrict__ sign, const uint16_t* __
         s = sign[v];
         k = idx[v];
         rq = rcode[v];
-        if (k >= (uint32_t)Layout<BITS>::K || rq > (BITS == kFmtW3V3 ? 7u : 15u)) {
+        if (k >= (uint32_t)Layout<BITS>::K || rq >= (1u << kV)) {
           bad = true;
           k = 0;
           rq = 0;
@@ -80,18 +87,25 @@ __global__ void pack_kernel(const uint8_t* __restrict__ sign, const uint16_t* __
       const int v8 = 2 * m + half;   // vector number within the lane, 0..7
       const int hs = 16 * half;      // B's index/radius fields sit 16 bits higher
       // sign bits 2p / 2p+1 go to bits (top - p) / (top - p + 16), where top is
-      // 15 for A and, below A's bits, 12 (W2) or 11 (W3) for B
-      const int top_bit = half == 0 ? 15 : (BITS == 2 ? 12 : 11);
-      const int npairs = BITS == 2 ? 3 : 4;
+      // 15 for A and, below A's pairs, 15 - (A's pairs in the word) for B
+      const int na = kSmall ? (kExtra <= 1 ? 4 : 3) : 4;
+      const int nb = kSmall ? (kExtra == 0 ? 4 : 3) : 4;
+      const int top_bit = half == 0 ? 15 : 15 - na;
+      const int npairs = half == 0 ? na : nb;
       uint32_t w = 0;
       for (int p = 0; p < npairs; ++p) {
         w |= ((s >> (2 * p)) & 1u) << (top_bit - p);
         w |= ((s >> (2 * p + 1)) & 1u) << (top_bit - p + 16);
       }
-      if (BITS == 2) {
-        w |= (rq | (k << 4)) << hs;
-        e_lo |= ((s >> 6) & 1u) << (7 - v8);
-        e_hi |= ((s >> 7) & 1u) << (7 - v8);
+      if (kSmall) {
+        w |= (rq | (k << kV)) << hs;
+        if (kExtra == 2) {
+          e_lo |= ((s >> 6) & 1u) << (7 - v8);
+          e_hi |= ((s >> 7) & 1u) << (7 - v8);
+        } else if (kExtra == 1 && half == 1) {
+          rword |= ((s >> 6) & 1u) << (15 - 4 * q - m);
+          rword |= ((s >> 7) & 1u) << (31 - 4 * q - m);
+        }
       } else if (BITS == kFmtW3V3) {
         w |= (k & 0xFFu) << hs;
         hw[m >> 1] |= (((k >> 8) & 0x1Fu) | (rq << 5)) << (8 * (2 * (m & 1) + half));
@@ -110,8 +124,8 @@ __global__ void pack_kernel(const uint8_t* __restrict__ sign, const uint16_t* __
   const int ra = rt * kRowsPerTile + gid, rb = ra + 8;
   if (ra < rows) pa = (uint32_t)scale[(size_t)ra * ng + g] | ((uint32_t)offset[(size_t)ra * ng + g] << 16);
   if (rb < rows) pb = (uint32_t)scale[(size_t)rb * ng + g] | ((uint32_t)offset[(size_t)rb * ng + g] << 16);
-  if (BITS == 2) {
-    uint8_t* rec = base + Layout<2>::kRecOff + gid * 16;
+  if constexpr (kSmall && kExtra == 2) {
+    uint8_t* rec = base + Layout<BITS>::kRecOff + gid * 16;
     uint8_t* sw = rec + 4 * (q >> 1);          // S01 or S23
     const int b0 = (q & 1) ? 0 : 1;            // even lane: bytes 1, 3; odd lane: bytes 0, 2
     sw[b0] = (uint8_t)e_lo;
@@ -120,7 +134,12 @@ __global__ void pack_kernel(const uint8_t* __restrict__ sign, const uint16_t* __
       *reinterpret_cast<uint32_t*>(rec + 8) = pa;
       *reinterpret_cast<uint32_t*>(rec + 12) = pb;
     }
-  } else if (BITS == kFmtW3V3) {
+  } else if constexpr (kSmall) {
+    if (kExtra == 1)
+      atomicOr(reinterpret_cast<unsigned*>(base + Layout<BITS>::kRecOff + gid * 4), rword);
+    if (q == 0)
+      *reinterpret_cast<uint2*>(base + Layout<BITS>::kParamOff + gid * 8) = make_uint2(pa, pb);
+  } else if constexpr (BITS == kFmtW3V3) {
     *reinterpret_cast<uint2*>(base + Layout<kFmtW3V3>::kHiOff + lane * 8) = make_uint2(hw[0], hw[1]);
     if (q == 0)
       *reinterpret_cast<uint2*>(base + Layout<kFmtW3V3>::kParamOff + gid * 8) = make_uint2(pa, pb);
@@ -154,14 +173,15 @@ __global__ void decode_kernel(const uint8_t* __restrict__ units, const uint8_t* 
   GlobalCodebook cb{codebook};
   uint4 sa, sb;
   uint32_t r;
-  if constexpr (BITS == 2) {
+  if constexpr (fmt_small(BITS)) {
     const uint32_t W = word_of(u.w, m);
-    directions_w2(W, w2_sign3(u, q), m, cb, 0u, false, sa, sb);
-    r = radius_pair(qpair_w2(W), params_delta(u.par.x, u.par.y), params_rmin(u.par.x, u.par.y));
+    directions_small<BITS>(W, sign_extra<BITS>(u, q), m, cb, 0u, false, sa, sb);
+    r = radius_pair<fmt_radius_bits(BITS)>(W, params_delta(u.par.x, u.par.y),
+                                           params_rmin(u.par.x, u.par.y));
   } else if constexpr (BITS == kFmtW3V3) {
     directions_w3v3(u, m, cb, sa, sb);
-    r = radius_pair(qpair_w3v3(u, m), params_delta(u.par.x, u.par.y),
-                    params_rmin(u.par.x, u.par.y));
+    r = radius_pair<3>(qpair_w3v3(u, m), params_delta(u.par.x, u.par.y),
+                       params_rmin(u.par.x, u.par.y));
   } else {
     directions_w3(u, m, q, cb, sa, sb);
     r = radius_pair(qpair_w3(u, m), params_delta(u.par.x, u.par.y),
@@ -247,11 +267,19 @@ sphq_status sphq_create_v(int rows, int cols, int bits, int radius_bits, int K,
                      "sphq_create: need rows >= 1 and cols a positive multiple of 128");
   if (bits != 2 && bits != 3)
     return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_create: bits must be 2 or 3");
-  if (K != (1 << (7 * bits - 8)))
-    return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_create: K must be 2^(7*bits-8)");
-  if (radius_bits != 4 && !(radius_bits == 3 && bits == 3))
+  // direction index bits D = log2 K: 13 for W3; 6 (the §3.1 rule), 7 or 8 (Tab. 4) for W2
+  int dbits = -1;
+  for (int d = 0; d < 31; ++d)
+    if (K == (1 << d)) dbits = d;
+  const bool k_ok = bits == 3 ? dbits == 13 : (dbits >= 6 && dbits <= 8);
+  if (!k_ok)
     return set_error(SPHQ_ERR_UNSUPPORTED,
-                     "sphq_create: radius_bits must be 4, or 3 with bits = 3");
+                     "sphq_create: K must be 8192 for bits = 3 and 64, 128 or 256 for bits = 2");
+  const int fmt = fmt_of_split(dbits, radius_bits);
+  if (fmt < 0)
+    return set_error(SPHQ_ERR_UNSUPPORTED,
+                     "sphq_create: unsupported split; sign/index/radius bits must be one of "
+                     "8/6/4, 8/6/3, 8/6/2, 8/7/3, 8/7/2, 8/8/2, 8/13/4, 8/13/3");
   if (!codebook || !scale || !offset)
     return set_error(SPHQ_ERR_INVALID_ARG, "sphq_create: NULL codebook/scale/offset");
   const long long nrt = (rows + kRowsPerTile - 1) / kRowsPerTile;
@@ -276,10 +304,9 @@ sphq_status sphq_create_v(int rows, int cols, int bits, int radius_bits, int K,
   h->device = dev;
   h->sm_count = prop.multiProcessorCount;
   h->vbits = radius_bits;
-  h->fmt = bits == 2 ? 2 : radius_bits == 3 ? kFmtW3V3 : 3;
-  h->unit_bytes = h->fmt == 2   ? Layout<2>::kUnitBytes
-                  : h->fmt == 3 ? Layout<3>::kUnitBytes
-                                : Layout<kFmtW3V3>::kUnitBytes;
+  h->dbits = dbits;
+  h->fmt = fmt;
+  h->unit_bytes = fmt_unit_bytes(fmt);
 
   auto fail = [&](sphq_status s) {
     free_handle(h);
@@ -308,8 +335,8 @@ sphq_status sphq_create_v(int rows, int cols, int bits, int radius_bits, int K,
     return fail(cuda_error(e, "memset zeros"));
   if ((e = cudaMemcpy(h->codebook, codebook, (size_t)K * 16, cudaMemcpyDefault)) != cudaSuccess)
     return fail(cuda_error(e, "copy codebook"));
-  if (bits == 2) {
-    // shared-memory image of the W2 GEMV: entry k, copy c at 128 k + 16 c
+  if (fmt_small(fmt)) {
+    // shared-memory image of the small-codebook GEMV: entry k, copy c at 128 k + 16 c
     if ((e = cudaMalloc(&h->cbimage, (size_t)K * 8 * 16)) != cudaSuccess)
       return fail(cuda_error(e, "cudaMalloc(codebook image)"));
     for (int c = 0; c < 8; ++c)
@@ -351,24 +378,24 @@ sphq_status sphq_pack(sphq_handle h, const uint8_t* sign, const uint16_t* idx,
   const long long threads = (long long)h->nrt * h->ng * 32;
   const int block = 256;
   const unsigned grid = (unsigned)((threads + block - 1) / block);
-  if (h->fmt == 2)
-    pack_kernel<2><<<grid, block, 0, s>>>(sign, idx, rcode, scale, offset,
-                                          (uint8_t*)h->units, h->rows, h->ng, h->nrt, h->flag);
-  else if (h->fmt == 3)
-    pack_kernel<3><<<grid, block, 0, s>>>(sign, idx, rcode, scale, offset,
-                                          (uint8_t*)h->units, h->rows, h->ng, h->nrt, h->flag);
-  else
-    pack_kernel<kFmtW3V3><<<grid, block, 0, s>>>(sign, idx, rcode, scale, offset,
-                                                 (uint8_t*)h->units, h->rows, h->ng, h->nrt,
-                                                 h->flag);
+  switch (h->fmt) {
+#define SPHQ_PACK_CASE(F)                                                                   \
+  case F:                                                                                   \
+    pack_kernel<F><<<grid, block, 0, s>>>(sign, idx, rcode, scale, offset,                  \
+                                          (uint8_t*)h->units, h->rows, h->ng, h->nrt, h->flag); \
+    break;
+    SPHQ_FOR_EACH_FMT(SPHQ_PACK_CASE)
+#undef SPHQ_PACK_CASE
+    default:
+      return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_pack: unknown format");
+  }
   SPHQ_CUDA(cudaGetLastError(), "pack kernel launch");
   int flag = 0;
   SPHQ_CUDA(cudaMemcpyAsync(&flag, h->flag, sizeof(int), cudaMemcpyDeviceToHost, s), "read flag");
   SPHQ_CUDA(cudaStreamSynchronize(s), "pack");
   if (flag)
     return set_error(SPHQ_ERR_INVALID_ARG,
-                     h->vbits == 3 ? "sphq_pack: a direction index >= K or a radius code > 7"
-                                   : "sphq_pack: a direction index >= K or a radius code > 15");
+                     "sphq_pack: a direction index >= K or a radius code >= 2^radius_bits");
   h->packed = true;
   return SPHQ_OK;
 }
@@ -383,16 +410,18 @@ sphq_status sphq_decode(sphq_handle h, void* w, sphq_stream stream) {
   const long long n = (long long)h->rows * (h->cols / kVec);
   const int block = 256;
   const unsigned grid = (unsigned)((n + block - 1) / block);
-  if (h->fmt == 2)
-    decode_kernel<2><<<grid, block, 0, s>>>((const uint8_t*)h->units, (const uint8_t*)h->codebook,
-                                            (uint16_t*)w, h->rows, h->cols, h->ng, h->nrt);
-  else if (h->fmt == 3)
-    decode_kernel<3><<<grid, block, 0, s>>>((const uint8_t*)h->units, (const uint8_t*)h->codebook,
-                                            (uint16_t*)w, h->rows, h->cols, h->ng, h->nrt);
-  else
-    decode_kernel<kFmtW3V3><<<grid, block, 0, s>>>((const uint8_t*)h->units,
-                                                   (const uint8_t*)h->codebook, (uint16_t*)w,
-                                                   h->rows, h->cols, h->ng, h->nrt);
+  switch (h->fmt) {
+#define SPHQ_DECODE_CASE(F)                                                                    \
+  case F:                                                                                      \
+    decode_kernel<F><<<grid, block, 0, s>>>((const uint8_t*)h->units,                          \
+                                            (const uint8_t*)h->codebook, (uint16_t*)w, h->rows, \
+                                            h->cols, h->ng, h->nrt);                           \
+    break;
+    SPHQ_FOR_EACH_FMT(SPHQ_DECODE_CASE)
+#undef SPHQ_DECODE_CASE
+    default:
+      return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_decode: unknown format");
+  }
   SPHQ_CUDA(cudaGetLastError(), "decode kernel launch");
   return SPHQ_OK;
 }
@@ -453,8 +482,8 @@ sphq_status sphq_gemv_host(sphq_handle h, const void* x_host, void* y_host, int 
 size_t sphq_bytes(sphq_handle h, int batch) {
   if (!h || batch < 1 || batch > SPHQ_MAX_BATCH) return 0;
   const size_t weights = (size_t)h->rows * h->cols;
-  // payload bits per 8-D vector: 8 signs + (7B-8) index bits + V radius bits
-  const size_t vec_bits = 8 + (7 * h->bits - 8) + h->vbits;
+  // payload bits per 8-D vector: 8 signs + D index bits + V radius bits
+  const size_t vec_bits = 8 + h->dbits + h->vbits;
   const size_t payload = weights / kVec * vec_bits / 8;
   const size_t params = (size_t)h->rows * h->ng * 4;
   const size_t codebook = (size_t)h->K * 16;

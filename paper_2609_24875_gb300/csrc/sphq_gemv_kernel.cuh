@@ -1,0 +1,688 @@
+// Fused spherical dequantize-GEMV kernel for decode (SPHQuant §3.4, App. D), sm_103a.
+//
+// y[n][r] = sum_j w_hat[r][j] x[n][j] for a batch of n <= 8 activation rows.
+//
+// Decode stays on the CUDA cores: each thread rebuilds whole 8-D blocks in
+// registers (codebook entry from shared memory, coordinate signs, radius of
+// Eq. (7)) and never writes them to memory.  The multiply-accumulate with the
+// activations runs on the tensor cores as m16n8k16 MMAs with fp32
+// accumulation; the thread/fragment mapping of the unit layout
+// (sphq_layout.cuh) puts the two blocks a thread decodes from word w_m
+// directly into the A fragment -- coordinates 0-3 feed one MMA and 4-7 the
+// next -- and the matching activations go in the B fragment.  Products of two
+// fp16 values are exact in fp32.
+//
+// Two ways of applying the radius, chosen by batch size:
+//  * batch 1-2 ("factored"): the A fragment holds the signed unit direction
+//    s (.) c_z and the B fragment is block diagonal -- column 2c + b carries
+//    batch row b of slot c only -- so every MMA pair returns, in the lane
+//    that decoded them, the per-vector dots d = (s (.) c_z) . x_b.  The lane
+//    then adds r_hat * d with one fp32 FMA (r_hat from the fp16 FMA of
+//    Eq. (7)).  This skips the four half-rate fp16 products per block; the
+//    result differs from the exact W_hat x by at most one fp16 rounding of
+//    each product r_hat * c (2^-11 relative), inside the stated tolerance.
+//  * batch 3-8 ("full"): the lane forms w_hat = RN16(r_hat * (s (.) c_z))
+//    exactly as Eq. (4) defines it and the MMA's N dimension is the batch.
+//
+// Work decomposition.  The row tiles (16 rows) are dealt to thread-block
+// clusters in contiguous, near-equal ranges; every CTA of a cluster takes the
+// same tiles and its own contiguous share of the radius groups (split-K
+// inside the cluster).  Inside a CTA the tiles are cut into strips of two: a
+// work item is (strip, group), i.e. the two units of one group below each
+// other, so the activations of a group are loaded once for two units.  The
+// items are dealt to the warps in contiguous ranges.  Sums are reduced on
+// chip only and in a fixed order, so results do not depend on scheduling:
+// when a warp leaves a strip it sends its quad-reduced sums of each of the
+// strip's tiles to the tile's owner CTA (tile index mod cluster size) with
+// st.async into the owner's shared memory, completing on the owner's
+// mbarrier; the owner adds the blocks of all covering warps in (rank, warp)
+// order and writes fp16 y.
+//
+// Staging.  The codebook image (W2: eight interleaved copies, 8 KiB; W3: the
+// 128 KiB table) and, for batch 1-2, the CTA's slice of the activations are
+// copied into shared memory by bulk asynchronous copies completing on
+// mbarriers.  Codes stream from HBM through registers (16-byte loads that
+// bypass L1) one work item ahead of use, and a bulk L2 prefetch runs two
+// items further ahead (an item's units are contiguous in memory).
+//
+// Programmatic dependent launch: the kernel lets the next kernel on the
+// stream launch at once, prefetches its codes, issues its first unit loads
+// and the codebook copy, and only then waits (griddepcontrol.wait) for the
+// previous kernel -- before it touches activations or outputs.  Codes and
+// codebook are immutable after sphq_pack, so this overlap is safe.
+//
+// Every wait on an mbarrier gives up after about two seconds, records an
+// error bit in the handle's device flag word and carries on, so a fault in
+// the exchange cannot hang the GPU.
+//
+// This header holds the device code; sphq_gemv.cu instantiates it for the W2
+// and W3 formats and holds the launch plans, sphq_gemv_splits.cu instantiates
+// the Tab. 4 splits.
+#pragma once
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+
+#include "sphq_internal.h"
+#include "sphq_layout.cuh"
+
+namespace sphq {
+
+constexpr int kStrip = 2;  // row tiles per work item (activation reuse)
+constexpr unsigned kStripMask = (1u << kStrip) - 1u;
+
+// Radius application modes.
+constexpr int kFactored1 = 1;  // batch 1
+constexpr int kFactored2 = 2;  // batch 2
+constexpr int kFull = 8;       // batch 3..8
+
+struct GemvArgs {
+  const uint8_t* units;
+  const uint8_t* cbimage;  // codebook image as laid out in shared memory
+  const uint16_t* x;
+  uint16_t* y;
+  int* flag;               // device error word: bit 1 = an mbarrier wait gave up
+  int rows, cols, ng, nrt;
+  int batch;
+  int nclusters;           // clusters holding tiles (grid = nclusters x cluster size)
+  uint32_t cb_bytes;       // codebook image bytes
+  uint32_t x_pitch;        // bytes between staged activation rows (factored modes)
+  uint32_t off_x, off_zero, off_recv, off_bar;  // dynamic smem offsets
+  const uint16_t* zeros;   // 256 B of zeros in global memory (batch 3-8 non-suppliers)
+};
+
+// ---------------------------------------------------------------------------
+// PTX wrappers
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+// Makes mbarrier initialisation visible to the async proxy and the cluster.
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+// Tests phase `parity` of a local mbarrier; while it is incomplete the thread
+// may sleep up to ~20 us (it wakes as soon as the phase completes), so a
+// waiting warp does not spin on the issue slots.
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity), "r"(20000u)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ uint64_t globaltimer() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Waits for phase `parity` of a local mbarrier; gives up after ~2 s.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer();
+  for (;;) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (globaltimer() - t0 > 2000000000ull) return false;
+  }
+}
+// Bulk copy global -> own shared memory, completing on a local mbarrier.
+// dst, src and bytes must be multiples of 16.
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes,
+                                         uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          dst),
+      "l"(src), "r"(bytes), "r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t cluster_id() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%clusterid.x;" : "=r"(r));
+  return r;
+}
+// Relaxed arrive: it orders nothing (the mbarrier initialisation is published
+// by fence.mbarrier_init), so it does not wait for this thread's loads in flight.
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() {
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Address of the same shared-memory location in cluster CTA `rank`.
+__device__ __forceinline__ uint32_t mapa(uint32_t addr, uint32_t rank) {
+  uint32_t d;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(d) : "r"(addr), "r"(rank));
+  return d;
+}
+// 16-byte store into another CTA's shared memory, completing on its mbarrier.
+__device__ __forceinline__ void st_async16(uint32_t raddr, float4 v, uint32_t rbar) {
+  asm volatile(
+      "st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1, %2, %3, %4}, "
+      "[%5];" ::"r"(raddr),
+      "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"(rbar)
+      : "memory");
+}
+__device__ __forceinline__ void st_async4(uint32_t raddr, float v, uint32_t rbar) {
+  asm volatile(
+      "st.async.shared::cluster.mbarrier::complete_tx::bytes.b32 [%0], %1, [%2];" ::"r"(raddr),
+      "r"(__float_as_uint(v)), "r"(rbar)
+      : "memory");
+}
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// The MMAs are pure register computations (no volatile), so the compiler may
+// interleave the words of a unit freely.
+__device__ __forceinline__ void mma16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                         uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 "
+      "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+// D = A B (C = 0)
+__device__ __forceinline__ void mma16816_zero(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                              uint32_t a3, uint32_t b0, uint32_t b1) {
+  const float z = 0.f;
+  asm("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 "
+      "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%10,%10,%10,%10};"
+      : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1), "f"(z));
+}
+
+// Activations of batch 3-8 are re-read by every strip: keep them in L1.
+__device__ __forceinline__ uint4 ldg_x16(const uint16_t* p) {
+  uint4 v;
+  asm volatile("ld.global.nc.L1::evict_last.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+
+__device__ __forceinline__ float h_lo_to_f32(uint32_t h2) {
+  float f;
+  asm("{\n\t.reg .f16 lo, hi;\n\tmov.b32 {lo, hi}, %1;\n\tcvt.f32.f16 %0, lo;\n\t}"
+      : "=f"(f)
+      : "r"(h2));
+  return f;
+}
+__device__ __forceinline__ float h_hi_to_f32(uint32_t h2) {
+  float f;
+  asm("{\n\t.reg .f16 lo, hi;\n\tmov.b32 {lo, hi}, %1;\n\tcvt.f32.f16 %0, hi;\n\t}"
+      : "=f"(f)
+      : "r"(h2));
+  return f;
+}
+
+// ---------------------------------------------------------------------------
+// Decode + multiply of one unit
+// ---------------------------------------------------------------------------
+
+template <int BITS>
+struct UnitConst {
+  uint32_t d2, m2, e;
+};
+
+template <int BITS>
+__device__ __forceinline__ UnitConst<BITS> unit_const(const Unit<BITS>& u, int q) {
+  UnitConst<BITS> c;
+  if constexpr (fmt_small(BITS)) {
+    c.d2 = params_delta(u.par.x, u.par.y);
+    c.m2 = params_rmin(u.par.x, u.par.y);
+    c.e = sign_extra<BITS>(u, q);
+  } else {
+    c.d2 = params_delta(u.par.x, u.par.y);
+    c.m2 = params_rmin(u.par.x, u.par.y);
+    c.e = 0;
+  }
+  return c;
+}
+
+template <int BITS>
+__device__ __forceinline__ void word_directions(const Unit<BITS>& u, const UnitConst<BITS>& k,
+                                                int m, int q, const SmemCodebook& cb, uint4& sa,
+                                                uint4& sb, uint32_t& qp) {
+  if constexpr (fmt_small(BITS)) {
+    const uint32_t W = word_of(u.w, m);
+    directions_small<BITS>(W, k.e, m, cb, cb.copyoff, true, sa, sb);
+    qp = W;
+  } else if constexpr (BITS == kFmtW3V3) {
+    directions_w3v3(u, m, cb, sa, sb);
+    qp = qpair_w3v3(u, m);
+  } else {
+    directions_w3(u, m, q, cb, sa, sb);
+    qp = qpair_w3(u, m);
+  }
+}
+
+// Accumulators of one warp for one row tile.
+template <int MODE>
+struct Acc {
+  static constexpr int NB = MODE == kFull ? 1 : MODE;
+  float f[NB][2];  // factored: [batch row][row gid / gid+8]
+  float d[4];      // full: MMA accumulator fragment
+  __device__ __forceinline__ void zero() {
+#pragma unroll
+    for (int i = 0; i < NB; ++i) f[i][0] = f[i][1] = 0.f;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) d[i] = 0.f;
+  }
+};
+
+// One unit (16 rows x 16 slots); xv[m] is this lane's B-fragment data for
+// word m (its activation row at slot 4m+q, or zeros).
+template <int BITS, int MODE>
+__device__ __forceinline__ void process_unit(const Unit<BITS>& cur, const uint4 (&xv)[4], int q,
+                                             const SmemCodebook& cb, Acc<MODE>& acc) {
+  const UnitConst<BITS> kc = unit_const<BITS>(cur, q);
+#pragma unroll
+  for (int m = 0; m < 4; ++m) {
+    uint4 sa, sb;
+    uint32_t qp;
+    word_directions<BITS>(cur, kc, m, q, cb, sa, sb, qp);
+    const uint32_t r = radius_pair<fmt_radius_bits(BITS)>(qp, kc.d2, kc.m2);
+    if constexpr (MODE == kFull) {
+      const uint4 wa = scale_block(sa, bcast_lo(r));
+      const uint4 wb = scale_block(sb, bcast_hi(r));
+      mma16816(acc.d, wa.x, wb.x, wa.y, wb.y, xv[m].x, xv[m].y);
+      mma16816(acc.d, wa.z, wb.z, wa.w, wb.w, xv[m].z, xv[m].w);
+    } else {
+      float d[4];
+      mma16816_zero(d, sa.x, sb.x, sa.y, sb.y, xv[m].x, xv[m].y);
+      mma16816(d, sa.z, sb.z, sa.w, sb.w, xv[m].z, xv[m].w);
+      const float rA = h_lo_to_f32(r), rB = h_hi_to_f32(r);
+      acc.f[0][0] = __fmaf_rn(rA, d[0], acc.f[0][0]);
+      acc.f[0][1] = __fmaf_rn(rB, d[2], acc.f[0][1]);
+      if constexpr (MODE == kFactored2) {
+        acc.f[1][0] = __fmaf_rn(rA, d[1], acc.f[1][0]);
+        acc.f[1][1] = __fmaf_rn(rB, d[3], acc.f[1][1]);
+      }
+    }
+  }
+}
+
+// Sends a warp's accumulators of one row tile to the tile's owner CTA:
+// 4-byte st.async stores into the owner's receive slot ([batch row][row]),
+// completing on the owner's receive mbarrier (raddr / rbar are addresses in
+// the owner's shared memory).
+template <int MODE>
+__device__ __forceinline__ void send_partial(uint32_t raddr, uint32_t rbar, Acc<MODE>& acc,
+                                             int lane, int batch) {
+  const int gid = lane >> 2, q = lane & 3;
+  if constexpr (MODE == kFull) {
+    // d[0..3] = D[gid][2q], D[gid][2q+1], D[gid+8][2q], D[gid+8][2q+1]
+    if (2 * q < batch) {
+      st_async4(raddr + 4u * ((2 * q) * kRowsPerTile + gid), acc.d[0], rbar);
+      st_async4(raddr + 4u * ((2 * q) * kRowsPerTile + gid + 8), acc.d[2], rbar);
+    }
+    if (2 * q + 1 < batch) {
+      st_async4(raddr + 4u * ((2 * q + 1) * kRowsPerTile + gid), acc.d[1], rbar);
+      st_async4(raddr + 4u * ((2 * q + 1) * kRowsPerTile + gid + 8), acc.d[3], rbar);
+    }
+  } else {
+    // sum the lane's slots, then the quad's four lanes (slots q = 0..3)
+#pragma unroll
+    for (int i = 0; i < MODE; ++i) {
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        float t = acc.f[i][h];
+        t += __shfl_xor_sync(0xFFFFFFFFu, t, 1);
+        t += __shfl_xor_sync(0xFFFFFFFFu, t, 2);
+        if (q == 0) st_async4(raddr + 4u * (i * kRowsPerTile + gid + 8 * h), t, rbar);
+      }
+    }
+  }
+}
+
+// First item of warp w when the items of a CTA are dealt to WARPS warps in
+// contiguous ranges of near-equal unit counts: items are (strip, group) in
+// strip-major order, ngc per strip, two units each except in the last strip
+// when the tile count T is odd (one unit).  The unit share of warp w starts
+// at unit U*w/WARPS, rounded to an item boundary.
+template <int WARPS>
+__device__ __forceinline__ int warp_item(int T, int ngc, int w) {
+  const int full = (T / kStrip) * ngc;    // items of two units
+  const int units = T * ngc;
+  const int u = (int)((unsigned)units * (unsigned)w / (unsigned)WARPS);
+  return u < 2 * full ? (u + 1) / 2 : full + (u - 2 * full);
+}
+
+// Warps of CTA `rank` (of csize) whose items cover strip ts, as a bit mask.
+template <int WARPS>
+__device__ __forceinline__ uint32_t cover_mask(int ng, int T, int rank, int csize, int ts) {
+  const int lo = (int)((unsigned)ng * rank / csize), hi = (int)((unsigned)ng * (rank + 1) / csize);
+  const int ngc = hi - lo;
+  uint32_t m = 0;
+  for (int w = 0; w < WARPS; ++w) {
+    const int a0 = warp_item<WARPS>(T, ngc, w), a1 = warp_item<WARPS>(T, ngc, w + 1);
+    if (a0 < a1 && a0 < (ts + 1) * ngc && a1 > ts * ngc) m |= 1u << w;
+  }
+  return m;
+}
+
+// ---------------------------------------------------------------------------
+// The kernel
+// ---------------------------------------------------------------------------
+
+// Contiguous near-equal share [lo, hi) of n items for part i of p (32-bit
+// arithmetic when n * p fits, which is every practical case).
+__device__ __forceinline__ int share_lo(int n, int i, int p) {
+  if ((unsigned)n < 65536u && (unsigned)p < 65536u) return (int)((unsigned)n * (unsigned)i / (unsigned)p);
+  return (int)(((long long)n * i) / p);
+}
+// The same for a compile-time number of parts (a shift for powers of two).
+template <int P>
+__device__ __forceinline__ int share_lo_c(int n, int i) {
+  return (int)((unsigned)n * (unsigned)i / (unsigned)P);
+}
+
+// One work item: the activations of one group (xp: this lane's 16 bytes of
+// word 0; words 1-3 follow at 64-byte steps) and the units of the strip's
+// SIZE row tiles below each other (u[j]).  Each unit's register slot is
+// refilled with the next item's unit j as soon as it is consumed: unit j of
+// the same strip at the next group (base nb), or, for the strip's LAST item,
+// the units in nmask of the warp's next strip.
+template <int BITS, int MODE, int SIZE, bool LAST>
+__device__ __forceinline__ void run_item(Unit<BITS> (&u)[kStrip], Acc<MODE> (&acc)[kStrip],
+                                         const uint8_t* xp, const uint8_t* nb, unsigned nmask,
+                                         int lane, int q, const SmemCodebook& cb) {
+  constexpr int UB = Layout<BITS>::kUnitBytes;
+  uint4 xv[4];
+#pragma unroll
+  for (int m = 0; m < 4; ++m) {
+    if constexpr (MODE == kFull)
+      xv[m] = ldg_x16(reinterpret_cast<const uint16_t*>(xp) + 32 * m);
+    else
+      xv[m] = *reinterpret_cast<const uint4*>(xp + 64 * m);
+  }
+#pragma unroll
+  for (int j = 0; j < kStrip; ++j) {
+    if (j < SIZE) process_unit<BITS, MODE>(u[j], xv, q, cb, acc[j]);
+    if (LAST) {
+      if (nmask >> j & 1u) u[j] = load_unit<BITS>(nb + j * UB, lane);
+    } else if (j < SIZE) {
+      u[j] = load_unit<BITS>(nb + j * UB, lane);
+    }
+  }
+}
+
+// cnt >= 1 items of one strip of SIZE tiles at consecutive groups, starting
+// at unit base ub and activations xp; the last item loads the next strip's
+// first units (base nb, mask nmask).
+template <int BITS, int MODE, int SIZE>
+__device__ __forceinline__ void run_segment(Unit<BITS> (&u)[kStrip], Acc<MODE> (&acc)[kStrip],
+                                            int cnt, const uint8_t* ub, size_t gstride,
+                                            const uint8_t* xp, int xstep, const uint8_t* nb,
+                                            unsigned nmask, int lane, int q,
+                                            const SmemCodebook& cb) {
+  constexpr uint32_t kBytes = SIZE * Layout<BITS>::kUnitBytes;
+  if constexpr (SIZE == 1) {
+    // One-tile strips use the two register slots as a two-item ring (slot
+    // c % 2 holds item c), so two units stay in flight.  The strip is the
+    // warp's last, so nothing is loaded past it (nmask is 0).
+    (void)nb;
+    (void)nmask;
+    if (cnt > 1) u[1] = load_unit<BITS>(ub + gstride, lane);
+    int c = 0;
+    for (; c + 1 < cnt; c += 2) {
+      // items c+2, c+3 go to registers below; c+4, c+5 toward L2
+      if (lane == 0 && c + 4 < cnt) prefetch_l2(ub + 4 * gstride, kBytes);
+      if (lane == 0 && c + 5 < cnt) prefetch_l2(ub + 5 * gstride, kBytes);
+      uint4 xv[4];
+#pragma unroll
+      for (int m = 0; m < 4; ++m) {
+        if constexpr (MODE == kFull)
+          xv[m] = ldg_x16(reinterpret_cast<const uint16_t*>(xp) + 32 * m);
+        else
+          xv[m] = *reinterpret_cast<const uint4*>(xp + 64 * m);
+      }
+      process_unit<BITS, MODE>(u[0], xv, q, cb, acc[0]);
+      if (c + 2 < cnt) u[0] = load_unit<BITS>(ub + 2 * gstride, lane);
+#pragma unroll
+      for (int m = 0; m < 4; ++m) {
+        if constexpr (MODE == kFull)
+          xv[m] = ldg_x16(reinterpret_cast<const uint16_t*>(xp + xstep) + 32 * m);
+        else
+          xv[m] = *reinterpret_cast<const uint4*>(xp + xstep + 64 * m);
+      }
+      process_unit<BITS, MODE>(u[1], xv, q, cb, acc[0]);
+      if (c + 3 < cnt) u[1] = load_unit<BITS>(ub + 3 * gstride, lane);
+      ub += 2 * gstride;
+      xp += 2 * xstep;
+    }
+    if (c < cnt) run_item<BITS, MODE, 1, true>(u, acc, xp, nb, 0u, lane, q, cb);
+    return;
+  }
+  if (lane == 0 && cnt > 1) prefetch_l2(ub + gstride, kBytes);
+  for (int c = 0; c + 1 < cnt; ++c) {
+    if (lane == 0 && c + 2 < cnt) prefetch_l2(ub + 2 * gstride, kBytes);
+    run_item<BITS, MODE, SIZE, false>(u, acc, xp, ub + gstride, 0u, lane, q, cb);
+    ub += gstride;
+    xp += xstep;
+  }
+  run_item<BITS, MODE, SIZE, true>(u, acc, xp, nb, nmask, lane, q, cb);
+}
+
+template <int BITS, int MODE, int WARPS, int MINB>
+__global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a) {
+  extern __shared__ __align__(128) uint8_t smem[];
+  pdl_launch_dependents();
+  constexpr int NBP = MODE == kFull ? kMaxBatch : MODE;  // floats per row in a partial block
+  constexpr int kBlk = kRowsPerTile * NBP;                // floats per partial block
+  constexpr int UB = Layout<BITS>::kUnitBytes;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int gid = lane >> 2, q = lane & 3;
+  const int csize = (int)(gridDim.x / (unsigned)a.nclusters);
+  const int crank = csize > 1 ? (int)cluster_rank() : 0;
+  const int cid = csize > 1 ? (int)cluster_id() : (int)blockIdx.x;
+
+  // this cluster's row tiles and this CTA's radius groups
+  const int t0 = share_lo(a.nrt, cid, a.nclusters);
+  const int T = share_lo(a.nrt, cid + 1, a.nclusters) - t0;
+  const int g0 = share_lo(a.ng, crank, csize);
+  const int ngc = share_lo(a.ng, crank + 1, csize) - g0;
+  const int nfull = T / kStrip;  // strips with all four tiles
+  const unsigned last_mask = (1u << (T - kStrip * nfull)) - 1u;
+  const int i0 = warp_item<WARPS>(T, ngc, warp), i1 = warp_item<WARPS>(T, ngc, warp + 1);
+
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + a.off_bar);
+  uint32_t* masks = reinterpret_cast<uint32_t*>(smem + a.off_bar + 32);  // [owned tile][rank]
+  const uint32_t bar_cb = smem_u32(&bars[0]), bar_x = smem_u32(&bars[1]),
+                 bar_recv = smem_u32(&bars[2]);
+  const int nown = crank < T ? (T - crank + csize - 1) / csize : 0;  // tiles this CTA owns
+
+  // units (t0 + 4s + j, g), j = 0..3, start at strip_base(s, g) + j * UB
+  const size_t gstride = (size_t)a.nrt * UB;
+  auto strip_base = [&](int s, int g) {
+    return a.units + ((size_t)g * a.nrt + t0 + kStrip * s) * UB;
+  };
+  auto strip_mask = [&](int s) { return s < nfull ? kStripMask : last_mask; };
+
+  // first item's units (codes are immutable: no wait needed)
+  Unit<BITS> u[kStrip] = {};
+  int s = i0 < i1 ? i0 / ngc : 0;
+  int g = i0 < i1 ? g0 + i0 % ngc : g0;
+  if (i0 < i1) {
+    const unsigned m0 = strip_mask(s);
+#pragma unroll
+    for (int j = 0; j < kStrip; ++j)
+      if (m0 >> j & 1u) u[j] = load_unit<BITS>(strip_base(s, g) + j * UB, lane);
+  }
+
+  if (threadIdx.x == 0) {
+    mbar_init(bar_cb, 1);
+    mbar_init(bar_x, 1);
+    mbar_init(bar_recv, 1);
+    fence_mbar_init();
+    mbar_arrive_expect_tx(bar_cb, a.cb_bytes);
+    for (uint32_t o = 0; o < a.cb_bytes; o += 32768u)
+      bulk_g2s(smem_u32(smem) + o, a.cbimage + o, min(32768u, a.cb_bytes - o), bar_cb);
+    // every warp of the cluster that covers an owned tile sends 64 * batch
+    // bytes for it; remember who, for the final sum
+    uint32_t bytes = 0;
+    for (int k = 0; k < nown; ++k)
+      for (int r = 0; r < csize; ++r) {
+        const uint32_t m = cover_mask<WARPS>(a.ng, T, r, csize, (crank + k * csize) / kStrip);
+        masks[k * csize + r] = m;
+        bytes += (uint32_t)__popc(m) * 64u * (uint32_t)a.batch;
+      }
+    mbar_arrive_expect_tx(bar_recv, bytes);
+  }
+  if (MODE != kFull && threadIdx.x < 16)  // zero block read by lanes that supply no activations
+    reinterpret_cast<uint4*>(smem + a.off_zero)[threadIdx.x] = make_uint4(0, 0, 0, 0);
+  __syncthreads();                  // mbarrier initialisation visible to the CTA
+  if (csize > 1) cluster_arrive_relaxed();  // ... and to the cluster (waited on below)
+
+  pdl_wait();  // the previous kernel's outputs (our activations) are complete
+  if (MODE != kFull && threadIdx.x == 0) {
+    const uint32_t row_bytes = (uint32_t)ngc * kGroupCols * 2;
+    mbar_arrive_expect_tx(bar_x, row_bytes * MODE);
+    for (int b = 0; b < MODE; ++b)
+      bulk_g2s(smem_u32(smem + a.off_x) + b * a.x_pitch,
+               a.x + (size_t)b * a.cols + (size_t)g0 * kGroupCols, row_bytes, bar_x);
+  }
+  if (csize > 1) cluster_wait();  // every CTA's receive mbarrier is initialised
+  bool ok = mbar_wait(bar_cb, 0);
+  if (MODE != kFull) ok &= mbar_wait(bar_x, 0);
+  if (!ok && lane == 0) atomicOr(a.flag, 2);
+
+  SmemCodebook cb;
+  cb.base = smem;
+  cb.copyoff = fmt_small(BITS) ? (uint32_t)(lane & 7) * 16u : 0u;
+
+  // The activation row this lane supplies to the B fragment; the other lanes
+  // read a zero block (stride 0), so the loop has no lane-dependent branch.
+  int xb;
+  bool provider;
+  if (MODE == kFull) {
+    xb = gid;
+    provider = gid < a.batch;
+  } else {
+    xb = gid - 2 * q;
+    provider = xb >= 0 && xb < MODE;
+  }
+  const uint8_t* x0;  // this lane's activation bytes of group g0
+  if (MODE == kFull)
+    x0 = provider ? reinterpret_cast<const uint8_t*>(a.x + (size_t)xb * a.cols + (size_t)g0 * kGroupCols)
+                  : reinterpret_cast<const uint8_t*>(a.zeros);
+  else
+    x0 = provider ? smem + a.off_x + xb * a.x_pitch : smem + a.off_zero;
+  x0 += q * 16;
+  const int xstep = provider ? kGroupCols * 2 : 0;
+
+  // receive slot of (owned tile k, rank r, warp w): ((k * csize + r) * WARPS + w) * kBlk floats
+  const uint32_t recv_base = smem_u32(smem + a.off_recv);
+
+  Acc<MODE> acc[kStrip];
+#pragma unroll
+  for (int j = 0; j < kStrip; ++j) acc[j].zero();
+
+  // Units of a strip at one group are contiguous: one bulk L2 prefetch per
+  // item, two items ahead inside the strip (the next item's units are already
+  // in flight to registers).
+  int left = i1 - i0;
+  while (left > 0) {
+    // the warp's items of strip s: groups g .. g + cnt - 1
+    const int cnt = min(left, g0 + ngc - g);
+    left -= cnt;
+    const uint8_t* ub = strip_base(s, g);
+    const uint8_t* xp = x0 + (g - g0) * xstep;
+    const uint8_t* nb = strip_base(s + 1, g0);
+    const unsigned nmask = left > 0 ? strip_mask(s + 1) : 0u;
+    static_assert(kStrip == 2, "strip sizes dispatched below");
+    if (s < nfull)
+      run_segment<BITS, MODE, 2>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask, lane, q, cb);
+    else
+      run_segment<BITS, MODE, 1>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask, lane, q, cb);
+#pragma unroll
+    for (int j = 0; j < kStrip; ++j) {
+      const int tau = s * kStrip + j;
+      if (tau < T) {
+        const int owner = tau % csize;
+        const uint32_t slot =
+            recv_base + 4u * (uint32_t)((((tau / csize) * csize + crank) * WARPS + warp) * kBlk);
+        send_partial<MODE>(mapa(slot, (uint32_t)owner), mapa(bar_recv, (uint32_t)owner), acc[j],
+                           lane, a.batch);
+      }
+      acc[j].zero();
+    }
+    ++s;
+    g = g0;
+  }
+  // Owned tiles (tau = crank + k * csize): wait for every covering warp of
+  // the cluster, then sum their blocks in (rank, warp) order and write y.
+  if (nown == 0) return;
+  if (!mbar_wait(bar_recv, 0) && threadIdx.x == 0) atomicOr(a.flag, 2);
+  const float* recv = reinterpret_cast<const float*>(smem + a.off_recv);
+  for (int e = threadIdx.x; e < nown * kBlk; e += WARPS * 32) {
+    const int k = e / kBlk, i = e % kBlk;
+    const int b = i / kRowsPerTile, r = (t0 + crank + k * csize) * kRowsPerTile + i % kRowsPerTile;
+    if (b >= a.batch || r >= a.rows) continue;
+    float sum = 0.f;
+    for (int rk = 0; rk < csize; ++rk) {
+      const uint32_t m = masks[k * csize + rk];
+#pragma unroll
+      for (int w = 0; w < WARPS; ++w)
+        if (m >> w & 1u) sum += recv[(((size_t)k * csize + rk) * WARPS + w) * kBlk + i];
+    }
+    a.y[(size_t)b * a.rows + r] = f32_to_h_rn(sum);
+  }
+}
+
+
+// Launch shape per format.  Small-codebook splits (W2 and Tab. 4): eight
+// interleaved codebook copies (K x 128 B) and two CTAs per SM.
+template <int BITS> struct KernelShape {
+  static constexpr int kWarps = 8;
+  static constexpr int kMinBlocks = 2;
+  static constexpr uint32_t kCbBytes = (uint32_t)Layout<BITS>::K * 8 * 16;
+};
+// W3: the 128 KiB codebook allows one CTA per SM; 8 warps with the whole
+// register file (up to 255 registers each) hide the codebook's bank-conflict
+// latency better than 16 warps at 128 (measured 9-15% faster).
+template <> struct KernelShape<3> {
+  static constexpr int kWarps = 8;
+  static constexpr int kMinBlocks = 1;
+  static constexpr uint32_t kCbBytes = (uint32_t)Layout<3>::K * 16;
+};
+template <> struct KernelShape<kFmtW3V3> : KernelShape<3> {};
+
+constexpr int kModes[3] = {kFactored1, kFactored2, kFull};
+
+template <int BITS, int MODE>
+inline const void* kptr() {
+  return reinterpret_cast<const void*>(
+      &gemv_kernel<BITS, MODE, KernelShape<BITS>::kWarps, KernelShape<BITS>::kMinBlocks>);
+}
+template <int FMT>
+inline const void* kptr_mode(int mode) {
+  return mode == kFactored1 ? kptr<FMT, kFactored1>() : mode == kFactored2 ? kptr<FMT, kFactored2>()
+                                                                           : kptr<FMT, kFull>();
+}
+
+// Kernels of the Tab. 4 splits (formats 5-9), instantiated in their own
+// translation unit; nullptr for other formats.
+const void* split_kernel(int fmt, int mode);
+
+}  // namespace sphq

@@ -31,6 +31,22 @@
 //   from bits 15/31 (the fp16 sign bits of a half2 register) and the two
 //   radius codes of a word one AND away from two fp16 integers.
 //
+// Small-codebook splits (Tab. 4: 8 sign bits, a D-bit direction index with
+// K = 2^D entries, D = 6..8, and V-bit radius codes, D + V <= 10).  The W2
+// unit above is the D = 6, V = 4 member; the others keep its word layout with
+// their field widths:
+//   word w_m, A in the low and B in the high 16 bits: radius code at bits
+//   0..V-1 (16..), direction index at V..V+D-1 (16+V..); then sign pairs from
+//   the top: A's pairs p at bits 15-p / 31-p, B's at (15-NA-p) / (31-NA-p),
+//   where NA = 4 if D + V <= 9 else 3, NB = 4 if D + V = 8 else 3.  Pairs that
+//   do not fit (D + V - 8 per vector) go to a record per quad:
+//     D + V = 10: the W2 record, { S01, S23, P_gid, P_gid+8 } at 512 + 16*gid
+//                 (640 B per unit)
+//     D + V = 9:  B's pair 3 only, one word R at 512 + 4*gid: bit 15-4q-m
+//                 = sign bit 6 and bit 31-4q-m = sign bit 7 of B of lane q's
+//                 word m; then { P_gid, P_gid+8 } at 544 + 8*gid (608 B)
+//     D + V = 8:  no record; { P_gid, P_gid+8 } at 512 + 8*gid (576 B)
+//
 // W3 unit (864 B = 256 x 3.125 bits + 64 B of group parameters):
 //   [0, 512)    lane l: words w_0..w_3, bits of w_m:
 //                 0-7 direction index bits 0-7 of A, 16-23 of B
@@ -71,16 +87,42 @@ __host__ __device__ __forceinline__ long long unit_index(int rt, int g, int nrt)
   return (long long)g * nrt + rt;
 }
 
-// Format ids used as template arguments: 2 = W2, 3 = W3, 4 = W3 with 3-bit
-// radius codes.  The codebook size follows the weight bit-width B.
+// Format ids used as template arguments, one per bit split (sign / direction
+// index / radius bits): 2 = W2 (8/6/4), 3 = W3 (8/13/4), 4 = W3 with 3-bit
+// radius codes (8/13/3), and the small-codebook splits of Tab. 4:
+// 5 = 8/6/2, 6 = 8/6/3, 7 = 8/7/2, 8 = 8/7/3, 9 = 8/8/2.
 constexpr int kFmtW3V3 = 4;
-__host__ __device__ constexpr int fmt_bits(int fmt) { return fmt == kFmtW3V3 ? 3 : fmt; }
+constexpr int kFmt862 = 5, kFmt863 = 6, kFmt872 = 7, kFmt873 = 8, kFmt882 = 9;
+__host__ __device__ constexpr int fmt_dir_bits(int fmt) {
+  return fmt == 3 || fmt == 4 ? 13 : fmt == 7 || fmt == 8 ? 7 : fmt == 9 ? 8 : 6;
+}
+__host__ __device__ constexpr int fmt_radius_bits(int fmt) {
+  return fmt == 2 || fmt == 3 ? 4 : fmt == 4 || fmt == 6 || fmt == 8 ? 3 : 2;
+}
+// formats whose codebook (K <= 256) is kept as eight interleaved copies
+__host__ __device__ constexpr bool fmt_small(int fmt) { return fmt == 2 || fmt >= 5; }
+// format id of a split, or -1
+__host__ __device__ constexpr int fmt_of_split(int dir_bits, int radius_bits) {
+  return dir_bits == 13 ? (radius_bits == 4 ? 3 : radius_bits == 3 ? 4 : -1)
+         : dir_bits == 6 ? (radius_bits == 4 ? 2 : radius_bits == 2 ? 5 : radius_bits == 3 ? 6 : -1)
+         : dir_bits == 7 ? (radius_bits == 2 ? 7 : radius_bits == 3 ? 8 : -1)
+         : dir_bits == 8 ? (radius_bits == 2 ? 9 : -1)
+                         : -1;
+}
 
-template <int BITS> struct Layout;
-template <> struct Layout<2> {
-  static constexpr int K = 64;
-  static constexpr int kUnitBytes = 640;
+// Small-codebook splits (W2 included).
+template <int BITS> struct Layout {
+  static_assert(fmt_small(BITS), "unknown format");
+  static constexpr int D = fmt_dir_bits(BITS), V = fmt_radius_bits(BITS);
+  static constexpr int K = 1 << D;
+  static constexpr int kExtra = D + V - 8;    // sign bits per vector kept outside the words
+  static constexpr int NA = kExtra <= 1 ? 4 : 3;  // sign pairs of A / B inside a word
+  static constexpr int NB = kExtra == 0 ? 4 : 3;
   static constexpr int kRecOff = 512;
+  static constexpr int kParamOff = kExtra == 2 ? 520 : kExtra == 1 ? 544 : 512;
+  static constexpr int kParamStride = kExtra == 2 ? 16 : 8;  // bytes between quads' params
+  static constexpr int kUnitBytes = kExtra == 2 ? 640 : kExtra == 1 ? 608 : 576;
+  static_assert(kExtra >= 0 && kExtra <= 2, "split does not fit the word layout");
 };
 template <> struct Layout<kFmtW3V3> {
   static constexpr int K = 8192;
@@ -96,11 +138,25 @@ template <> struct Layout<3> {
   static constexpr int kTopOff = 832;
 };
 
+// Unit bytes of a format (host-side mirror of Layout<F>::kUnitBytes).
+__host__ __device__ constexpr int fmt_unit_bytes(int fmt) {
+  return fmt == 3 ? Layout<3>::kUnitBytes
+         : fmt == kFmtW3V3 ? Layout<kFmtW3V3>::kUnitBytes
+         : fmt_dir_bits(fmt) + fmt_radius_bits(fmt) == 10 ? 640
+         : fmt_dir_bits(fmt) + fmt_radius_bits(fmt) == 9 ? 608
+                                                          : 576;
+}
+static_assert(fmt_unit_bytes(2) == Layout<2>::kUnitBytes && fmt_unit_bytes(5) == Layout<5>::kUnitBytes &&
+                  fmt_unit_bytes(6) == Layout<6>::kUnitBytes && fmt_unit_bytes(7) == Layout<7>::kUnitBytes &&
+                  fmt_unit_bytes(8) == Layout<8>::kUnitBytes && fmt_unit_bytes(9) == Layout<9>::kUnitBytes,
+              "unit sizes");
+
 // Per-lane data of one unit.
-template <int BITS> struct Unit;
-template <> struct Unit<2> {
+// Small-codebook splits: s is the lane's word of the quad's sign record (W2
+// record: S01 for q < 2, S23 otherwise; one extra bit: R; none: 0).
+template <int BITS> struct Unit {
   uint4 w;      // words w_0..w_3
-  uint32_t s;   // the lane's sign word of the quad record: S01 (q < 2) or S23
+  uint32_t s;
   uint2 par;    // {P_gid, P_gid+8}
 };
 template <> struct Unit<kFmtW3V3> {
@@ -134,16 +190,23 @@ __device__ __forceinline__ uint32_t ldg_stream4(const void* p) {
   return v;
 }
 
+// Small-codebook splits (the W3 formats are specialised below).
 template <int BITS>
-__device__ __forceinline__ Unit<BITS> load_unit(const uint8_t* unit, int lane);
-
-template <>
-__device__ __forceinline__ Unit<2> load_unit<2>(const uint8_t* unit, int lane) {
-  Unit<2> u;
+__device__ __forceinline__ Unit<BITS> load_unit(const uint8_t* unit, int lane) {
+  using L = Layout<BITS>;
+  Unit<BITS> u;
   u.w = ldg_stream16(unit + lane * 16);
-  const uint8_t* rec = unit + Layout<2>::kRecOff + (lane >> 2) * 16;
-  u.s = ldg_stream4(rec + 4 * ((lane >> 1) & 1));
-  u.par = ldg_stream8(rec + 8);
+  if constexpr (L::kExtra == 2) {
+    const uint8_t* rec = unit + L::kRecOff + (lane >> 2) * 16;
+    u.s = ldg_stream4(rec + 4 * ((lane >> 1) & 1));
+    u.par = ldg_stream8(rec + 8);
+  } else if constexpr (L::kExtra == 1) {
+    u.s = ldg_stream4(unit + L::kRecOff + (lane >> 2) * 4);
+    u.par = ldg_stream8(unit + L::kParamOff + (lane >> 2) * 8);
+  } else {
+    u.s = 0;
+    u.par = ldg_stream8(unit + L::kParamOff + (lane >> 2) * 8);
+  }
   return u;
 }
 
@@ -224,11 +287,14 @@ __device__ __forceinline__ uint16_t f32_to_h_rn(float v) {
 }
 
 // Radius pair of one word, Eq. (7): r_hat = RN16(q * Delta + r_min) with one
-// fp16 fused multiply-add per vector.  qpair holds the codes of A (bits 0-3)
-// and B (bits 16-19); 1024 + q is an exact fp16 value (bits 0x6400 | q), so
+// fp16 fused multiply-add per vector.  qpair holds the V-bit codes of A (bits
+// 0..V-1) and B (bits 16..16+V-1); 1024 + q is an exact fp16 value (bits 0x6400 | q), so
 // subtracting 1024 gives q exactly.  d2 / m2: (Delta, r_min) of rows (A, B).
+// V < 4: only bits 0..V-1 (16..16+V-1) are codes.
+template <int V = 4>
 __device__ __forceinline__ uint32_t radius_pair(uint32_t qpair, uint32_t d2, uint32_t m2) {
-  const uint32_t qh = (qpair & 0x000F000Fu) | 0x64006400u;
+  constexpr uint32_t kMask = ((1u << V) - 1u) * 0x00010001u;
+  const uint32_t qh = (qpair & kMask) | 0x64006400u;
   return hfma2_rn(hsub2_rn(qh, 0x64006400u), d2, m2);
 }
 
@@ -277,35 +343,56 @@ struct GlobalCodebook {
   }
 };
 
-// Signed directions of the two vectors of word m of a W2 unit (A = row gid,
-// B = row gid+8).  `e` is the lane's pair-3 sign word aligned to bits 8-15 /
-// 24-31.  Codebook offsets: 128*k + copy offset (interleaved smem copies) or
-// 16*k (a plain table).
-template <class CB>
-__device__ __forceinline__ void directions_w2(uint32_t W, uint32_t e, int m, const CB& cb,
-                                              uint32_t copyoff, bool interleaved, uint4& sa,
-                                              uint4& sb) {
-  const uint32_t w3 = shl_fma<3>(W);
+// Signed directions of the two vectors of word m of a small-codebook unit
+// (W2 and the other splits of Tab. 4; A = row gid, B = row gid+8).  `e` is
+// the lane's sign_extra word.  Codebook offsets: 128*k + copy offset
+// (interleaved shared-memory copies) or 16*k (a plain table).
+template <int FMT, class CB>
+__device__ __forceinline__ void directions_small(uint32_t W, uint32_t e, int m, const CB& cb,
+                                                 uint32_t copyoff, bool interleaved, uint4& sa,
+                                                 uint4& sb) {
+  using L = Layout<FMT>;
+  constexpr int V = L::V, NA = L::NA;
+  constexpr uint32_t kIdx = (uint32_t)L::K - 1u;
   uint32_t offA, offB;
   if (interleaved) {
-    offA = (w3 & 0x1F80u) | copyoff;
-    offB = ((W >> 13) & 0x1F80u) | copyoff;
+    offA = (shl_fma<7 - V>(W) & (kIdx << 7)) | copyoff;
+    offB = ((W >> (9 + V)) & (kIdx << 7)) | copyoff;
   } else {
-    offA = (W & 0x3F0u);
-    offB = (W >> 16) & 0x3F0u;
+    offA = shl_fma<4 - V>(W) & (kIdx << 4);
+    offB = (W >> (12 + V)) & (kIdx << 4);
   }
   const uint4 ca = cb.at(offA);
   const uint4 cbv = cb.at(offB);
-  const uint32_t ea = shl_fma_rt(e, 2 * m);
-  const uint32_t eb = shl_fma_rt(e, 2 * m + 1);
-  sa = apply_signs(ca, W, shl_fma<1>(W), shl_fma<2>(W), ea);
-  sb = apply_signs(cbv, w3, shl_fma<4>(W), shl_fma<5>(W), eb);
+  // pair 3 of A: in the word (NA = 4) or in the W2 record; pair 3 of B: in
+  // the word (NB = 4), in R (one extra bit) or in the W2 record
+  uint32_t a3, b3;
+  if constexpr (L::kExtra == 2) {
+    a3 = shl_fma_rt(e, 2 * m);
+    b3 = shl_fma_rt(e, 2 * m + 1);
+  } else if constexpr (L::kExtra == 1) {
+    a3 = shl_fma<3>(W);
+    b3 = shl_fma_rt(e, m);
+  } else {
+    a3 = shl_fma<3>(W);
+    b3 = shl_fma<7>(W);
+  }
+  sa = apply_signs(ca, W, shl_fma<1>(W), shl_fma<2>(W), a3);
+  sb = apply_signs(cbv, shl_fma<NA>(W), shl_fma<NA + 1>(W), shl_fma<NA + 2>(W), b3);
 }
 
-// The lane's pair-3 sign word of a W2 unit, aligned to bits 8-15 / 24-31.
-__device__ __forceinline__ uint32_t w2_sign3(const Unit<2>& u, int q) {
-  const uint32_t s = u.s;
-  return (q & 1) ? (s << 8) : s;
+// The lane's sign word for the pairs kept outside the words: the W2 record
+// word aligned to bits 8-15 / 24-31, or R shifted by 4q; zero without a record.
+template <int FMT>
+__device__ __forceinline__ uint32_t sign_extra(const Unit<FMT>& u, int q) {
+  if constexpr (Layout<FMT>::kExtra == 2) {
+    const uint32_t s = u.s;
+    return (q & 1) ? (s << 8) : s;
+  } else if constexpr (Layout<FMT>::kExtra == 1) {
+    return shl_fma_rt(u.s, 4 * q);
+  } else {
+    return 0u;
+  }
 }
 __device__ __forceinline__ uint32_t params_delta(uint32_t pa, uint32_t pb) {
   return prmt<0x5410u>(pa, pb);
@@ -363,8 +450,8 @@ __device__ __forceinline__ uint32_t qpair_w3v3(const Unit<kFmtW3V3>& u, int m) {
   return w3v3_hi(u, m) >> 13;
 }
 
-// Radius codes of word m as a pair (A at bits 0-3, B at bits 16-19).
-__device__ __forceinline__ uint32_t qpair_w2(uint32_t W) { return W; }
+// Radius codes of word m as a pair (A at bits 0-3, B at bits 16-19); the
+// small-codebook words carry their codes at bits 0 / 16 already.
 __device__ __forceinline__ uint32_t qpair_w3(const Unit<3>& u, int m) { return u.mq.y >> (4 * m); }
 
 }  // namespace sphq

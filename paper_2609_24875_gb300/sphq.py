@@ -103,10 +103,13 @@ class SphqMatrix:
     """
 
     def __init__(self, rows: int, cols: int, bits: int, codebook, scale, offset,
-                 radius_bits: int = 4):
+                 radius_bits: int = 4, K: int | None = None):
+        """bits 2 or 3; K defaults to 2^(7*bits - 8) (64 / 8192); the Tab. 4 splits
+        take K = 128 or 256 at bits = 2 and radius_bits 2 or 3 (sphq_create_v)."""
         import torch
         L = load()
-        K = 1 << (7 * bits - 8)
+        if K is None:
+            K = 1 << (7 * bits - 8)
         cb = codebook.contiguous()
         sc = scale.contiguous()
         of = offset.contiguous()

@@ -89,13 +89,15 @@ def make_x(rng: np.random.Generator, B: int, cols: int) -> np.ndarray:
 
 
 def random_codes(bits: int, rows: int, cols: int, seed: int, B: int = 1,
-                 codebook: np.ndarray | None = None, radius_bits: int = RADIUS_BITS):
+                 codebook: np.ndarray | None = None, radius_bits: int = RADIUS_BITS,
+                 K: int | None = None):
     """Uniformly random codes (configurations 0, 2, 3, 4), radius codes drawn
-    from U{0..2^radius_bits - 1}.  Returns (Codes, x)."""
+    from U{0..2^radius_bits - 1}, direction indices from U{0..K-1} (K defaults
+    to the codebook size of `bits`).  Returns (Codes, x)."""
     if cols % GROUP_COLS:
         raise ValueError("cols must be a multiple of 128")
     rng = np.random.Generator(np.random.PCG64(seed))
-    K = bits_to_K(bits)
+    K = bits_to_K(bits) if K is None else K
     cb = make_codebook(rng, K)
     if codebook is not None:
         cb = codebook

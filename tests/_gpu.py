@@ -18,7 +18,8 @@ def to_dev(a):
 
 def make_matrix(codes: inp.Codes) -> SphqMatrix:
     m = SphqMatrix(codes.rows, codes.cols, codes.bits, to_dev(codes.codebook),
-                   to_dev(codes.scale), to_dev(codes.offset), radius_bits=codes.vbits)
+                   to_dev(codes.scale), to_dev(codes.offset), radius_bits=codes.vbits,
+                   K=codes.K)
     m.pack(to_dev(codes.sign), to_dev(codes.idx), to_dev(codes.rcode))
     return m
 

@@ -78,7 +78,7 @@ def test_pack_rejects_radius_codes_above_seven():
 
 def test_unsupported_splits_are_refused():
     codes, _ = inp.random_codes(2, 16, 128, seed=1)
-    for bits, vb in ((2, 3), (3, 2), (3, 5), (2, 0)):
+    for bits, vb in ((3, 2), (3, 5), (2, 0), (2, 5)):
         cb = codes.codebook if bits == 2 else inp.random_codes(3, 16, 128, seed=1)[0].codebook
         with pytest.raises(SphqError) as e:
             SphqMatrix(16, 128, bits, G.to_dev(cb), G.to_dev(codes.scale),

@@ -30,6 +30,7 @@ def test_budget(kind, kw, expected):
         assert oracle.payload_bits_per_weight(kw["bits"], kw["V"]) == expected
     elif kind == "split":
         assert (kw["sign"] + kw["dir"] + kw["radius"]) / 8 == expected
+        assert oracle.split_bits_per_weight(kw["dir"], kw["radius"]) == expected
         # §3.2: the same budget is 2 + (V - 2)/8 when the index keeps 6 bits
         if kw["dir"] == 6:
             assert 2 + (kw["radius"] - 2) / 8 == expected
