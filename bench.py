@@ -607,23 +607,23 @@ def run_report(args):
     flush = torch.empty(2 * L2 // 4, dtype=torch.float32, device=dev)
     t = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int16) if a.dtype == np.uint16 else a)).to(dev)
 
-    def pool_for(bits, rows, cols, seed, batch, vbits=4):
-        codes, x = inp.random_codes(bits, rows, cols, seed=seed, B=batch, radius_bits=vbits)
-        one = (7 * bits + vbits) * rows * cols // 64
+    def pool_for(bits, rows, cols, seed, batch, vbits=4, K=None):
+        codes, x = inp.random_codes(bits, rows, cols, seed=seed, B=batch, radius_bits=vbits, K=K)
+        one = (8 + int(np.log2(codes.K)) + vbits) * rows * cols // 64
         P = min(512, max(2, int(np.ceil(2 * L2 / one)) + 1))
         cb, sc, of = t(codes.codebook), t(codes.scale), t(codes.offset)
         sg, ix, rc = t(codes.sign), t(codes.idx), t(codes.rcode)
         mats = []
         for _ in range(P):
-            m = SphqMatrix(rows, cols, bits, cb, sc, of, radius_bits=vbits)
+            m = SphqMatrix(rows, cols, bits, cb, sc, of, radius_bits=vbits, K=codes.K)
             m.pack(sg, ix, rc)
             mats.append(m)
         xd = t(x).view(torch.float16)
         ys = [torch.empty((batch, rows), dtype=torch.float16, device=dev) for _ in mats]
         return mats, xd, ys
 
-    def entry(bits, rows, cols, seed, batch, cold=False, vbits=4):
-        mats, xd, ys = pool_for(bits, rows, cols, seed, batch, vbits)
+    def entry(bits, rows, cols, seed, batch, cold=False, vbits=4, K=None):
+        mats, xd, ys = pool_for(bits, rows, cols, seed, batch, vbits, K)
         b = mats[0].bytes(batch)
         us = steady_us(mats, xd, ys, batch, stream)
         e = {"us": round(us, 3), "GB/s": round(b / us / 1e3, 1),
@@ -646,10 +646,15 @@ def run_report(args):
     rep["cfg3_w3_proj_batch"] = {f"{nm} {r}x{c} B{bt}": entry(3, r, c, inp.seed_for(3, i), bt)
                                  for i, (nm, r, c) in enumerate(inp.DECODER_PROJ)
                                  if nm in ("q", "k", "gate", "down") for bt in (1, 2, 4, 8)}
-    # general bit split: W3 with 3-bit radius codes (3.00 bits per weight)
+    # general bit splits: W3 with 3-bit radius codes (3.00 bits per weight) and
+    # the small-codebook splits of the bit-allocation ablation (sign/index/radius)
     rep["w3v3_square"] = {f"W3V3 {n}x{n} B{bt}": entry(3, n, n, inp.seed_for(1, 10 + i), bt,
                                                        cold=bt == 1, vbits=3)
                           for i, n in enumerate((4096, 8192)) for bt in (1, 4)}
+    rep["tab4_splits_8192"] = {f"8/{d}/{v} 8192x8192 B1": entry(2, 8192, 8192,
+                                                               inp.seed_for(1, 20 + 10 * d + v),
+                                                               1, vbits=v, K=1 << d)
+                               for d, v in ((6, 2), (6, 3), (7, 2), (7, 3), (8, 2), (6, 4))}
     # CPU oracle on the 1024^2 matrix: single thread and all cores
     import oracle
     codes, x = inp.random_codes(2, 1024, 1024, seed=inp.seed_for(0, 0))

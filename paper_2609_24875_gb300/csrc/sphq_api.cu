@@ -1,5 +1,5 @@
 // C ABI of the sphq library: handle lifetime, packing, decode, errors.
-// The GEMV kernels and their launch plans live in sphq_gemv.cu.
+// The GEMV kernels live in sphq_gemv_kernel.cuh, their launch plans in sphq_gemv.cu.
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 

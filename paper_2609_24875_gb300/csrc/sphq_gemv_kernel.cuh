@@ -38,8 +38,9 @@
 // mbarrier; the owner adds the blocks of all covering warps in (rank, warp)
 // order and writes fp16 y.
 //
-// Staging.  The codebook image (W2: eight interleaved copies, 8 KiB; W3: the
-// 128 KiB table) and, for batch 1-2, the CTA's slice of the activations are
+// Staging.  The codebook image (W2 and the other small-codebook splits: eight
+// interleaved copies, K x 128 B; W3: the 128 KiB table) and, for batch 1-2, the
+// CTA's slice of the activations are
 // copied into shared memory by bulk asynchronous copies completing on
 // mbarriers.  Codes stream from HBM through registers (16-byte loads that
 // bypass L1) one work item ahead of use, and a bulk L2 prefetch runs two
