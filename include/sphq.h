@@ -56,10 +56,12 @@ typedef enum sphq_status {
   SPHQ_ERR_NOT_PACKED = 3,    /* gemv/decode before a successful sphq_pack   */
   SPHQ_ERR_CUDA = 4,          /* a CUDA runtime call failed                  */
   SPHQ_ERR_OOM = 5,           /* device allocation failed                    */
-  SPHQ_ERR_DEVICE = 6         /* no usable sm_103 device                     */
+  SPHQ_ERR_DEVICE = 6,        /* no usable sm_103 device                     */
+  SPHQ_ERR_TIMEOUT = 7        /* a kernel gave up an on-chip wait (sphq_check) */
 } sphq_status;
 
 #define SPHQ_MAX_BATCH 8
+#define SPHQ_GEMM_MAX_BATCH (1 << 22)
 #define SPHQ_GROUP_COLS 128   /* scalars per radius group (§3.1)   */
 #define SPHQ_VECTOR_DIM 8     /* 8-D vectors (§3.1)                */
 
@@ -201,6 +203,34 @@ sphq_status sphq_gemv_host(sphq_handle h, const void* x_host, void* y_host, int 
  */
 sphq_status sphq_gemv_noalloc(sphq_handle h, const void* x, void* y, int batch,
                               sphq_stream stream);
+
+/*
+ * sphq_gemm -- Y = X W_hat^T for any batch (prefill), on the tensor cores.
+ * (The paper's kernel serves decode only; this is the large-batch form of the
+ * same product, §3.4 with W_hat from Eq. (7) and Eq. (4).)
+ *
+ *   x      batch x cols fp16, device pointer, 16-byte aligned.
+ *   y      batch x rows fp16, device pointer, 2-byte aligned; written in full.
+ *   batch  1..SPHQ_GEMM_MAX_BATCH; efficient from a few dozen rows up (tiles
+ *          of 128 activation rows); sphq_gemv is the fast path for batch <= 8.
+ *
+ * Asynchronous on `stream`, no allocation (graph-capturable).  Numerics: each
+ * weight is the exact fp16 W_hat of sphq_decode, products are exact in fp32,
+ * fp32 accumulation, fp16 output rounded to nearest: the same bound as
+ * sphq_gemv.  Concurrency as for sphq_gemv (the handle's error word).
+ */
+sphq_status sphq_gemm(sphq_handle h, const void* x, void* y, int batch, sphq_stream stream);
+
+/*
+ * sphq_check -- synchronise `stream`, then read and clear the handle's device
+ * error word.  Every on-chip wait in the GEMV and GEMM kernels (mbarriers of
+ * the staged copies, the cluster exchange, the tensor-core pipeline) gives up
+ * after about two seconds instead of hanging, sets the word and lets the
+ * kernel finish; the output of such a launch is invalid.  Returns
+ * SPHQ_ERR_TIMEOUT if the word was set since the last check, SPHQ_OK
+ * otherwise (or SPHQ_ERR_CUDA if the stream itself reports an error).
+ */
+sphq_status sphq_check(sphq_handle h, sphq_stream stream);
 
 /*
  * sphq_decode -- write the decoded weights W_hat (rows x cols fp16, device

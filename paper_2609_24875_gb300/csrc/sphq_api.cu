@@ -199,7 +199,7 @@ using namespace sphq;
 
 extern "C" {
 
-int sphq_version(void) { return 10100; }
+int sphq_version(void) { return 10200; }
 
 sphq_status sphq_get_plan(sphq_handle h, int batch, sphq_plan_info* out) {
   g_last_error.clear();
@@ -437,6 +437,34 @@ sphq_status sphq_gemv(sphq_handle h, const void* x, void* y, int batch, sphq_str
     return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemv: y must be a 4-byte aligned pointer");
   if (!h->packed) return set_error(SPHQ_ERR_NOT_PACKED, "sphq_gemv: handle not packed");
   return launch_gemv(h, x, y, batch, reinterpret_cast<cudaStream_t>(stream));
+}
+
+sphq_status sphq_gemm(sphq_handle h, const void* x, void* y, int batch, sphq_stream stream) {
+  g_last_error.clear();
+  if (!h) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemm: NULL handle");
+  if (batch < 1 || batch > SPHQ_GEMM_MAX_BATCH)
+    return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm: batch must be 1..SPHQ_GEMM_MAX_BATCH");
+  if (!x || reinterpret_cast<uintptr_t>(x) % 16)
+    return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemm: x must be a 16-byte aligned pointer");
+  if (!y || reinterpret_cast<uintptr_t>(y) % 2)
+    return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemm: y must be a 2-byte aligned pointer");
+  if (!h->packed) return set_error(SPHQ_ERR_NOT_PACKED, "sphq_gemm: handle not packed");
+  return launch_gemm(h, x, y, batch, reinterpret_cast<cudaStream_t>(stream));
+}
+
+sphq_status sphq_check(sphq_handle h, sphq_stream stream) {
+  g_last_error.clear();
+  if (!h) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_check: NULL handle");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  int word = 0;
+  SPHQ_CUDA(cudaMemcpyAsync(&word, h->flag + 1, sizeof(int), cudaMemcpyDeviceToHost, s),
+            "read error word");
+  SPHQ_CUDA(cudaMemsetAsync(h->flag + 1, 0, sizeof(int), s), "clear error word");
+  SPHQ_CUDA(cudaStreamSynchronize(s), "sphq_check");
+  if (word)
+    return set_error(SPHQ_ERR_TIMEOUT,
+                     "sphq_check: a kernel gave up waiting on an mbarrier (results invalid)");
+  return SPHQ_OK;
 }
 
 // Device address of a page-locked, mapped host buffer, or null for any other

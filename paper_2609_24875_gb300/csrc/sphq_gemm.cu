@@ -1,0 +1,374 @@
+// Prefill / large-batch product Y = X W_hat^T on the fifth-generation tensor
+// cores (tcgen05), sm_103a.
+//
+// For batches above the decode GEMV's eight rows the product is a dense
+// contraction (2 * batch * rows * cols flops against rows * cols decoded
+// weights), so it runs as a tensor-core GEMM whose B operand is decoded on
+// the fly: W_hat is rebuilt exactly as Eq. (7) and Eq. (4) define it (the
+// decode of the GEMV's batch 3-8 mode) straight into shared memory, never to
+// HBM.
+//
+// Tiles: an output tile is 128 activation rows (the MMA's M; tokens) x 256
+// weight rows (the MMA's N; 16 row tiles of the unit layout), accumulated in
+// fp32 in tensor memory over the columns in steps of 64.  Per step:
+//  * one TMA warp loads the 128 x 64 activation tile (A operand, K-major,
+//    128-byte swizzle; rows past the batch read zeros);
+//  * eight decode warps each rebuild two 16 x 64 slices of W_hat (half a unit
+//    of two row tiles) into the B operand tile in the same swizzled K-major
+//    layout, fence them to the async proxy and arrive on the stage's
+//    mbarrier;
+//  * one MMA warp issues four 128 x 256 x 16 tcgen05.mma (fp16 x fp16 ->
+//    fp32) when both halves of the stage are in, and commits their completion
+//    to the stage's "empty" mbarrier, which releases the buffers.
+// Stages rotate through a ring of buffers (two to four, as shared memory
+// allows next to the codebook).  After the last step the decode warps read
+// the accumulators from tensor memory (warp w: lanes 32 (w % 4).., columns
+// 128 (w / 4)..), round to fp16 and store Y.
+//
+// Every mbarrier wait gives up after about two seconds and records bit 1 in
+// the handle's device error word, so a fault cannot hang the GPU.
+#include <cuda.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+
+#include <mutex>
+
+#include "sphq_gemv_kernel.cuh"
+#include "sphq_umma.cuh"
+
+namespace sphq {
+
+constexpr int kGemmBM = 128;                    // activation rows per tile (MMA M)
+constexpr int kGemmBN = 256;                    // weight rows per tile (MMA N)
+constexpr int kGemmBK = 64;                     // columns per pipeline stage
+constexpr int kGemmTilesN = kGemmBN / kRowsPerTile;
+constexpr int kGemmDecodeWarps = 8;             // two row tiles each
+constexpr int kGemmThreads = (kGemmDecodeWarps + 2) * 32;
+constexpr int kGemmMmaWarp = kGemmDecodeWarps;
+constexpr int kGemmTmaWarp = kGemmDecodeWarps + 1;
+constexpr uint32_t kTileA = kGemmBM * kGemmBK * 2;  // 16 KiB
+constexpr uint32_t kTileB = kGemmBN * kGemmBK * 2;  // 32 KiB
+static_assert(kGemmTilesN == 2 * kGemmDecodeWarps, "two row tiles per decode warp");
+
+struct GemmArgs {
+  const uint8_t* units;
+  const uint8_t* cbimage;  // codebook as laid out in shared memory
+  uint16_t* y;             // batch x rows fp16
+  int* flag;               // device error word: bit 1 = an mbarrier wait gave up
+  int rows, cols, nrt, batch;
+  int stages;              // ring depth
+  uint32_t cb_bytes;
+  uint32_t off_b, off_cb, off_bar;  // from the 1024-byte aligned base; A tiles at 0
+};
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void sts16(uint32_t addr, uint4 v) {
+  asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x), "r"(v.y),
+               "r"(v.z), "r"(v.w)
+               : "memory");
+}
+
+// Decodes words M and M+1 (the stage's 64 columns) of the lane's unit and
+// stores its four 16-byte blocks into the B tile: vector (row, slot) goes to
+// tile row n and 16-byte chunk c = slot % 8, at chunk position c ^ (n % 8).
+template <int FMT, int M>
+__device__ __forceinline__ void decode_half(const Unit<FMT>& u, const UnitConst<FMT>& kc, int q,
+                                            int gid, int jt, const SmemCodebook& cb,
+                                            uint32_t btile) {
+#pragma unroll
+  for (int mm = 0; mm < 2; ++mm) {
+    uint4 sa, sb;
+    uint32_t qp;
+    word_directions<FMT>(u, kc, M + mm, q, cb, sa, sb, qp);
+    const uint32_t r = radius_pair<fmt_radius_bits(FMT)>(qp, kc.d2, kc.m2);
+    const uint4 wa = scale_block(sa, bcast_lo(r));
+    const uint4 wb = scale_block(sb, bcast_hi(r));
+    const int c = 4 * mm + q;
+    const int nA = kRowsPerTile * jt + gid, nB = nA + 8;
+    sts16(btile + nA * 128 + ((c ^ (nA & 7)) << 4), wa);
+    sts16(btile + nB * 128 + ((c ^ (nB & 7)) << 4), wb);
+  }
+}
+
+template <int FMT>
+__global__ void __launch_bounds__(kGemmThreads, 1)
+    gemm_kernel(const GemmArgs a, const __grid_constant__ CUtensorMap tmap) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  const uint32_t sbase = smem_u32(smem);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int S = a.stages;
+  const int nk = a.cols / kGemmBK;
+  const int ng = a.cols / kGroupCols;
+  const uint32_t full0 = sbase + a.off_bar;  // full[S], empty[S], acc, cb, tmem slot
+  const uint32_t empty0 = full0 + 8u * S;
+  const uint32_t acc_bar = empty0 + 8u * S;
+  const uint32_t cb_bar = acc_bar + 8u;
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + a.off_bar + 16u * S + 16u);
+  const int rt0 = blockIdx.x * kGemmTilesN;
+  const int tok0 = blockIdx.y * kGemmBM;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(full0 + 8u * s, kGemmDecodeWarps + 1);
+      mbar_init(empty0 + 8u * s, 1);
+    }
+    mbar_init(acc_bar, 1);
+    mbar_init(cb_bar, 1);
+    fence_mbar_init();
+    mbar_arrive_expect_tx(cb_bar, a.cb_bytes);
+    for (uint32_t o = 0; o < a.cb_bytes; o += 32768u)
+      bulk_g2s(sbase + a.off_cb + o, a.cbimage + o, min(32768u, a.cb_bytes - o), cb_bar);
+  }
+  if (warp == kGemmMmaWarp) {
+    umma::tmem_alloc(smem_u32(tslot), kGemmBN);
+    umma::tmem_relinquish();
+  }
+  umma::fence_before_sync();
+  __syncthreads();
+  umma::fence_after_sync();
+  const uint32_t taddr = *tslot;
+
+  if (warp == kGemmTmaWarp) {
+    if (lane == 0) {
+      umma::prefetch_tmap(&tmap);
+      for (int i = 0, s = 0, r = 0; i < nk; ++i) {
+        if (r > 0 && !mbar_wait(empty0 + 8u * s, (r - 1) & 1)) atomicOr(a.flag, 2);
+        mbar_arrive_expect_tx(full0 + 8u * s, kTileA);
+        umma::tma_load_2d(sbase + s * kTileA, &tmap, i * kGemmBK, tok0, full0 + 8u * s);
+        if (++s == S) s = 0, ++r;
+      }
+    }
+    __syncwarp();
+  } else if (warp == kGemmMmaWarp) {
+    if (lane == 0) {
+      constexpr uint32_t idesc = umma::idesc_f16_f32(kGemmBM, kGemmBN);
+      for (int i = 0, s = 0, r = 0; i < nk; ++i) {
+        if (!mbar_wait(full0 + 8u * s, r & 1)) atomicOr(a.flag, 2);
+        umma::fence_after_sync();
+        const uint32_t at = sbase + s * kTileA, bt = sbase + a.off_b + s * kTileB;
+#pragma unroll
+        for (int kk = 0; kk < kGemmBK / 16; ++kk)
+          umma::mma_f16(taddr, umma::smem_desc_sw128(at + 32u * kk),
+                        umma::smem_desc_sw128(bt + 32u * kk), idesc, (i | kk) != 0);
+        umma::commit(empty0 + 8u * s);
+        if (++s == S) s = 0, ++r;
+      }
+      umma::commit(acc_bar);
+    }
+    __syncwarp();
+  } else {
+    // ---- decode warps: W_hat slices into the B tiles ----
+    const int q = lane & 3, gid = lane >> 2;
+    constexpr int UB = Layout<FMT>::kUnitBytes;
+    SmemCodebook cb;
+    cb.base = smem + a.off_cb;
+    cb.copyoff = fmt_small(FMT) ? (uint32_t)(lane & 7) * 16u : 0u;
+    const int j0 = 2 * warp;
+    const bool ok0 = rt0 + j0 < a.nrt, ok1 = rt0 + j0 + 1 < a.nrt;
+    const uint8_t* ub0 = a.units + (size_t)(rt0 + j0) * UB;  // group 0; + g * nrt * UB
+    const size_t gstride = (size_t)a.nrt * UB;
+    Unit<FMT> cur[2] = {}, nxt[2] = {};
+    if (ok0) nxt[0] = load_unit<FMT>(ub0, lane);
+    if (ok1) nxt[1] = load_unit<FMT>(ub0 + UB, lane);
+    if (!mbar_wait(cb_bar, 0) && lane == 0) atomicOr(a.flag, 2);
+    for (int i = 0, s = 0, r = 0; i < nk; ++i) {
+      const int g = i >> 1;
+      if ((i & 1) == 0) {
+        cur[0] = nxt[0];
+        cur[1] = nxt[1];
+        if (g + 1 < ng) {
+          const uint8_t* nb = ub0 + (size_t)(g + 1) * gstride;
+          if (ok0) nxt[0] = load_unit<FMT>(nb, lane);
+          if (ok1) nxt[1] = load_unit<FMT>(nb + UB, lane);
+        }
+      }
+      if (r > 0 && !mbar_wait(empty0 + 8u * s, (r - 1) & 1) && lane == 0) atomicOr(a.flag, 2);
+      const uint32_t bt = sbase + a.off_b + s * kTileB;
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        if (!(j ? ok1 : ok0)) continue;
+        const UnitConst<FMT> kc = unit_const<FMT>(cur[j], q);
+        if (i & 1)
+          decode_half<FMT, 2>(cur[j], kc, q, gid, j0 + j, cb, bt);
+        else
+          decode_half<FMT, 0>(cur[j], kc, q, gid, j0 + j, cb, bt);
+      }
+      umma::fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(full0 + 8u * s);
+      if (++s == S) s = 0, ++r;
+    }
+
+    // ---- epilogue: accumulators -> fp16 Y ----
+    if (!mbar_wait(acc_bar, 0) && lane == 0) atomicOr(a.flag, 2);
+    umma::fence_after_sync();
+    const int quarter = warp & 3;
+    const int token = tok0 + 32 * quarter + lane;
+#pragma unroll 1
+    for (int cc = 0; cc < 4; ++cc) {
+      const int c0 = (warp >> 2) * (kGemmBN / 2) + 32 * cc;
+      uint32_t v[32];
+      umma::ld_32x32b_x32(taddr + ((uint32_t)(32 * quarter) << 16) + (uint32_t)c0, v);
+      umma::wait_ld();
+      const int row0 = rt0 * kRowsPerTile + c0;
+      if (token < a.batch && row0 < a.rows) {
+        uint16_t* dst = a.y + (size_t)token * a.rows + row0;
+        if (row0 + 32 <= a.rows && (reinterpret_cast<uintptr_t>(dst) & 15u) == 0) {
+          uint32_t hv[16];
+#pragma unroll
+          for (int t = 0; t < 16; ++t) {
+            const __half2 p = __floats2half2_rn(__uint_as_float(v[2 * t]),
+                                                __uint_as_float(v[2 * t + 1]));
+            hv[t] = *reinterpret_cast<const uint32_t*>(&p);
+          }
+#pragma unroll
+          for (int t = 0; t < 4; ++t)
+            reinterpret_cast<uint4*>(dst)[t] =
+                make_uint4(hv[4 * t], hv[4 * t + 1], hv[4 * t + 2], hv[4 * t + 3]);
+        } else {
+#pragma unroll
+          for (int t = 0; t < 32; ++t)
+            if (row0 + t < a.rows) dst[t] = f32_to_h_rn(__uint_as_float(v[t]));
+        }
+      }
+    }
+  }
+  umma::fence_before_sync();
+  __syncthreads();
+  if (warp == kGemmMmaWarp) {
+    umma::fence_after_sync();
+    umma::tmem_dealloc(taddr, kGemmBN);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+    else
+      (void)cudaGetLastError();
+  });
+  return fn;
+}
+
+static const void* gemm_kernel_ptr(int fmt) {
+  switch (fmt) {
+#define SPHQ_GEMM_PTR(F) \
+  case F:                \
+    return reinterpret_cast<const void*>(&gemm_kernel<F>);
+    SPHQ_GEMM_PTR(2)
+    SPHQ_GEMM_PTR(3)
+    SPHQ_GEMM_PTR(4)
+    SPHQ_GEMM_PTR(5)
+    SPHQ_GEMM_PTR(6)
+    SPHQ_GEMM_PTR(7)
+    SPHQ_GEMM_PTR(8)
+    SPHQ_GEMM_PTR(9)
+#undef SPHQ_GEMM_PTR
+    default:
+      return nullptr;
+  }
+}
+
+static size_t align_to(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+// Shared-memory layout of the GEMM for a handle: ring depth and offsets.
+struct GemmSmem {
+  int stages = 0;
+  uint32_t cb_bytes = 0, off_b = 0, off_cb = 0, off_bar = 0;
+  size_t total = 0;
+};
+
+static GemmSmem gemm_smem(const sphq_handle_s* h, int optin) {
+  GemmSmem L;
+  L.cb_bytes = fmt_small(h->fmt) ? (uint32_t)h->K * 8u * 16u : (uint32_t)h->K * 16u;
+  for (int S = 4; S >= 2; --S) {
+    const size_t off_b = (size_t)S * kTileA;
+    const size_t off_cb = off_b + (size_t)S * kTileB;
+    const size_t off_bar = align_to(off_cb + L.cb_bytes, 16);
+    const size_t total = 1024 + off_bar + 16u * S + 16u + 16u;  // alignment slack + barriers + slot
+    if (total <= (size_t)optin) {
+      L.stages = S;
+      L.off_b = (uint32_t)off_b;
+      L.off_cb = (uint32_t)off_cb;
+      L.off_bar = (uint32_t)off_bar;
+      L.total = total;
+      return L;
+    }
+  }
+  return L;
+}
+
+sphq_status launch_gemm(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return set_error(SPHQ_ERR_CUDA, "sphq_gemm: cuTensorMapEncodeTiled unavailable");
+  int optin = 0;
+  cudaError_t e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, h->device);
+  if (e != cudaSuccess) return cuda_error(e, "cudaDeviceGetAttribute");
+  const GemmSmem L = gemm_smem(h, optin);
+  if (L.stages == 0) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm: shared memory too small");
+  const void* kfn = gemm_kernel_ptr(h->fmt);
+  if (!kfn) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm: unknown format");
+  {
+    static std::mutex mu;
+    static bool done[16] = {};
+    std::lock_guard<std::mutex> lock(mu);
+    if (!done[h->fmt]) {
+      e = cudaFuncSetAttribute(kfn, cudaFuncAttributeMaxDynamicSharedMemorySize, optin);
+      if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(gemm)");
+      done[h->fmt] = true;
+    }
+  }
+  // activations: a batch x cols fp16 tensor, boxes of 128 rows x 64 columns
+  CUtensorMap tmap;
+  const cuuint64_t gdim[2] = {(cuuint64_t)h->cols, (cuuint64_t)batch};
+  const cuuint64_t gstride[1] = {(cuuint64_t)h->cols * 2};
+  const cuuint32_t box[2] = {(cuuint32_t)kGemmBK, (cuuint32_t)kGemmBM};
+  const cuuint32_t estride[2] = {1, 1};
+  CUresult cr = enc(&tmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(x), gdim, gstride,
+                    box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (cr != CUDA_SUCCESS)
+    return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemm: cuTensorMapEncodeTiled rejected x");
+  GemmArgs a;
+  a.units = (const uint8_t*)h->units;
+  a.cbimage = (const uint8_t*)(fmt_small(h->fmt) ? h->cbimage : h->codebook);
+  a.y = (uint16_t*)y;
+  a.flag = h->flag + 1;
+  a.rows = h->rows;
+  a.cols = h->cols;
+  a.nrt = h->nrt;
+  a.batch = batch;
+  a.stages = L.stages;
+  a.cb_bytes = L.cb_bytes;
+  a.off_b = L.off_b;
+  a.off_cb = L.off_cb;
+  a.off_bar = L.off_bar;
+  const dim3 grid((unsigned)((h->nrt + kGemmTilesN - 1) / kGemmTilesN),
+                  (unsigned)((batch + kGemmBM - 1) / kGemmBM));
+  void* args[] = {&a, &tmap};
+  e = cudaLaunchKernel(kfn, grid, dim3(kGemmThreads), args, L.total, s);
+  if (e != cudaSuccess) return cuda_error(e, "gemm launch");
+  return SPHQ_OK;
+}
+
+}  // namespace sphq

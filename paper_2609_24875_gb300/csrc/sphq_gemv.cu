@@ -222,7 +222,7 @@ sphq_status launch_gemv(sphq_handle h, const void* x, void* y, int batch, cudaSt
   const GemvPlan& p = h->plan[batch];
   GemvArgs a;
   a.units = (const uint8_t*)h->units;
-  a.cbimage = (const uint8_t*)(h->bits == 2 ? h->cbimage : h->codebook);
+  a.cbimage = (const uint8_t*)(fmt_small(h->fmt) ? h->cbimage : h->codebook);
   a.x = (const uint16_t*)x;
   a.y = (uint16_t*)y;
   a.flag = h->flag + 1;

@@ -42,7 +42,7 @@ struct sphq_handle_s {
   uint32_t* params = nullptr;  // rows * ng words: Delta | r_min << 16
   float* ws = nullptr;         // split-K partial sums of plans that need them (none today)
   size_t ws_floats = 0;
-  int* flag = nullptr;         // [0] pack validation, [1] gemv wait timeouts
+  int* flag = nullptr;         // [0] pack validation, [1] kernel wait timeouts (gemv, gemm)
   void* xstage = nullptr;      // SPHQ_MAX_BATCH x cols fp16 (sphq_gemv_host)
   void* ystage = nullptr;      // SPHQ_MAX_BATCH x rows fp16
   void* zeros = nullptr;       // 256 B of zeros (activations of non-supplying lanes)
@@ -61,6 +61,8 @@ sphq_status make_gemv_plans(sphq_handle h);
 sphq_status set_gemv_cluster_size(sphq_handle h, int batch, int csize);
 // Enqueues the GEMV (validated arguments).
 sphq_status launch_gemv(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s);
+// Enqueues the tensor-core product for any batch (validated arguments).
+sphq_status launch_gemm(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s);
 // Enqueues the GEMV with caller-provided split-K scratch: `ws` holds at least
 // h->ws_floats floats and `tickets` h->nrt zeroed counters.
 sphq_status launch_gemv_scratch(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s,

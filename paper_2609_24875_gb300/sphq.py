@@ -56,6 +56,10 @@ def load() -> ctypes.CDLL:
         L.sphq_pack.restype = i32
         L.sphq_gemv.argtypes = [vp, vp, vp, i32, vp]
         L.sphq_gemv.restype = i32
+        L.sphq_gemm.argtypes = [vp, vp, vp, i32, vp]
+        L.sphq_gemm.restype = i32
+        L.sphq_check.argtypes = [vp, vp]
+        L.sphq_check.restype = i32
         L.sphq_gemv_host.argtypes = [vp, vp, vp, i32, vp]
         L.sphq_gemv_host.restype = i32
         L.sphq_decode.argtypes = [vp, vp, vp]
@@ -153,6 +157,30 @@ class SphqMatrix:
             y = torch.empty((B, self.rows), dtype=torch.float16, device=x.device)
         _check(load().sphq_gemv(self._h, x.data_ptr(), y.data_ptr(), B, _stream_ptr(stream)))
         return y
+
+    def gemm(self, x, y=None, stream=None):
+        """Y = X W_hat^T on the tensor cores for any batch (prefill).
+        x: (batch, cols) fp16 on the device; returns (batch, rows) fp16."""
+        import torch
+        if x.dim() == 1:
+            x = x.unsqueeze(0)
+        B = x.shape[0]
+        if x.shape[1] != self.cols or x.element_size() != 2 or not x.is_cuda:
+            raise ValueError("x must be a (batch, cols) 2-byte CUDA tensor")
+        x = x.contiguous()
+        if y is None:
+            y = torch.empty((B, self.rows), dtype=torch.float16, device=x.device)
+        _check(load().sphq_gemm(self._h, x.data_ptr(), y.data_ptr(), B, _stream_ptr(stream)))
+        return y
+
+    def gemm_ptr(self, x_ptr: int, y_ptr: int, batch: int, stream_ptr: int) -> None:
+        """Raw-pointer sphq_gemm (no tensor checks)."""
+        _check(load().sphq_gemm(self._h, x_ptr, y_ptr, batch, stream_ptr))
+
+    def check(self, stream=None) -> None:
+        """sphq_check: synchronise the stream and raise if a kernel on this
+        handle gave up an on-chip wait since the last check."""
+        _check(load().sphq_check(self._h, _stream_ptr(stream)))
 
     def gemv_ptr(self, x_ptr: int, y_ptr: int, batch: int, stream_ptr: int) -> None:
         """Raw-pointer call (no tensor checks), for graph capture and benchmarks."""
