@@ -56,7 +56,8 @@ UNIT = "GB/s"
 # from ncu captures of the 8192x8192 batch-1 launches (profiles/
 # gemv_w2_8192_b1_full.md, gemv_w3_8192_b1_full.md), valid for the kernel
 # sources with this digest only; the roofline reports traffic null otherwise.
-TRAFFIC_SOURCES = ("paper_2609_24875_gb300/csrc/sphq_gemv.cu",
+TRAFFIC_SOURCES = ("paper_2609_24875_gb300/csrc/sphq_gemv_kernel.cuh",
+                   "paper_2609_24875_gb300/csrc/sphq_gemv.cu",
                    "paper_2609_24875_gb300/csrc/sphq_layout.cuh")
 TRAFFIC_DIGEST = "16baa0ff9a5899d0:154cf99e178b8279"
 TRAFFIC_RATIO = {2: 21042432 / 21005312, 3: 28503552 / 28475392}
@@ -516,23 +517,24 @@ def run_reference(args, world, rank):
 def run_case(spec: str, pool: int, launches: int):
     """Profiling driver: `bits:n[:batch]` -> `pool` distinct packed n x n
     matrices, `launches` GEMVs round robin on one stream, no timing (for
-    running under ncu).  bits `3v3` selects W3 with 3-bit radius codes."""
+    running under ncu).  bits `3v3` selects W3 with 3-bit radius codes, `dDvV`
+    the 8/D/V split (e.g. `d7v2`)."""
     import torch
 
     head, *rest = spec.split(":")
-    bits, vbits = (3, 3) if head == "3v3" else (int(head), 4)
+    bits, vbits, K = parse_split(head)
     parts = [int(v) for v in rest]
     n = parts[0]
     batch = parts[1] if len(parts) > 1 else 1
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     from paper_2609_24875_gb300 import SphqMatrix
-    codes, x = inp.random_codes(bits, n, n, seed=1, B=batch, radius_bits=vbits)
+    codes, x = inp.random_codes(bits, n, n, seed=1, B=batch, radius_bits=vbits, K=K)
     t = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int16) if a.dtype == np.uint16 else a)).to(dev)
     mats = []
     for _ in range(pool):
         m = SphqMatrix(n, n, bits, t(codes.codebook), t(codes.scale), t(codes.offset),
-                       radius_bits=vbits)
+                       radius_bits=vbits, K=K)
         m.pack(t(codes.sign), t(codes.idx), t(codes.rcode))
         mats.append(m)
     xd = t(x).view(torch.float16)
@@ -543,6 +545,107 @@ def run_case(spec: str, pool: int, launches: int):
     torch.cuda.synchronize()
     print(f"case W{bits} V={vbits} {n}x{n} batch {batch}: {launches} launches over {pool} "
           "matrices done")
+
+
+def parse_split(head: str):
+    """bits token of the profiling drivers -> (bits, radius bits, K): "2", "3",
+    "3v3" (W3, 3-bit radius codes) or "2:D:V" style "d7v2" (8/7/2)."""
+    if head == "3v3":
+        return 3, 3, 8192
+    if head.startswith("d"):
+        d, v = head[1:].split("v")
+        return 2, int(v), 1 << int(d)
+    b = int(head)
+    return b, 4, 1 << (7 * b - 8)
+
+
+def run_gemm_case(spec: str, launches: int):
+    """Profiling driver of the prefill GEMM: `bits:rows:cols:batch` ->
+    `launches` sphq_gemm calls on one matrix, no timing (for ncu)."""
+    import torch
+
+    head, *rest = spec.split(":")
+    bits, vbits, K = parse_split(head)
+    rows, cols, batch = (int(v) for v in rest)
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    from paper_2609_24875_gb300 import SphqMatrix
+    codes, x = inp.random_codes(bits, rows, cols, seed=1, B=batch, radius_bits=vbits, K=K)
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int16) if a.dtype == np.uint16 else a)).to(dev)
+    m = SphqMatrix(rows, cols, bits, t(codes.codebook), t(codes.scale), t(codes.offset),
+                   radius_bits=vbits, K=K)
+    m.pack(t(codes.sign), t(codes.idx), t(codes.rcode))
+    xd = t(x).view(torch.float16)
+    y = torch.empty((batch, rows), dtype=torch.float16, device=dev)
+    s = torch.cuda.current_stream()
+    for _ in range(launches):
+        m.gemm_ptr(xd.data_ptr(), y.data_ptr(), batch, s.cuda_stream)
+    m.check()
+    print(f"gemm case W{bits} V={vbits} K={K} {rows}x{cols} batch {batch}: {launches} launches done")
+
+
+def gemm_report(hbm_peak):
+    """Prefill GEMM (sphq_gemm) against the tensor-core roofline: TFLOP/s =
+    2 * batch * rows * cols / time (median of 10 timed calls after warm-up,
+    events on the launching stream), fraction of the measured bf16 dense peak
+    (fp16 runs at the bf16 rate); a dense fp16 cuBLAS GEMM on the decoded
+    weights of the same shape is timed beside it as context."""
+    import torch
+
+    from paper_2609_24875_gb300 import SphqMatrix
+    dev = torch.device("cuda", 0)
+    peaks = {}
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            peaks = json.load(f)
+    except OSError:
+        pass
+    tf_peak = float(peaks.get("bf16_tflops", 1900.0))
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int16) if a.dtype == np.uint16 else a)).to(dev)
+    stream = torch.cuda.Stream(device=dev)
+
+    def timed(fn, reps=10):
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                fn()
+        stream.synchronize()
+        times = []
+        for _ in range(reps):
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            with torch.cuda.stream(stream):
+                e0.record(stream)
+                fn()
+                e1.record(stream)
+            stream.synchronize()
+            times.append(e0.elapsed_time(e1) * 1e3)
+        return statistics.median(times)
+
+    out = {"peak_tflops": tf_peak}
+    for name, (bits, v, K) in (("W2", (2, 4, 64)), ("W3", (3, 4, 8192)), ("W3V3", (3, 3, 8192)),
+                               ("8/8/2", (2, 2, 256))):
+        for rows, cols, batch in ((3584, 3584, 512), (18944, 3584, 2048), (8192, 8192, 4096)):
+            codes, _ = inp.random_codes(bits, rows, cols, seed=inp.seed_for(5, rows % 97),
+                                        radius_bits=v, K=K)
+            m = SphqMatrix(rows, cols, bits, t(codes.codebook), t(codes.scale), t(codes.offset),
+                           radius_bits=v, K=K)
+            m.pack(t(codes.sign), t(codes.idx), t(codes.rcode))
+            x = torch.randn(batch, cols, device=dev).half()
+            y = torch.empty(batch, rows, device=dev, dtype=torch.half)
+            us = timed(lambda: m.gemm_ptr(x.data_ptr(), y.data_ptr(), batch, stream.cuda_stream))
+            m.check(stream)
+            wd = m.decode()
+            torch.cuda.synchronize()
+            us_d = timed(lambda: torch.matmul(x, wd.t()))
+            fl = 2.0 * batch * rows * cols
+            out[f"{name} {rows}x{cols} B{batch}"] = {
+                "us": round(us, 2), "TF/s": round(fl / us / 1e6, 1),
+                "tensor_frac": round(fl / us / 1e6 / tf_peak, 4),
+                "dense_fp16_cublas_us": round(us_d, 2)}
+            m.close()
+            del wd, x, y
+            torch.cuda.empty_cache()
+    return out
 
 
 def steady_us(mats, xd, ys, batch, stream, reps=20):
@@ -655,6 +758,7 @@ def run_report(args):
                                                                inp.seed_for(1, 20 + 10 * d + v),
                                                                1, vbits=v, K=1 << d)
                                for d, v in ((6, 2), (6, 3), (7, 2), (7, 3), (8, 2), (6, 4))}
+    rep["prefill_gemm"] = gemm_report(hbm_peak)
     # CPU oracle on the 1024^2 matrix: single thread and all cores
     import oracle
     codes, x = inp.random_codes(2, 1024, 1024, seed=inp.seed_for(0, 0))
@@ -685,11 +789,16 @@ def main():
     ap.add_argument("--case", default="", help="profiling driver: bits:n[:batch], no timing")
     ap.add_argument("--pool", type=int, default=4, help="--case: distinct matrices")
     ap.add_argument("--launches", type=int, default=8, help="--case: GEMV launches")
+    ap.add_argument("--gemm-case", default="",
+                    help="prefill GEMM profiling driver: bits:rows:cols:batch, no timing")
     ap.add_argument("--report", action="store_true",
                     help="supplementary per-configuration table (one JSON object)")
     args = ap.parse_args()
     if args.case:
         run_case(args.case, args.pool, args.launches)
+        return
+    if args.gemm_case:
+        run_gemm_case(args.gemm_case, args.launches)
         return
     if args.report:
         run_report(args)

@@ -8,22 +8,27 @@
 // decode of the GEMV's batch 3-8 mode) straight into shared memory, never to
 // HBM.
 //
-// Tiles: an output tile is 128 activation rows (the MMA's M; tokens) x 256
-// weight rows (the MMA's N; 16 row tiles of the unit layout), accumulated in
-// fp32 in tensor memory over the columns in steps of 64.  Per step:
-//  * one TMA warp loads the 128 x 64 activation tile (A operand, K-major,
-//    128-byte swizzle; rows past the batch read zeros);
+// Tiles: an output tile is 128 or 256 activation rows (one or two MMAs of
+// M = 128; tokens) x 256 weight rows (the MMA's N; 16 row tiles of the unit
+// layout), accumulated in fp32 in tensor memory (256 or all 512 columns) over
+// the columns in steps of 64.  Two activation tiles per decoded weight tile
+// halve the decode and shared-memory traffic per flop; they are used when the
+// batch exceeds 128 and two ring stages still fit next to the codebook (not
+// for the 128 KiB W3 table).  Per step:
+//  * one TMA warp loads the 128 (256) x 64 activation tile (A operand,
+//    K-major, 128-byte swizzle; rows past the batch read zeros);
 //  * eight decode warps each rebuild two 16 x 64 slices of W_hat (half a unit
 //    of two row tiles) into the B operand tile in the same swizzled K-major
 //    layout, fence them to the async proxy and arrive on the stage's
 //    mbarrier;
-//  * one MMA warp issues four 128 x 256 x 16 tcgen05.mma (fp16 x fp16 ->
-//    fp32) when both halves of the stage are in, and commits their completion
+//  * one MMA warp issues four (eight) 128 x 256 x 16 tcgen05.mma (fp16 x
+//    fp16 -> fp32) when both halves of the stage are in, and commits their completion
 //    to the stage's "empty" mbarrier, which releases the buffers.
 // Stages rotate through a ring of buffers (two to four, as shared memory
 // allows next to the codebook).  After the last step the decode warps read
-// the accumulators from tensor memory (warp w: lanes 32 (w % 4).., columns
-// 128 (w / 4)..), round to fp16 and store Y.
+// the accumulators from tensor memory (warp w: lanes 32 (w % 4).. of
+// accumulator w / 4, or of column half w / 4 with one accumulator), round to
+// fp16 and store Y.
 //
 // Every mbarrier wait gives up after about two seconds and records bit 1 in
 // the handle's device error word, so a fault cannot hang the GPU.
@@ -46,7 +51,7 @@ constexpr int kGemmDecodeWarps = 8;             // two row tiles each
 constexpr int kGemmThreads = (kGemmDecodeWarps + 2) * 32;
 constexpr int kGemmMmaWarp = kGemmDecodeWarps;
 constexpr int kGemmTmaWarp = kGemmDecodeWarps + 1;
-constexpr uint32_t kTileA = kGemmBM * kGemmBK * 2;  // 16 KiB
+constexpr uint32_t kTileA = kGemmBM * kGemmBK * 2;  // 16 KiB per 128 activation rows
 constexpr uint32_t kTileB = kGemmBN * kGemmBK * 2;  // 32 KiB
 static_assert(kGemmTilesN == 2 * kGemmDecodeWarps, "two row tiles per decode warp");
 
@@ -70,31 +75,47 @@ __device__ __forceinline__ void sts16(uint32_t addr, uint4 v) {
                : "memory");
 }
 
+__device__ __forceinline__ uint4 sel4(bool p, uint4 a, uint4 b) {
+  return make_uint4(p ? a.x : b.x, p ? a.y : b.y, p ? a.z : b.z, p ? a.w : b.w);
+}
+
 // Decodes words M and M+1 (the stage's 64 columns) of the lane's unit and
 // stores its four 16-byte blocks into the B tile: vector (row, slot) goes to
 // tile row n and 16-byte chunk c = slot % 8, at chunk position c ^ (n % 8).
+// Lanes of odd gid store word M+1 first: the two gids of a quarter warp then
+// write disjoint chunk positions ({q ^ gid} and {(4 + q) ^ (gid + 1)}), so
+// each 16-byte store is free of bank conflicts.
 template <int FMT, int M>
 __device__ __forceinline__ void decode_half(const Unit<FMT>& u, const UnitConst<FMT>& kc, int q,
                                             int gid, int jt, const SmemCodebook& cb,
                                             uint32_t btile) {
+  uint4 wa[2], wb[2];
 #pragma unroll
   for (int mm = 0; mm < 2; ++mm) {
     uint4 sa, sb;
     uint32_t qp;
     word_directions<FMT>(u, kc, M + mm, q, cb, sa, sb, qp);
     const uint32_t r = radius_pair<fmt_radius_bits(FMT)>(qp, kc.d2, kc.m2);
-    const uint4 wa = scale_block(sa, bcast_lo(r));
-    const uint4 wb = scale_block(sb, bcast_hi(r));
-    const int c = 4 * mm + q;
-    const int nA = kRowsPerTile * jt + gid, nB = nA + 8;
-    sts16(btile + nA * 128 + ((c ^ (nA & 7)) << 4), wa);
-    sts16(btile + nB * 128 + ((c ^ (nB & 7)) << 4), wb);
+    wa[mm] = scale_block(sa, bcast_lo(r));
+    wb[mm] = scale_block(sb, bcast_hi(r));
   }
+  const bool odd = gid & 1;
+  const int nA = kRowsPerTile * jt + gid, nB = nA + 8;
+  const uint32_t rowA = btile + nA * 128, rowB = btile + nB * 128;
+  const int c0 = (odd ? 4 : 0) + q, c1 = c0 ^ 4;  // first / second chunk stored
+  sts16(rowA + ((c0 ^ (nA & 7)) << 4), sel4(odd, wa[1], wa[0]));
+  sts16(rowB + ((c0 ^ (nB & 7)) << 4), sel4(odd, wb[1], wb[0]));
+  sts16(rowA + ((c1 ^ (nA & 7)) << 4), sel4(odd, wa[0], wa[1]));
+  sts16(rowB + ((c1 ^ (nB & 7)) << 4), sel4(odd, wb[0], wb[1]));
 }
 
-template <int FMT>
+// MT activation tiles of 128 rows share each decoded B tile (MT accumulators
+// of 256 tensor-memory columns).
+template <int FMT, int MT>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_kernel(const GemmArgs a, const __grid_constant__ CUtensorMap tmap) {
+  constexpr uint32_t kStageA = MT * kTileA;
+  constexpr uint32_t kCols = MT * kGemmBN;  // tensor-memory columns
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -109,7 +130,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   const uint32_t cb_bar = acc_bar + 8u;
   uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + a.off_bar + 16u * S + 16u);
   const int rt0 = blockIdx.x * kGemmTilesN;
-  const int tok0 = blockIdx.y * kGemmBM;
+  const int tok0 = blockIdx.y * kGemmBM * MT;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -124,7 +145,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       bulk_g2s(sbase + a.off_cb + o, a.cbimage + o, min(32768u, a.cb_bytes - o), cb_bar);
   }
   if (warp == kGemmMmaWarp) {
-    umma::tmem_alloc(smem_u32(tslot), kGemmBN);
+    umma::tmem_alloc(smem_u32(tslot), kCols);
     umma::tmem_relinquish();
   }
   umma::fence_before_sync();
@@ -137,8 +158,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       umma::prefetch_tmap(&tmap);
       for (int i = 0, s = 0, r = 0; i < nk; ++i) {
         if (r > 0 && !mbar_wait(empty0 + 8u * s, (r - 1) & 1)) atomicOr(a.flag, 2);
-        mbar_arrive_expect_tx(full0 + 8u * s, kTileA);
-        umma::tma_load_2d(sbase + s * kTileA, &tmap, i * kGemmBK, tok0, full0 + 8u * s);
+        mbar_arrive_expect_tx(full0 + 8u * s, kStageA);
+        umma::tma_load_2d(sbase + s * kStageA, &tmap, i * kGemmBK, tok0, full0 + 8u * s);
         if (++s == S) s = 0, ++r;
       }
     }
@@ -149,11 +170,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       for (int i = 0, s = 0, r = 0; i < nk; ++i) {
         if (!mbar_wait(full0 + 8u * s, r & 1)) atomicOr(a.flag, 2);
         umma::fence_after_sync();
-        const uint32_t at = sbase + s * kTileA, bt = sbase + a.off_b + s * kTileB;
+        const uint32_t at = sbase + s * kStageA, bt = sbase + a.off_b + s * kTileB;
 #pragma unroll
-        for (int kk = 0; kk < kGemmBK / 16; ++kk)
-          umma::mma_f16(taddr, umma::smem_desc_sw128(at + 32u * kk),
-                        umma::smem_desc_sw128(bt + 32u * kk), idesc, (i | kk) != 0);
+        for (int t = 0; t < MT; ++t)
+#pragma unroll
+          for (int kk = 0; kk < kGemmBK / 16; ++kk)
+            umma::mma_f16(taddr + t * kGemmBN, umma::smem_desc_sw128(at + t * kTileA + 32u * kk),
+                          umma::smem_desc_sw128(bt + 32u * kk), idesc, (i | kk) != 0);
         umma::commit(empty0 + 8u * s);
         if (++s == S) s = 0, ++r;
       }
@@ -186,7 +209,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           if (ok1) nxt[1] = load_unit<FMT>(nb + UB, lane);
         }
       }
-      if (r > 0 && !mbar_wait(empty0 + 8u * s, (r - 1) & 1) && lane == 0) atomicOr(a.flag, 2);
+      // one lane polls the stage's release (the MMAs that read it are
+      // complete); the warp's stores follow it through __syncwarp
+      if (r > 0 && lane == 0 && !mbar_wait(empty0 + 8u * s, (r - 1) & 1)) atomicOr(a.flag, 2);
+      __syncwarp();
       const uint32_t bt = sbase + a.off_b + s * kTileB;
 #pragma unroll
       for (int j = 0; j < 2; ++j) {
@@ -206,15 +232,19 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     // ---- epilogue: accumulators -> fp16 Y ----
     if (!mbar_wait(acc_bar, 0) && lane == 0) atomicOr(a.flag, 2);
     umma::fence_after_sync();
-    const int quarter = warp & 3;
-    const int token = tok0 + 32 * quarter + lane;
+    // warp w reads lanes 32 (w % 4).. of accumulator w / 4 (MT = 2), or of
+    // the single accumulator's column half w / 4 (MT = 1)
+    const int quarter = warp & 3, hi = warp >> 2;
+    const int token = tok0 + (MT == 2 ? kGemmBM * hi : 0) + 32 * quarter + lane;
+    constexpr int kChunks = MT == 2 ? kGemmBN / 32 : kGemmBN / 64;
 #pragma unroll 1
-    for (int cc = 0; cc < 4; ++cc) {
-      const int c0 = (warp >> 2) * (kGemmBN / 2) + 32 * cc;
+    for (int cc = 0; cc < kChunks; ++cc) {
+      const int col = (MT == 2 ? 0 : hi * (kGemmBN / 2)) + 32 * cc;  // within the accumulator
+      const uint32_t tcol = (uint32_t)((MT == 2 ? hi * kGemmBN : 0) + col);
       uint32_t v[32];
-      umma::ld_32x32b_x32(taddr + ((uint32_t)(32 * quarter) << 16) + (uint32_t)c0, v);
+      umma::ld_32x32b_x32(taddr + ((uint32_t)(32 * quarter) << 16) + tcol, v);
       umma::wait_ld();
-      const int row0 = rt0 * kRowsPerTile + c0;
+      const int row0 = rt0 * kRowsPerTile + col;
       if (token < a.batch && row0 < a.rows) {
         uint16_t* dst = a.y + (size_t)token * a.rows + row0;
         if (row0 + 32 <= a.rows && (reinterpret_cast<uintptr_t>(dst) & 15u) == 0) {
@@ -241,7 +271,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   __syncthreads();
   if (warp == kGemmMmaWarp) {
     umma::fence_after_sync();
-    umma::tmem_dealloc(taddr, kGemmBN);
+    umma::tmem_dealloc(taddr, kCols);
   }
 }
 
@@ -270,11 +300,17 @@ static EncodeTiledFn encode_fn() {
   return fn;
 }
 
-static const void* gemm_kernel_ptr(int fmt) {
+template <int FMT>
+static const void* gemm_ptr_mt(int mt) {
+  return mt == 2 ? reinterpret_cast<const void*>(&gemm_kernel<FMT, 2>)
+                 : reinterpret_cast<const void*>(&gemm_kernel<FMT, 1>);
+}
+
+static const void* gemm_kernel_ptr(int fmt, int mt) {
   switch (fmt) {
 #define SPHQ_GEMM_PTR(F) \
   case F:                \
-    return reinterpret_cast<const void*>(&gemm_kernel<F>);
+    return gemm_ptr_mt<F>(mt);
     SPHQ_GEMM_PTR(2)
     SPHQ_GEMM_PTR(3)
     SPHQ_GEMM_PTR(4)
@@ -298,11 +334,11 @@ struct GemmSmem {
   size_t total = 0;
 };
 
-static GemmSmem gemm_smem(const sphq_handle_s* h, int optin) {
+static GemmSmem gemm_smem(const sphq_handle_s* h, int optin, int mt) {
   GemmSmem L;
   L.cb_bytes = fmt_small(h->fmt) ? (uint32_t)h->K * 8u * 16u : (uint32_t)h->K * 16u;
   for (int S = 4; S >= 2; --S) {
-    const size_t off_b = (size_t)S * kTileA;
+    const size_t off_b = (size_t)S * mt * kTileA;
     const size_t off_cb = off_b + (size_t)S * kTileB;
     const size_t off_bar = align_to(off_cb + L.cb_bytes, 16);
     const size_t total = 1024 + off_bar + 16u * S + 16u + 16u;  // alignment slack + barriers + slot
@@ -324,25 +360,29 @@ sphq_status launch_gemm(sphq_handle h, const void* x, void* y, int batch, cudaSt
   int optin = 0;
   cudaError_t e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, h->device);
   if (e != cudaSuccess) return cuda_error(e, "cudaDeviceGetAttribute");
-  const GemmSmem L = gemm_smem(h, optin);
+  // two activation tiles per decoded weight tile when the batch fills them
+  // and two ring stages still fit next to the codebook
+  int mt = batch > kGemmBM ? 2 : 1;
+  GemmSmem L = gemm_smem(h, optin, mt);
+  if (L.stages == 0 && mt == 2) L = gemm_smem(h, optin, mt = 1);
   if (L.stages == 0) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm: shared memory too small");
-  const void* kfn = gemm_kernel_ptr(h->fmt);
+  const void* kfn = gemm_kernel_ptr(h->fmt, mt);
   if (!kfn) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm: unknown format");
   {
     static std::mutex mu;
-    static bool done[16] = {};
+    static bool done[16][3] = {};
     std::lock_guard<std::mutex> lock(mu);
-    if (!done[h->fmt]) {
+    if (!done[h->fmt][mt]) {
       e = cudaFuncSetAttribute(kfn, cudaFuncAttributeMaxDynamicSharedMemorySize, optin);
       if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(gemm)");
-      done[h->fmt] = true;
+      done[h->fmt][mt] = true;
     }
   }
   // activations: a batch x cols fp16 tensor, boxes of 128 rows x 64 columns
   CUtensorMap tmap;
   const cuuint64_t gdim[2] = {(cuuint64_t)h->cols, (cuuint64_t)batch};
   const cuuint64_t gstride[1] = {(cuuint64_t)h->cols * 2};
-  const cuuint32_t box[2] = {(cuuint32_t)kGemmBK, (cuuint32_t)kGemmBM};
+  const cuuint32_t box[2] = {(cuuint32_t)kGemmBK, (cuuint32_t)(kGemmBM * mt)};
   const cuuint32_t estride[2] = {1, 1};
   CUresult cr = enc(&tmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(x), gdim, gstride,
                     box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -364,7 +404,7 @@ sphq_status launch_gemm(sphq_handle h, const void* x, void* y, int batch, cudaSt
   a.off_cb = L.off_cb;
   a.off_bar = L.off_bar;
   const dim3 grid((unsigned)((h->nrt + kGemmTilesN - 1) / kGemmTilesN),
-                  (unsigned)((batch + kGemmBM - 1) / kGemmBM));
+                  (unsigned)((batch + kGemmBM * mt - 1) / (kGemmBM * mt)));
   void* args[] = {&a, &tmap};
   e = cudaLaunchKernel(kfn, grid, dim3(kGemmThreads), args, L.total, s);
   if (e != cudaSuccess) return cuda_error(e, "gemm launch");
