@@ -11,15 +11,16 @@
 // Tiles: an output tile is 128 or 256 activation rows (one or two MMAs of
 // M = 128; tokens) x 256 weight rows (the MMA's N; 16 row tiles of the unit
 // layout), accumulated in fp32 in tensor memory (256 or all 512 columns) over
-// the columns in steps of 64.  Two activation tiles per decoded weight tile
-// halve the decode and shared-memory traffic per flop; they are used when the
-// batch exceeds 128 and two ring stages still fit next to the codebook (not
-// for the 128 KiB W3 table).  Per step:
-//  * one TMA warp loads the 128 (256) x 64 activation tile (A operand,
-//    K-major, 128-byte swizzle; rows past the batch read zeros);
-//  * eight decode warps each rebuild two 16 x 64 slices of W_hat (half a unit
-//    of two row tiles) into the B operand tile in the same swizzled K-major
-//    layout, fence them to the async proxy and arrive on the stage's
+// the columns in steps of 64 (128-byte swizzled operand rows) or 32 (64-byte
+// swizzle).  Two activation tiles per decoded weight tile halve the decode
+// and shared-memory traffic per flop; they are used when the batch exceeds
+// 128.  Next to the 128 KiB W3 codebook only 32-column steps leave room for a
+// ring of three stages with two activation tiles.  Per step:
+//  * one TMA warp loads the 128 (256) x BK activation tile (A operand,
+//    K-major, swizzled; rows past the batch read zeros);
+//  * eight decode warps each rebuild two 16 x BK slices of W_hat (half or a
+//    quarter of a unit of two row tiles) into the B operand tile in the same
+//    swizzled K-major layout, fence them to the async proxy and arrive on the stage's
 //    mbarrier;
 //  * one MMA warp issues four (eight) 128 x 256 x 16 tcgen05.mma (fp16 x
 //    fp16 -> fp32) when both halves of the stage are in, and commits their completion
@@ -45,14 +46,14 @@ namespace sphq {
 
 constexpr int kGemmBM = 128;                    // activation rows per tile (MMA M)
 constexpr int kGemmBN = 256;                    // weight rows per tile (MMA N)
-constexpr int kGemmBK = 64;                     // columns per pipeline stage
 constexpr int kGemmTilesN = kGemmBN / kRowsPerTile;
 constexpr int kGemmDecodeWarps = 8;             // two row tiles each
 constexpr int kGemmThreads = (kGemmDecodeWarps + 2) * 32;
 constexpr int kGemmMmaWarp = kGemmDecodeWarps;
 constexpr int kGemmTmaWarp = kGemmDecodeWarps + 1;
-constexpr uint32_t kTileA = kGemmBM * kGemmBK * 2;  // 16 KiB per 128 activation rows
-constexpr uint32_t kTileB = kGemmBN * kGemmBK * 2;  // 32 KiB
+// operand tile bytes for a stage of BK columns
+constexpr uint32_t tile_a_bytes(int bk) { return (uint32_t)kGemmBM * bk * 2; }  // per 128 rows
+constexpr uint32_t tile_b_bytes(int bk) { return (uint32_t)kGemmBN * bk * 2; }
 static_assert(kGemmTilesN == 2 * kGemmDecodeWarps, "two row tiles per decode warp");
 
 struct GemmArgs {
@@ -109,20 +110,40 @@ __device__ __forceinline__ void decode_half(const Unit<FMT>& u, const UnitConst<
   sts16(rowB + ((c1 ^ (nB & 7)) << 4), sel4(odd, wb[0], wb[1]));
 }
 
+// Decodes word M (a stage of 32 columns) of the lane's unit into a B tile of
+// 64-byte rows in the 64-byte swizzle: chunk q of row n at q ^ ((n / 2) % 4).
+// Rows gid and gid + 1 of a quarter warp are 64 bytes apart, so the eight
+// lanes hit distinct 16-byte bank groups.
+template <int FMT, int M>
+__device__ __forceinline__ void decode_word(const Unit<FMT>& u, const UnitConst<FMT>& kc, int q,
+                                            int gid, int jt, const SmemCodebook& cb,
+                                            uint32_t btile) {
+  uint4 sa, sb;
+  uint32_t qp;
+  word_directions<FMT>(u, kc, M, q, cb, sa, sb, qp);
+  const uint32_t r = radius_pair<fmt_radius_bits(FMT)>(qp, kc.d2, kc.m2);
+  const int nA = kRowsPerTile * jt + gid, nB = nA + 8;
+  sts16(btile + nA * 64 + ((q ^ ((nA >> 1) & 3)) << 4), scale_block(sa, bcast_lo(r)));
+  sts16(btile + nB * 64 + ((q ^ ((nB >> 1) & 3)) << 4), scale_block(sb, bcast_hi(r)));
+}
+
 // MT activation tiles of 128 rows share each decoded B tile (MT accumulators
-// of 256 tensor-memory columns).
-template <int FMT, int MT>
+// of 256 tensor-memory columns); BK columns per stage: 64 (128-byte swizzle)
+// or 32 (64-byte swizzle, half the ring memory, for the 128 KiB W3 codebook).
+template <int FMT, int MT, int BK>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_kernel(const GemmArgs a, const __grid_constant__ CUtensorMap tmap) {
+  constexpr uint32_t kTileA = tile_a_bytes(BK), kTileB = tile_b_bytes(BK);
   constexpr uint32_t kStageA = MT * kTileA;
   constexpr uint32_t kCols = MT * kGemmBN;  // tensor-memory columns
+  constexpr int kStepsPerGroup = kGroupCols / BK;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   const uint32_t sbase = smem_u32(smem);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int S = a.stages;
-  const int nk = a.cols / kGemmBK;
+  const int nk = a.cols / BK;
   const int ng = a.cols / kGroupCols;
   const uint32_t full0 = sbase + a.off_bar;  // full[S], empty[S], acc, cb, tmem slot
   const uint32_t empty0 = full0 + 8u * S;
@@ -159,7 +180,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       for (int i = 0, s = 0, r = 0; i < nk; ++i) {
         if (r > 0 && !mbar_wait(empty0 + 8u * s, (r - 1) & 1)) atomicOr(a.flag, 2);
         mbar_arrive_expect_tx(full0 + 8u * s, kStageA);
-        umma::tma_load_2d(sbase + s * kStageA, &tmap, i * kGemmBK, tok0, full0 + 8u * s);
+        umma::tma_load_2d(sbase + s * kStageA, &tmap, i * BK, tok0, full0 + 8u * s);
         if (++s == S) s = 0, ++r;
       }
     }
@@ -174,9 +195,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 #pragma unroll
         for (int t = 0; t < MT; ++t)
 #pragma unroll
-          for (int kk = 0; kk < kGemmBK / 16; ++kk)
-            umma::mma_f16(taddr + t * kGemmBN, umma::smem_desc_sw128(at + t * kTileA + 32u * kk),
-                          umma::smem_desc_sw128(bt + 32u * kk), idesc, (i | kk) != 0);
+          for (int kk = 0; kk < BK / 16; ++kk) {
+            const uint32_t ad = at + t * kTileA + 32u * kk, bd = bt + 32u * kk;
+            umma::mma_f16(taddr + t * kGemmBN,
+                          BK == 64 ? umma::smem_desc_sw128(ad) : umma::smem_desc_sw64(ad),
+                          BK == 64 ? umma::smem_desc_sw128(bd) : umma::smem_desc_sw64(bd), idesc,
+                          (i | kk) != 0);
+          }
         umma::commit(empty0 + 8u * s);
         if (++s == S) s = 0, ++r;
       }
@@ -199,8 +224,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     if (ok1) nxt[1] = load_unit<FMT>(ub0 + UB, lane);
     if (!mbar_wait(cb_bar, 0) && lane == 0) atomicOr(a.flag, 2);
     for (int i = 0, s = 0, r = 0; i < nk; ++i) {
-      const int g = i >> 1;
-      if ((i & 1) == 0) {
+      const int g = i / kStepsPerGroup;
+      const int step = i % kStepsPerGroup;
+      if (step == 0) {
         cur[0] = nxt[0];
         cur[1] = nxt[1];
         if (g + 1 < ng) {
@@ -218,10 +244,21 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       for (int j = 0; j < 2; ++j) {
         if (!(j ? ok1 : ok0)) continue;
         const UnitConst<FMT> kc = unit_const<FMT>(cur[j], q);
-        if (i & 1)
-          decode_half<FMT, 2>(cur[j], kc, q, gid, j0 + j, cb, bt);
-        else
-          decode_half<FMT, 0>(cur[j], kc, q, gid, j0 + j, cb, bt);
+        if constexpr (BK == 64) {
+          if (step)
+            decode_half<FMT, 2>(cur[j], kc, q, gid, j0 + j, cb, bt);
+          else
+            decode_half<FMT, 0>(cur[j], kc, q, gid, j0 + j, cb, bt);
+        } else {
+          if (step == 0)
+            decode_word<FMT, 0>(cur[j], kc, q, gid, j0 + j, cb, bt);
+          else if (step == 1)
+            decode_word<FMT, 1>(cur[j], kc, q, gid, j0 + j, cb, bt);
+          else if (step == 2)
+            decode_word<FMT, 2>(cur[j], kc, q, gid, j0 + j, cb, bt);
+          else
+            decode_word<FMT, 3>(cur[j], kc, q, gid, j0 + j, cb, bt);
+        }
       }
       umma::fence_proxy_async_smem();
       __syncwarp();
@@ -301,16 +338,22 @@ static EncodeTiledFn encode_fn() {
 }
 
 template <int FMT>
-static const void* gemm_ptr_mt(int mt) {
-  return mt == 2 ? reinterpret_cast<const void*>(&gemm_kernel<FMT, 2>)
-                 : reinterpret_cast<const void*>(&gemm_kernel<FMT, 1>);
+static const void* gemm_ptr(int mt, int bk) {
+  if constexpr (!fmt_small(FMT)) {
+    if (bk == 32)
+      return mt == 2 ? reinterpret_cast<const void*>(&gemm_kernel<FMT, 2, 32>)
+                     : reinterpret_cast<const void*>(&gemm_kernel<FMT, 1, 32>);
+  }
+  if (bk != 64) return nullptr;
+  return mt == 2 ? reinterpret_cast<const void*>(&gemm_kernel<FMT, 2, 64>)
+                 : reinterpret_cast<const void*>(&gemm_kernel<FMT, 1, 64>);
 }
 
-static const void* gemm_kernel_ptr(int fmt, int mt) {
+static const void* gemm_kernel_ptr(int fmt, int mt, int bk) {
   switch (fmt) {
 #define SPHQ_GEMM_PTR(F) \
   case F:                \
-    return gemm_ptr_mt<F>(mt);
+    return gemm_ptr<F>(mt, bk);
     SPHQ_GEMM_PTR(2)
     SPHQ_GEMM_PTR(3)
     SPHQ_GEMM_PTR(4)
@@ -334,12 +377,12 @@ struct GemmSmem {
   size_t total = 0;
 };
 
-static GemmSmem gemm_smem(const sphq_handle_s* h, int optin, int mt) {
+static GemmSmem gemm_smem(const sphq_handle_s* h, int optin, int mt, int bk) {
   GemmSmem L;
   L.cb_bytes = fmt_small(h->fmt) ? (uint32_t)h->K * 8u * 16u : (uint32_t)h->K * 16u;
   for (int S = 4; S >= 2; --S) {
-    const size_t off_b = (size_t)S * mt * kTileA;
-    const size_t off_cb = off_b + (size_t)S * kTileB;
+    const size_t off_b = (size_t)S * mt * tile_a_bytes(bk);
+    const size_t off_cb = off_b + (size_t)S * tile_b_bytes(bk);
     const size_t off_bar = align_to(off_cb + L.cb_bytes, 16);
     const size_t total = 1024 + off_bar + 16u * S + 16u + 16u;  // alignment slack + barriers + slot
     if (total <= (size_t)optin) {
@@ -360,32 +403,50 @@ sphq_status launch_gemm(sphq_handle h, const void* x, void* y, int batch, cudaSt
   int optin = 0;
   cudaError_t e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, h->device);
   if (e != cudaSuccess) return cuda_error(e, "cudaDeviceGetAttribute");
-  // two activation tiles per decoded weight tile when the batch fills them
-  // and two ring stages still fit next to the codebook
-  int mt = batch > kGemmBM ? 2 : 1;
-  GemmSmem L = gemm_smem(h, optin, mt);
-  if (L.stages == 0 && mt == 2) L = gemm_smem(h, optin, mt = 1);
-  if (L.stages == 0) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm: shared memory too small");
-  const void* kfn = gemm_kernel_ptr(h->fmt, mt);
-  if (!kfn) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm: unknown format");
+  // Shape: two activation tiles per decoded weight tile when the batch fills
+  // them and the grid still has a wave's worth of CTAs (estimated time per
+  // CTA: 1.6 with two tiles against 1 with one, times the waves); 64-column
+  // stages unless they leave no room for a ring of two next to the codebook
+  // (W3 with two activation tiles, which takes 32-column stages, three deep).
+  const long long tiles_n = (h->nrt + kGemmTilesN - 1) / kGemmTilesN;
+  const int sms = h->sm_count > 0 ? h->sm_count : 1;
+  auto waves = [&](int m) {
+    const long long ctas = tiles_n * ((batch + kGemmBM * m - 1) / (kGemmBM * m));
+    return (double)((ctas + sms - 1) / sms);
+  };
+  const bool two = batch > kGemmBM && 1.6 * waves(2) < waves(1);
+  static const int kCand2[4][2] = {{2, 64}, {2, 32}, {1, 64}, {1, 32}};
+  static const int kCand1[2][2] = {{1, 64}, {1, 32}};
+  const int (*cand)[2] = two ? kCand2 : kCand1;
+  const int ncand = two ? 4 : 2;
+  int mt = 0, bk = 0;
+  GemmSmem L;
+  for (int c = 0; c < ncand && !mt; ++c) {
+    if (!gemm_kernel_ptr(h->fmt, cand[c][0], cand[c][1])) continue;
+    const GemmSmem T = gemm_smem(h, optin, cand[c][0], cand[c][1]);
+    if (T.stages >= 2) mt = cand[c][0], bk = cand[c][1], L = T;
+  }
+  if (!mt) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm: shared memory too small");
+  const void* kfn = gemm_kernel_ptr(h->fmt, mt, bk);
   {
     static std::mutex mu;
-    static bool done[16][3] = {};
+    static bool done[16][3][2] = {};
     std::lock_guard<std::mutex> lock(mu);
-    if (!done[h->fmt][mt]) {
+    if (!done[h->fmt][mt][bk == 64]) {
       e = cudaFuncSetAttribute(kfn, cudaFuncAttributeMaxDynamicSharedMemorySize, optin);
       if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(gemm)");
-      done[h->fmt][mt] = true;
+      done[h->fmt][mt][bk == 64] = true;
     }
   }
   // activations: a batch x cols fp16 tensor, boxes of 128 rows x 64 columns
   CUtensorMap tmap;
   const cuuint64_t gdim[2] = {(cuuint64_t)h->cols, (cuuint64_t)batch};
   const cuuint64_t gstride[1] = {(cuuint64_t)h->cols * 2};
-  const cuuint32_t box[2] = {(cuuint32_t)kGemmBK, (cuuint32_t)(kGemmBM * mt)};
+  const cuuint32_t box[2] = {(cuuint32_t)bk, (cuuint32_t)(kGemmBM * mt)};
   const cuuint32_t estride[2] = {1, 1};
   CUresult cr = enc(&tmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(x), gdim, gstride,
-                    box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                    bk == 64 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B,
                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (cr != CUDA_SUCCESS)
     return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemm: cuTensorMapEncodeTiled rejected x");

@@ -4,13 +4,15 @@
 // layout, the instruction descriptor of an fp16 x fp16 -> fp32 MMA, MMA issue
 // and completion, tensor-memory loads, and 2-D tiled TMA loads.
 //
-// Operand layout used throughout (both operands K-major, 128-byte swizzle):
-// a tile of R rows x 64 fp16 (128 bytes per row) at a 1024-byte aligned base;
-// row r occupies bytes [128 r, 128 r + 128), and its 16-byte chunk c (fp16
-// columns 8c..8c+7) is stored at chunk position c ^ (r % 8).  Eight rows form
-// one 1024-byte swizzle atom; atoms follow each other (stride 1024 bytes).
-// This is the layout a TMA load with CU_TENSOR_MAP_SWIZZLE_128B and a box of
-// 64 fp16 columns writes, and the one the descriptor below describes.
+// Operand layouts (both operands K-major): a tile of R rows x 64 fp16 (128
+// bytes per row) at a 1024-byte aligned base; row r occupies bytes
+// [128 r, 128 r + 128), and its 16-byte chunk c (fp16 columns 8c..8c+7) is
+// stored at chunk position c ^ (r % 8).  Eight rows form one 1024-byte
+// swizzle atom; atoms follow each other (stride 1024 bytes).  This is the
+// layout a TMA load with CU_TENSOR_MAP_SWIZZLE_128B and a box of 64 fp16
+// columns writes.  With 32 fp16 per row (64 bytes) the 64-byte swizzle puts
+// chunk c of row r at c ^ ((r / 2) % 4), 512-byte atoms
+// (CU_TENSOR_MAP_SWIZZLE_64B, a box of 32 columns).
 #pragma once
 #include <cstdint>
 
@@ -33,6 +35,14 @@ namespace umma {
 __host__ __device__ constexpr uint64_t smem_desc_sw128(uint32_t saddr) {
   return (uint64_t)((saddr >> 4) & 0x3FFFu) | ((uint64_t)1u << 16) | ((uint64_t)(1024u >> 4) << 32) |
          ((uint64_t)1u << 46) | ((uint64_t)2u << 61);
+}
+
+// The same for rows of 64 bytes (32 fp16) in the 64-byte swizzle: chunk c
+// (0..3) of row r at chunk position c ^ ((r / 2) % 4), 8-row atoms of 512
+// bytes (stride byte offset 512), layout 4 = 64-byte swizzle.
+__host__ __device__ constexpr uint64_t smem_desc_sw64(uint32_t saddr) {
+  return (uint64_t)((saddr >> 4) & 0x3FFFu) | ((uint64_t)1u << 16) | ((uint64_t)(512u >> 4) << 32) |
+         ((uint64_t)1u << 46) | ((uint64_t)4u << 61);
 }
 
 // Instruction descriptor (32 bits) of tcgen05.mma .kind::f16 with fp16 A and
