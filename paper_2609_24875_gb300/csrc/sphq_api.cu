@@ -452,6 +452,26 @@ sphq_status sphq_gemm(sphq_handle h, const void* x, void* y, int batch, sphq_str
   return launch_gemm(h, x, y, batch, reinterpret_cast<cudaStream_t>(stream));
 }
 
+sphq_status sphq_get_gemm_shape(sphq_handle h, int batch, sphq_gemm_info* out) {
+  g_last_error.clear();
+  if (!h || !out) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_get_gemm_shape: NULL argument");
+  if (batch < 1 || batch > SPHQ_GEMM_MAX_BATCH)
+    return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_get_gemm_shape: batch out of range");
+  return gemm_shape_info(h, batch, out);
+}
+
+sphq_status sphq_set_gemm_shape(sphq_handle h, int act_tiles, int weight_rows) {
+  g_last_error.clear();
+  if (!h) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_set_gemm_shape: NULL handle");
+  if (act_tiles < 0 || act_tiles > 2 || (weight_rows != 0 && weight_rows != 128 && weight_rows != 256) ||
+      (act_tiles == 2 && weight_rows == 128))
+    return set_error(SPHQ_ERR_INVALID_ARG,
+                     "sphq_set_gemm_shape: act_tiles 0..2, weight_rows 0/128/256, not 2 x 128");
+  h->gemm_mt = act_tiles;
+  h->gemm_bn = weight_rows;
+  return SPHQ_OK;
+}
+
 sphq_status sphq_check(sphq_handle h, sphq_stream stream) {
   g_last_error.clear();
   if (!h) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_check: NULL handle");

@@ -9,8 +9,9 @@
 // HBM.
 //
 // Tiles: an output tile is 128 or 256 activation rows (one or two MMAs of
-// M = 128; tokens) x 256 weight rows (the MMA's N; 16 row tiles of the unit
-// layout), accumulated in fp32 in tensor memory (256 or all 512 columns) over
+// M = 128; tokens) x 256 or 128 weight rows (the MMA's N; 16 or 8 row tiles
+// of the unit layout; 128 only with one activation tile, for grids that
+// would otherwise leave SMs idle), accumulated in fp32 in tensor memory (256 or all 512 columns) over
 // the columns in steps of 64 (128-byte swizzled operand rows) or 32 (64-byte
 // swizzle).  Two activation tiles per decoded weight tile halve the decode
 // and shared-memory traffic per flop; they are used when the batch exceeds
@@ -18,12 +19,12 @@
 // ring of three stages with two activation tiles.  Per step:
 //  * one TMA warp loads the 128 (256) x BK activation tile (A operand,
 //    K-major, swizzled; rows past the batch read zeros);
-//  * eight decode warps each rebuild two 16 x BK slices of W_hat (half or a
-//    quarter of a unit of two row tiles) into the B operand tile in the same
+//  * eight decode warps each rebuild one or two 16 x BK slices of W_hat (half
+//    or a quarter of a unit of each of their row tiles) into the B operand tile in the same
 //    swizzled K-major layout, fence them to the async proxy and arrive on the stage's
 //    mbarrier;
-//  * one MMA warp issues four (eight) 128 x 256 x 16 tcgen05.mma (fp16 x
-//    fp16 -> fp32) when both halves of the stage are in, and commits their completion
+//  * one MMA warp issues BK / 16 (times the activation tiles) 128 x BN x 16
+//    tcgen05.mma (fp16 x fp16 -> fp32) when both halves of the stage are in, and commits their completion
 //    to the stage's "empty" mbarrier, which releases the buffers.
 // Stages rotate through a ring of buffers (two to four, as shared memory
 // allows next to the codebook).  After the last step the decode warps read
@@ -45,16 +46,13 @@
 namespace sphq {
 
 constexpr int kGemmBM = 128;                    // activation rows per tile (MMA M)
-constexpr int kGemmBN = 256;                    // weight rows per tile (MMA N)
-constexpr int kGemmTilesN = kGemmBN / kRowsPerTile;
 constexpr int kGemmDecodeWarps = 8;             // two row tiles each
 constexpr int kGemmThreads = (kGemmDecodeWarps + 2) * 32;
 constexpr int kGemmMmaWarp = kGemmDecodeWarps;
 constexpr int kGemmTmaWarp = kGemmDecodeWarps + 1;
 // operand tile bytes for a stage of BK columns
 constexpr uint32_t tile_a_bytes(int bk) { return (uint32_t)kGemmBM * bk * 2; }  // per 128 rows
-constexpr uint32_t tile_b_bytes(int bk) { return (uint32_t)kGemmBN * bk * 2; }
-static_assert(kGemmTilesN == 2 * kGemmDecodeWarps, "two row tiles per decode warp");
+constexpr uint32_t tile_b_bytes(int bk, int bn) { return (uint32_t)bn * bk * 2; }
 
 struct GemmArgs {
   const uint8_t* units;
@@ -130,12 +128,15 @@ __device__ __forceinline__ void decode_word(const Unit<FMT>& u, const UnitConst<
 // MT activation tiles of 128 rows share each decoded B tile (MT accumulators
 // of 256 tensor-memory columns); BK columns per stage: 64 (128-byte swizzle)
 // or 32 (64-byte swizzle, half the ring memory, for the 128 KiB W3 codebook).
-template <int FMT, int MT, int BK>
+template <int FMT, int MT, int BK, int BN>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_kernel(const GemmArgs a, const __grid_constant__ CUtensorMap tmap) {
-  constexpr uint32_t kTileA = tile_a_bytes(BK), kTileB = tile_b_bytes(BK);
+  constexpr int kTilesN = BN / kRowsPerTile;          // row tiles per weight tile
+  constexpr int kTPW = kTilesN / kGemmDecodeWarps;    // row tiles per decode warp (2 or 1)
+  static_assert(kTPW * kGemmDecodeWarps == kTilesN && (kTPW == 1 || kTPW == 2), "tile split");
+  constexpr uint32_t kTileA = tile_a_bytes(BK), kTileB = tile_b_bytes(BK, BN);
   constexpr uint32_t kStageA = MT * kTileA;
-  constexpr uint32_t kCols = MT * kGemmBN;  // tensor-memory columns
+  constexpr uint32_t kCols = MT * BN;  // tensor-memory columns
   constexpr int kStepsPerGroup = kGroupCols / BK;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -150,7 +151,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   const uint32_t acc_bar = empty0 + 8u * S;
   const uint32_t cb_bar = acc_bar + 8u;
   uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + a.off_bar + 16u * S + 16u);
-  const int rt0 = blockIdx.x * kGemmTilesN;
+  const int rt0 = blockIdx.x * kTilesN;
   const int tok0 = blockIdx.y * kGemmBM * MT;
 
   if (threadIdx.x == 0) {
@@ -187,7 +188,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     __syncwarp();
   } else if (warp == kGemmMmaWarp) {
     if (lane == 0) {
-      constexpr uint32_t idesc = umma::idesc_f16_f32(kGemmBM, kGemmBN);
+      constexpr uint32_t idesc = umma::idesc_f16_f32(kGemmBM, BN);
       for (int i = 0, s = 0, r = 0; i < nk; ++i) {
         if (!mbar_wait(full0 + 8u * s, r & 1)) atomicOr(a.flag, 2);
         umma::fence_after_sync();
@@ -197,7 +198,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk) {
             const uint32_t ad = at + t * kTileA + 32u * kk, bd = bt + 32u * kk;
-            umma::mma_f16(taddr + t * kGemmBN,
+            umma::mma_f16(taddr + t * BN,
                           BK == 64 ? umma::smem_desc_sw128(ad) : umma::smem_desc_sw64(ad),
                           BK == 64 ? umma::smem_desc_sw128(bd) : umma::smem_desc_sw64(bd), idesc,
                           (i | kk) != 0);
@@ -215,8 +216,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     SmemCodebook cb;
     cb.base = smem + a.off_cb;
     cb.copyoff = fmt_small(FMT) ? (uint32_t)(lane & 7) * 16u : 0u;
-    const int j0 = 2 * warp;
-    const bool ok0 = rt0 + j0 < a.nrt, ok1 = rt0 + j0 + 1 < a.nrt;
+    const int j0 = kTPW * warp;
+    const bool ok0 = rt0 + j0 < a.nrt, ok1 = kTPW == 2 && rt0 + j0 + 1 < a.nrt;
     const uint8_t* ub0 = a.units + (size_t)(rt0 + j0) * UB;  // group 0; + g * nrt * UB
     const size_t gstride = (size_t)a.nrt * UB;
     Unit<FMT> cur[2] = {}, nxt[2] = {};
@@ -273,11 +274,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     // the single accumulator's column half w / 4 (MT = 1)
     const int quarter = warp & 3, hi = warp >> 2;
     const int token = tok0 + (MT == 2 ? kGemmBM * hi : 0) + 32 * quarter + lane;
-    constexpr int kChunks = MT == 2 ? kGemmBN / 32 : kGemmBN / 64;
+    constexpr int kChunks = MT == 2 ? BN / 32 : BN / 64;
 #pragma unroll 1
     for (int cc = 0; cc < kChunks; ++cc) {
-      const int col = (MT == 2 ? 0 : hi * (kGemmBN / 2)) + 32 * cc;  // within the accumulator
-      const uint32_t tcol = (uint32_t)((MT == 2 ? hi * kGemmBN : 0) + col);
+      const int col = (MT == 2 ? 0 : hi * (BN / 2)) + 32 * cc;  // within the accumulator
+      const uint32_t tcol = (uint32_t)((MT == 2 ? hi * BN : 0) + col);
       uint32_t v[32];
       umma::ld_32x32b_x32(taddr + ((uint32_t)(32 * quarter) << 16) + tcol, v);
       umma::wait_ld();
@@ -337,23 +338,30 @@ static EncodeTiledFn encode_fn() {
   return fn;
 }
 
+// Instantiated shapes (MT, BK, BN): 128-row weight tiles only with one
+// activation tile; 32-column stages only for the W3 tables.
 template <int FMT>
-static const void* gemm_ptr(int mt, int bk) {
-  if constexpr (!fmt_small(FMT)) {
-    if (bk == 32)
-      return mt == 2 ? reinterpret_cast<const void*>(&gemm_kernel<FMT, 2, 32>)
-                     : reinterpret_cast<const void*>(&gemm_kernel<FMT, 1, 32>);
+static const void* gemm_ptr(int mt, int bk, int bn) {
+  const void* p = nullptr;
+  if (bn == 256) {
+    if (bk == 64) p = mt == 2 ? (const void*)&gemm_kernel<FMT, 2, 64, 256>
+                              : (const void*)&gemm_kernel<FMT, 1, 64, 256>;
+    if constexpr (!fmt_small(FMT))
+      if (bk == 32) p = mt == 2 ? (const void*)&gemm_kernel<FMT, 2, 32, 256>
+                                : (const void*)&gemm_kernel<FMT, 1, 32, 256>;
+  } else if (bn == 128 && mt == 1) {
+    if (bk == 64) p = (const void*)&gemm_kernel<FMT, 1, 64, 128>;
+    if constexpr (!fmt_small(FMT))
+      if (bk == 32) p = (const void*)&gemm_kernel<FMT, 1, 32, 128>;
   }
-  if (bk != 64) return nullptr;
-  return mt == 2 ? reinterpret_cast<const void*>(&gemm_kernel<FMT, 2, 64>)
-                 : reinterpret_cast<const void*>(&gemm_kernel<FMT, 1, 64>);
+  return p;
 }
 
-static const void* gemm_kernel_ptr(int fmt, int mt, int bk) {
+static const void* gemm_kernel_ptr(int fmt, int mt, int bk, int bn) {
   switch (fmt) {
 #define SPHQ_GEMM_PTR(F) \
   case F:                \
-    return gemm_ptr<F>(mt, bk);
+    return gemm_ptr<F>(mt, bk, bn);
     SPHQ_GEMM_PTR(2)
     SPHQ_GEMM_PTR(3)
     SPHQ_GEMM_PTR(4)
@@ -377,12 +385,12 @@ struct GemmSmem {
   size_t total = 0;
 };
 
-static GemmSmem gemm_smem(const sphq_handle_s* h, int optin, int mt, int bk) {
+static GemmSmem gemm_smem(const sphq_handle_s* h, int optin, int mt, int bk, int bn) {
   GemmSmem L;
   L.cb_bytes = fmt_small(h->fmt) ? (uint32_t)h->K * 8u * 16u : (uint32_t)h->K * 16u;
   for (int S = 4; S >= 2; --S) {
     const size_t off_b = (size_t)S * mt * tile_a_bytes(bk);
-    const size_t off_cb = off_b + (size_t)S * tile_b_bytes(bk);
+    const size_t off_cb = off_b + (size_t)S * tile_b_bytes(bk, bn);
     const size_t off_bar = align_to(off_cb + L.cb_bytes, 16);
     const size_t total = 1024 + off_bar + 16u * S + 16u + 16u;  // alignment slack + barriers + slot
     if (total <= (size_t)optin) {
@@ -397,45 +405,86 @@ static GemmSmem gemm_smem(const sphq_handle_s* h, int optin, int mt, int bk) {
   return L;
 }
 
+struct GemmShape {
+  int mt = 0, bk = 0, bn = 0;
+  GemmSmem L;
+};
+
+// Shape (MT activation tiles, BN weight rows per CTA): the least estimated
+// time = waves of CTAs x time per CTA, the latter relative to the work of one
+// CTA (MT x BN) over its measured efficiency (two tiles of 256 rows: 1, one:
+// 0.64, one of 128 rows: 0.5), unless sphq_set_gemm_shape fixed MT / BN; a
+// candidate needs a ring of two stages next to the codebook, with 64-column
+// stages if they fit, else 32-column ones (W3 with two activation tiles).
+static GemmShape select_gemm_shape(const sphq_handle_s* h, int batch, int optin) {
+  const int sms = h->sm_count > 0 ? h->sm_count : 1;
+  static const int kShapes[3][2] = {{2, 256}, {1, 256}, {1, 128}};
+  static const double kEff[3] = {1.0, 0.64, 0.5};
+  GemmShape best;
+  double best_t = 0;
+  for (int c = 0; c < 3; ++c) {
+    const int m = kShapes[c][0], n = kShapes[c][1];
+    if (h->gemm_mt ? m != h->gemm_mt : (m == 2 && batch <= kGemmBM)) continue;
+    if (h->gemm_bn && n != h->gemm_bn) continue;
+    for (int k : {64, 32}) {
+      if (!gemm_kernel_ptr(h->fmt, m, k, n)) continue;
+      const GemmSmem T = gemm_smem(h, optin, m, k, n);
+      if (T.stages < 2) continue;
+      const long long ctas = (long long)((h->nrt + n / kRowsPerTile - 1) / (n / kRowsPerTile)) *
+                             ((batch + kGemmBM * m - 1) / (kGemmBM * m));
+      const double t = (double)((ctas + sms - 1) / sms) * (m * n) / kEff[c];
+      if (!best.mt || t < best_t - 1e-9) {
+        best.mt = m, best.bk = k, best.bn = n, best.L = T;
+        best_t = t;
+      }
+      break;  // 64-column stages when they fit
+    }
+  }
+  return best;
+}
+
+static sphq_status device_smem_optin(const sphq_handle_s* h, int* optin) {
+  cudaError_t e = cudaDeviceGetAttribute(optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, h->device);
+  if (e != cudaSuccess) return cuda_error(e, "cudaDeviceGetAttribute");
+  return SPHQ_OK;
+}
+
+sphq_status gemm_shape_info(sphq_handle h, int batch, sphq_gemm_info* out) {
+  int optin = 0;
+  sphq_status st = device_smem_optin(h, &optin);
+  if (st != SPHQ_OK) return st;
+  const GemmShape g = select_gemm_shape(h, batch, optin);
+  if (!g.mt) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm: no shape fits this device");
+  out->act_tiles = g.mt;
+  out->weight_rows = g.bn;
+  out->stage_cols = g.bk;
+  out->stages = g.L.stages;
+  out->grid_x = (h->nrt + g.bn / kRowsPerTile - 1) / (g.bn / kRowsPerTile);
+  out->grid_y = (batch + kGemmBM * g.mt - 1) / (kGemmBM * g.mt);
+  out->smem_bytes = (long long)g.L.total;
+  return SPHQ_OK;
+}
+
 sphq_status launch_gemm(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s) {
   EncodeTiledFn enc = encode_fn();
   if (!enc) return set_error(SPHQ_ERR_CUDA, "sphq_gemm: cuTensorMapEncodeTiled unavailable");
   int optin = 0;
-  cudaError_t e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, h->device);
-  if (e != cudaSuccess) return cuda_error(e, "cudaDeviceGetAttribute");
-  // Shape: two activation tiles per decoded weight tile when the batch fills
-  // them and the grid still has a wave's worth of CTAs (estimated time per
-  // CTA: 1.6 with two tiles against 1 with one, times the waves); 64-column
-  // stages unless they leave no room for a ring of two next to the codebook
-  // (W3 with two activation tiles, which takes 32-column stages, three deep).
-  const long long tiles_n = (h->nrt + kGemmTilesN - 1) / kGemmTilesN;
-  const int sms = h->sm_count > 0 ? h->sm_count : 1;
-  auto waves = [&](int m) {
-    const long long ctas = tiles_n * ((batch + kGemmBM * m - 1) / (kGemmBM * m));
-    return (double)((ctas + sms - 1) / sms);
-  };
-  const bool two = batch > kGemmBM && 1.6 * waves(2) < waves(1);
-  static const int kCand2[4][2] = {{2, 64}, {2, 32}, {1, 64}, {1, 32}};
-  static const int kCand1[2][2] = {{1, 64}, {1, 32}};
-  const int (*cand)[2] = two ? kCand2 : kCand1;
-  const int ncand = two ? 4 : 2;
-  int mt = 0, bk = 0;
-  GemmSmem L;
-  for (int c = 0; c < ncand && !mt; ++c) {
-    if (!gemm_kernel_ptr(h->fmt, cand[c][0], cand[c][1])) continue;
-    const GemmSmem T = gemm_smem(h, optin, cand[c][0], cand[c][1]);
-    if (T.stages >= 2) mt = cand[c][0], bk = cand[c][1], L = T;
-  }
-  if (!mt) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm: shared memory too small");
-  const void* kfn = gemm_kernel_ptr(h->fmt, mt, bk);
+  sphq_status st = device_smem_optin(h, &optin);
+  if (st != SPHQ_OK) return st;
+  const GemmShape g = select_gemm_shape(h, batch, optin);
+  if (!g.mt) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm: no shape fits this device");
+  const int mt = g.mt, bk = g.bk, bn = g.bn;
+  const GemmSmem& L = g.L;
+  cudaError_t e;
+  const void* kfn = gemm_kernel_ptr(h->fmt, mt, bk, bn);
   {
     static std::mutex mu;
-    static bool done[16][3][2] = {};
+    static bool done[16][3][2][2] = {};
     std::lock_guard<std::mutex> lock(mu);
-    if (!done[h->fmt][mt][bk == 64]) {
+    if (!done[h->fmt][mt][bk == 64][bn == 256]) {
       e = cudaFuncSetAttribute(kfn, cudaFuncAttributeMaxDynamicSharedMemorySize, optin);
       if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(gemm)");
-      done[h->fmt][mt][bk == 64] = true;
+      done[h->fmt][mt][bk == 64][bn == 256] = true;
     }
   }
   // activations: a batch x cols fp16 tensor, boxes of 128 rows x 64 columns
@@ -464,7 +513,7 @@ sphq_status launch_gemm(sphq_handle h, const void* x, void* y, int batch, cudaSt
   a.off_b = L.off_b;
   a.off_cb = L.off_cb;
   a.off_bar = L.off_bar;
-  const dim3 grid((unsigned)((h->nrt + kGemmTilesN - 1) / kGemmTilesN),
+  const dim3 grid((unsigned)((h->nrt + bn / kRowsPerTile - 1) / (bn / kRowsPerTile)),
                   (unsigned)((batch + kGemmBM * mt - 1) / (kGemmBM * mt)));
   void* args[] = {&a, &tmap};
   e = cudaLaunchKernel(kfn, grid, dim3(kGemmThreads), args, L.total, s);

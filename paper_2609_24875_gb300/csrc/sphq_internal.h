@@ -46,6 +46,8 @@ struct sphq_handle_s {
   void* xstage = nullptr;      // SPHQ_MAX_BATCH x cols fp16 (sphq_gemv_host)
   void* ystage = nullptr;      // SPHQ_MAX_BATCH x rows fp16
   void* zeros = nullptr;       // 256 B of zeros (activations of non-supplying lanes)
+  int gemm_mt = 0;             // sphq_set_gemm_shape: activation tiles (0 = automatic)
+  int gemm_bn = 0;             //   weight rows per CTA tile (0 = automatic)
   bool packed = false;
   sphq::GemvPlan plan[SPHQ_MAX_BATCH + 1];
 };
@@ -61,6 +63,8 @@ sphq_status make_gemv_plans(sphq_handle h);
 sphq_status set_gemv_cluster_size(sphq_handle h, int batch, int csize);
 // Enqueues the GEMV (validated arguments).
 sphq_status launch_gemv(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s);
+// Launch shape sphq_gemm would use for `batch`.
+sphq_status gemm_shape_info(sphq_handle h, int batch, sphq_gemm_info* out);
 // Enqueues the tensor-core product for any batch (validated arguments).
 sphq_status launch_gemm(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s);
 // Enqueues the GEMV with caller-provided split-K scratch: `ws` holds at least

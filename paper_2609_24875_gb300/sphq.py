@@ -38,6 +38,14 @@ class PlanInfo(ctypes.Structure):
                 ("staged_x", ctypes.c_int)]
 
 
+class GemmInfo(ctypes.Structure):
+    """sphq_gemm_info: the prefill GEMM launch shape for one batch size."""
+    _fields_ = [("act_tiles", ctypes.c_int), ("weight_rows", ctypes.c_int),
+                ("stage_cols", ctypes.c_int), ("stages", ctypes.c_int),
+                ("grid_x", ctypes.c_int), ("grid_y", ctypes.c_int),
+                ("smem_bytes", ctypes.c_longlong)]
+
+
 def load() -> ctypes.CDLL:
     """Load libsphq.so (built by __graft_entry__.build()); raises if missing."""
     global _lib
@@ -60,6 +68,10 @@ def load() -> ctypes.CDLL:
         L.sphq_gemm.restype = i32
         L.sphq_check.argtypes = [vp, vp]
         L.sphq_check.restype = i32
+        L.sphq_get_gemm_shape.argtypes = [vp, i32, ctypes.POINTER(GemmInfo)]
+        L.sphq_get_gemm_shape.restype = i32
+        L.sphq_set_gemm_shape.argtypes = [vp, i32, i32]
+        L.sphq_set_gemm_shape.restype = i32
         L.sphq_gemv_host.argtypes = [vp, vp, vp, i32, vp]
         L.sphq_gemv_host.restype = i32
         L.sphq_decode.argtypes = [vp, vp, vp]
@@ -176,6 +188,17 @@ class SphqMatrix:
     def gemm_ptr(self, x_ptr: int, y_ptr: int, batch: int, stream_ptr: int) -> None:
         """Raw-pointer sphq_gemm (no tensor checks)."""
         _check(load().sphq_gemm(self._h, x_ptr, y_ptr, batch, stream_ptr))
+
+    def gemm_shape(self, batch: int) -> dict:
+        """The launch shape sphq_gemm uses for `batch` (sphq_get_gemm_shape)."""
+        info = GemmInfo()
+        _check(load().sphq_get_gemm_shape(self._h, batch, ctypes.byref(info)))
+        return {name: getattr(info, name) for name, _ in GemmInfo._fields_}
+
+    def set_gemm_shape(self, act_tiles: int = 0, weight_rows: int = 0) -> None:
+        """Fix sphq_gemm's activation tiles per CTA (1, 2) and weight rows per
+        CTA (128, 256); 0 = automatic."""
+        _check(load().sphq_set_gemm_shape(self._h, act_tiles, weight_rows))
 
     def check(self, stream=None) -> None:
         """sphq_check: synchronise the stream and raise if a kernel on this

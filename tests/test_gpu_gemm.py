@@ -51,6 +51,43 @@ def test_small_shapes(fmt, rows, cols, batch):
     m.close()
 
 
+# every launch shape (activation tiles, weight rows per CTA) the library has,
+# forced with sphq_set_gemm_shape, on shapes with ragged edges in every dimension
+SHAPES = [(1, 128), (1, 256), (2, 256)]
+
+
+@pytest.mark.parametrize("fmt", FORMATS, ids=FIDS)
+@pytest.mark.parametrize("shape", SHAPES, ids=[f"mt{m}-bn{n}" for m, n in SHAPES])
+def test_every_launch_shape(fmt, shape):
+    bits, v, K = fmt
+    rows, cols, batch = 1000, 1024, 300
+    codes, x = inp.random_codes(bits, rows, cols, seed=55 + bits + v + shape[1], B=batch,
+                                radius_bits=v, K=K)
+    m = G.make_matrix(codes)
+    m.set_gemm_shape(*shape)
+    info = m.gemm_shape(batch)
+    assert (info["act_tiles"], info["weight_rows"]) == shape
+    assert info["stages"] >= 2 and info["stage_cols"] in (32, 64)
+    assert info["grid_x"] == -(-((rows + 15) // 16) // (shape[1] // 16))
+    assert info["grid_y"] == -(-batch // (128 * shape[0]))
+    check_gemm(m, codes, x)
+    m.check()
+    m.set_gemm_shape(0, 0)
+    m.close()
+
+
+def test_shape_choice_and_invalid_shapes():
+    codes, _ = inp.random_codes(2, 8192, 1024, seed=6)
+    m = G.make_matrix(codes)
+    assert m.gemm_shape(4096)["act_tiles"] == 2          # many tiles: two per CTA
+    small = m.gemm_shape(64)
+    assert small["act_tiles"] == 1
+    for bad in ((3, 0), (2, 128), (0, 64), (-1, 0)):
+        with pytest.raises(SphqError):
+            m.set_gemm_shape(*bad)
+    m.close()
+
+
 def test_matches_gemv_within_tolerance_for_small_batches():
     codes, x = inp.random_codes(2, 3584, 3584, seed=41, B=8)
     m = G.make_matrix(codes)
