@@ -19,18 +19,17 @@
 // ring of three stages with two activation tiles.  Per step:
 //  * one TMA warp loads the 128 (256) x BK activation tile (A operand,
 //    K-major, swizzled; rows past the batch read zeros);
-//  * eight decode warps each rebuild one or two 16 x BK slices of W_hat (half
-//    or a quarter of a unit of each of their row tiles) into the B operand tile in the same
-//    swizzled K-major layout, fence them to the async proxy and arrive on the stage's
+//  * one decode warp per 16-row tile (16 or 8 warps) rebuilds its 16 x BK
+//    slice of W_hat (half or a quarter of a unit) into the B operand tile in
+//    the same swizzled K-major layout, fence them to the async proxy and arrive on the stage's
 //    mbarrier;
 //  * one MMA warp issues BK / 16 (times the activation tiles) 128 x BN x 16
 //    tcgen05.mma (fp16 x fp16 -> fp32) when both halves of the stage are in, and commits their completion
 //    to the stage's "empty" mbarrier, which releases the buffers.
 // Stages rotate through a ring of buffers (two to four, as shared memory
 // allows next to the codebook).  After the last step the decode warps read
-// the accumulators from tensor memory (warp w: lanes 32 (w % 4).. of
-// accumulator w / 4, or of column half w / 4 with one accumulator), round to
-// fp16 and store Y.
+// the accumulators from tensor memory (warp w: lanes 32 (w % 4).., the warps
+// of one lane quarter splitting the columns), round to fp16 and store Y.
 //
 // Every mbarrier wait gives up after about two seconds and records bit 1 in
 // the handle's device error word, so a fault cannot hang the GPU.
@@ -46,10 +45,9 @@
 namespace sphq {
 
 constexpr int kGemmBM = 128;                    // activation rows per tile (MMA M)
-constexpr int kGemmDecodeWarps = 8;             // two row tiles each
-constexpr int kGemmThreads = (kGemmDecodeWarps + 2) * 32;
-constexpr int kGemmMmaWarp = kGemmDecodeWarps;
-constexpr int kGemmTmaWarp = kGemmDecodeWarps + 1;
+// One decode warp per 16-row tile of the weight tile (16 or 8), then the MMA
+// warp and the TMA warp.
+constexpr int gemm_threads(int bn) { return (bn / kRowsPerTile + 2) * 32; }
 // operand tile bytes for a stage of BK columns
 constexpr uint32_t tile_a_bytes(int bk) { return (uint32_t)kGemmBM * bk * 2; }  // per 128 rows
 constexpr uint32_t tile_b_bytes(int bk, int bn) { return (uint32_t)bn * bk * 2; }
@@ -129,11 +127,11 @@ __device__ __forceinline__ void decode_word(const Unit<FMT>& u, const UnitConst<
 // of 256 tensor-memory columns); BK columns per stage: 64 (128-byte swizzle)
 // or 32 (64-byte swizzle, half the ring memory, for the 128 KiB W3 codebook).
 template <int FMT, int MT, int BK, int BN>
-__global__ void __launch_bounds__(kGemmThreads, 1)
+__global__ void __launch_bounds__(gemm_threads(BN), 1)
     gemm_kernel(const GemmArgs a, const __grid_constant__ CUtensorMap tmap) {
-  constexpr int kTilesN = BN / kRowsPerTile;          // row tiles per weight tile
-  constexpr int kTPW = kTilesN / kGemmDecodeWarps;    // row tiles per decode warp (2 or 1)
-  static_assert(kTPW * kGemmDecodeWarps == kTilesN && (kTPW == 1 || kTPW == 2), "tile split");
+  constexpr int kTilesN = BN / kRowsPerTile;  // row tiles per weight tile
+  constexpr int kDecodeWarps = kTilesN;       // one row tile each
+  constexpr int kMmaWarp = kDecodeWarps, kTmaWarp = kDecodeWarps + 1;
   constexpr uint32_t kTileA = tile_a_bytes(BK), kTileB = tile_b_bytes(BK, BN);
   constexpr uint32_t kStageA = MT * kTileA;
   constexpr uint32_t kCols = MT * BN;  // tensor-memory columns
@@ -156,7 +154,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
-      mbar_init(full0 + 8u * s, kGemmDecodeWarps + 1);
+      mbar_init(full0 + 8u * s, kDecodeWarps + 1);
       mbar_init(empty0 + 8u * s, 1);
     }
     mbar_init(acc_bar, 1);
@@ -166,7 +164,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     for (uint32_t o = 0; o < a.cb_bytes; o += 32768u)
       bulk_g2s(sbase + a.off_cb + o, a.cbimage + o, min(32768u, a.cb_bytes - o), cb_bar);
   }
-  if (warp == kGemmMmaWarp) {
+  if (warp == kMmaWarp) {
     umma::tmem_alloc(smem_u32(tslot), kCols);
     umma::tmem_relinquish();
   }
@@ -175,7 +173,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   umma::fence_after_sync();
   const uint32_t taddr = *tslot;
 
-  if (warp == kGemmTmaWarp) {
+  if (warp == kTmaWarp) {
     if (lane == 0) {
       umma::prefetch_tmap(&tmap);
       for (int i = 0, s = 0, r = 0; i < nk; ++i) {
@@ -186,7 +184,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       }
     }
     __syncwarp();
-  } else if (warp == kGemmMmaWarp) {
+  } else if (warp == kMmaWarp) {
     if (lane == 0) {
       constexpr uint32_t idesc = umma::idesc_f16_f32(kGemmBM, BN);
       for (int i = 0, s = 0, r = 0; i < nk; ++i) {
@@ -216,49 +214,41 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     SmemCodebook cb;
     cb.base = smem + a.off_cb;
     cb.copyoff = fmt_small(FMT) ? (uint32_t)(lane & 7) * 16u : 0u;
-    const int j0 = kTPW * warp;
-    const bool ok0 = rt0 + j0 < a.nrt, ok1 = kTPW == 2 && rt0 + j0 + 1 < a.nrt;
-    const uint8_t* ub0 = a.units + (size_t)(rt0 + j0) * UB;  // group 0; + g * nrt * UB
+    const int jt = warp;  // this warp's row tile within the weight tile
+    const bool ok = rt0 + jt < a.nrt;
+    const uint8_t* ub0 = a.units + (size_t)(rt0 + jt) * UB;  // group 0; + g * nrt * UB
     const size_t gstride = (size_t)a.nrt * UB;
-    Unit<FMT> cur[2] = {}, nxt[2] = {};
-    if (ok0) nxt[0] = load_unit<FMT>(ub0, lane);
-    if (ok1) nxt[1] = load_unit<FMT>(ub0 + UB, lane);
+    Unit<FMT> cur = {}, nxt = {};
+    if (ok) nxt = load_unit<FMT>(ub0, lane);
     if (!mbar_wait(cb_bar, 0) && lane == 0) atomicOr(a.flag, 2);
     for (int i = 0, s = 0, r = 0; i < nk; ++i) {
       const int g = i / kStepsPerGroup;
       const int step = i % kStepsPerGroup;
       if (step == 0) {
-        cur[0] = nxt[0];
-        cur[1] = nxt[1];
-        if (g + 1 < ng) {
-          const uint8_t* nb = ub0 + (size_t)(g + 1) * gstride;
-          if (ok0) nxt[0] = load_unit<FMT>(nb, lane);
-          if (ok1) nxt[1] = load_unit<FMT>(nb + UB, lane);
-        }
+        cur = nxt;
+        if (ok && g + 1 < ng) nxt = load_unit<FMT>(ub0 + (size_t)(g + 1) * gstride, lane);
       }
       // one lane polls the stage's release (the MMAs that read it are
       // complete); the warp's stores follow it through __syncwarp
       if (r > 0 && lane == 0 && !mbar_wait(empty0 + 8u * s, (r - 1) & 1)) atomicOr(a.flag, 2);
       __syncwarp();
       const uint32_t bt = sbase + a.off_b + s * kTileB;
-#pragma unroll
-      for (int j = 0; j < 2; ++j) {
-        if (!(j ? ok1 : ok0)) continue;
-        const UnitConst<FMT> kc = unit_const<FMT>(cur[j], q);
+      if (ok) {
+        const UnitConst<FMT> kc = unit_const<FMT>(cur, q);
         if constexpr (BK == 64) {
           if (step)
-            decode_half<FMT, 2>(cur[j], kc, q, gid, j0 + j, cb, bt);
+            decode_half<FMT, 2>(cur, kc, q, gid, jt, cb, bt);
           else
-            decode_half<FMT, 0>(cur[j], kc, q, gid, j0 + j, cb, bt);
+            decode_half<FMT, 0>(cur, kc, q, gid, jt, cb, bt);
         } else {
           if (step == 0)
-            decode_word<FMT, 0>(cur[j], kc, q, gid, j0 + j, cb, bt);
+            decode_word<FMT, 0>(cur, kc, q, gid, jt, cb, bt);
           else if (step == 1)
-            decode_word<FMT, 1>(cur[j], kc, q, gid, j0 + j, cb, bt);
+            decode_word<FMT, 1>(cur, kc, q, gid, jt, cb, bt);
           else if (step == 2)
-            decode_word<FMT, 2>(cur[j], kc, q, gid, j0 + j, cb, bt);
+            decode_word<FMT, 2>(cur, kc, q, gid, jt, cb, bt);
           else
-            decode_word<FMT, 3>(cur[j], kc, q, gid, j0 + j, cb, bt);
+            decode_word<FMT, 3>(cur, kc, q, gid, jt, cb, bt);
         }
       }
       umma::fence_proxy_async_smem();
@@ -270,15 +260,19 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     // ---- epilogue: accumulators -> fp16 Y ----
     if (!mbar_wait(acc_bar, 0) && lane == 0) atomicOr(a.flag, 2);
     umma::fence_after_sync();
-    // warp w reads lanes 32 (w % 4).. of accumulator w / 4 (MT = 2), or of
-    // the single accumulator's column half w / 4 (MT = 1)
-    const int quarter = warp & 3, hi = warp >> 2;
-    const int token = tok0 + (MT == 2 ? kGemmBM * hi : 0) + 32 * quarter + lane;
-    constexpr int kChunks = MT == 2 ? BN / 32 : BN / 64;
+    // warp w reads lanes 32 (w % 4).. (its quarter of tensor memory); the
+    // kDecodeWarps / 4 warps of a quarter split the MT x BN columns evenly
+    constexpr int kParts = kDecodeWarps / 4;
+    constexpr int kColsPerWarp = MT * BN / kParts;
+    static_assert(kColsPerWarp <= BN && kColsPerWarp % 32 == 0, "epilogue split");
+    const int quarter = warp & 3, part = warp >> 2;
+    const int start = part * kColsPerWarp;
+    const int acc = start / BN;
+    const int token = tok0 + kGemmBM * acc + 32 * quarter + lane;
 #pragma unroll 1
-    for (int cc = 0; cc < kChunks; ++cc) {
-      const int col = (MT == 2 ? 0 : hi * (BN / 2)) + 32 * cc;  // within the accumulator
-      const uint32_t tcol = (uint32_t)((MT == 2 ? hi * BN : 0) + col);
+    for (int cc = 0; cc < kColsPerWarp / 32; ++cc) {
+      const int col = start % BN + 32 * cc;  // within the accumulator
+      const uint32_t tcol = (uint32_t)(acc * BN + col);
       uint32_t v[32];
       umma::ld_32x32b_x32(taddr + ((uint32_t)(32 * quarter) << 16) + tcol, v);
       umma::wait_ld();
@@ -307,7 +301,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   }
   umma::fence_before_sync();
   __syncthreads();
-  if (warp == kGemmMmaWarp) {
+  if (warp == kMmaWarp) {
     umma::fence_after_sync();
     umma::tmem_dealloc(taddr, kCols);
   }
@@ -516,7 +510,7 @@ sphq_status launch_gemm(sphq_handle h, const void* x, void* y, int batch, cudaSt
   const dim3 grid((unsigned)((h->nrt + bn / kRowsPerTile - 1) / (bn / kRowsPerTile)),
                   (unsigned)((batch + kGemmBM * mt - 1) / (kGemmBM * mt)));
   void* args[] = {&a, &tmap};
-  e = cudaLaunchKernel(kfn, grid, dim3(kGemmThreads), args, L.total, s);
+  e = cudaLaunchKernel(kfn, grid, dim3(gemm_threads(bn)), args, L.total, s);
   if (e != cudaSuccess) return cuda_error(e, "gemm launch");
   return SPHQ_OK;
 }
