@@ -84,6 +84,9 @@ def lib() -> ctypes.CDLL:
             L.sphqo_pack_w2_words.restype = i32
             L.sphqo_unpack_w2_words.argtypes = [i32, i32, u16, u32, u8, u16, u8]
             L.sphqo_unpack_w2_words.restype = i32
+            L.sphqo_encode_f32.argtypes = [i32, i32, i32, i32, u16, ctypes.POINTER(ctypes.c_float),
+                                           u8, u16, u8, u16, u16]
+            L.sphqo_encode_f32.restype = i32
             L.sphqo_set_threads.argtypes = [i32]
             L.sphqo_get_threads.restype = i32
             L.sphqo_max_threads.restype = i32
@@ -327,6 +330,31 @@ def encode(w, codebook, V: int = 4, chunk: int = 1 << 14):
     q = np.clip(qf, 0, levels).astype(np.uint8).reshape(rows, cols // VEC)
     return dict(sign=sign, idx=z.astype(np.uint16), rcode=q, scale=scale16,
                 offset=offset16, r_tilde=r_tilde)
+
+
+def encode_fp32(w, codebook, V: int = 4):
+    """The encoder of `encode` (Eqs. (3), (5), (6), (7)) with every decision in
+    IEEE single precision and a fixed operation order (fused multiply-adds in
+    coordinate order, correctly rounded sqrt and division; see the C source),
+    so that a single-precision implementation elsewhere can match it bit for
+    bit.  w: float32 (rows, cols).  Returns dict(sign, idx, rcode, scale, offset)."""
+    w = np.ascontiguousarray(np.asarray(w, np.float32))
+    rows, cols = w.shape
+    cb = _c(codebook, np.uint16)
+    K = cb.shape[0]
+    nv = cols // VEC
+    sign = np.empty((rows, nv), np.uint8)
+    idx = np.empty((rows, nv), np.uint16)
+    rcode = np.empty((rows, nv), np.uint8)
+    scale = np.empty((rows, cols // GROUP), np.uint16)
+    offset = np.empty((rows, cols // GROUP), np.uint16)
+    rc = lib().sphqo_encode_f32(rows, cols, K, V, _p(cb, ctypes.c_uint16),
+                                _p(w, ctypes.c_float), _p(sign, ctypes.c_uint8),
+                                _p(idx, ctypes.c_uint16), _p(rcode, ctypes.c_uint8),
+                                _p(scale, ctypes.c_uint16), _p(offset, ctypes.c_uint16))
+    if rc != 0:
+        raise ValueError("oracle encode_fp32: bad arguments")
+    return dict(sign=sign, idx=idx, rcode=rcode, scale=scale, offset=offset)
 
 
 # ---------------------------------------------------------------------------

@@ -315,3 +315,93 @@ int sphqo_unpack_w2_words(int rows, int cols, const uint16_t* base, const uint32
   }
   return 0;
 }
+
+/* ------------------------------------------------------------------------- */
+/* Eqs. (3), (5), (6), (7) in IEEE binary32: the encoder                      */
+/* ------------------------------------------------------------------------- */
+
+/*
+ * The encoder of §3.1 (Eq. (3) decomposition, Eq. (5) nearest direction,
+ * Eq. (6) radius projection, Eq. (7) group quantisation) with every decision
+ * taken in single precision, in this order (the float64 encoder in
+ * oracle/__init__.py is the same algorithm in double precision):
+ *   p_j = |w_j|, sign bit j = (w_j < 0)
+ *   r = sqrt(fma(p_7, p_7, ... fma(p_0, p_0, 0)))     (correctly rounded sqrt)
+ *   d_j = p_j / max(r, 1e-12)                          (correctly rounded division)
+ *   score_k = fma(d_7, c_k7, ... fma(d_0, c_k0, 0)); z = argmax, ties -> lowest k
+ *   r~ = fma(p_7, c_z7, ... fma(p_0, c_z0, 0))
+ *   per group of 16 vectors: Delta = (max r~ - min r~) / (2^V - 1),
+ *   Delta16 = RN16(Delta), m16 = RN16(min r~),
+ *   q = 0 if Delta16 = 0, else clip(floor((r~ - m16) / Delta16 + 0.5), 0, 2^V - 1)
+ * fma is the fused multiply-add (one rounding).  `codebook` is K x 8 binary16.
+ */
+static float sphqo_half_to_float(uint16_t h) { return (float)sphqo_half_to_double(h); }
+
+int sphqo_encode_f32(int rows, int cols, int K, int V, const uint16_t* codebook, const float* w,
+                     uint8_t* sign, uint16_t* idx, uint8_t* rcode, uint16_t* scale,
+                     uint16_t* offset) {
+  if (rows < 0 || cols % (SPHQO_VEC * SPHQO_GROUP) != 0 || K < 1 || V < 1 || V > 8) return -1;
+  const int nv = cols / SPHQO_VEC;
+  const int ng = nv / SPHQO_GROUP;
+  const int qmax = (1 << V) - 1;
+  float* cf = (float*)malloc(sizeof(float) * (size_t)K * SPHQO_VEC);
+  if (!cf) return -2;
+  for (int64_t i = 0; i < (int64_t)K * SPHQO_VEC; ++i) cf[i] = sphqo_half_to_float(codebook[i]);
+#pragma omp parallel for schedule(dynamic, 4) num_threads(g_threads)
+  for (int row = 0; row < rows; ++row) {
+    for (int g = 0; g < ng; ++g) {
+      float rt[SPHQO_GROUP];
+      for (int v = 0; v < SPHQO_GROUP; ++v) {
+        const int64_t t = (int64_t)row * nv + (int64_t)g * SPHQO_GROUP + v;
+        const float* x = w + t * SPHQO_VEC;
+        float p[SPHQO_VEC], d[SPHQO_VEC];
+        uint8_t s = 0;
+        float acc = 0.0f;
+        for (int j = 0; j < SPHQO_VEC; ++j) {
+          p[j] = fabsf(x[j]);
+          if (x[j] < 0.0f) s |= (uint8_t)(1u << j);
+          acc = fmaf(p[j], p[j], acc);
+        }
+        const float r = sqrtf(acc);
+        const float den = r > 1e-12f ? r : 1e-12f;
+        for (int j = 0; j < SPHQO_VEC; ++j) d[j] = p[j] / den;
+        int best = 0;
+        float bs = 0.0f;
+        for (int k = 0; k < K; ++k) {
+          float sc = 0.0f;
+          for (int j = 0; j < SPHQO_VEC; ++j) sc = fmaf(d[j], cf[(int64_t)k * SPHQO_VEC + j], sc);
+          if (k == 0 || sc > bs) {
+            bs = sc;
+            best = k;
+          }
+        }
+        float rr = 0.0f;
+        for (int j = 0; j < SPHQO_VEC; ++j) rr = fmaf(p[j], cf[(int64_t)best * SPHQO_VEC + j], rr);
+        rt[v] = rr;
+        sign[t] = s;
+        idx[t] = (uint16_t)best;
+      }
+      float mn = rt[0], mx = rt[0];
+      for (int v = 1; v < SPHQO_GROUP; ++v) {
+        mn = fminf(mn, rt[v]);
+        mx = fmaxf(mx, rt[v]);
+      }
+      const float delta = (mx - mn) / (float)qmax;
+      const uint16_t d16 = sphqo_round_half((double)delta);
+      const uint16_t m16 = sphqo_round_half((double)mn);
+      const float df = sphqo_half_to_float(d16), mf = sphqo_half_to_float(m16);
+      scale[(int64_t)row * ng + g] = d16;
+      offset[(int64_t)row * ng + g] = m16;
+      for (int v = 0; v < SPHQO_GROUP; ++v) {
+        int q = 0;
+        if (df != 0.0f) {
+          const float u = floorf((rt[v] - mf) / df + 0.5f);
+          q = u < 0.0f ? 0 : (u > (float)qmax ? qmax : (int)u);
+        }
+        rcode[(int64_t)row * nv + (int64_t)g * SPHQO_GROUP + v] = (uint8_t)q;
+      }
+    }
+  }
+  free(cf);
+  return 0;
+}
