@@ -128,6 +128,26 @@ sphq_status sphq_pack(sphq_handle h, const uint8_t* sign, const uint16_t* idx,
                       const uint8_t* rcode, sphq_stream stream);
 
 /*
+ * sphq_encode -- quantise a weight matrix with the handle's codebook (§3.1:
+ * Eq. (3) signs / radius / direction, Eq. (5) nearest codebook direction,
+ * Eq. (6) radius projection, Eq. (7) per-group radius codes) and pack it.
+ *
+ *   w       rows x cols fp32, device pointer, 16-byte aligned.
+ *   sign    rows x (cols/8) uint8 out, idx uint16 out (2-byte aligned), rcode
+ *           uint8 out: the canonical codes sphq_pack takes (device pointers).
+ *   scale, offset  rows x (cols/128) fp16 out (Delta16, m16), or NULL.
+ *
+ * Every decision is taken in IEEE single precision in a fixed order (see
+ * sphq_encode.cu): the codes equal those of a single-precision CPU encoder
+ * bit for bit.  The handle's group parameters are replaced by the encoder's
+ * and the codes are packed (as sphq_pack), so the handle is ready for
+ * sphq_gemv / sphq_gemm on return.  Synchronous; allocates a temporary
+ * rows x cols/8 fp32 buffer.  Errors as sphq_pack, plus SPHQ_ERR_TIMEOUT.
+ */
+sphq_status sphq_encode(sphq_handle h, const float* w, uint8_t* sign, uint16_t* idx,
+                        uint8_t* rcode, void* scale, void* offset, sphq_stream stream);
+
+/*
  * sphq_gemv -- y = W_hat x for a batch of activation rows (§3.4, App. D).
  *
  *   x      batch x cols fp16, device pointer, 16-byte aligned.

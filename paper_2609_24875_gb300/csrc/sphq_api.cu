@@ -360,15 +360,9 @@ sphq_status sphq_create_v(int rows, int cols, int bits, int radius_bits, int K,
   return SPHQ_OK;
 }
 
-sphq_status sphq_pack(sphq_handle h, const uint8_t* sign, const uint16_t* idx,
-                      const uint8_t* rcode, sphq_stream stream) {
-  g_last_error.clear();
-  if (!h) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_pack: NULL handle");
-  if (!sign || !idx || !rcode)
-    return set_error(SPHQ_ERR_INVALID_ARG, "sphq_pack: NULL code pointer");
-  if (reinterpret_cast<uintptr_t>(idx) % 2)
-    return set_error(SPHQ_ERR_INVALID_ARG, "sphq_pack: idx must be 2-byte aligned");
-  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+// Validates and packs canonical device codes into the handle (synchronous).
+static sphq_status pack_codes(sphq_handle h, const uint8_t* sign, const uint16_t* idx,
+                              const uint8_t* rcode, cudaStream_t s) {
   h->packed = false;
   const uint16_t* scale = reinterpret_cast<const uint16_t*>(h->params);
   const uint16_t* offset = scale + (size_t)h->rows * h->ng;
@@ -398,6 +392,55 @@ sphq_status sphq_pack(sphq_handle h, const uint8_t* sign, const uint16_t* idx,
                      "sphq_pack: a direction index >= K or a radius code >= 2^radius_bits");
   h->packed = true;
   return SPHQ_OK;
+}
+
+sphq_status sphq_pack(sphq_handle h, const uint8_t* sign, const uint16_t* idx,
+                      const uint8_t* rcode, sphq_stream stream) {
+  g_last_error.clear();
+  if (!h) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_pack: NULL handle");
+  if (!sign || !idx || !rcode)
+    return set_error(SPHQ_ERR_INVALID_ARG, "sphq_pack: NULL code pointer");
+  if (reinterpret_cast<uintptr_t>(idx) % 2)
+    return set_error(SPHQ_ERR_INVALID_ARG, "sphq_pack: idx must be 2-byte aligned");
+  return pack_codes(h, sign, idx, rcode, reinterpret_cast<cudaStream_t>(stream));
+}
+
+sphq_status sphq_encode(sphq_handle h, const float* w, uint8_t* sign, uint16_t* idx,
+                        uint8_t* rcode, void* scale, void* offset, sphq_stream stream) {
+  g_last_error.clear();
+  if (!h) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_encode: NULL handle");
+  if (!w || reinterpret_cast<uintptr_t>(w) % 16)
+    return set_error(SPHQ_ERR_INVALID_ARG, "sphq_encode: w must be a 16-byte aligned pointer");
+  if (!sign || !idx || !rcode || reinterpret_cast<uintptr_t>(idx) % 2)
+    return set_error(SPHQ_ERR_INVALID_ARG, "sphq_encode: NULL or misaligned code pointer");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const size_t nvec = (size_t)h->rows * (h->cols / kVec);
+  float* rtilde = nullptr;
+  SPHQ_CUDA(cudaMalloc(&rtilde, nvec * sizeof(float)), "cudaMalloc(radii)");
+  sphq_status st = launch_encode(h, w, sign, idx, rcode, rtilde, s);
+  if (st == SPHQ_OK) {
+    const size_t np = (size_t)h->rows * h->ng;
+    const uint16_t* p16 = reinterpret_cast<const uint16_t*>(h->params);
+    cudaError_t e = cudaSuccess;
+    if (scale) e = cudaMemcpyAsync(scale, p16, np * 2, cudaMemcpyDefault, s);
+    if (e == cudaSuccess && offset) e = cudaMemcpyAsync(offset, p16 + np, np * 2, cudaMemcpyDefault, s);
+    if (e != cudaSuccess) st = cuda_error(e, "copy group parameters");
+  }
+  if (st == SPHQ_OK) st = pack_codes(h, sign, idx, rcode, s);  // synchronises s
+  cudaError_t e = cudaStreamSynchronize(s);
+  cudaFree(rtilde);
+  if (st == SPHQ_OK && e != cudaSuccess) st = cuda_error(e, "sphq_encode");
+  if (st == SPHQ_OK) {
+    int word = 0;
+    e = cudaMemcpy(&word, h->flag + 1, sizeof(int), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_error(e, "read error word");
+    if (word) {
+      cudaMemset(h->flag + 1, 0, sizeof(int));
+      h->packed = false;
+      return set_error(SPHQ_ERR_TIMEOUT, "sphq_encode: a kernel gave up an on-chip wait");
+    }
+  }
+  return st;
 }
 
 sphq_status sphq_decode(sphq_handle h, void* w, sphq_stream stream) {

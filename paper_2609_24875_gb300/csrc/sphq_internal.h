@@ -63,6 +63,10 @@ sphq_status make_gemv_plans(sphq_handle h);
 sphq_status set_gemv_cluster_size(sphq_handle h, int batch, int csize);
 // Enqueues the GEMV (validated arguments).
 sphq_status launch_gemv(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s);
+// Enqueues the encoder: codes and per-vector radii, then the group
+// parameters into the handle's parameter planes.
+sphq_status launch_encode(sphq_handle h, const float* w, uint8_t* sign, uint16_t* idx,
+                          uint8_t* rcode, float* rtilde, cudaStream_t s);
 // Launch shape sphq_gemm would use for `batch`.
 sphq_status gemm_shape_info(sphq_handle h, int batch, sphq_gemm_info* out);
 // Enqueues the tensor-core product for any batch (validated arguments).

@@ -68,6 +68,8 @@ def load() -> ctypes.CDLL:
         L.sphq_gemm.restype = i32
         L.sphq_check.argtypes = [vp, vp]
         L.sphq_check.restype = i32
+        L.sphq_encode.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp]
+        L.sphq_encode.restype = i32
         L.sphq_get_gemm_shape.argtypes = [vp, i32, ctypes.POINTER(GemmInfo)]
         L.sphq_get_gemm_shape.restype = i32
         L.sphq_set_gemm_shape.argtypes = [vp, i32, i32]
@@ -169,6 +171,27 @@ class SphqMatrix:
             y = torch.empty((B, self.rows), dtype=torch.float16, device=x.device)
         _check(load().sphq_gemv(self._h, x.data_ptr(), y.data_ptr(), B, _stream_ptr(stream)))
         return y
+
+    def encode(self, w, stream=None):
+        """sphq_encode: quantise w ((rows, cols) float32 CUDA tensor) with this
+        matrix's codebook and pack it.  Returns the canonical codes and group
+        parameters as CUDA tensors: sign, idx, rcode (rows, cols/8) and scale,
+        offset (rows, cols/128, fp16 bits as int16)."""
+        import torch
+        if (tuple(w.shape) != (self.rows, self.cols) or w.dtype != torch.float32
+                or not w.is_cuda or not w.is_contiguous()):
+            raise ValueError("w must be a contiguous (rows, cols) float32 CUDA tensor")
+        nv, ng = self.cols // 8, self.cols // 128
+        dev = w.device
+        sign = torch.empty((self.rows, nv), dtype=torch.uint8, device=dev)
+        idx = torch.empty((self.rows, nv), dtype=torch.int16, device=dev)
+        rcode = torch.empty((self.rows, nv), dtype=torch.uint8, device=dev)
+        scale = torch.empty((self.rows, ng), dtype=torch.int16, device=dev)
+        offset = torch.empty((self.rows, ng), dtype=torch.int16, device=dev)
+        _check(load().sphq_encode(self._h, w.data_ptr(), sign.data_ptr(), idx.data_ptr(),
+                                  rcode.data_ptr(), scale.data_ptr(), offset.data_ptr(),
+                                  _stream_ptr(stream)))
+        return sign, idx, rcode, scale, offset
 
     def gemm(self, x, y=None, stream=None):
         """Y = X W_hat^T on the tensor cores for any batch (prefill).
