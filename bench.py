@@ -584,6 +584,72 @@ def run_gemm_case(spec: str, launches: int):
     print(f"gemm case W{bits} V={vbits} K={K} {rows}x{cols} batch {batch}: {launches} launches done")
 
 
+def run_encode_case(spec: str, launches: int):
+    """Profiling driver of the encoder: `bits:rows:cols` (bits token as for
+    --case) -> `launches` sphq_encode calls on N(0, 0.02^2) weights, no timing."""
+    import torch
+
+    head, *rest = spec.split(":")
+    bits, vbits, K = parse_split(head)
+    rows, cols = (int(v) for v in rest)
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    from paper_2609_24875_gb300 import SphqMatrix
+    cb = inp.make_codebook(np.random.Generator(np.random.PCG64(1)), K)
+    ones = inp.to_f16_bits(np.ones((rows, cols // 128)))
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int16))).to(dev)
+    m = SphqMatrix(rows, cols, bits, t(cb), t(ones), t(ones), radius_bits=vbits, K=K)
+    w = torch.from_numpy(inp.gaussian_weights(rows, cols, seed=1).astype(np.float32)).to(dev)
+    for _ in range(launches):
+        m.encode(w)
+    torch.cuda.synchronize()
+    print(f"encode case W{bits} V={vbits} K={K} {rows}x{cols}: {launches} calls done")
+
+
+def encode_report():
+    """GPU encoder (sphq_encode) throughput on N(0, 0.02^2) weights: ms per
+    matrix (min of 3 calls after one warm-up, host clock around a synchronous
+    call), 8-D vectors and coarse scores per second, and the tensor-core share
+    (two passes of one 128 x 256 x 16 MMA per 256 entries); the single-
+    precision CPU oracle encoder on a 64-row sample for comparison."""
+    import torch
+
+    import oracle
+    from paper_2609_24875_gb300 import SphqMatrix
+    dev = torch.device("cuda", 0)
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int16))).to(dev)
+    out = {}
+    for name, (bits, v, K) in (("W2", (2, 4, 64)), ("8/8/2", (2, 2, 256)), ("W3", (3, 4, 8192))):
+        cb = inp.make_codebook(np.random.Generator(np.random.PCG64(1)), K)
+        for n in (4096, 8192):
+            ones = inp.to_f16_bits(np.ones((n, n // 128)))
+            m = SphqMatrix(n, n, bits, t(cb), t(ones), t(ones), radius_bits=v, K=K)
+            w = (torch.randn(n, n, device=dev) * 0.02).float()
+            m.encode(w)
+            torch.cuda.synchronize()
+            ts = []
+            for _ in range(3):
+                t0 = time.perf_counter()
+                m.encode(w)
+                torch.cuda.synchronize()
+                ts.append(time.perf_counter() - t0)
+            ms = min(ts) * 1e3
+            nv = n * n / 8
+            out[f"{name} {n}x{n}"] = {"ms": round(ms, 3), "Gvec/s": round(nv / ms / 1e6, 3),
+                                      "Tscores/s": round(nv * K / ms / 1e9, 3)}
+            m.close()
+            del w
+            torch.cuda.empty_cache()
+        wc = inp.gaussian_weights(64, 4096, seed=2).astype(np.float32)
+        oracle.set_threads(oracle.max_threads())
+        t0 = time.perf_counter()
+        oracle.encode_fp32(wc, cb, v)
+        cpu_s = time.perf_counter() - t0
+        out[f"{name} cpu_oracle_fp32"] = {"Gvec/s": round(64 * 512 / cpu_s / 1e9, 6),
+                                          "threads": oracle.max_threads()}
+    return out
+
+
 def gemm_report(hbm_peak):
     """Prefill GEMM (sphq_gemm) against the tensor-core roofline: TFLOP/s =
     2 * batch * rows * cols / time (median of 10 timed calls after warm-up,
@@ -759,6 +825,7 @@ def run_report(args):
                                                                1, vbits=v, K=1 << d)
                                for d, v in ((6, 2), (6, 3), (7, 2), (7, 3), (8, 2), (6, 4))}
     rep["prefill_gemm"] = gemm_report(hbm_peak)
+    rep["encode"] = encode_report()
     # CPU oracle on the 1024^2 matrix: single thread and all cores
     import oracle
     codes, x = inp.random_codes(2, 1024, 1024, seed=inp.seed_for(0, 0))
@@ -791,6 +858,8 @@ def main():
     ap.add_argument("--launches", type=int, default=8, help="--case: GEMV launches")
     ap.add_argument("--gemm-case", default="",
                     help="prefill GEMM profiling driver: bits:rows:cols:batch, no timing")
+    ap.add_argument("--encode-case", default="",
+                    help="encoder profiling driver: bits:rows:cols, no timing")
     ap.add_argument("--report", action="store_true",
                     help="supplementary per-configuration table (one JSON object)")
     args = ap.parse_args()
@@ -799,6 +868,9 @@ def main():
         return
     if args.gemm_case:
         run_gemm_case(args.gemm_case, args.launches)
+        return
+    if args.encode_case:
+        run_encode_case(args.encode_case, args.launches)
         return
     if args.report:
         run_report(args)

@@ -19,10 +19,11 @@
 //     operand reads each entry twice (the K-major no-swizzle layout with a
 //     zero leading-dimension offset), so no [c | c] copy is needed.  The
 //     coarse score is within 3e-6 of the single-precision score.
-//  2. exact choice: each thread keeps the entries whose coarse score is within
-//     kDelta (1e-5) of its running maximum, in increasing k; after the scan it
-//     re-scores them with the single-precision fused multiply-add chain and
-//     takes the largest, lowest k on ties.  The single-precision argmax is
+//  2. exact choice: a first pass over the coarse scores takes their maximum,
+//     a second (the MMAs repeated) keeps, in increasing k, the entries within
+//     kDelta (1e-5, relative above 1) of it; they are re-scored with the
+//     single-precision fused multiply-add chain and the largest is taken,
+//     lowest k on ties.  The single-precision argmax is
 //     always among them (its coarse score is within 2 x 3e-6 of the coarse
 //     maximum).  If more than kCand entries qualify (degenerate codebooks,
 //     zero vectors) the thread re-scores all K entries the same way.
@@ -135,13 +136,14 @@ __global__ void __launch_bounds__(kEncThreads, 1) encode_vectors_kernel(const En
       for (long long tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
         if (!mbar_wait(a_full, it & 1)) atomicOr(a.flag, 2);
         umma::fence_after_sync();
-        for (int c = 0; c < nchunks; ++c, ++u) {
+        for (int c = 0; c < 2 * nchunks; ++c, ++u) {  // two passes over the entries
           const int b = (int)(u & 1);
+          const int ch = c < nchunks ? c : c - nchunks;
           if (u >= 2 && !mbar_wait(t_free0 + 8u * b, (uint32_t)((u / 2 - 1) & 1)))
             atomicOr(a.flag, 2);
           umma::fence_after_sync();
           umma::mma_f16(taddr + (uint32_t)(b * kEncChunk), desc_noswizzle(abase, kEncPlane),
-                        desc_noswizzle(sbase + (uint32_t)(c * a.chunk) * 16u, 0u), idesc, 0u);
+                        desc_noswizzle(sbase + (uint32_t)(ch * a.chunk) * 16u, 0u), idesc, 0u);
           umma::commit(t_full0 + 8u * b);
         }
       }
@@ -196,50 +198,49 @@ __global__ void __launch_bounds__(kEncThreads, 1) encode_vectors_kernel(const En
       __syncwarp();
       if (lane == 0) enc_arrive(a_full);
 
-      // scan the coarse scores, keeping the entries within kDelta of the max
-      float best = -INFINITY;
+      // Two passes over the coarse scores (the MMAs are repeated, which is
+      // cheap): the first takes the maximum, the second collects, in
+      // increasing k, the entries within the window below it.  Each block of
+      // 32 scores is reduced to its maximum first, so a score costs about one
+      // instruction per pass and only the block holding the maximum (or a
+      // near tie) is inspected element by element.
+      float cmax = -INFINITY, thr = -INFINITY;
       int ck[kCand];
-      float cs[kCand];
       int nc = 0;
       bool overflow = false;
-      for (int c = 0; c < nchunks; ++c, ++u) {
+      for (int c = 0; c < 2 * nchunks; ++c, ++u) {
+        const bool collect = c >= nchunks;
+        if (c == nchunks) thr = cmax - kDelta * fmaxf(1.f, fabsf(cmax));
         const int b = (int)(u & 1);
         if (!mbar_wait(t_full0 + 8u * b, (uint32_t)((u / 2) & 1)) && lane == 0)
           atomicOr(a.flag, 2);
         umma::fence_after_sync();
+        const int kc = (collect ? c - nchunks : c) * a.chunk;
         for (int cc = 0; cc < a.chunk / 32; ++cc) {
           uint32_t sv[32];
           umma::ld_32x32b_x32(taddr + ((uint32_t)(32 * warp) << 16) +
                                   (uint32_t)(b * kEncChunk + 32 * cc),
                               sv);
           umma::wait_ld();
-          const int k0 = c * a.chunk + 32 * cc;
+          float m8[8];
 #pragma unroll
-          for (int jj = 0; jj < 32; ++jj) {
-            const float s = __uint_as_float(sv[jj]);
-            if (s >= best - kDelta * fmaxf(1.f, fabsf(best))) {
-              if (s > best) {
-                best = s;
-                // drop candidates that fell out of the window (order kept)
-                const float thr = best - kDelta * fmaxf(1.f, fabsf(best));
-                int m = 0;
+          for (int i = 0; i < 8; ++i)
+            m8[i] = fmaxf(fmaxf(__uint_as_float(sv[4 * i]), __uint_as_float(sv[4 * i + 1])),
+                          fmaxf(__uint_as_float(sv[4 * i + 2]), __uint_as_float(sv[4 * i + 3])));
+          const float bm = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
+                                 fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
+          if (!collect) {
+            cmax = fmaxf(cmax, bm);
+          } else if (bm >= thr) {
+            const int k0 = kc + 32 * cc;
 #pragma unroll
-                for (int i = 0; i < kCand; ++i)
-                  if (i < nc && cs[i] >= thr) {
-                    ck[m] = ck[i];
-                    cs[m] = cs[i];
-                    ++m;
-                  }
-                nc = m;
+            for (int jj = 0; jj < 32; ++jj)
+              if (__uint_as_float(sv[jj]) >= thr) {
+                if (nc < kCand)
+                  ck[nc++] = k0 + jj;
+                else
+                  overflow = true;
               }
-              if (nc < kCand) {
-                ck[nc] = k0 + jj;
-                cs[nc] = s;
-                ++nc;
-              } else {
-                overflow = true;
-              }
-            }
           }
         }
         umma::fence_before_sync();
