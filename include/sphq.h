@@ -269,6 +269,34 @@ sphq_status sphq_set_gemm_shape(sphq_handle h, int act_tiles, int weight_rows);
 sphq_status sphq_check(sphq_handle h, sphq_stream stream);
 
 /*
+ * sphq_export / sphq_import -- the packed device image of a handle as one
+ * host blob and back (checkpointing quantised weights without re-packing).
+ * (No counterpart in the paper.)
+ *
+ *   sphq_export(h, buf, capacity, &size): *size = blob bytes; with buf NULL
+ *     only the size is returned.  Otherwise writes the blob (a 48-byte header
+ *     "SPHQ" / format 1 / shape / split, then codebook, group parameters and
+ *     the packed units) into host memory `buf` of `capacity` bytes
+ *     (SPHQ_ERR_INVALID_ARG if smaller); the handle must be packed.
+ *     Synchronous.
+ *   sphq_import(buf, size, &h): a new packed handle on the current device
+ *     from a blob (SPHQ_ERR_INVALID_ARG for a malformed or truncated blob).
+ *     Blobs are tied to this library's layout version (format 1).
+ */
+sphq_status sphq_export(sphq_handle h, void* buf, size_t capacity, size_t* size);
+sphq_status sphq_import(const void* buf, size_t size, sphq_handle* out);
+
+/*
+ * sphq_selftest_wait_timeout -- exercises the bounded-wait path: launches on
+ * `stream` a one-CTA kernel whose single on-chip wait (an mbarrier nothing
+ * arrives on) can never complete.  It gives up after about two seconds like
+ * every wait of the library, sets the handle's error word and exits; the
+ * next sphq_check returns SPHQ_ERR_TIMEOUT and the context stays usable.
+ * For tests of the failure detection.  (No counterpart in the paper.)
+ */
+sphq_status sphq_selftest_wait_timeout(sphq_handle h, sphq_stream stream);
+
+/*
  * sphq_decode -- write the decoded weights W_hat (rows x cols fp16, device
  * pointer, 16-byte aligned) on `stream`.  Bit-exact with Eq. (7) + Eq. (4) as
  * stated at the top of this header.  For verification; the GEMV never

@@ -19,6 +19,8 @@ static thread_local std::string g_last_error;
 // zero block read by GEMV lanes that supply no activations (4 words x 4 lanes x 16 B)
 constexpr size_t kZeroBytes = 256;
 
+void clear_error() { g_last_error.clear(); }
+
 sphq_status set_error(sphq_status s, const std::string& msg) {
   g_last_error = msg;
   return s;

@@ -54,6 +54,7 @@ struct sphq_handle_s {
 
 namespace sphq {
 
+void clear_error();
 sphq_status set_error(sphq_status s, const std::string& msg);
 sphq_status cuda_error(cudaError_t e, const char* what);
 

@@ -18,7 +18,7 @@ HEADER = os.path.join(os.path.dirname(HERE), "include", "sphq.h")
 SPHQ_OK = 0
 STATUS = {0: "SPHQ_OK", 1: "SPHQ_ERR_INVALID_ARG", 2: "SPHQ_ERR_UNSUPPORTED",
           3: "SPHQ_ERR_NOT_PACKED", 4: "SPHQ_ERR_CUDA", 5: "SPHQ_ERR_OOM",
-          6: "SPHQ_ERR_DEVICE"}
+          6: "SPHQ_ERR_DEVICE", 7: "SPHQ_ERR_TIMEOUT"}
 MAX_BATCH = 8
 
 _lib = None
@@ -68,6 +68,12 @@ def load() -> ctypes.CDLL:
         L.sphq_gemm.restype = i32
         L.sphq_check.argtypes = [vp, vp]
         L.sphq_check.restype = i32
+        L.sphq_export.argtypes = [vp, vp, sz, ctypes.POINTER(sz)]
+        L.sphq_export.restype = i32
+        L.sphq_import.argtypes = [vp, sz, ctypes.POINTER(vp)]
+        L.sphq_import.restype = i32
+        L.sphq_selftest_wait_timeout.argtypes = [vp, vp]
+        L.sphq_selftest_wait_timeout.restype = i32
         L.sphq_encode.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp]
         L.sphq_encode.restype = i32
         L.sphq_get_gemm_shape.argtypes = [vp, i32, ctypes.POINTER(GemmInfo)]
@@ -171,6 +177,36 @@ class SphqMatrix:
             y = torch.empty((B, self.rows), dtype=torch.float16, device=x.device)
         _check(load().sphq_gemv(self._h, x.data_ptr(), y.data_ptr(), B, _stream_ptr(stream)))
         return y
+
+    def export(self) -> bytes:
+        """sphq_export: the packed device image as a host blob."""
+        L = load()
+        size = ctypes.c_size_t()
+        _check(L.sphq_export(self._h, None, 0, ctypes.byref(size)))
+        buf = ctypes.create_string_buffer(size.value)
+        _check(L.sphq_export(self._h, buf, size.value, ctypes.byref(size)))
+        return buf.raw
+
+    @classmethod
+    def from_blob(cls, blob: bytes) -> "SphqMatrix":
+        """sphq_import: a packed matrix on the current device from a blob."""
+        import struct
+
+        import torch
+        L = load()
+        h = ctypes.c_void_p()
+        _check(L.sphq_import(blob, len(blob), ctypes.byref(h)))
+        _, _, rows, cols, bits, vbits, K, _ = struct.unpack_from("<4sIiiiiii", blob, 0)
+        m = cls.__new__(cls)
+        m._h = h
+        m.rows, m.cols, m.bits, m.K, m.radius_bits = rows, cols, bits, K, vbits
+        m.device = torch.device("cuda", torch.cuda.current_device())
+        return m
+
+    def selftest_wait_timeout(self, stream=None) -> None:
+        """sphq_selftest_wait_timeout: a kernel whose one wait never completes
+        (it gives up after ~2 s and sets the error word; see check())."""
+        _check(load().sphq_selftest_wait_timeout(self._h, _stream_ptr(stream)))
 
     def encode(self, w, stream=None):
         """sphq_encode: quantise w ((rows, cols) float32 CUDA tensor) with this
