@@ -84,6 +84,9 @@ def lib() -> ctypes.CDLL:
             L.sphqo_pack_w2_words.restype = i32
             L.sphqo_unpack_w2_words.argtypes = [i32, i32, u16, u32, u8, u16, u8]
             L.sphqo_unpack_w2_words.restype = i32
+            L.sphqo_decode_dim.argtypes = [i32, i32, i32, i32, i32, u16, u16, u16, u16, u16, u8,
+                                           u16]
+            L.sphqo_decode_dim.restype = i32
             L.sphqo_encode_f32.argtypes = [i32, i32, i32, i32, u16, ctypes.POINTER(ctypes.c_float),
                                            u8, u16, u8, u16, u16]
             L.sphqo_encode_f32.restype = i32
@@ -156,6 +159,28 @@ def decode(codebook, scale, offset, sign, idx, rcode) -> np.ndarray:
                             _p(rcode, ctypes.c_uint8), _p(out, ctypes.c_uint16))
     if rc != 0:
         raise ValueError("oracle decode: bad shape or out-of-range code")
+    return out
+
+
+def decode_dim(codebook, scale, offset, sign, idx, rcode, V: int = 4) -> np.ndarray:
+    """W_hat for vectors of dim = 4, 8 or 16 coordinates (Tab. 7; Eq. (7),
+    Eq. (4)); radius groups of 128 scalars.  codebook (K, dim) binary16 bits;
+    sign (rows, cols/dim) u16; idx u16; rcode u8."""
+    codebook = _c(codebook, np.uint16)
+    sign, idx, rcode = _c(sign, np.uint16), _c(idx, np.uint16), _c(rcode, np.uint8)
+    scale, offset = _c(scale, np.uint16), _c(offset, np.uint16)
+    K, dim = codebook.shape
+    rows, nv = sign.shape
+    cols = nv * dim
+    assert idx.shape == rcode.shape == sign.shape
+    assert scale.shape == offset.shape == (rows, cols // GROUP)
+    out = np.empty((rows, cols), np.uint16)
+    rc = lib().sphqo_decode_dim(rows, cols, dim, K, V, _p(codebook, ctypes.c_uint16),
+                                _p(scale, ctypes.c_uint16), _p(offset, ctypes.c_uint16),
+                                _p(sign, ctypes.c_uint16), _p(idx, ctypes.c_uint16),
+                                _p(rcode, ctypes.c_uint8), _p(out, ctypes.c_uint16))
+    if rc != 0:
+        raise ValueError("oracle decode_dim: bad shape or out-of-range code")
     return out
 
 

@@ -405,3 +405,46 @@ int sphqo_encode_f32(int rows, int cols, int K, int V, const uint16_t* codebook,
   free(cf);
   return 0;
 }
+
+/* ------------------------------------------------------------------------- */
+/* Eq. (7) and Eq. (4) for vectors of `dim` coordinates (Tab. 7)               */
+/* ------------------------------------------------------------------------- */
+
+/*
+ * The decode of sphqo_decode for vectors of dim = 4, 8 or 16 coordinates (§3.1
+ * with k = dim; the 4-D and 16-D configurations of Tab. 7).  Radius groups
+ * span 128 scalars (128 / dim vectors) as for 8-D vectors; radius codes have V
+ * bits.  sign is rows x (cols/dim) u16 (bit j = coordinate j negative),
+ * idx u16, rcode u8; codebook is K x dim binary16.
+ */
+int sphqo_decode_dim(int rows, int cols, int dim, int K, int V, const uint16_t* codebook,
+                     const uint16_t* scale, const uint16_t* offset, const uint16_t* sign,
+                     const uint16_t* idx, const uint8_t* rcode, uint16_t* w_out) {
+  if (rows < 0 || cols < 0 || cols % 128 != 0 || K <= 0 || V < 1 || V > 8 ||
+      (dim != 4 && dim != 8 && dim != 16))
+    return -1;
+  const int nv = cols / dim;
+  const int ng = cols / 128;
+  const int per_group = 128 / dim;
+  int bad = 0;
+#pragma omp parallel for schedule(static) reduction(| : bad)
+  for (int row = 0; row < rows; ++row) {
+    for (int t = 0; t < nv; ++t) {
+      const int64_t v = (int64_t)row * nv + t;
+      const int64_t g = (int64_t)row * ng + t / per_group;
+      const int k = idx[v];
+      const int q = rcode[v];
+      if (k >= K || q >= (1 << V)) {
+        bad = 1;
+        continue;
+      }
+      const double r = sphqo_half_to_double(sphqo_radius(q, scale[g], offset[g]));
+      for (int j = 0; j < dim; ++j) {
+        uint16_t w = sphqo_round_half(r * sphqo_half_to_double(codebook[(int64_t)k * dim + j]));
+        if ((sign[v] >> j) & 1) w ^= 0x8000u;
+        w_out[(int64_t)row * cols + (int64_t)t * dim + j] = w;
+      }
+    }
+  }
+  return bad ? -1 : 0;
+}

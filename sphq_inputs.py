@@ -71,8 +71,8 @@ def to_f16_bits(a) -> np.ndarray:
     return np.asarray(a, np.float64).astype(np.float16).view(np.uint16)
 
 
-def make_codebook(rng: np.random.Generator, K: int) -> np.ndarray:
-    c = np.abs(rng.standard_normal((K, VEC)))
+def make_codebook(rng: np.random.Generator, K: int, dim: int = VEC) -> np.ndarray:
+    c = np.abs(rng.standard_normal((K, dim)))
     c /= np.linalg.norm(c, axis=1, keepdims=True)
     return to_f16_bits(c)
 
@@ -108,6 +108,51 @@ def random_codes(bits: int, rows: int, cols: int, seed: int, B: int = 1,
     rcode = rng.integers(0, 1 << radius_bits, size=(rows, nv), dtype=np.uint8)
     x = make_x(rng, B, cols)
     return Codes(bits, cb, scale, offset, sign, idx, rcode, radius_bits), x
+
+
+@dataclass
+class CodesDim:
+    """Canonical codes of a matrix of dim-D vectors (Tab. 7: dim 4, 8, 16)."""
+    dim: int
+    bits: int
+    codebook: np.ndarray  # (K, dim) uint16 fp16 bits
+    scale: np.ndarray     # (rows, cols/128) uint16 fp16 bits
+    offset: np.ndarray
+    sign: np.ndarray      # (rows, cols/dim) uint16, bit j = coordinate j negative
+    idx: np.ndarray       # (rows, cols/dim) uint16
+    rcode: np.ndarray     # (rows, cols/dim) uint8
+    vbits: int = RADIUS_BITS
+
+    @property
+    def rows(self) -> int:
+        return self.sign.shape[0]
+
+    @property
+    def cols(self) -> int:
+        return self.sign.shape[1] * self.dim
+
+    @property
+    def K(self) -> int:
+        return self.codebook.shape[0]
+
+
+def random_codes_dim(dim: int, bits: int, rows: int, cols: int, seed: int, B: int = 1,
+                     radius_bits: int = RADIUS_BITS):
+    """Uniformly random codes of dim-D vectors: K = 2^((dim-1) bits - dim) entries
+    of |N(0, I_dim)| normalised, same draw order as random_codes.  Returns
+    (CodesDim, x)."""
+    if cols % GROUP_COLS:
+        raise ValueError("cols must be a multiple of 128")
+    rng = np.random.Generator(np.random.PCG64(seed))
+    K = 1 << ((dim - 1) * bits - dim)
+    cb = make_codebook(rng, K, dim)
+    scale, offset = make_params(rng, rows, cols)
+    nv = cols // dim
+    sign = rng.integers(0, 1 << dim, size=(rows, nv), dtype=np.uint32).astype(np.uint16)
+    idx = rng.integers(0, K, size=(rows, nv), dtype=np.uint16)
+    rcode = rng.integers(0, 1 << radius_bits, size=(rows, nv), dtype=np.uint8)
+    x = make_x(rng, B, cols)
+    return CodesDim(dim, bits, cb, scale, offset, sign, idx, rcode, radius_bits), x
 
 
 def gaussian_weights(rows: int, cols: int, seed: int, std: float = 0.02,
