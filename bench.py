@@ -824,6 +824,30 @@ def run_report(args):
                                                                inp.seed_for(1, 20 + 10 * d + v),
                                                                1, vbits=v, K=1 << d)
                                for d, v in ((6, 2), (6, 3), (7, 2), (7, 3), (8, 2), (6, 4))}
+    # 4-D vectors (the vector-dimension comparison at the W2 allocation)
+    rep["dim4"] = {}
+    for i, n in enumerate((4096, 8192)):
+        for bt in (1, 4):
+            codes, x = inp.random_codes_dim(4, 2, n, n, seed=inp.seed_for(1, 30 + i), B=bt)
+            one = n * n * 10 // 32
+            P = min(512, max(2, int(np.ceil(2 * L2 / one)) + 1))
+            cb, sc, of = t(codes.codebook), t(codes.scale), t(codes.offset)
+            sg, ix, rc = t(codes.sign.astype(np.uint8)), t(codes.idx), t(codes.rcode)
+            mats = []
+            for _ in range(P):
+                m = SphqMatrix(n, n, 2, cb, sc, of, radius_bits=4, K=4, dim=4)
+                m.pack(sg, ix, rc)
+                mats.append(m)
+            xd = t(x).view(torch.float16)
+            ys = [torch.empty((bt, n), dtype=torch.float16, device=dev) for _ in mats]
+            b = mats[0].bytes(bt)
+            us = steady_us(mats, xd, ys, bt, stream)
+            rep["dim4"][f"4-D {n}x{n} B{bt}"] = {
+                "us": round(us, 3), "GB/s": round(b / us / 1e3, 1),
+                "hbm_frac": round(b / us / 1e3 / hbm_peak, 4), "bytes": b, "pool": P}
+            for m in mats:
+                m.close()
+            torch.cuda.empty_cache()
     rep["prefill_gemm"] = gemm_report(hbm_peak)
     rep["encode"] = encode_report()
     # CPU oracle on the 1024^2 matrix: single thread and all cores

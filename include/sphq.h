@@ -109,11 +109,31 @@ sphq_status sphq_create_v(int rows, int cols, int bits, int radius_bits, int K,
                           sphq_handle* out);
 
 /*
+ * sphq_create_dim -- sphq_create_v for vectors of `dim` coordinates (§3.1
+ * with k = dim; the vector-dimension comparison of Tab. 7).
+ *
+ *   dim 8   as sphq_create_v.
+ *   dim 4   bits = 2, K = 4 (3B - 4 = 2 index bits), radius_bits = 4: 4 sign
+ *           bits + 2 + 4 = 10 bits per 4 weights (2.5 bits per weight);
+ *           codebook K x 4 fp16; radius groups of 128 scalars (32 vectors);
+ *           sphq_pack takes sign bytes with bits 0-3 (values above 15 are
+ *           rejected) and rows x cols/4 codes.  sphq_gemv, sphq_gemv_host,
+ *           sphq_decode, sphq_export support it; sphq_gemm and sphq_encode
+ *           do not (SPHQ_ERR_UNSUPPORTED).
+ *   dim 16  SPHQ_ERR_UNSUPPORTED: the W2 codebook (2^14 entries x 32 B =
+ *           512 KiB) exceeds an SM's shared memory.
+ */
+sphq_status sphq_create_dim(int rows, int cols, int dim, int bits, int radius_bits, int K,
+                            const void* codebook, const void* scale, const void* offset,
+                            sphq_handle* out);
+
+/*
  * sphq_pack -- convert canonical codes into the library's device layout
  * (the finalise-and-pack step, App. A step 10).
  *
  *   sign   rows x (cols/8) uint8, bit j set <=> coordinate j of the vector is
- *          negative (§3.1, Eq. (3)); vector t of a row covers columns 8t..8t+7.
+ *          negative (§3.1, Eq. (3)); vector t of a row covers columns 8t..8t+7
+ *          (4-D handles: rows x (cols/4), columns 4t..4t+3, bits 0-3).
  *   idx    rows x (cols/8) uint16, direction index z < K (Eq. (5)).
  *   rcode  rows x (cols/8) uint8, radius code q < 2^V (Eq. (7); V = 4, or
  *          the handle's radius_bits).

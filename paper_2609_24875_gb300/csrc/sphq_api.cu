@@ -153,6 +153,91 @@ __global__ void pack_kernel(const uint8_t* __restrict__ sign, const uint16_t* __
   }
 }
 
+// 4-D vectors: one thread per (unit, lane) composes the lane's five words
+// (layout in sphq_layout.cuh).  sign: rows x cols/4 bytes (bits 0-3).
+__global__ void pack4_kernel(const uint8_t* __restrict__ sign, const uint16_t* __restrict__ idx,
+                             const uint8_t* __restrict__ rcode, const uint16_t* __restrict__ scale,
+                             const uint16_t* __restrict__ offset, uint8_t* __restrict__ units,
+                             int rows, int ng, int nrt, int* __restrict__ flag) {
+  const long long tid = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (tid >= (long long)nrt * ng * 32) return;
+  const int lane = (int)(tid & 31);
+  const long long unit = tid >> 5;
+  const int rt = (int)(unit % nrt), g = (int)(unit / nrt);
+  const int gid = lane >> 2, q = lane & 3;
+  const int nv = ng * 32;
+  uint8_t* base = units + (size_t)unit * Layout<kFmt4D>::kUnitBytes;
+  uint32_t R[2] = {0, 0}, I = 0, S[2] = {0, 0};
+  bool bad = false;
+  for (int s = 0; s < 8; ++s) {
+    for (int half = 0; half < 2; ++half) {
+      const int row = rt * kRowsPerTile + gid + 8 * half;
+      if (row >= rows) continue;
+      const size_t v = (size_t)row * nv + (size_t)g * 32 + 4 * s + q;
+      uint32_t sg = sign[v], k = idx[v], rq = rcode[v];
+      if (k >= 4u || rq > 15u || sg > 15u) {
+        bad = true;
+        sg = k = rq = 0;
+      }
+      const int j = s & 3;
+      const int top = (half ? 7 : 15) - 2 * j;  // coordinate 0's bit
+      R[s >> 2] |= rq << (4 * j + 16 * half);
+      I |= k << (2 * s + 16 * half);
+      S[s >> 2] |= ((sg & 1u) << top) | (((sg >> 1) & 1u) << (top + 16)) |
+                   (((sg >> 2) & 1u) << (top - 1)) | (((sg >> 3) & 1u) << (top + 15));
+    }
+  }
+  if (bad) atomicOr(flag, 1);
+  *reinterpret_cast<uint4*>(base + lane * 16) = make_uint4(R[0], R[1], I, S[0]);
+  *reinterpret_cast<uint32_t*>(base + Layout<kFmt4D>::kS1Off + lane * 4) = S[1];
+  if (q == 0) {
+    uint32_t pa = 0, pb = 0;
+    const int ra = rt * kRowsPerTile + gid, rb = ra + 8;
+    if (ra < rows) pa = (uint32_t)scale[(size_t)ra * ng + g] | ((uint32_t)offset[(size_t)ra * ng + g] << 16);
+    if (rb < rows) pb = (uint32_t)scale[(size_t)rb * ng + g] | ((uint32_t)offset[(size_t)rb * ng + g] << 16);
+    *reinterpret_cast<uint2*>(base + Layout<kFmt4D>::kParamOff + gid * 8) = make_uint2(pa, pb);
+  }
+}
+
+template <int S>
+__device__ __forceinline__ void decode4_pair(const Unit<kFmt4D>& u, const GlobalCodebook& cb,
+                                             uint2& wa, uint2& wb) {
+  uint2 sa, sb;
+  directions_4d<S>(u.w, u.s1, cb, 0u, false, sa, sb);
+  const uint32_t r = radius_pair<4>(qpair_4d<S>(u.w), params_delta(u.par.x, u.par.y),
+                                    params_rmin(u.par.x, u.par.y));
+  const uint32_t ra = bcast_lo(r), rb = bcast_hi(r);
+  wa = make_uint2(hmul2_rn(ra, sa.x), hmul2_rn(ra, sa.y));
+  wb = make_uint2(hmul2_rn(rb, sb.x), hmul2_rn(rb, sb.y));
+}
+
+// W_hat of a 4-D matrix: one thread per vector.
+__global__ void decode4_kernel(const uint8_t* __restrict__ units, const uint8_t* __restrict__ codebook,
+                               uint16_t* __restrict__ w, int rows, int cols, int nrt) {
+  const long long tid = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  const int nv = cols / 4;
+  if (tid >= (long long)rows * nv) return;
+  const int row = (int)(tid / nv), t = (int)(tid % nv);
+  const int rt = row / kRowsPerTile, r16 = row % kRowsPerTile;
+  const int gid = r16 & 7, half = r16 >> 3;
+  const int g = t / 32, s = (t % 32) / 4, q = t % 4;
+  const Unit<kFmt4D> u = load_unit<kFmt4D>(
+      units + (size_t)unit_index(rt, g, nrt) * Layout<kFmt4D>::kUnitBytes, 4 * gid + q);
+  const GlobalCodebook cb{codebook};
+  uint2 wa, wb;
+  switch (s) {
+    case 0: decode4_pair<0>(u, cb, wa, wb); break;
+    case 1: decode4_pair<1>(u, cb, wa, wb); break;
+    case 2: decode4_pair<2>(u, cb, wa, wb); break;
+    case 3: decode4_pair<3>(u, cb, wa, wb); break;
+    case 4: decode4_pair<4>(u, cb, wa, wb); break;
+    case 5: decode4_pair<5>(u, cb, wa, wb); break;
+    case 6: decode4_pair<6>(u, cb, wa, wb); break;
+    default: decode4_pair<7>(u, cb, wa, wb); break;
+  }
+  *reinterpret_cast<uint2*>(w + (size_t)row * cols + (size_t)t * 4) = half ? wb : wa;
+}
+
 // ---------------------------------------------------------------------------
 // decode: W_hat (rows x cols fp16), through the same unpack/reconstruct code
 // ---------------------------------------------------------------------------
@@ -258,9 +343,9 @@ sphq_status sphq_create(int rows, int cols, int bits, int K, const void* codeboo
   return sphq_create_v(rows, cols, bits, 4, K, codebook, scale, offset, out);
 }
 
-sphq_status sphq_create_v(int rows, int cols, int bits, int radius_bits, int K,
-                          const void* codebook, const void* scale, const void* offset,
-                          sphq_handle* out) {
+static sphq_status create_impl(int rows, int cols, int dim, int bits, int radius_bits, int K,
+                               const void* codebook, const void* scale, const void* offset,
+                               sphq_handle* out) {
   g_last_error.clear();
   if (!out) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_create: out is NULL");
   *out = nullptr;
@@ -269,19 +354,34 @@ sphq_status sphq_create_v(int rows, int cols, int bits, int radius_bits, int K,
                      "sphq_create: need rows >= 1 and cols a positive multiple of 128");
   if (bits != 2 && bits != 3)
     return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_create: bits must be 2 or 3");
-  // direction index bits D = log2 K: 13 for W3; 6 (the §3.1 rule), 7 or 8 (Tab. 4) for W2
   int dbits = -1;
   for (int d = 0; d < 31; ++d)
     if (K == (1 << d)) dbits = d;
-  const bool k_ok = bits == 3 ? dbits == 13 : (dbits >= 6 && dbits <= 8);
-  if (!k_ok)
+  int fmt = -1;
+  if (dim == 4) {
+    // Tab. 7, W2 allocation: 3B - 4 = 2 index bits (K = 4), V = 4
+    if (bits != 2 || K != 4 || radius_bits != 4)
+      return set_error(SPHQ_ERR_UNSUPPORTED,
+                       "sphq_create_dim: 4-D vectors take bits = 2, K = 4, radius_bits = 4");
+    fmt = kFmt4D;
+  } else if (dim == 8) {
+    // direction index bits D = log2 K: 13 for W3; 6 (the §3.1 rule), 7 or 8 (Tab. 4) for W2
+    const bool k_ok = bits == 3 ? dbits == 13 : (dbits >= 6 && dbits <= 8);
+    if (!k_ok)
+      return set_error(SPHQ_ERR_UNSUPPORTED,
+                       "sphq_create: K must be 8192 for bits = 3 and 64, 128 or 256 for bits = 2");
+    fmt = fmt_of_split(dbits, radius_bits);
+    if (fmt < 0)
+      return set_error(SPHQ_ERR_UNSUPPORTED,
+                       "sphq_create: unsupported split; sign/index/radius bits must be one of "
+                       "8/6/4, 8/6/3, 8/6/2, 8/7/3, 8/7/2, 8/8/2, 8/13/4, 8/13/3");
+  } else {
     return set_error(SPHQ_ERR_UNSUPPORTED,
-                     "sphq_create: K must be 8192 for bits = 3 and 64, 128 or 256 for bits = 2");
-  const int fmt = fmt_of_split(dbits, radius_bits);
-  if (fmt < 0)
-    return set_error(SPHQ_ERR_UNSUPPORTED,
-                     "sphq_create: unsupported split; sign/index/radius bits must be one of "
-                     "8/6/4, 8/6/3, 8/6/2, 8/7/3, 8/7/2, 8/8/2, 8/13/4, 8/13/3");
+                     dim == 16 ? "sphq_create_dim: 16-D vectors are not supported (their W2 "
+                                 "codebook is 512 KiB, beyond shared memory)"
+                               : "sphq_create_dim: dim must be 4 or 8");
+  }
+  const size_t cb_bytes = (size_t)K * dim * 2;
   if (!codebook || !scale || !offset)
     return set_error(SPHQ_ERR_INVALID_ARG, "sphq_create: NULL codebook/scale/offset");
   const long long nrt = (rows + kRowsPerTile - 1) / kRowsPerTile;
@@ -307,6 +407,7 @@ sphq_status sphq_create_v(int rows, int cols, int bits, int radius_bits, int K,
   h->sm_count = prop.multiProcessorCount;
   h->vbits = radius_bits;
   h->dbits = dbits;
+  h->dim = dim;
   h->fmt = fmt;
   h->unit_bytes = fmt_unit_bytes(fmt);
 
@@ -319,7 +420,7 @@ sphq_status sphq_create_v(int rows, int cols, int bits, int radius_bits, int K,
   // past a warp's span without bounds checks
   if ((e = cudaMalloc(&h->units, ((size_t)nrt * ng + 2) * h->unit_bytes)) != cudaSuccess)
     return fail(cuda_error(e, "cudaMalloc(units)"));
-  if ((e = cudaMalloc(&h->codebook, (size_t)K * 16)) != cudaSuccess)
+  if ((e = cudaMalloc(&h->codebook, cb_bytes)) != cudaSuccess)
     return fail(cuda_error(e, "cudaMalloc(codebook)"));
   if ((e = cudaMalloc(&h->params, (size_t)rows * ng * 4)) != cudaSuccess)
     return fail(cuda_error(e, "cudaMalloc(params)"));
@@ -335,8 +436,17 @@ sphq_status sphq_create_v(int rows, int cols, int bits, int radius_bits, int K,
     return fail(cuda_error(e, "cudaMalloc(zeros)"));
   if ((e = cudaMemset(h->zeros, 0, kZeroBytes)) != cudaSuccess)
     return fail(cuda_error(e, "memset zeros"));
-  if ((e = cudaMemcpy(h->codebook, codebook, (size_t)K * 16, cudaMemcpyDefault)) != cudaSuccess)
+  if ((e = cudaMemcpy(h->codebook, codebook, cb_bytes, cudaMemcpyDefault)) != cudaSuccess)
     return fail(cuda_error(e, "copy codebook"));
+  if (fmt == kFmt4D) {
+    // shared-memory image of the 4-D GEMV: entry k, copy c (0..15) at 128 k + 8 c
+    if ((e = cudaMalloc(&h->cbimage, (size_t)K * 128)) != cudaSuccess)
+      return fail(cuda_error(e, "cudaMalloc(codebook image)"));
+    for (int c = 0; c < 16; ++c)
+      if ((e = cudaMemcpy2D(static_cast<uint8_t*>(h->cbimage) + 8 * c, 128, h->codebook, 8, 8,
+                            (size_t)K, cudaMemcpyDeviceToDevice)) != cudaSuccess)
+        return fail(cuda_error(e, "codebook image"));
+  }
   if (fmt_small(fmt)) {
     // shared-memory image of the small-codebook GEMV: entry k, copy c at 128 k + 16 c
     if ((e = cudaMalloc(&h->cbimage, (size_t)K * 8 * 16)) != cudaSuccess)
@@ -362,6 +472,18 @@ sphq_status sphq_create_v(int rows, int cols, int bits, int radius_bits, int K,
   return SPHQ_OK;
 }
 
+sphq_status sphq_create_v(int rows, int cols, int bits, int radius_bits, int K,
+                          const void* codebook, const void* scale, const void* offset,
+                          sphq_handle* out) {
+  return create_impl(rows, cols, 8, bits, radius_bits, K, codebook, scale, offset, out);
+}
+
+sphq_status sphq_create_dim(int rows, int cols, int dim, int bits, int radius_bits, int K,
+                            const void* codebook, const void* scale, const void* offset,
+                            sphq_handle* out) {
+  return create_impl(rows, cols, dim, bits, radius_bits, K, codebook, scale, offset, out);
+}
+
 // Validates and packs canonical device codes into the handle (synchronous).
 static sphq_status pack_codes(sphq_handle h, const uint8_t* sign, const uint16_t* idx,
                               const uint8_t* rcode, cudaStream_t s) {
@@ -374,7 +496,10 @@ static sphq_status pack_codes(sphq_handle h, const uint8_t* sign, const uint16_t
   const long long threads = (long long)h->nrt * h->ng * 32;
   const int block = 256;
   const unsigned grid = (unsigned)((threads + block - 1) / block);
-  switch (h->fmt) {
+  if (h->fmt == kFmt4D) {
+    pack4_kernel<<<grid, block, 0, s>>>(sign, idx, rcode, scale, offset, (uint8_t*)h->units,
+                                        h->rows, h->ng, h->nrt, h->flag);
+  } else switch (h->fmt) {
 #define SPHQ_PACK_CASE(F)                                                                   \
   case F:                                                                                   \
     pack_kernel<F><<<grid, block, 0, s>>>(sign, idx, rcode, scale, offset,                  \
@@ -391,7 +516,10 @@ static sphq_status pack_codes(sphq_handle h, const uint8_t* sign, const uint16_t
   SPHQ_CUDA(cudaStreamSynchronize(s), "pack");
   if (flag)
     return set_error(SPHQ_ERR_INVALID_ARG,
-                     "sphq_pack: a direction index >= K or a radius code >= 2^radius_bits");
+                     h->dim == 4 ? "sphq_pack: a direction index >= K, a radius code >= "
+                                   "2^radius_bits or a sign above 15"
+                                 : "sphq_pack: a direction index >= K or a radius code >= "
+                                   "2^radius_bits");
   h->packed = true;
   return SPHQ_OK;
 }
@@ -415,6 +543,7 @@ sphq_status sphq_encode(sphq_handle h, const float* w, uint8_t* sign, uint16_t* 
     return set_error(SPHQ_ERR_INVALID_ARG, "sphq_encode: w must be a 16-byte aligned pointer");
   if (!sign || !idx || !rcode || reinterpret_cast<uintptr_t>(idx) % 2)
     return set_error(SPHQ_ERR_INVALID_ARG, "sphq_encode: NULL or misaligned code pointer");
+  if (h->dim != 8) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_encode: 8-D vectors only");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   const size_t nvec = (size_t)h->rows * (h->cols / kVec);
   float* rtilde = nullptr;
@@ -455,7 +584,12 @@ sphq_status sphq_decode(sphq_handle h, void* w, sphq_stream stream) {
   const long long n = (long long)h->rows * (h->cols / kVec);
   const int block = 256;
   const unsigned grid = (unsigned)((n + block - 1) / block);
-  switch (h->fmt) {
+  if (h->fmt == kFmt4D) {
+    const long long nv4 = (long long)h->rows * (h->cols / 4);
+    decode4_kernel<<<(unsigned)((nv4 + 255) / 256), 256, 0, s>>>(
+        (const uint8_t*)h->units, (const uint8_t*)h->codebook, (uint16_t*)w, h->rows, h->cols,
+        h->nrt);
+  } else switch (h->fmt) {
 #define SPHQ_DECODE_CASE(F)                                                                    \
   case F:                                                                                      \
     decode_kernel<F><<<grid, block, 0, s>>>((const uint8_t*)h->units,                          \
@@ -494,6 +628,7 @@ sphq_status sphq_gemm(sphq_handle h, const void* x, void* y, int batch, sphq_str
   if (!y || reinterpret_cast<uintptr_t>(y) % 2)
     return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemm: y must be a 2-byte aligned pointer");
   if (!h->packed) return set_error(SPHQ_ERR_NOT_PACKED, "sphq_gemm: handle not packed");
+  if (h->dim != 8) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm: 8-D vectors only");
   return launch_gemm(h, x, y, batch, reinterpret_cast<cudaStream_t>(stream));
 }
 
@@ -575,11 +710,11 @@ sphq_status sphq_gemv_host(sphq_handle h, const void* x_host, void* y_host, int 
 size_t sphq_bytes(sphq_handle h, int batch) {
   if (!h || batch < 1 || batch > SPHQ_MAX_BATCH) return 0;
   const size_t weights = (size_t)h->rows * h->cols;
-  // payload bits per 8-D vector: 8 signs + D index bits + V radius bits
-  const size_t vec_bits = 8 + h->dbits + h->vbits;
-  const size_t payload = weights / kVec * vec_bits / 8;
+  // payload bits per dim-D vector: dim signs + D index bits + V radius bits
+  const size_t vec_bits = (size_t)h->dim + h->dbits + h->vbits;
+  const size_t payload = weights / h->dim * vec_bits / 8;
   const size_t params = (size_t)h->rows * h->ng * 4;
-  const size_t codebook = (size_t)h->K * 16;
+  const size_t codebook = (size_t)h->K * h->dim * 2;
   const size_t io = 2 * (size_t)batch * (h->cols + h->rows);
   return payload + params + codebook + io;
 }

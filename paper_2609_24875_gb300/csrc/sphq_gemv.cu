@@ -15,10 +15,13 @@ namespace sphq {
 // ---------------------------------------------------------------------------
 
 static int warps_for(int fmt) {
-  return fmt_small(fmt) ? KernelShape<2>::kWarps : KernelShape<3>::kWarps;
+  return fmt_small(fmt) || fmt == kFmt4D ? KernelShape<2>::kWarps : KernelShape<3>::kWarps;
 }
+// shared-memory codebook image: interleaved copies (128 bytes per entry) for
+// the small codebooks and 4-D, the plain 128 KiB table for W3
 static uint32_t cb_bytes_for(int fmt) {
-  return fmt_small(fmt) ? (uint32_t)(1u << fmt_dir_bits(fmt)) * 8u * 16u : KernelShape<3>::kCbBytes;
+  return fmt_small(fmt) || fmt == kFmt4D ? (uint32_t)(1u << fmt_dir_bits(fmt)) * 128u
+                                         : KernelShape<3>::kCbBytes;
 }
 
 static int mode_for(int batch) { return batch == 1 ? kFactored1 : batch == 2 ? kFactored2 : kFull; }
@@ -39,7 +42,7 @@ static sphq_status allow_max_smem(int device, int optin) {
   std::lock_guard<std::mutex> lock(mu);
   if (device < 0 || device >= 64) return set_error(SPHQ_ERR_DEVICE, "device index out of range");
   if (done[device]) return SPHQ_OK;
-  for (int fmt = 2; fmt <= kFmt882; ++fmt)
+  for (int fmt = 2; fmt <= kFmt4D; ++fmt)
     for (int mode : kModes) {
       cudaError_t e = cudaFuncSetAttribute(select_kernel(fmt, mode),
                                            cudaFuncAttributeMaxDynamicSharedMemorySize, optin);
@@ -222,7 +225,7 @@ sphq_status launch_gemv(sphq_handle h, const void* x, void* y, int batch, cudaSt
   const GemvPlan& p = h->plan[batch];
   GemvArgs a;
   a.units = (const uint8_t*)h->units;
-  a.cbimage = (const uint8_t*)(fmt_small(h->fmt) ? h->cbimage : h->codebook);
+  a.cbimage = (const uint8_t*)(h->cbimage ? h->cbimage : h->codebook);
   a.x = (const uint16_t*)x;
   a.y = (uint16_t*)y;
   a.flag = h->flag + 1;

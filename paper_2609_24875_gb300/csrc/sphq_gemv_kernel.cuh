@@ -291,12 +291,84 @@ struct Acc {
   }
 };
 
-// One unit (16 rows x 16 slots); xv[m] is this lane's B-fragment data for
-// word m (its activation row at slot 4m+q, or zeros).
+// The lane's B-fragment data of one group: 8-D, v[m] = its activation row
+// at slot 4m+q (16 bytes); 4-D, v[s] = at vector 4s+q (8 bytes); or zeros.
+template <int BITS> struct XFrag { uint4 v[4]; };
+template <> struct XFrag<kFmt4D> { uint2 v[8]; };
+
+// 8-byte activation load kept in L1 (batch 3-8, 4-D vectors)
+__device__ __forceinline__ uint2 ldg_x8(const uint8_t* p) {
+  uint2 v;
+  asm volatile("ld.global.nc.L1::evict_last.v2.u32 {%0,%1}, [%2];" : "=r"(v.x), "=r"(v.y) : "l"(p));
+  return v;
+}
+
+// xp: this lane's first activation bytes of the group (8-D: slot q at 16 q,
+// words 64 bytes apart; 4-D: vector q at 8 q, pairs 32 bytes apart).
 template <int BITS, int MODE>
-__device__ __forceinline__ void process_unit(const Unit<BITS>& cur, const uint4 (&xv)[4], int q,
+__device__ __forceinline__ void load_x(XFrag<BITS>& xv, const uint8_t* xp) {
+  if constexpr (BITS == kFmt4D) {
+#pragma unroll
+    for (int s = 0; s < 8; ++s) {
+      if constexpr (MODE == kFull)
+        xv.v[s] = ldg_x8(xp + 32 * s);
+      else
+        xv.v[s] = *reinterpret_cast<const uint2*>(xp + 32 * s);
+    }
+  } else {
+#pragma unroll
+    for (int m = 0; m < 4; ++m) {
+      if constexpr (MODE == kFull)
+        xv.v[m] = ldg_x16(reinterpret_cast<const uint16_t*>(xp) + 32 * m);
+      else
+        xv.v[m] = *reinterpret_cast<const uint4*>(xp + 64 * m);
+    }
+  }
+}
+
+// One pair s of a 4-D unit: one MMA for the two 4-D vectors of the lane.
+template <int MODE, int S>
+__device__ __forceinline__ void process_pair_4d(const Unit<kFmt4D>& cur,
+                                                const UnitConst<kFmt4D>& kc,
+                                                const XFrag<kFmt4D>& xv, const SmemCodebook& cb,
+                                                Acc<MODE>& acc) {
+  uint2 sa, sb;
+  directions_4d<S>(cur.w, cur.s1, cb, cb.copyoff, true, sa, sb);
+  const uint32_t r = radius_pair<4>(qpair_4d<S>(cur.w), kc.d2, kc.m2);
+  if constexpr (MODE == kFull) {
+    const uint32_t ra = bcast_lo(r), rb = bcast_hi(r);
+    mma16816(acc.d, hmul2_rn(ra, sa.x), hmul2_rn(rb, sb.x), hmul2_rn(ra, sa.y),
+             hmul2_rn(rb, sb.y), xv.v[S].x, xv.v[S].y);
+  } else {
+    float d[4];
+    mma16816_zero(d, sa.x, sb.x, sa.y, sb.y, xv.v[S].x, xv.v[S].y);
+    const float rA = h_lo_to_f32(r), rB = h_hi_to_f32(r);
+    acc.f[0][0] = __fmaf_rn(rA, d[0], acc.f[0][0]);
+    acc.f[0][1] = __fmaf_rn(rB, d[2], acc.f[0][1]);
+    if constexpr (MODE == kFactored2) {
+      acc.f[1][0] = __fmaf_rn(rA, d[1], acc.f[1][0]);
+      acc.f[1][1] = __fmaf_rn(rB, d[3], acc.f[1][1]);
+    }
+  }
+}
+
+// One unit (16 rows x 128 columns).
+template <int BITS, int MODE>
+__device__ __forceinline__ void process_unit(const Unit<BITS>& cur, const XFrag<BITS>& xf, int q,
                                              const SmemCodebook& cb, Acc<MODE>& acc) {
   const UnitConst<BITS> kc = unit_const<BITS>(cur, q);
+  if constexpr (BITS == kFmt4D) {
+    process_pair_4d<MODE, 0>(cur, kc, xf, cb, acc);
+    process_pair_4d<MODE, 1>(cur, kc, xf, cb, acc);
+    process_pair_4d<MODE, 2>(cur, kc, xf, cb, acc);
+    process_pair_4d<MODE, 3>(cur, kc, xf, cb, acc);
+    process_pair_4d<MODE, 4>(cur, kc, xf, cb, acc);
+    process_pair_4d<MODE, 5>(cur, kc, xf, cb, acc);
+    process_pair_4d<MODE, 6>(cur, kc, xf, cb, acc);
+    process_pair_4d<MODE, 7>(cur, kc, xf, cb, acc);
+    return;
+  } else {
+  const auto& xv = xf.v;
 #pragma unroll
   for (int m = 0; m < 4; ++m) {
     uint4 sa, sb;
@@ -320,6 +392,7 @@ __device__ __forceinline__ void process_unit(const Unit<BITS>& cur, const uint4 
         acc.f[1][1] = __fmaf_rn(rB, d[3], acc.f[1][1]);
       }
     }
+  }
   }
 }
 
@@ -409,14 +482,8 @@ __device__ __forceinline__ void run_item(Unit<BITS> (&u)[kStrip], Acc<MODE> (&ac
                                          const uint8_t* xp, const uint8_t* nb, unsigned nmask,
                                          int lane, int q, const SmemCodebook& cb) {
   constexpr int UB = Layout<BITS>::kUnitBytes;
-  uint4 xv[4];
-#pragma unroll
-  for (int m = 0; m < 4; ++m) {
-    if constexpr (MODE == kFull)
-      xv[m] = ldg_x16(reinterpret_cast<const uint16_t*>(xp) + 32 * m);
-    else
-      xv[m] = *reinterpret_cast<const uint4*>(xp + 64 * m);
-  }
+  XFrag<BITS> xv;
+  load_x<BITS, MODE>(xv, xp);
 #pragma unroll
   for (int j = 0; j < kStrip; ++j) {
     if (j < SIZE) process_unit<BITS, MODE>(u[j], xv, q, cb, acc[j]);
@@ -450,23 +517,11 @@ __device__ __forceinline__ void run_segment(Unit<BITS> (&u)[kStrip], Acc<MODE> (
       // items c+2, c+3 go to registers below; c+4, c+5 toward L2
       if (lane == 0 && c + 4 < cnt) prefetch_l2(ub + 4 * gstride, kBytes);
       if (lane == 0 && c + 5 < cnt) prefetch_l2(ub + 5 * gstride, kBytes);
-      uint4 xv[4];
-#pragma unroll
-      for (int m = 0; m < 4; ++m) {
-        if constexpr (MODE == kFull)
-          xv[m] = ldg_x16(reinterpret_cast<const uint16_t*>(xp) + 32 * m);
-        else
-          xv[m] = *reinterpret_cast<const uint4*>(xp + 64 * m);
-      }
+      XFrag<BITS> xv;
+      load_x<BITS, MODE>(xv, xp);
       process_unit<BITS, MODE>(u[0], xv, q, cb, acc[0]);
       if (c + 2 < cnt) u[0] = load_unit<BITS>(ub + 2 * gstride, lane);
-#pragma unroll
-      for (int m = 0; m < 4; ++m) {
-        if constexpr (MODE == kFull)
-          xv[m] = ldg_x16(reinterpret_cast<const uint16_t*>(xp + xstep) + 32 * m);
-        else
-          xv[m] = *reinterpret_cast<const uint4*>(xp + xstep + 64 * m);
-      }
+      load_x<BITS, MODE>(xv, xp + xstep);
       process_unit<BITS, MODE>(u[1], xv, q, cb, acc[0]);
       if (c + 3 < cnt) u[1] = load_unit<BITS>(ub + 3 * gstride, lane);
       ub += 2 * gstride;
@@ -570,7 +625,9 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
 
   SmemCodebook cb;
   cb.base = smem;
-  cb.copyoff = fmt_small(BITS) ? (uint32_t)(lane & 7) * 16u : 0u;
+  cb.copyoff = fmt_small(BITS) ? (uint32_t)(lane & 7) * 16u
+                : BITS == kFmt4D ? (uint32_t)(lane & 15) * 8u
+                                 : 0u;
 
   // The activation row this lane supplies to the B fragment; the other lanes
   // read a zero block (stride 0), so the loop has no lane-dependent branch.
@@ -589,7 +646,7 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
                   : reinterpret_cast<const uint8_t*>(a.zeros);
   else
     x0 = provider ? smem + a.off_x + xb * a.x_pitch : smem + a.off_zero;
-  x0 += q * 16;
+  x0 += q * (BITS == kFmt4D ? 8 : 16);
   const int xstep = provider ? kGroupCols * 2 : 0;
 
   // receive slot of (owned tile k, rank r, warp w): ((k * csize + r) * WARPS + w) * kBlk floats

@@ -30,6 +30,7 @@ struct sphq_handle_s {
   int rows = 0, cols = 0, bits = 0, K = 0;
   int vbits = 4;           // radius code bits V
   int dbits = 6;           // direction index bits D = log2 K
+  int dim = 8;             // vector dimension (8, or 4)
   int fmt = 0;             // device format id (sphq_layout.cuh), one per bit split
   int nrt = 0;             // row tiles of 16 rows
   int ng = 0;              // radius groups per row (cols / 128)

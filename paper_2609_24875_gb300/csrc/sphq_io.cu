@@ -10,13 +10,14 @@
 namespace sphq {
 
 // Blob layout (little-endian host memory):
-//   header  48 B: "SPHQ", format 1 (u32), rows, cols, bits, radius_bits, K
-//           (i32), 4 B zero, unit bytes (u64), packed-units bytes (u64)
-//   codebook K x 8 fp16 | scale rows x ng fp16 | offset rows x ng fp16 | units
+//   header  48 B: "SPHQ", format 1 (u32), rows, cols, bits, radius_bits, K,
+//           vector dimension (i32; 0 reads as 8), unit bytes (u64),
+//           packed-units bytes (u64)
+//   codebook K x dim fp16 | scale rows x ng fp16 | offset rows x ng fp16 | units
 struct BlobHeader {
   char magic[4];
   uint32_t format;
-  int32_t rows, cols, bits, radius_bits, K, pad;
+  int32_t rows, cols, bits, radius_bits, K, dim;
   uint64_t unit_bytes, units_bytes;
 };
 static_assert(sizeof(BlobHeader) == 48, "blob header");
@@ -25,7 +26,7 @@ constexpr uint32_t kBlobFormat = 1;
 static size_t blob_size(const sphq_handle_s* h, size_t* units_bytes) {
   const size_t ub = (size_t)h->nrt * h->ng * h->unit_bytes;
   if (units_bytes) *units_bytes = ub;
-  return sizeof(BlobHeader) + (size_t)h->K * 16 + 2 * (size_t)h->rows * h->ng * 2 + ub;
+  return sizeof(BlobHeader) + (size_t)h->K * h->dim * 2 + 2 * (size_t)h->rows * h->ng * 2 + ub;
 }
 
 // The one wait of this kernel can never complete (nothing arrives on the
@@ -64,14 +65,16 @@ sphq_status sphq_export(sphq_handle h, void* buf, size_t capacity, size_t* size)
   hd.bits = h->bits;
   hd.radius_bits = h->vbits;
   hd.K = h->K;
+  hd.dim = h->dim;
   hd.unit_bytes = h->unit_bytes;
   hd.units_bytes = ub;
   uint8_t* p = static_cast<uint8_t*>(buf);
   std::memcpy(p, &hd, sizeof(hd));
   p += sizeof(hd);
   const size_t np = (size_t)h->rows * h->ng;
-  cudaError_t e = cudaMemcpy(p, h->codebook, (size_t)h->K * 16, cudaMemcpyDeviceToHost);
-  p += (size_t)h->K * 16;
+  const size_t cbb = (size_t)h->K * h->dim * 2;
+  cudaError_t e = cudaMemcpy(p, h->codebook, cbb, cudaMemcpyDeviceToHost);
+  p += cbb;
   if (e == cudaSuccess) e = cudaMemcpy(p, h->params, 2 * np * 2, cudaMemcpyDeviceToHost);
   p += 2 * np * 2;
   if (e == cudaSuccess) e = cudaMemcpy(p, h->units, ub, cudaMemcpyDeviceToHost);
@@ -93,12 +96,15 @@ sphq_status sphq_import(const void* buf, size_t size, sphq_handle* out) {
       (long long)hd.rows * hd.cols > (1LL << 40))
     return set_error(SPHQ_ERR_INVALID_ARG, "sphq_import: bad shape in header");
   const uint8_t* p = static_cast<const uint8_t*>(buf) + sizeof(BlobHeader);
+  const int dim = hd.dim == 0 ? 8 : hd.dim;
+  if (dim != 4 && dim != 8) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_import: bad dimension");
   const size_t np = (size_t)hd.rows * (hd.cols / 128);
-  const size_t fixed = sizeof(BlobHeader) + (size_t)hd.K * 16 + 2 * np * 2;
+  const size_t cbb = (size_t)hd.K * dim * 2;
+  const size_t fixed = sizeof(BlobHeader) + cbb + 2 * np * 2;
   if (size < fixed) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_import: blob truncated");
   sphq_handle h = nullptr;
-  sphq_status st = sphq_create_v(hd.rows, hd.cols, hd.bits, hd.radius_bits, hd.K, p,
-                                 p + (size_t)hd.K * 16, p + (size_t)hd.K * 16 + np * 2, &h);
+  sphq_status st = sphq_create_dim(hd.rows, hd.cols, dim, hd.bits, hd.radius_bits, hd.K, p,
+                                   p + cbb, p + cbb + np * 2, &h);
   if (st != SPHQ_OK) return st;
   size_t ub = 0;
   const size_t need = blob_size(h, &ub);
@@ -106,7 +112,7 @@ sphq_status sphq_import(const void* buf, size_t size, sphq_handle* out) {
     sphq_destroy(h);
     return set_error(SPHQ_ERR_INVALID_ARG, "sphq_import: blob size does not match its header");
   }
-  cudaError_t e = cudaMemcpy(h->units, p + (size_t)hd.K * 16 + 2 * np * 2, ub,
+  cudaError_t e = cudaMemcpy(h->units, p + cbb + 2 * np * 2, ub,
                              cudaMemcpyHostToDevice);
   if (e != cudaSuccess) {
     sphq_destroy(h);

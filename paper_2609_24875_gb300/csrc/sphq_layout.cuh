@@ -68,6 +68,20 @@
 //                 radius code (0..7) in bits 5-7
 //   [768, 832)  quad gid: 8 B = { P_gid, P_gid+8 }
 //
+// 4-D vectors (format id 10, Tab. 7 at the W2 allocation: 4 sign bits, a
+// 2-bit index into K = 4 directions, a 4-bit radius code; 704 B = 512
+// vectors x 10 bits + 64 B params).  Lane l = 4*gid + q owns rows gid (A) and
+// gid+8 (B) at the group's vectors 4s+q, s = 0..7 ("pair s"); pair s fills
+// the lane's K slots of the s-th MMA (one 4-D vector per lane and row):
+//   [0, 512)    lane l: 16 B = { R0, R1, I, S0 }
+//   [512, 640)  lane l: 4 B = S1
+//   [640, 704)  quad gid: { P_gid, P_gid+8 }
+//   R_{s/4}: radius code of A at bits 4(s%4)..+3, of B 16 bits higher
+//   I: index of A at bits 2s..2s+1, of B at 16+2s..
+//   S_{s/4}, j = s % 4: sign bits of A: coordinate 0 at 15-2j, 1 at 31-2j,
+//     2 at 14-2j, 3 at 30-2j; of B: 0 at 7-2j, 1 at 23-2j, 2 at 6-2j, 3 at 22-2j
+//     (each coordinate pair is one shift away from bits 15 / 31)
+//
 // No byte beyond the algorithmic payload is stored; padded rows hold zero
 // codes and parameters.
 #pragma once
@@ -93,14 +107,19 @@ __host__ __device__ __forceinline__ long long unit_index(int rt, int g, int nrt)
 // 5 = 8/6/2, 6 = 8/6/3, 7 = 8/7/2, 8 = 8/7/3, 9 = 8/8/2.
 constexpr int kFmtW3V3 = 4;
 constexpr int kFmt862 = 5, kFmt863 = 6, kFmt872 = 7, kFmt873 = 8, kFmt882 = 9;
+// 4-D vectors at the W2 allocation (Tab. 7): 4 sign bits, a 2-bit index into
+// K = 4 directions, a 4-bit radius code (2.5 bits per weight).
+constexpr int kFmt4D = 10;
 __host__ __device__ constexpr int fmt_dir_bits(int fmt) {
-  return fmt == 3 || fmt == 4 ? 13 : fmt == 7 || fmt == 8 ? 7 : fmt == 9 ? 8 : 6;
+  return fmt == 3 || fmt == 4 ? 13 : fmt == 7 || fmt == 8 ? 7 : fmt == 9 ? 8 : fmt == kFmt4D ? 2 : 6;
 }
 __host__ __device__ constexpr int fmt_radius_bits(int fmt) {
-  return fmt == 2 || fmt == 3 ? 4 : fmt == 4 || fmt == 6 || fmt == 8 ? 3 : 2;
+  return fmt == 2 || fmt == 3 || fmt == kFmt4D ? 4 : fmt == 4 || fmt == 6 || fmt == 8 ? 3 : 2;
 }
+// vector dimension of a format
+__host__ __device__ constexpr int fmt_dim(int fmt) { return fmt == kFmt4D ? 4 : 8; }
 // formats whose codebook (K <= 256) is kept as eight interleaved copies
-__host__ __device__ constexpr bool fmt_small(int fmt) { return fmt == 2 || fmt >= 5; }
+__host__ __device__ constexpr bool fmt_small(int fmt) { return fmt == 2 || (fmt >= 5 && fmt <= 9); }
 // format id of a split, or -1
 __host__ __device__ constexpr int fmt_of_split(int dir_bits, int radius_bits) {
   return dir_bits == 13 ? (radius_bits == 4 ? 3 : radius_bits == 3 ? 4 : -1)
@@ -130,6 +149,14 @@ template <> struct Layout<kFmtW3V3> {
   static constexpr int kHiOff = 512;
   static constexpr int kParamOff = 768;
 };
+// 4-D unit: 704 B = 512 vectors x 10 bits + 16 x 4 B params; see the
+// format description at the top.
+template <> struct Layout<kFmt4D> {
+  static constexpr int K = 4;
+  static constexpr int kUnitBytes = 704;
+  static constexpr int kS1Off = 512;
+  static constexpr int kParamOff = 640;
+};
 template <> struct Layout<3> {
   static constexpr int K = 8192;
   static constexpr int kUnitBytes = 864;
@@ -142,6 +169,7 @@ template <> struct Layout<3> {
 __host__ __device__ constexpr int fmt_unit_bytes(int fmt) {
   return fmt == 3 ? Layout<3>::kUnitBytes
          : fmt == kFmtW3V3 ? Layout<kFmtW3V3>::kUnitBytes
+         : fmt == kFmt4D ? Layout<kFmt4D>::kUnitBytes
          : fmt_dir_bits(fmt) + fmt_radius_bits(fmt) == 10 ? 640
          : fmt_dir_bits(fmt) + fmt_radius_bits(fmt) == 9 ? 608
                                                           : 576;
@@ -162,6 +190,11 @@ template <int BITS> struct Unit {
 template <> struct Unit<kFmtW3V3> {
   uint4 w;
   uint2 hi;     // {H0, H1}
+  uint2 par;    // {P_gid, P_gid+8}
+};
+template <> struct Unit<kFmt4D> {
+  uint4 w;      // {R0, R1, I, S0}
+  uint32_t s1;  // S1
   uint2 par;    // {P_gid, P_gid+8}
 };
 template <> struct Unit<3> {
@@ -226,6 +259,15 @@ __device__ __forceinline__ Unit<kFmtW3V3> load_unit<kFmtW3V3>(const uint8_t* uni
   u.w = ldg_stream16(unit + lane * 16);
   u.hi = ldg_stream8(unit + Layout<kFmtW3V3>::kHiOff + lane * 8);
   u.par = ldg_stream8(unit + Layout<kFmtW3V3>::kParamOff + (lane >> 2) * 8);
+  return u;
+}
+
+template <>
+__device__ __forceinline__ Unit<kFmt4D> load_unit<kFmt4D>(const uint8_t* unit, int lane) {
+  Unit<kFmt4D> u;
+  u.w = ldg_stream16(unit + lane * 16);
+  u.s1 = ldg_stream4(unit + Layout<kFmt4D>::kS1Off + lane * 4);
+  u.par = ldg_stream8(unit + Layout<kFmt4D>::kParamOff + (lane >> 2) * 8);
   return u;
 }
 
@@ -329,19 +371,63 @@ __device__ __forceinline__ uint4 lds16(uint32_t saddr) {
 // quarter-warp then touch eight distinct 16-byte bank groups).  W3: a single
 // copy, entry k at byte 16*k.  `base` is a shared-memory address, or for the
 // global-memory variant used by the decode kernel a generic pointer.
+// 4-D: sixteen interleaved copies of the 8-byte entries, entry k of copy c at
+// 128*k + 8*c; lane l uses copy l % 16 (a half warp's 8-byte loads then touch
+// sixteen distinct bank pairs).
 struct SmemCodebook {
   const uint8_t* base;  // the shared-memory table (a __shared__ array)
-  uint32_t copyoff;     // W2: 16 * (lane % 8), W3: 0
+  uint32_t copyoff;     // W2: 16 * (lane % 8), 4-D: 8 * (lane % 16), W3: 0
   __device__ __forceinline__ uint4 at(uint32_t off) const {
     return *reinterpret_cast<const uint4*>(base + off);
+  }
+  __device__ __forceinline__ uint2 at8(uint32_t off) const {
+    return *reinterpret_cast<const uint2*>(base + off);
   }
 };
 struct GlobalCodebook {
-  const uint8_t* base;  // K x 16 B
+  const uint8_t* base;  // K x 16 B (4-D: K x 8 B)
   __device__ __forceinline__ uint4 at(uint32_t off) const {
     return *reinterpret_cast<const uint4*>(base + off);
   }
+  __device__ __forceinline__ uint2 at8(uint32_t off) const {
+    return *reinterpret_cast<const uint2*>(base + off);
+  }
 };
+
+// Signed directions of pair s of a 4-D unit (A = row gid, B = row gid+8):
+// two half2 registers per vector (coordinates 0-1, 2-3).  Codebook offsets
+// 128*k + copy offset, or 8*k for a plain table.
+template <int S, class CB>
+__device__ __forceinline__ void directions_4d(const uint4& w, uint32_t s1, const CB& cb,
+                                              uint32_t copyoff, bool interleaved, uint2& sa,
+                                              uint2& sb) {
+  const uint32_t I = w.z;
+  const uint32_t Sw = S < 4 ? w.w : s1;
+  constexpr int j = S & 3;
+  // index of A at bits 2S..2S+1, of B at 16+2S..
+  uint32_t ia, ib;
+  if constexpr (2 * S <= 7) ia = shl_fma<7 - 2 * S>(I) & 0x180u;
+  else ia = (I >> (2 * S - 7)) & 0x180u;
+  ib = (I >> (9 + 2 * S)) & 0x180u;
+  uint32_t offA, offB;
+  if (interleaved) {
+    offA = ia | copyoff;
+    offB = ib | copyoff;
+  } else {
+    offA = ia >> 4;
+    offB = ib >> 4;
+  }
+  const uint2 ca = cb.at8(offA);
+  const uint2 cbv = cb.at8(offB);
+  sa = make_uint2(ca.x ^ (shl_fma<2 * j>(Sw) & kSignMask), ca.y ^ (shl_fma<2 * j + 1>(Sw) & kSignMask));
+  sb = make_uint2(cbv.x ^ (shl_fma<8 + 2 * j>(Sw) & kSignMask),
+                  cbv.y ^ (shl_fma<9 + 2 * j>(Sw) & kSignMask));
+}
+// Radius codes of pair s (A at bits 0-3, B at 16-19).
+template <int S>
+__device__ __forceinline__ uint32_t qpair_4d(const uint4& w) {
+  return (S < 4 ? w.x : w.y) >> (4 * (S & 3));
+}
 
 // Signed directions of the two vectors of word m of a small-codebook unit
 // (W2 and the other splits of Tab. 4; A = row gid, B = row gid+8).  `e` is

@@ -60,6 +60,9 @@ def load() -> ctypes.CDLL:
         L.sphq_create.restype = i32
         L.sphq_create_v.argtypes = [i32, i32, i32, i32, i32, vp, vp, vp, ctypes.POINTER(vp)]
         L.sphq_create_v.restype = i32
+        L.sphq_create_dim.argtypes = [i32, i32, i32, i32, i32, i32, vp, vp, vp,
+                                      ctypes.POINTER(vp)]
+        L.sphq_create_dim.restype = i32
         L.sphq_pack.argtypes = [vp, vp, vp, vp, vp]
         L.sphq_pack.restype = i32
         L.sphq_gemv.argtypes = [vp, vp, vp, i32, vp]
@@ -127,26 +130,27 @@ class SphqMatrix:
     """
 
     def __init__(self, rows: int, cols: int, bits: int, codebook, scale, offset,
-                 radius_bits: int = 4, K: int | None = None):
-        """bits 2 or 3; K defaults to 2^(7*bits - 8) (64 / 8192); the Tab. 4 splits
-        take K = 128 or 256 at bits = 2 and radius_bits 2 or 3 (sphq_create_v)."""
+                 radius_bits: int = 4, K: int | None = None, dim: int = 8):
+        """bits 2 or 3; K defaults to 2^((dim-1)*bits - dim) (64 / 8192 for 8-D);
+        the Tab. 4 splits take K = 128 or 256 at bits = 2 and radius_bits 2 or 3
+        (sphq_create_v); dim = 4 takes bits 2, K 4 (sphq_create_dim)."""
         import torch
         L = load()
         if K is None:
-            K = 1 << (7 * bits - 8)
+            K = 1 << ((dim - 1) * bits - dim)
         cb = codebook.contiguous()
         sc = scale.contiguous()
         of = offset.contiguous()
-        for t, shape in ((cb, (K, 8)), (sc, (rows, cols // 128)), (of, (rows, cols // 128))):
+        for t, shape in ((cb, (K, dim)), (sc, (rows, cols // 128)), (of, (rows, cols // 128))):
             if tuple(t.shape) != shape or t.element_size() != 2:
                 raise ValueError(f"expected a 2-byte tensor of shape {shape}, got "
                                  f"{tuple(t.shape)} {t.dtype}")
         h = ctypes.c_void_p()
-        _check(L.sphq_create_v(rows, cols, bits, radius_bits, K, cb.data_ptr(), sc.data_ptr(),
-                               of.data_ptr(), ctypes.byref(h)))
+        _check(L.sphq_create_dim(rows, cols, dim, bits, radius_bits, K, cb.data_ptr(),
+                                 sc.data_ptr(), of.data_ptr(), ctypes.byref(h)))
         self._h = h
         self.rows, self.cols, self.bits, self.K = rows, cols, bits, K
-        self.radius_bits = radius_bits
+        self.radius_bits, self.dim = radius_bits, dim
         self.device = torch.device("cuda", torch.cuda.current_device())
 
     @property
@@ -154,8 +158,8 @@ class SphqMatrix:
         return self._h.value
 
     def pack(self, sign, idx, rcode, stream=None) -> None:
-        """sign/idx/rcode: (rows, cols/8) uint8 / uint16(int16) / uint8 device tensors."""
-        nv = self.cols // 8
+        """sign/idx/rcode: (rows, cols/dim) uint8 / uint16(int16) / uint8 device tensors."""
+        nv = self.cols // self.dim
         for t in (sign, idx, rcode):
             if tuple(t.shape) != (self.rows, nv) or not t.is_cuda or not t.is_contiguous():
                 raise ValueError("codes must be contiguous CUDA tensors of shape (rows, cols/8)")
@@ -196,10 +200,11 @@ class SphqMatrix:
         L = load()
         h = ctypes.c_void_p()
         _check(L.sphq_import(blob, len(blob), ctypes.byref(h)))
-        _, _, rows, cols, bits, vbits, K, _ = struct.unpack_from("<4sIiiiiii", blob, 0)
+        _, _, rows, cols, bits, vbits, K, dim = struct.unpack_from("<4sIiiiiii", blob, 0)
         m = cls.__new__(cls)
         m._h = h
         m.rows, m.cols, m.bits, m.K, m.radius_bits = rows, cols, bits, K, vbits
+        m.dim = dim or 8
         m.device = torch.device("cuda", torch.cuda.current_device())
         return m
 
