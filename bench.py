@@ -848,6 +848,15 @@ def run_report(args):
             for m in mats:
                 m.close()
             torch.cuda.empty_cache()
+    # 16-D study: random 32-byte entry reads from a 512 KiB codebook
+    from paper_2609_24875_gb300 import sphq as _sphq
+    rates = {name: _sphq.study_gather16(mode) for mode, name in
+             ((0, "l2"), (1, "cluster_dsmem_4"), (2, "local_smem"))}
+    # 16-D W2 payload per vector: 16 sign + 14 index + 4 radius bits + params
+    need = hbm_peak * 1e9 / (34 / 8 + 4 * 16 / 128)
+    rep["gather16_study"] = {k: {"G_entries/s": round(v / 1e9, 1),
+                                 "max_hbm_frac_16d": round(min(1.0, v / need), 3)}
+                             for k, v in rates.items()}
     rep["prefill_gemm"] = gemm_report(hbm_peak)
     rep["encode"] = encode_report()
     # CPU oracle on the 1024^2 matrix: single thread and all cores

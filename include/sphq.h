@@ -317,6 +317,20 @@ sphq_status sphq_import(const void* buf, size_t size, sphq_handle* out);
 sphq_status sphq_selftest_wait_timeout(sphq_handle h, sphq_stream stream);
 
 /*
+ * sphq_study_gather16 -- measurement behind the 16-D decision (Tab. 7): the
+ * rate, in entries per second over the whole GPU, of random 32-byte reads
+ * from a 2^14-entry (512 KiB) table -- the 16-D W2 codebook -- held
+ *   mode 0: in global memory (L2-resident),
+ *   mode 1: split over a thread-block cluster of 4 CTAs (128 KiB of shared
+ *           memory each) and read through distributed shared memory,
+ *   mode 2: as mode 1 but every CTA reads its own quarter only (the local
+ *           shared-memory gather of the 8-D kernels, for reference).
+ * `iters` reads per thread; synchronous; allocates and frees its buffers.
+ * (No counterpart in the paper.)
+ */
+sphq_status sphq_study_gather16(int mode, int iters, double* entries_per_s);
+
+/*
  * sphq_decode -- write the decoded weights W_hat (rows x cols fp16, device
  * pointer, 16-byte aligned) on `stream`.  Bit-exact with Eq. (7) + Eq. (4) as
  * stated at the top of this header.  For verification; the GEMV never

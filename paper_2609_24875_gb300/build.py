@@ -16,7 +16,7 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libsphq.so")
 SOURCES = ["sphq_api.cu", "sphq_gemv.cu", "sphq_gemv_splits.cu", "sphq_gemm.cu",
-           "sphq_encode.cu", "sphq_io.cu", "sphq_noalloc.cu"]
+           "sphq_encode.cu", "sphq_io.cu", "sphq_study.cu", "sphq_noalloc.cu"]
 HEADERS = ["sphq_layout.cuh", "sphq_gemv_kernel.cuh", "sphq_umma.cuh", "sphq_internal.h"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xptxas", "-v",

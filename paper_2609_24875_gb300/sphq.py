@@ -75,6 +75,8 @@ def load() -> ctypes.CDLL:
         L.sphq_export.restype = i32
         L.sphq_import.argtypes = [vp, sz, ctypes.POINTER(vp)]
         L.sphq_import.restype = i32
+        L.sphq_study_gather16.argtypes = [i32, i32, ctypes.POINTER(ctypes.c_double)]
+        L.sphq_study_gather16.restype = i32
         L.sphq_selftest_wait_timeout.argtypes = [vp, vp]
         L.sphq_selftest_wait_timeout.restype = i32
         L.sphq_encode.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp]
@@ -336,3 +338,11 @@ class SphqMatrix:
             self.close()
         except Exception:
             pass
+
+
+def study_gather16(mode: int, iters: int = 4096) -> float:
+    """sphq_study_gather16: random 32-byte reads per second from a 512 KiB
+    table (0: L2, 1: cluster shared memory, 2: local shared memory)."""
+    rate = ctypes.c_double()
+    _check(load().sphq_study_gather16(mode, iters, ctypes.byref(rate)))
+    return rate.value
