@@ -192,9 +192,10 @@ sphq_status sphq_gemv(sphq_handle h, const void* x, void* y, int batch, sphq_str
  *
  * With page-locked (pinned) host buffers that are mapped into the device
  * address space (cudaHostAlloc / cudaHostRegister with mapping, the default
- * on this platform) and aligned like sphq_gemv's (x 16 bytes, y 4 bytes), the
- * GEMV kernel reads x and writes y in host memory directly over the
- * CPU-GPU link: one launch on `stream`, no copy operations.  Otherwise it
+ * on this platform) and aligned like sphq_gemv's (x 16 bytes, y 4 bytes), a
+ * small kernel reads x once over the CPU-GPU link into a device staging
+ * buffer owned by the handle and the GEMV writes y in host memory directly:
+ * two launches on `stream`, no copy operations.  Otherwise it
  * enqueues a copy of x into a device staging buffer owned by the handle, the
  * GEMV, and a copy of y back to y_host; with pageable buffers the CUDA runtime
  * makes those copies synchronous.  Either way the call returns without

@@ -667,6 +667,13 @@ sphq_status sphq_check(sphq_handle h, sphq_stream stream) {
   return SPHQ_OK;
 }
 
+// Copies n16 16-byte words from host memory (a mapped pinned buffer read over
+// the CPU-GPU link) into a device buffer.
+__global__ void stage_x_kernel(const uint4* __restrict__ src, uint4* __restrict__ dst, int n16) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n16) dst[i] = src[i];
+}
+
 // Device address of a page-locked, mapped host buffer, or null for any other
 // pointer (pageable memory, device memory, or an error from the query).
 static const void* mapped_device_pointer(const void* p) {
@@ -690,14 +697,21 @@ sphq_status sphq_gemv_host(sphq_handle h, const void* x_host, void* y_host, int 
   if (!x_host || !y_host) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemv_host: NULL buffer");
   if (!h->packed) return set_error(SPHQ_ERR_NOT_PACKED, "sphq_gemv_host: handle not packed");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  // Page-locked host buffers mapped into the device address space: the
-  // kernel reads x and writes y over the CPU-GPU link directly (coherent on
-  // Grace-Blackwell), with no separate copy operations on the stream.
+  // Page-locked host buffers mapped into the device address space: one small
+  // kernel reads x over the CPU-GPU link (coherent on Grace-Blackwell) into
+  // the handle's device staging buffer -- once, instead of every CTA of the
+  // GEMV fetching its slice across the link -- and the GEMV writes y into
+  // host memory directly.  No copy-engine operations on the stream.
   const void* xd = mapped_device_pointer(x_host);
   void* yd = const_cast<void*>(mapped_device_pointer(y_host));
   if (xd && yd && reinterpret_cast<uintptr_t>(xd) % 16 == 0 &&
-      reinterpret_cast<uintptr_t>(yd) % 4 == 0)
-    return launch_gemv(h, xd, yd, batch, s);
+      reinterpret_cast<uintptr_t>(yd) % 4 == 0) {
+    const int n16 = batch * h->cols * 2 / 16;
+    stage_x_kernel<<<(n16 + 255) / 256, 256, 0, s>>>(static_cast<const uint4*>(xd),
+                                                    static_cast<uint4*>(h->xstage), n16);
+    SPHQ_CUDA(cudaGetLastError(), "stage x");
+    return launch_gemv(h, h->xstage, yd, batch, s);
+  }
   SPHQ_CUDA(cudaMemcpyAsync(h->xstage, x_host, (size_t)batch * h->cols * 2,
                             cudaMemcpyHostToDevice, s), "copy x to device");
   sphq_status st = launch_gemv(h, h->xstage, h->ystage, batch, s);
