@@ -39,6 +39,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <mutex>
 
 #include "sphq_gemv_kernel.cuh"
 #include "sphq_umma.cuh"
@@ -331,12 +332,18 @@ sphq_status launch_encode(sphq_handle h, const float* w, uint8_t* sign, uint16_t
   const size_t need = 1024 + (size_t)a.off_bar + 64;
   const size_t smem = std::max(need, (size_t)120 * 1024);
   if (smem > (size_t)optin) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_encode: shared memory");
-  static bool attr_done = false;
-  if (!attr_done) {
-    e = cudaFuncSetAttribute(encode_vectors_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             optin);
-    if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(encode)");
-    attr_done = true;
+  {
+    // once per device (the attribute belongs to the kernel on the current device)
+    static std::mutex mu;
+    static bool done[64] = {};
+    std::lock_guard<std::mutex> lock(mu);
+    if (h->device < 0 || h->device >= 64) return set_error(SPHQ_ERR_DEVICE, "device index out of range");
+    if (!done[h->device]) {
+      e = cudaFuncSetAttribute(encode_vectors_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               optin);
+      if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(encode)");
+      done[h->device] = true;
+    }
   }
   const long long ntiles = (a.nvec + kEncTile - 1) / kEncTile;
   const unsigned grid = (unsigned)std::max(1LL, std::min<long long>(ntiles, h->sm_count));

@@ -472,13 +472,17 @@ sphq_status launch_gemm(sphq_handle h, const void* x, void* y, int batch, cudaSt
   cudaError_t e;
   const void* kfn = gemm_kernel_ptr(h->fmt, mt, bk, bn);
   {
+    // the attribute belongs to the kernel on the current device: once per
+    // (device, kernel)
     static std::mutex mu;
-    static bool done[16][3][2][2] = {};
+    static bool done[64][16][3][2][2] = {};
     std::lock_guard<std::mutex> lock(mu);
-    if (!done[h->fmt][mt][bk == 64][bn == 256]) {
+    if (h->device < 0 || h->device >= 64) return set_error(SPHQ_ERR_DEVICE, "device index out of range");
+    bool& d = done[h->device][h->fmt][mt][bk == 64][bn == 256];
+    if (!d) {
       e = cudaFuncSetAttribute(kfn, cudaFuncAttributeMaxDynamicSharedMemorySize, optin);
       if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(gemm)");
-      done[h->fmt][mt][bk == 64][bn == 256] = true;
+      d = true;
     }
   }
   // activations: a batch x cols fp16 tensor, boxes of 128 rows x 64 columns
