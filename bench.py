@@ -50,6 +50,8 @@ import numpy as np  # noqa: E402
 import sphq_inputs as inp  # noqa: E402
 
 METRIC = "batch-1 W2/W3 GEMV effective GB/s and % of GB300 HBM peak; µs/token for linear stack"
+WORKLOAD = ("W2+W3 GEMV sweep 4096^2 and 8192^2 + 28-layer W2/W3 decoder linear stack, "
+            "batch 1")
 UNIT = "GB/s"
 
 # DRAM traffic of the GEMV kernel per launch relative to its algorithmic bytes,
@@ -341,8 +343,7 @@ def run_gpu(args, world, rank, local):
         "steps": K, "warmup": args.warmup, "ms_per_step": round(total_ms / K, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "fp16 in, fp32 accumulate (2.25/3.125-bit codes)", "data": "synthetic",
-        "config": {"workload": "W2+W3 GEMV sweep 4096^2 and 8192^2 + 28-layer W2/W3 "
-                               "decoder linear stack, batch 1",
+        "config": {"workload": WORKLOAD,
                    "pools": {s["name"]: s["P"] for s in shapes},
                    "l2_policy": "inputs larger than L2: each pool > 2x L2 and each stack "
                                 "> 10x L2, distinct buffers per GEMV",
@@ -455,31 +456,37 @@ def make_stack(args, bits, dev, stream, fused=False):
 
 def oracle_sample(seconds: float, threads: int):
     """Times the float64 oracle (decode + matvec, row by row) on row samples of
-    the sweep's four shapes until about `seconds` have elapsed.  Returns
+    the step's matrices -- the sweep's four shapes and the W2 / W3 decoder
+    projections of the stack -- until about `seconds` have elapsed.  Returns
     (GB/s over the sampled rows' share of the algorithmic bytes, description)."""
     import oracle
     oracle.set_threads(threads)
     per_shape = []
     for sid, (bits, n) in enumerate(inp.SQUARE_SWEEP):
-        rows = 64
-        codes, x = inp.random_codes(bits, rows, n, seed=inp.seed_for(1, sid))
-        per_shape.append((bits, n, codes, x))
+        codes, x = inp.random_codes(bits, 64, n, seed=inp.seed_for(1, sid))
+        per_shape.append((bits, n, n, codes, x))
+    for bits in (2, 3):
+        for i, (_, rows, cols) in enumerate(inp.DECODER_PROJ):
+            codes, x = inp.random_codes(bits, 32, cols, seed=inp.seed_for(4, 10 * bits + i))
+            per_shape.append((bits, rows, cols, codes, x))
     done_bytes, t_total, rows_done = 0.0, 0.0, 0
     budget = seconds / len(per_shape)
-    for bits, n, codes, x in per_shape:
-        full_bytes = n * n * (7 * bits + 4) / 64 + n * n / 128 * 4 + (1 << (7 * bits - 8)) * 16 + 4 * n
+    for bits, rows, cols, codes, x in per_shape:
+        full_bytes = (rows * cols * (7 * bits + 4) / 64 + rows * cols / 128 * 4
+                      + (1 << (7 * bits - 8)) * 16 + 2 * (rows + cols))
         t0 = time.perf_counter()
         while True:
             oracle.decode_gemv(codes.codebook, codes.scale, codes.offset, codes.sign,
                                codes.idx, codes.rcode, x)
             rows_done += codes.rows
-            done_bytes += full_bytes * codes.rows / n
+            done_bytes += full_bytes * codes.rows / rows
             if time.perf_counter() - t0 > budget:
                 break
         t_total += time.perf_counter() - t0
     gbs = done_bytes / t_total / 1e9
-    desc = (f"float64 oracle decode+matvec on 64-row samples of the W2/W3 4096^2 and 8192^2 "
-            f"matrices, {rows_done} rows in {t_total:.1f} s, bytes scaled to the rows' share")
+    desc = (f"float64 oracle decode+matvec on row samples (64 / 32 rows) of the W2/W3 4096^2 and "
+            f"8192^2 matrices and the W2/W3 decoder projections, {rows_done} rows in "
+            f"{t_total:.1f} s, bytes scaled to the rows' share")
     return gbs, desc, t_total
 
 
@@ -504,8 +511,7 @@ def run_reference(args, world, rank):
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(dt / args.steps * 1e3, 2), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": "W2+W3 GEMV sweep 4096^2 and 8192^2, batch 1",
-                   "parallelism": "cpu oracle"},
+        "config": {"workload": WORKLOAD, "parallelism": "cpu oracle"},
         "hbm_frac": round(value / hbm_peak, 6),
         "cpu_baseline": {"value": round(value, 4), "unit": UNIT, "cores": threads,
                          "kind": "oracle", "sample": desc},
