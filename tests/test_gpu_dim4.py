@@ -123,3 +123,14 @@ def test_code_validation_and_unsupported_entry_points():
     with pytest.raises(SphqError) as e:
         SphqMatrix(16, 128, 2, G.to_dev(cb16), G.to_dev(sc), G.to_dev(sc), K=1 << 14, dim=16)
     assert e.value.status == 2
+
+
+def test_8192_square_sampled_rows():
+    n = 8192
+    codes, x = inp.random_codes_dim(4, 2, n, n, seed=48, B=4)
+    m = make4(codes)
+    rs = G.sample_rows(n, 64, seed=5)
+    assert np.array_equal(G.decoded_bits(m, rs), ref_decode(codes, rs))
+    for B in (1, 4):
+        check(m, codes, x[:B], rs)
+    m.close()

@@ -106,3 +106,14 @@ def test_argument_errors():
     with pytest.raises(ValueError):
         m.encode(w)
     m.close()
+
+
+def test_8192_square_w3_sampled_rows():
+    # the size `bench.py --report` times (encode), checked on sampled rows
+    bits, v, K = 3, 4, 8192
+    n = 8192
+    cb = _codebook(K, 12)
+    w = inp.gaussian_weights(n, n, seed=inp.seed_for(1, 4)).astype(np.float32)
+    m = _matrix(bits, v, K, n, n, cb)
+    _check(m, w, cb, v, rows=G.sample_rows(n, 12, seed=n))
+    m.close()

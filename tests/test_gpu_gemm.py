@@ -154,3 +154,20 @@ def test_argument_errors():
         m.gemm_ptr(xb.data_ptr(), y.data_ptr(), 0, 0)
     assert e.value.status == 2
     m.close()
+
+
+@pytest.mark.parametrize("fmt", FORMATS[:3], ids=FIDS[:3])
+@pytest.mark.parametrize("rows,cols,batch", [(8192, 8192, 4096), (18944, 3584, 2048)])
+def test_report_sizes_sampled(fmt, rows, cols, batch):
+    # the sizes `bench.py --report` times (prefill_gemm), in the launch shape
+    # the library chooses for them, checked on sampled rows
+    bits, v, K = fmt
+    codes, _ = inp.random_codes(bits, rows, cols, seed=31 + rows + v, radius_bits=v, K=K)
+    rng = np.random.default_rng(rows + bits)
+    x = inp.to_f16_bits(rng.standard_normal((batch, cols)))
+    m = G.make_matrix(codes)
+    assert m.gemm_shape(batch)["act_tiles"] == 2
+    check_gemm(m, codes, x, G.sample_rows(rows, 24, seed=rows))
+    m.check()
+    m.close()
+    torch.cuda.empty_cache()
