@@ -256,11 +256,13 @@ def run_gpu(args, world, rank, local):
 
     def step(evs=None):
         for i, s in enumerate(parts):
+            torch.cuda.nvtx.range_push(s["name"])   # NVTX ranges for timeline tools
             if evs is not None:
                 evs[i][0].record(stream)
             s["graph"].replay()
             if evs is not None:
                 evs[i][1].record(stream)
+            torch.cuda.nvtx.range_pop()
 
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):

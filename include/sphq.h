@@ -42,6 +42,10 @@
 extern "C" {
 #endif
 
+/* Host logging: with the environment variable SPHQ_LOG set (and not "0"),
+ * sphq_create prints the format and the GEMV launch plans and sphq_gemm its
+ * launch shape to stderr. */
+
 /* Opaque handle to one quantised weight matrix resident in device memory. */
 typedef struct sphq_handle_s* sphq_handle;
 

@@ -4,6 +4,7 @@
 #include <cuda_runtime.h>
 
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <string>
 
@@ -20,6 +21,16 @@ static thread_local std::string g_last_error;
 constexpr size_t kZeroBytes = 256;
 
 void clear_error() { g_last_error.clear(); }
+
+// Host logging to stderr when the environment variable SPHQ_LOG is set
+// (to anything but "0").
+bool log_enabled() {
+  static const bool on = [] {
+    const char* v = std::getenv("SPHQ_LOG");
+    return v && *v && std::strcmp(v, "0") != 0;
+  }();
+  return on;
+}
 
 sphq_status set_error(sphq_status s, const std::string& msg) {
   g_last_error = msg;
@@ -465,6 +476,17 @@ static sphq_status create_impl(int rows, int cols, int dim, int bits, int radius
     return fail(cuda_error(e, "copy offset"));
   sphq_status st = make_gemv_plans(h);
   if (st != SPHQ_OK) return fail(st);
+  if (log_enabled()) {
+    std::fprintf(stderr, "sphq: matrix %d x %d, %d-D, split %d/%d/%d (format %d), unit %zu B\n",
+                 rows, cols, dim, dim, dbits, radius_bits, fmt, h->unit_bytes);
+    for (int b = 1; b <= SPHQ_MAX_BATCH; ++b) {
+      const GemvPlan& p = h->plan[b];
+      std::fprintf(stderr,
+                   "sphq:   gemv batch %d: grid %d, cluster %d x %d, <= %d row tiles per cluster, "
+                   "%d warps, %zu B shared, mode %d\n",
+                   b, p.grid, p.nclusters, p.csize, p.tmax, p.warps_per_cta, p.smem, p.mode);
+    }
+  }
   if (h->ws_floats > 0 &&
       (e = cudaMalloc(&h->ws, h->ws_floats * sizeof(float))) != cudaSuccess)
     return fail(cuda_error(e, "cudaMalloc(workspace)"));

@@ -37,6 +37,7 @@
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 
+#include <cstdio>
 #include <mutex>
 
 #include "sphq_gemv_kernel.cuh"
@@ -469,6 +470,11 @@ sphq_status launch_gemm(sphq_handle h, const void* x, void* y, int batch, cudaSt
   if (!g.mt) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm: no shape fits this device");
   const int mt = g.mt, bk = g.bk, bn = g.bn;
   const GemmSmem& L = g.L;
+  if (log_enabled())
+    std::fprintf(stderr,
+                 "sphq: gemm %d x %d, batch %d: %d activation tile(s) x %d weight rows, "
+                 "%d-column stages x %d, %zu B shared\n",
+                 h->rows, h->cols, batch, mt, bn, bk, L.stages, L.total);
   cudaError_t e;
   const void* kfn = gemm_kernel_ptr(h->fmt, mt, bk, bn);
   {

@@ -56,6 +56,7 @@ struct sphq_handle_s {
 namespace sphq {
 
 void clear_error();
+bool log_enabled();  // SPHQ_LOG set: host logging to stderr
 sphq_status set_error(sphq_status s, const std::string& msg);
 sphq_status cuda_error(cudaError_t e, const char* what);
 
