@@ -808,13 +808,19 @@ def run_report(args):
         if cold:
             cu = cold_us(mats[0], xd, ys[0], batch, stream, flush)
             e["cold_us"] = round(cu, 3)
+            # the same graph of back-to-back launches without programmatic
+            # dependent launch (each GEMV waits for the previous to finish)
+            for m in mats:
+                m.set_pdl(False)
+            e["us_no_pdl"] = round(steady_us(mats, xd, ys, batch, stream), 3)
         for m in mats:
             m.close()
         torch.cuda.empty_cache()
         return e
 
     rep = {"steady": "median of 20 graph replays over a pool > 2x L2, back-to-back with PDL",
-           "cold": "one call after writing a 2x L2 buffer, events around the call"}
+           "cold": "one call after writing a 2x L2 buffer, events around the call",
+           "us_no_pdl": "steady state with plain stream-ordered launches (sphq_set_pdl 0)"}
     rep["cfg0_w2_1024"] = entry(2, 1024, 1024, inp.seed_for(0, 0), 1, cold=True)
     rep["cfg1_sweep"] = {f"W{b} {n}x{n}": entry(b, n, n, inp.seed_for(1, i), 1, cold=True)
                          for i, (b, n) in enumerate(inp.SQUARE_SWEEP)}

@@ -385,6 +385,19 @@ sphq_status sphq_get_plan(sphq_handle h, int batch, sphq_plan_info* out);
  */
 sphq_status sphq_set_cluster_size(sphq_handle h, int batch, int cluster_size);
 
+/*
+ * sphq_set_pdl -- launch this handle's GEMVs as programmatic dependent
+ * launches (enabled = 1, the default) or as plain stream-ordered launches
+ * (0).  (No counterpart in the paper: a launch option.)  With it, a GEMV's
+ * CTAs may start while the previous kernel on the stream is finishing and
+ * load their codes and codebook before waiting for it; the activations are
+ * read only after that kernel completes, so results are the same either way
+ * (bit for bit).  Applies to sphq_gemv, sphq_gemv_noalloc and
+ * sphq_gemv_host; launches already enqueued or captured keep their setting.
+ * SPHQ_ERR_INVALID_ARG for a NULL handle or another value.
+ */
+sphq_status sphq_set_pdl(sphq_handle h, int enabled);
+
 /* Release the handle and its device memory.  NULL is accepted.  The caller
  * ensures no kernel using the handle is still running. */
 sphq_status sphq_destroy(sphq_handle h);

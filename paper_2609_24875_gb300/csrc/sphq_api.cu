@@ -297,7 +297,7 @@ using namespace sphq;
 
 extern "C" {
 
-int sphq_version(void) { return 10200; }
+int sphq_version(void) { return 10300; }
 
 sphq_status sphq_get_plan(sphq_handle h, int batch, sphq_plan_info* out) {
   g_last_error.clear();
@@ -331,6 +331,15 @@ sphq_status sphq_set_cluster_size(sphq_handle h, int batch, int cluster_size) {
   if (dev != h->device)
     return set_error(SPHQ_ERR_DEVICE, "sphq_set_cluster_size: current device is not the handle's");
   return set_gemv_cluster_size(h, batch, cluster_size);
+}
+
+sphq_status sphq_set_pdl(sphq_handle h, int enabled) {
+  g_last_error.clear();
+  if (!h) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_set_pdl: NULL handle");
+  if (enabled != 0 && enabled != 1)
+    return set_error(SPHQ_ERR_INVALID_ARG, "sphq_set_pdl: enabled must be 0 or 1");
+  h->pdl = enabled != 0;
+  return SPHQ_OK;
 }
 
 const char* sphq_last_error(void) { return g_last_error.c_str(); }

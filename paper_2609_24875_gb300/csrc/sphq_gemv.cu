@@ -86,21 +86,23 @@ static SmemLayout smem_layout(const sphq_handle_s* h, int mode, int warps, int c
   return L;
 }
 
+// Without `pdl` the launch waits for the previous work on the stream to
+// finish; the kernel's dependency wait then returns at once.
 static cudaLaunchConfig_t launch_config(const GemvPlan& p, cudaStream_t s,
-                                        cudaLaunchAttribute (&attr)[2]) {
+                                        cudaLaunchAttribute (&attr)[2], bool pdl = true) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.grid);
   cfg.blockDim = dim3(p.warps_per_cta * 32);
   cfg.dynamicSmemBytes = p.smem;
   cfg.stream = s;
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  attr[1].id = cudaLaunchAttributeClusterDimension;
-  attr[1].val.clusterDim.x = (unsigned)p.csize;
-  attr[1].val.clusterDim.y = 1;
-  attr[1].val.clusterDim.z = 1;
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)p.csize;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 2;
+  cfg.numAttrs = pdl ? 2 : 1;
   return cfg;
 }
 
@@ -243,7 +245,7 @@ sphq_status launch_gemv(sphq_handle h, const void* x, void* y, int batch, cudaSt
   a.off_recv = p.off_recv;
   a.off_bar = p.off_bar;
   cudaLaunchAttribute attr[2];
-  cudaLaunchConfig_t cfg = launch_config(p, s, attr);
+  cudaLaunchConfig_t cfg = launch_config(p, s, attr, h->pdl);
   void* args[] = {&a};
   cudaError_t e = cudaLaunchKernelExC(&cfg, select_kernel(h->fmt, p.mode), args);
   if (e != cudaSuccess) return cuda_error(e, "gemv launch");

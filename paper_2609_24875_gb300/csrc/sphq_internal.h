@@ -47,6 +47,7 @@ struct sphq_handle_s {
   void* xstage = nullptr;      // SPHQ_MAX_BATCH x cols fp16 (sphq_gemv_host)
   void* ystage = nullptr;      // SPHQ_MAX_BATCH x rows fp16
   void* zeros = nullptr;       // 256 B of zeros (activations of non-supplying lanes)
+  bool pdl = true;             // sphq_set_pdl: GEMV launched as a programmatic dependent
   int gemm_mt = 0;             // sphq_set_gemm_shape: activation tiles (0 = automatic)
   int gemm_bn = 0;             //   weight rows per CTA tile (0 = automatic)
   bool packed = false;

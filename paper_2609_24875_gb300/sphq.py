@@ -101,6 +101,8 @@ def load() -> ctypes.CDLL:
         L.sphq_get_plan.restype = i32
         L.sphq_set_cluster_size.argtypes = [vp, i32, i32]
         L.sphq_set_cluster_size.restype = i32
+        L.sphq_set_pdl.argtypes = [vp, i32]
+        L.sphq_set_pdl.restype = i32
         _lib = L
     return _lib
 
@@ -327,6 +329,10 @@ class SphqMatrix:
     def set_cluster_size(self, batch: int, cluster_size: int) -> None:
         """Fix the cluster size of the launch shape for `batch` (0: automatic)."""
         _check(load().sphq_set_cluster_size(self._h, batch, cluster_size))
+
+    def set_pdl(self, enabled: bool) -> None:
+        """GEMVs as programmatic dependent launches (default) or plain ones."""
+        _check(load().sphq_set_pdl(self._h, 1 if enabled else 0))
 
     def close(self) -> None:
         if getattr(self, "_h", None) is not None and self._h.value:

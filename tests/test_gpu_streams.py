@@ -157,3 +157,35 @@ def test_sphq_log_reports_formats_and_launch_shapes():
                        timeout=300)
     assert r.returncode == 0, r.stderr[-2000:]
     assert "sphq:" not in r.stderr
+
+
+@pytest.mark.parametrize("bits,rows,cols,batch", [(2, 1000, 2048, 1), (3, 720, 1024, 2),
+                                                  (3, 512, 1536, 8)])
+def test_pdl_off_gives_the_same_result(bits, rows, cols, batch):
+    """sphq_set_pdl(0): plain stream-ordered launches, same result bit for bit,
+    also inside a captured graph of back-to-back GEMVs that feed each other."""
+    codes, x = inp.random_codes(bits, rows, cols, seed=4400 + rows + batch, B=batch)
+    m = G.make_matrix(codes)
+    xd = G.x_dev(x)
+    y_on = _lone(m, xd)
+    m.set_pdl(False)
+    y_off = _lone(m, xd)
+    assert torch.equal(y_on, y_off)
+    # a chain: each GEMV reads the previous one's output (square matrix)
+    sq, _ = inp.random_codes(bits, 256, 256, seed=4500 + batch, B=batch)
+    ms = G.make_matrix(sq)
+    x0 = G.x_dev(inp.make_x(np.random.default_rng(batch), batch, 256))
+    outs = {}
+    for pdl in (True, False):
+        ms.set_pdl(pdl)
+        bufs = [x0.clone()] + [torch.empty_like(x0) for _ in range(4)]
+        for i in range(4):
+            ms.gemv(bufs[i], y=bufs[i + 1])
+        torch.cuda.synchronize()
+        outs[pdl] = [b.clone() for b in bufs]
+    for a, b in zip(outs[True], outs[False]):
+        # bit patterns: late links of the chain may overflow fp16
+        assert torch.equal(a.view(torch.int16), b.view(torch.int16))
+    for m_ in (m, ms):
+        m_.check()
+        m_.close()
