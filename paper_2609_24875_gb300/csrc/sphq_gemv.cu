@@ -159,16 +159,17 @@ static sphq_status make_plan(sphq_handle h, int batch, int forced, int optin, Ge
           continue;
         }
         const int waves = (nclusters + ncl - 1) / ncl;
-        // Estimated time per launch (us), from GB300 measurements of
-        // back-to-back launches: a fixed part (launch, staging, reduction,
-        // and the wait for the slowest CTA of a cluster, which grows with the
-        // cluster size) plus ~0.06 us per unit per CTA; strips of fewer than
-        // four tiles keep fewer units in flight per warp (about twice the time
-        // per unit with one tile per cluster).
-        const double fixed = csize == 1 ? 2.6 : csize == 2 ? 3.7 : csize == 4 ? 4.6 : 5.3;
-        const double shallow = 1.0 + 0.33 * (kStrip - std::min(tmax, kStrip));
+        // Estimated time per launch (us), fitted to GB300 measurements of
+        // back-to-back launches at every cluster size on the decoder and
+        // square shapes (W2 and W3, batch 1, 2, 8): a fixed part (launch,
+        // staging, reduction, and the wait for the slowest CTA of a cluster)
+        // plus ~0.05 us per unit per CTA; one-tile strips do not share
+        // activation loads between two units and keep fewer units in flight
+        // per warp.
+        const double fixed = csize == 1 ? 2.6 : csize == 2 ? 3.6 : csize == 4 ? 3.6 : 5.0;
+        const double shallow = 1.0 + 0.66 * (kStrip - std::min(tmax, kStrip));
         const double cost =
-            fixed + waves * 0.06 * tmax * ((h->ng + csize - 1) / csize) * shallow;
+            fixed + waves * 0.05 * tmax * ((h->ng + csize - 1) / csize) * shallow;
         if (best.grid == 0 || cost < best_cost - 1e-9) {
           p.grid = nclusters * csize;
           p.nclusters = nclusters;
