@@ -523,35 +523,34 @@ def run_reference(args, world, rank):
 
 
 def run_case(spec: str, pool: int, launches: int):
-    """Profiling driver: `bits:n[:batch]` -> `pool` distinct packed n x n
-    matrices, `launches` GEMVs round robin on one stream, no timing (for
-    running under ncu).  bits `3v3` selects W3 with 3-bit radius codes, `dDvV`
-    the 8/D/V split (e.g. `d7v2`)."""
+    """Profiling driver: `bits:n[:batch]` or `bits:RxC[:batch]` -> `pool`
+    distinct packed n x n (R x C) matrices, `launches` GEMVs round robin on one
+    stream, no timing (for running under ncu).  bits `3v3` selects W3 with
+    3-bit radius codes, `dDvV` the 8/D/V split (e.g. `d7v2`)."""
     import torch
 
-    head, *rest = spec.split(":")
+    head, size, *rest = spec.split(":")
     bits, vbits, K = parse_split(head)
-    parts = [int(v) for v in rest]
-    n = parts[0]
-    batch = parts[1] if len(parts) > 1 else 1
+    rows, n = (int(v) for v in size.split("x")) if "x" in size else (int(size), int(size))
+    batch = int(rest[0]) if rest else 1
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     from paper_2609_24875_gb300 import SphqMatrix
-    codes, x = inp.random_codes(bits, n, n, seed=1, B=batch, radius_bits=vbits, K=K)
+    codes, x = inp.random_codes(bits, rows, n, seed=1, B=batch, radius_bits=vbits, K=K)
     t = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int16) if a.dtype == np.uint16 else a)).to(dev)
     mats = []
     for _ in range(pool):
-        m = SphqMatrix(n, n, bits, t(codes.codebook), t(codes.scale), t(codes.offset),
+        m = SphqMatrix(rows, n, bits, t(codes.codebook), t(codes.scale), t(codes.offset),
                        radius_bits=vbits, K=K)
         m.pack(t(codes.sign), t(codes.idx), t(codes.rcode))
         mats.append(m)
     xd = t(x).view(torch.float16)
-    ys = [torch.empty((batch, n), dtype=torch.float16, device=dev) for _ in mats]
+    ys = [torch.empty((batch, rows), dtype=torch.float16, device=dev) for _ in mats]
     s = torch.cuda.current_stream()
     for i in range(launches):
         mats[i % pool].gemv_ptr(xd.data_ptr(), ys[i % pool].data_ptr(), batch, s.cuda_stream)
     torch.cuda.synchronize()
-    print(f"case W{bits} V={vbits} {n}x{n} batch {batch}: {launches} launches over {pool} "
+    print(f"case W{bits} V={vbits} {rows}x{n} batch {batch}: {launches} launches over {pool} "
           "matrices done")
 
 
@@ -900,7 +899,7 @@ def main():
     ap.add_argument("--no-stack", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
-    ap.add_argument("--case", default="", help="profiling driver: bits:n[:batch], no timing")
+    ap.add_argument("--case", default="", help="profiling driver: bits:n[:batch] or bits:RxC[:batch], no timing")
     ap.add_argument("--pool", type=int, default=4, help="--case: distinct matrices")
     ap.add_argument("--launches", type=int, default=8, help="--case: GEMV launches")
     ap.add_argument("--gemm-case", default="",

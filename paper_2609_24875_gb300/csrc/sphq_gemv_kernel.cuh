@@ -442,17 +442,13 @@ __device__ __forceinline__ int warp_item(int T, int ngc, int w) {
   return u < 2 * full ? (u + 1) / 2 : full + (u - 2 * full);
 }
 
-// Warps of CTA `rank` (of csize) whose items cover strip ts, as a bit mask.
+// Whether warp w of CTA `rank` (of csize) has items in strip ts.
 template <int WARPS>
-__device__ __forceinline__ uint32_t cover_mask(int ng, int T, int rank, int csize, int ts) {
+__device__ __forceinline__ bool covers(int ng, int T, int rank, int csize, int ts, int w) {
   const int lo = (int)((unsigned)ng * rank / csize), hi = (int)((unsigned)ng * (rank + 1) / csize);
   const int ngc = hi - lo;
-  uint32_t m = 0;
-  for (int w = 0; w < WARPS; ++w) {
-    const int a0 = warp_item<WARPS>(T, ngc, w), a1 = warp_item<WARPS>(T, ngc, w + 1);
-    if (a0 < a1 && a0 < (ts + 1) * ngc && a1 > ts * ngc) m |= 1u << w;
-  }
-  return m;
+  const int a0 = warp_item<WARPS>(T, ngc, w), a1 = warp_item<WARPS>(T, ngc, w + 1);
+  return a0 < a1 && a0 < (ts + 1) * ngc && a1 > ts * ngc;
 }
 
 // ---------------------------------------------------------------------------
@@ -594,20 +590,37 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
     mbar_arrive_expect_tx(bar_cb, a.cb_bytes);
     for (uint32_t o = 0; o < a.cb_bytes; o += 32768u)
       bulk_g2s(smem_u32(smem) + o, a.cbimage + o, min(32768u, a.cb_bytes - o), bar_cb);
-    // every warp of the cluster that covers an owned tile sends 64 * batch
-    // bytes for it; remember who, for the final sum
-    uint32_t bytes = 0;
-    for (int k = 0; k < nown; ++k)
-      for (int r = 0; r < csize; ++r) {
-        const uint32_t m = cover_mask<WARPS>(a.ng, T, r, csize, (crank + k * csize) / kStrip);
-        masks[k * csize + r] = m;
-        bytes += (uint32_t)__popc(m) * 64u * (uint32_t)a.batch;
+  }
+  // Who covers each owned tile, for the final sum: bit w of
+  // masks[k * csize + r] is set if warp w of rank r has items in the strip of
+  // owned tile k.  One thread per bit (a single thread took microseconds for
+  // the tens of masks of a long tile range); a ballot gathers each mask.
+  static_assert(WARPS < 32 && 32 % WARPS == 0, "masks are groups of a ballot");
+  {
+    const int total = nown * csize * WARPS;
+    for (int base = warp * 32; base < total; base += WARPS * 32) {
+      const int j = base + lane;
+      bool bit = false;
+      if (j < total) {
+        const int kr = j / WARPS;
+        bit = covers<WARPS>(a.ng, T, kr % csize, csize, (crank + (kr / csize) * csize) / kStrip,
+                            j % WARPS);
       }
-    mbar_arrive_expect_tx(bar_recv, bytes);
+      const uint32_t b = __ballot_sync(0xFFFFFFFFu, bit);
+      if (j < total && j % WARPS == 0)
+        masks[j / WARPS] = (b >> (lane & ~(WARPS - 1))) & ((1u << WARPS) - 1u);
+    }
   }
   if (MODE != kFull && threadIdx.x < 16)  // zero block read by lanes that supply no activations
     reinterpret_cast<uint4*>(smem + a.off_zero)[threadIdx.x] = make_uint4(0, 0, 0, 0);
-  __syncthreads();                  // mbarrier initialisation visible to the CTA
+  __syncthreads();                  // mbarrier initialisation and masks visible to the CTA
+  if (threadIdx.x == 0) {
+    // every covering warp of the cluster sends 64 * batch bytes per owned tile
+    uint32_t n = 0;
+    for (int i = 0; i < nown * csize; ++i) n += (uint32_t)__popc(masks[i]);
+    mbar_arrive_expect_tx(bar_recv, n * 64u * (uint32_t)a.batch);
+  }
+  __syncwarp();
   if (csize > 1) cluster_arrive_relaxed();  // ... and to the cluster (waited on below)
 
   pdl_wait();  // the previous kernel's outputs (our activations) are complete
