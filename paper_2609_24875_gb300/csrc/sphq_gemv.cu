@@ -165,8 +165,13 @@ static sphq_status make_plan(sphq_handle h, int batch, int forced, int optin, Ge
         // staging, reduction, and the wait for the slowest CTA of a cluster)
         // plus ~0.05 us per unit per CTA; one-tile strips do not share
         // activation loads between two units and keep fewer units in flight
-        // per warp.
-        const double fixed = csize == 1 ? 2.6 : csize == 2 ? 3.6 : csize == 4 ? 3.6 : 5.0;
+        // per warp.  Batch 3-8 (full mode: activations read from global
+        // memory, eight partial sums per row through the cluster) pay more
+        // for clusters: one CTA per cluster is the measured best there except
+        // on long rows (3584 x 18944).
+        const double fixed = mode == kFull
+                                 ? (csize == 1 ? 2.6 : csize == 8 ? 5.8 : 4.4)
+                                 : (csize == 1 ? 2.6 : csize == 2 ? 3.6 : csize == 4 ? 3.6 : 5.0);
         const double shallow = 1.0 + 0.66 * (kStrip - std::min(tmax, kStrip));
         const double cost =
             fixed + waves * 0.05 * tmax * ((h->ng + csize - 1) / csize) * shallow;
