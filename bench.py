@@ -55,9 +55,9 @@ WORKLOAD = ("W2+W3 GEMV sweep 4096^2 and 8192^2 + 28-layer W2/W3 decoder linear 
 UNIT = "GB/s"
 
 # DRAM traffic of the GEMV kernel per launch relative to its algorithmic bytes,
-# from ncu captures of the 8192x8192 batch-1 launches (profiles/
-# gemv_w2_8192_b1_full.md, gemv_w3_8192_b1_full.md), valid for the kernel
-# sources with this digest only; the roofline reports traffic null otherwise.
+# from one-pass ncu captures (dram__bytes_read.sum + dram__bytes_write.sum) of
+# the 8192x8192 batch-1 launches, valid for the kernel sources with this
+# digest only; the roofline reports traffic null otherwise.
 TRAFFIC_SOURCES = ("paper_2609_24875_gb300/csrc/sphq_gemv_kernel.cuh",
                    "paper_2609_24875_gb300/csrc/sphq_gemv.cu",
                    "paper_2609_24875_gb300/csrc/sphq_layout.cuh")
@@ -102,7 +102,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "50"],
+                 "--format=csv,noheader,nounits", "-lms", "10"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.t = threading.Thread(target=self._read, daemon=True)
             self.t.start()
@@ -721,6 +721,21 @@ def gemm_report(hbm_peak):
     return out
 
 
+def study_gather16(mode: int, iters: int = 4096) -> float:
+    """Random 32-byte reads per second from a 512 KiB table (0: L2, 1: cluster
+    shared memory, 2: local shared memory), from the profiling library
+    libsphq_study.so (built next to libsphq.so, not part of its C ABI)."""
+    import ctypes
+    lib = ctypes.CDLL(os.path.join(ROOT, "paper_2609_24875_gb300", "libsphq_study.so"))
+    lib.sphq_study_gather16.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.POINTER(ctypes.c_double)]
+    lib.sphq_study_gather16.restype = ctypes.c_int
+    rate = ctypes.c_double()
+    rc = lib.sphq_study_gather16(mode, iters, ctypes.byref(rate))
+    if rc != 0:
+        raise RuntimeError(f"sphq_study_gather16 failed ({rc})")
+    return rate.value
+
+
 def steady_us(mats, xd, ys, batch, stream, reps=20):
     """Median over `reps` graph replays of the mean time per GEMV of a CUDA
     graph of back-to-back launches over the pool."""
@@ -862,8 +877,7 @@ def run_report(args):
                 m.close()
             torch.cuda.empty_cache()
     # 16-D study: random 32-byte entry reads from a 512 KiB codebook
-    from paper_2609_24875_gb300 import sphq as _sphq
-    rates = {name: _sphq.study_gather16(mode) for mode, name in
+    rates = {name: study_gather16(mode) for mode, name in
              ((0, "l2"), (1, "cluster_dsmem_4"), (2, "local_smem"))}
     # 16-D W2 payload per vector: 16 sign + 14 index + 4 radius bits + params
     need = hbm_peak * 1e9 / (34 / 8 + 4 * 16 / 128)

@@ -231,11 +231,12 @@ sphq_status sphq_gemv_host(sphq_handle h, const void* x_host, void* y_host, int 
  * launch.)
  *
  * Arguments, numerics and asynchrony are those of sphq_gemv.  It calls no
- * cudaMalloc, cudaFree or other allocating routine.  Limits: the matrix may
- * have at most 16384 row tiles (rows <= 262144) and may need at most
- * 4128768 bytes of partial sums; larger shapes return SPHQ_ERR_UNSUPPORTED
- * with a message naming the limit.  The current device must be the handle's
- * device (else SPHQ_ERR_DEVICE).
+ * cudaMalloc, cudaFree or other allocating routine.  Limits: a launch plan
+ * that reduces through the array may cover at most 16384 row tiles (rows <=
+ * 262144) and need at most 4128768 bytes of partial sums; beyond that the
+ * call returns SPHQ_ERR_UNSUPPORTED with a message naming the limit.  The
+ * current plans reduce on chip, so every shape sphq_gemv takes is accepted.
+ * The current device must be the handle's device (else SPHQ_ERR_DEVICE).
  *
  * The first call on each device looks up the array's device address (one
  * cudaGetSymbolAddress with that device current) and caches it; make that
@@ -320,20 +321,6 @@ sphq_status sphq_import(const void* buf, size_t size, sphq_handle* out);
  * For tests of the failure detection.  (No counterpart in the paper.)
  */
 sphq_status sphq_selftest_wait_timeout(sphq_handle h, sphq_stream stream);
-
-/*
- * sphq_study_gather16 -- measurement behind the 16-D decision (Tab. 7): the
- * rate, in entries per second over the whole GPU, of random 32-byte reads
- * from a 2^14-entry (512 KiB) table -- the 16-D W2 codebook -- held
- *   mode 0: in global memory (L2-resident),
- *   mode 1: split over a thread-block cluster of 4 CTAs (128 KiB of shared
- *           memory each) and read through distributed shared memory,
- *   mode 2: as mode 1 but every CTA reads its own quarter only (the local
- *           shared-memory gather of the 8-D kernels, for reference).
- * `iters` reads per thread; synchronous; allocates and frees its buffers.
- * (No counterpart in the paper.)
- */
-sphq_status sphq_study_gather16(int mode, int iters, double* entries_per_s);
 
 /*
  * sphq_decode -- write the decoded weights W_hat (rows x cols fp16, device

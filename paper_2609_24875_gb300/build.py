@@ -1,4 +1,5 @@
-"""Builds libsphq.so, the sm_103a CUDA library behind include/sphq.h.
+"""Builds libsphq.so, the sm_103a CUDA library behind include/sphq.h, and
+libsphq_study.so, the benchmark's 16-D gather-rate study (not part of the C ABI).
 
 Plain nvcc, one translation unit per source compiled in parallel, static CUDA
 runtime, no cmake.  The output lands next to this file (in-tree) and is
@@ -16,7 +17,9 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libsphq.so")
 SOURCES = ["sphq_api.cu", "sphq_gemv.cu", "sphq_gemv_splits.cu", "sphq_gemm.cu",
-           "sphq_encode.cu", "sphq_io.cu", "sphq_study.cu", "sphq_noalloc.cu"]
+           "sphq_encode.cu", "sphq_io.cu", "sphq_noalloc.cu"]
+STUDY_SRC = os.path.join(CSRC, "study", "gather16.cu")
+STUDY_LIB = os.path.join(HERE, "libsphq_study.so")
 HEADERS = ["sphq_layout.cuh", "sphq_gemv_kernel.cuh", "sphq_umma.cuh", "sphq_internal.h"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xptxas", "-v",
@@ -37,11 +40,11 @@ def _inputs():
 
 
 def up_to_date() -> bool:
-    if not os.path.exists(LIB):
+    if not os.path.exists(LIB) or not os.path.exists(STUDY_LIB):
         return False
     srcs, hdrs = _inputs()
-    t = os.path.getmtime(LIB)
-    return all(os.path.getmtime(p) <= t for p in srcs + hdrs + [__file__])
+    t = min(os.path.getmtime(LIB), os.path.getmtime(STUDY_LIB))
+    return all(os.path.getmtime(p) <= t for p in srcs + hdrs + [STUDY_SRC, __file__])
 
 
 def build(force: bool = False, verbose: bool = False) -> str:
@@ -61,8 +64,18 @@ def build(force: bool = False, verbose: bool = False) -> str:
             f.write(r.stdout + r.stderr)
         return obj
 
-    with cf.ThreadPoolExecutor(max_workers=len(srcs)) as ex:
+    def study():
+        tmp = STUDY_LIB + f".tmp{os.getpid()}"
+        cmd = [cc, *ARCH, *FLAGS, "-shared", "-o", tmp, STUDY_SRC, "-cudart", "static"]
+        r = subprocess.run(cmd, capture_output=True, text=True)
+        if r.returncode != 0:
+            raise RuntimeError(f"nvcc failed on {STUDY_SRC}:\n{r.stdout}\n{r.stderr}")
+        os.replace(tmp, STUDY_LIB)
+
+    with cf.ThreadPoolExecutor(max_workers=len(srcs) + 1) as ex:
+        fut = ex.submit(study)
         objs = list(ex.map(compile_one, srcs))
+        fut.result()
     tmp = LIB + f".tmp{os.getpid()}"
     cmd = [cc, *ARCH, "-shared", "-o", tmp, *objs, "-cudart", "static"]
     r = subprocess.run(cmd, capture_output=True, text=True)

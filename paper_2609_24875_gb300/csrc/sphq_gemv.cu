@@ -81,7 +81,7 @@ static SmemLayout smem_layout(const sphq_handle_s* h, int mode, int warps, int c
   o += (size_t)nown_max * csize * warps * blk;
   o = align_up(o, 8);
   L.bar = o;
-  o += 32 + 4 * (size_t)nown_max * csize;  // three mbarriers, then the cover masks
+  o += 32;  // three mbarriers
   L.total = align_up(o, 16);
   return L;
 }
@@ -250,6 +250,17 @@ sphq_status launch_gemv(sphq_handle h, const void* x, void* y, int batch, cudaSt
   a.zeros = (const uint16_t*)h->zeros;
   a.off_recv = p.off_recv;
   a.off_bar = p.off_bar;
+  int cshift = 0;
+  while ((1 << cshift) < p.csize) ++cshift;
+  a.cshift = cshift;
+  a.tq = h->nrt / p.nclusters;
+  a.tr = h->nrt % p.nclusters;
+  a.gq = h->ng >> cshift;
+  a.gr = h->ng & (p.csize - 1);
+  for (int k = 0; k < 2; ++k) {
+    const unsigned long long d = (unsigned long long)std::max(1, a.gq + k);
+    a.ngc_m[k] = ((1ull << 32) + d - 1) / d;
+  }
   cudaLaunchAttribute attr[2];
   cudaLaunchConfig_t cfg = launch_config(p, s, attr, h->pdl);
   void* args[] = {&a};
@@ -259,11 +270,18 @@ sphq_status launch_gemv(sphq_handle h, const void* x, void* y, int batch, cudaSt
 }
 
 // The kernel reduces on chip and needs no global scratch; the caller's
-// scratch is accepted and left untouched.
+// scratch is accepted and left untouched.  A plan that asked for scratch
+// (ws_floats > 0) would have to pass `ws` and `tickets` to its kernel; no
+// kernel takes them, so such a plan is refused rather than launched on the
+// handle's own buffer.
 sphq_status launch_gemv_scratch(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s,
                                 float* ws, unsigned* tickets) {
   (void)ws;
   (void)tickets;
+  if (h->ws_floats > 0)
+    return set_error(SPHQ_ERR_UNSUPPORTED,
+                     "sphq_gemv_noalloc: this launch plan reduces through scratch that the "
+                     "kernel does not take from the caller");
   return launch_gemv(h, x, y, batch, s);
 }
 

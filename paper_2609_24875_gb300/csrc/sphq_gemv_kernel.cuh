@@ -54,7 +54,13 @@
 //
 // Every wait on an mbarrier gives up after about two seconds, records an
 // error bit in the handle's device flag word and carries on, so a fault in
-// the exchange cannot hang the GPU.
+// the exchange cannot hang the GPU.  On that failure path an owner CTA that
+// gave up may exit while a peer's st.async into its shared memory is still in
+// flight; a remote store to an exited CTA is undefined, so after a reported
+// timeout the results are void and the context should be treated as suspect
+// (the path is never taken when every covering warp sends, which the byte
+// count of the receive barrier guarantees in a correct launch).  A cluster
+// barrier before exit would close the gap but cannot be bounded in time.
 //
 // This header holds the device code; sphq_gemv.cu instantiates it for the W2
 // and W3 formats and holds the launch plans, sphq_gemv_splits.cu instantiates
@@ -89,6 +95,13 @@ struct GemvArgs {
   uint32_t x_pitch;        // bytes between staged activation rows (factored modes)
   uint32_t off_x, off_zero, off_recv, off_bar;  // dynamic smem offsets
   const uint16_t* zeros;   // 256 B of zeros in global memory (batch 3-8 non-suppliers)
+  // Work split, precomputed on the host so that the prologue has no runtime
+  // division: cluster c holds tiles [c*tq + min(c, tr), +tq + (c < tr));
+  // rank r of a cluster holds groups [r*gq + min(r, gr), +gq + (r < gr));
+  // clusters have 2^cshift CTAs; ngc_m[k] = ceil(2^32 / (gq + k)) divides
+  // item indices by the group count.
+  int tq, tr, gq, gr, cshift;
+  unsigned long long ngc_m[2];
 };
 
 // ---------------------------------------------------------------------------
@@ -134,6 +147,28 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
   const uint64_t t0 = globaltimer();
   for (;;) {
     if (mbar_try_wait(bar, parity)) return true;
+    if (globaltimer() - t0 > 2000000000ull) return false;
+  }
+}
+// The same wait without the suspend hint: the thread polls, so it resumes as
+// soon as the phase completes (the GEMV's few one-off waits sit on its
+// critical path).  Gives up after ~2 s.
+__device__ __forceinline__ bool mbar_try_wait_poll(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ bool mbar_wait_poll(uint32_t bar, uint32_t parity) {
+  if (mbar_try_wait_poll(bar, parity)) return true;
+  const uint64_t t0 = globaltimer();
+  for (;;) {
+    if (mbar_try_wait_poll(bar, parity)) return true;
     if (globaltimer() - t0 > 2000000000ull) return false;
   }
 }
@@ -442,15 +477,6 @@ __device__ __forceinline__ int warp_item(int T, int ngc, int w) {
   return u < 2 * full ? (u + 1) / 2 : full + (u - 2 * full);
 }
 
-// Whether warp w of CTA `rank` (of csize) has items in strip ts.
-template <int WARPS>
-__device__ __forceinline__ bool covers(int ng, int T, int rank, int csize, int ts, int w) {
-  const int lo = (int)((unsigned)ng * rank / csize), hi = (int)((unsigned)ng * (rank + 1) / csize);
-  const int ngc = hi - lo;
-  const int a0 = warp_item<WARPS>(T, ngc, w), a1 = warp_item<WARPS>(T, ngc, w + 1);
-  return a0 < a1 && a0 < (ts + 1) * ngc && a1 > ts * ngc;
-}
-
 // ---------------------------------------------------------------------------
 // The kernel
 // ---------------------------------------------------------------------------
@@ -545,43 +571,21 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
   constexpr int UB = Layout<BITS>::kUnitBytes;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int gid = lane >> 2, q = lane & 3;
-  const int csize = (int)(gridDim.x / (unsigned)a.nclusters);
+  const int cshift = a.cshift, csize = 1 << cshift;
   const int crank = csize > 1 ? (int)cluster_rank() : 0;
   const int cid = csize > 1 ? (int)cluster_id() : (int)blockIdx.x;
 
-  // this cluster's row tiles and this CTA's radius groups
-  const int t0 = share_lo(a.nrt, cid, a.nclusters);
-  const int T = share_lo(a.nrt, cid + 1, a.nclusters) - t0;
-  const int g0 = share_lo(a.ng, crank, csize);
-  const int ngc = share_lo(a.ng, crank + 1, csize) - g0;
-  const int nfull = T / kStrip;  // strips with all four tiles
-  const unsigned last_mask = (1u << (T - kStrip * nfull)) - 1u;
-  const int i0 = warp_item<WARPS>(T, ngc, warp), i1 = warp_item<WARPS>(T, ngc, warp + 1);
-
+  // this cluster's row tiles
+  const int t0 = cid * a.tq + min(cid, a.tr);
+  const int T = a.tq + (cid < a.tr ? 1 : 0);
+  const int nown = crank < T ? (T - crank + csize - 1) >> cshift : 0;  // tiles this CTA owns
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + a.off_bar);
-  uint32_t* masks = reinterpret_cast<uint32_t*>(smem + a.off_bar + 32);  // [owned tile][rank]
   const uint32_t bar_cb = smem_u32(&bars[0]), bar_x = smem_u32(&bars[1]),
                  bar_recv = smem_u32(&bars[2]);
-  const int nown = crank < T ? (T - crank + csize - 1) / csize : 0;  // tiles this CTA owns
-
-  // units (t0 + 4s + j, g), j = 0..3, start at strip_base(s, g) + j * UB
-  const size_t gstride = (size_t)a.nrt * UB;
-  auto strip_base = [&](int s, int g) {
-    return a.units + ((size_t)g * a.nrt + t0 + kStrip * s) * UB;
-  };
-  auto strip_mask = [&](int s) { return s < nfull ? kStripMask : last_mask; };
-
-  // first item's units (codes are immutable: no wait needed)
-  Unit<BITS> u[kStrip] = {};
-  int s = i0 < i1 ? i0 / ngc : 0;
-  int g = i0 < i1 ? g0 + i0 % ngc : g0;
-  if (i0 < i1) {
-    const unsigned m0 = strip_mask(s);
-#pragma unroll
-    for (int j = 0; j < kStrip; ++j)
-      if (m0 >> j & 1u) u[j] = load_unit<BITS>(strip_base(s, g) + j * UB, lane);
-  }
-
+  // The codebook copy goes first: it is the longest transfer of the
+  // prologue.  Every warp of the cluster sends one block per tile of the
+  // cluster (its partial sums, or -0.0, the additive identity, for tiles
+  // outside its items), so the receive barrier expects a fixed byte count.
   if (threadIdx.x == 0) {
     mbar_init(bar_cb, 1);
     mbar_init(bar_x, 1);
@@ -590,37 +594,44 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
     mbar_arrive_expect_tx(bar_cb, a.cb_bytes);
     for (uint32_t o = 0; o < a.cb_bytes; o += 32768u)
       bulk_g2s(smem_u32(smem) + o, a.cbimage + o, min(32768u, a.cb_bytes - o), bar_cb);
+    mbar_arrive_expect_tx(bar_recv, (uint32_t)(nown * csize * WARPS) * 64u * (uint32_t)a.batch);
   }
-  // Who covers each owned tile, for the final sum: bit w of
-  // masks[k * csize + r] is set if warp w of rank r has items in the strip of
-  // owned tile k.  One thread per bit (a single thread took microseconds for
-  // the tens of masks of a long tile range); a ballot gathers each mask.
-  static_assert(WARPS < 32 && 32 % WARPS == 0, "masks are groups of a ballot");
-  {
-    const int total = nown * csize * WARPS;
-    for (int base = warp * 32; base < total; base += WARPS * 32) {
-      const int j = base + lane;
-      bool bit = false;
-      if (j < total) {
-        const int kr = j / WARPS;
-        bit = covers<WARPS>(a.ng, T, kr % csize, csize, (crank + (kr / csize) * csize) / kStrip,
-                            j % WARPS);
-      }
-      const uint32_t b = __ballot_sync(0xFFFFFFFFu, bit);
-      if (j < total && j % WARPS == 0)
-        masks[j / WARPS] = (b >> (lane & ~(WARPS - 1))) & ((1u << WARPS) - 1u);
-    }
+
+  // this CTA's radius groups and this warp's items
+  const int g0 = crank * a.gq + min(crank, a.gr);
+  const int ngc = a.gq + (crank < a.gr ? 1 : 0);
+  const unsigned long long ngc_m = a.ngc_m[crank < a.gr ? 1 : 0];
+  // v / ngc for 0 <= v < T * ngc: a multiply by the rounded-up reciprocal,
+  // corrected by one where it overshoots
+  auto div_ngc = [&](int v) {
+    int d = (int)(((unsigned long long)(unsigned)v * ngc_m) >> 32);
+    return d * ngc > v ? d - 1 : d;
+  };
+  const int nfull = T / kStrip;  // strips with all kStrip tiles
+  const unsigned last_mask = (1u << (T - kStrip * nfull)) - 1u;
+  const int i0 = warp_item<WARPS>(T, ngc, warp), i1 = warp_item<WARPS>(T, ngc, warp + 1);
+
+  // units (t0 + kStrip s + j, g), j < kStrip, start at strip_base(s, g) + j * UB
+  const size_t gstride = (size_t)a.nrt * UB;
+  auto strip_base = [&](int s, int g) {
+    return a.units + ((size_t)g * a.nrt + t0 + kStrip * s) * UB;
+  };
+  auto strip_mask = [&](int s) { return s < nfull ? kStripMask : last_mask; };
+
+  // first item's units (codes are immutable: no wait needed)
+  Unit<BITS> u[kStrip] = {};
+  int s = i0 < i1 ? div_ngc(i0) : 0;
+  int g = i0 < i1 ? g0 + (i0 - s * ngc) : g0;
+  if (i0 < i1) {
+    const unsigned m0 = strip_mask(s);
+#pragma unroll
+    for (int j = 0; j < kStrip; ++j)
+      if (m0 >> j & 1u) u[j] = load_unit<BITS>(strip_base(s, g) + j * UB, lane);
   }
+
   if (MODE != kFull && threadIdx.x < 16)  // zero block read by lanes that supply no activations
     reinterpret_cast<uint4*>(smem + a.off_zero)[threadIdx.x] = make_uint4(0, 0, 0, 0);
-  __syncthreads();                  // mbarrier initialisation and masks visible to the CTA
-  if (threadIdx.x == 0) {
-    // every covering warp of the cluster sends 64 * batch bytes per owned tile
-    uint32_t n = 0;
-    for (int i = 0; i < nown * csize; ++i) n += (uint32_t)__popc(masks[i]);
-    mbar_arrive_expect_tx(bar_recv, n * 64u * (uint32_t)a.batch);
-  }
-  __syncwarp();
+  __syncthreads();                  // mbarrier initialisation visible to the CTA
   if (csize > 1) cluster_arrive_relaxed();  // ... and to the cluster (waited on below)
 
   pdl_wait();  // the previous kernel's outputs (our activations) are complete
@@ -632,8 +643,8 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
                a.x + (size_t)b * a.cols + (size_t)g0 * kGroupCols, row_bytes, bar_x);
   }
   if (csize > 1) cluster_wait();  // every CTA's receive mbarrier is initialised
-  bool ok = mbar_wait(bar_cb, 0);
-  if (MODE != kFull) ok &= mbar_wait(bar_x, 0);
+  bool ok = mbar_wait_poll(bar_cb, 0);
+  if (MODE != kFull) ok &= mbar_wait_poll(bar_x, 0);
   if (!ok && lane == 0) atomicOr(a.flag, 2);
 
   SmemCodebook cb;
@@ -690,9 +701,9 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
     for (int j = 0; j < kStrip; ++j) {
       const int tau = s * kStrip + j;
       if (tau < T) {
-        const int owner = tau % csize;
+        const int owner = tau & (csize - 1);
         const uint32_t slot =
-            recv_base + 4u * (uint32_t)((((tau / csize) * csize + crank) * WARPS + warp) * kBlk);
+            recv_base + 4u * (uint32_t)(((((tau >> cshift) << cshift) + crank) * WARPS + warp) * kBlk);
         send_partial<MODE>(mapa(slot, (uint32_t)owner), mapa(bar_recv, (uint32_t)owner), acc[j],
                            lane, a.batch);
       }
@@ -701,10 +712,27 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
     ++s;
     g = g0;
   }
-  // Owned tiles (tau = crank + k * csize): wait for every covering warp of
-  // the cluster, then sum their blocks in (rank, warp) order and write y.
+  // -0.0 blocks for the cluster's tiles outside this warp's items (tiles
+  // [tau_lo, tau_hi) got its partial sums): 16 bytes per lane, 64 bytes per
+  // batch row
+  {
+    const int w0 = warp_item<WARPS>(T, ngc, warp), w1 = warp_item<WARPS>(T, ngc, warp + 1);
+    const int tau_lo = w0 < w1 ? div_ngc(w0) * kStrip : 0;
+    const int tau_hi = w0 < w1 ? min(T, (div_ngc(w1 - 1) + 1) * kStrip) : 0;
+  for (int tau = 0; tau < T; ++tau) {
+    if (tau >= tau_lo && tau < tau_hi) continue;
+    const uint32_t slot =
+        recv_base + 4u * (uint32_t)(((((tau >> cshift) << cshift) + crank) * WARPS + warp) * kBlk);
+    const uint32_t owner = (uint32_t)(tau & (csize - 1));
+    if (lane < 4 * a.batch)
+      st_async16(mapa(slot, owner) + 16u * (uint32_t)lane, make_float4(-0.f, -0.f, -0.f, -0.f),
+                 mapa(bar_recv, owner));
+  }
+  }
+  // Owned tiles (tau = crank + k * csize): wait for every warp of the
+  // cluster, then sum their blocks in (rank, warp) order and write y.
   if (nown == 0) return;
-  if (!mbar_wait(bar_recv, 0) && threadIdx.x == 0) atomicOr(a.flag, 2);
+  if (!mbar_wait_poll(bar_recv, 0) && threadIdx.x == 0) atomicOr(a.flag, 2);
   const float* recv = reinterpret_cast<const float*>(smem + a.off_recv);
   for (int e = threadIdx.x; e < nown * kBlk; e += WARPS * 32) {
     const int k = e / kBlk, i = e % kBlk;
@@ -712,10 +740,8 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
     if (b >= a.batch || r >= a.rows) continue;
     float sum = 0.f;
     for (int rk = 0; rk < csize; ++rk) {
-      const uint32_t m = masks[k * csize + rk];
 #pragma unroll
-      for (int w = 0; w < WARPS; ++w)
-        if (m >> w & 1u) sum += recv[(((size_t)k * csize + rk) * WARPS + w) * kBlk + i];
+      for (int w = 0; w < WARPS; ++w) sum += recv[(((size_t)k * csize + rk) * WARPS + w) * kBlk + i];
     }
     a.y[(size_t)b * a.rows + r] = f32_to_h_rn(sum);
   }

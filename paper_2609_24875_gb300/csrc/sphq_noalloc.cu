@@ -57,8 +57,10 @@ extern "C" sphq_status sphq_gemv_noalloc(sphq_handle h, const void* x, void* y, 
   if (!y || reinterpret_cast<uintptr_t>(y) % 4)
     return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemv_noalloc: y must be a 4-byte aligned pointer");
   if (!h->packed) return set_error(SPHQ_ERR_NOT_PACKED, "sphq_gemv_noalloc: handle not packed");
-  if ((size_t)h->nrt * sizeof(unsigned) > kTicketBytes ||
-      h->ws_floats * sizeof(float) > kPartialBytes)
+  // The limit binds only a plan that reduces through global scratch; the
+  // current plans reduce on chip and take any shape sphq_gemv takes.
+  if (h->ws_floats > 0 && ((size_t)h->nrt * sizeof(unsigned) > kTicketBytes ||
+                           h->ws_floats * sizeof(float) > kPartialBytes))
     return set_error(SPHQ_ERR_UNSUPPORTED,
                      "sphq_gemv_noalloc: the matrix needs more split-K scratch than the fixed "
                      "4 MiB device array holds (at most 16384 row tiles of 16 rows and "

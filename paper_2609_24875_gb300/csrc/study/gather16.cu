@@ -4,11 +4,34 @@
 // shared memory of a thread-block cluster.  These kernels measure the rate of
 // random 32-byte entry reads each way, next to the local shared-memory gather
 // the 8-D kernels use, on a table of that size.  No counterpart in the paper.
+//
+// A profiling tool of the benchmark (`bench.py --report`), built as its own
+// library (libsphq_study.so); it is not part of the sphq C ABI.
 #include <cuda_runtime.h>
 
-#include "sphq_gemv_kernel.cuh"
+#include <cstdint>
 
-namespace sphq {
+namespace sphq_study {
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() {
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ uint32_t mapa(uint32_t addr, uint32_t rank) {
+  uint32_t d;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(d) : "r"(addr), "r"(rank));
+  return d;
+}
 
 constexpr int kStudyThreads = 256;
 constexpr uint32_t kStudyEntries = 1u << 14;   // 16-D W2 codebook: 2^14 x 32 B
@@ -82,31 +105,30 @@ __global__ void __launch_bounds__(kStudyThreads) study_dsmem_kernel(const uint4*
   if (acc == 0x12345678u) out[tid] = acc;
 }
 
-}  // namespace sphq
+}  // namespace sphq_study
 
-using namespace sphq;
+using namespace sphq_study;
 
 extern "C" {
 
 // Runs study `mode` (0: L2, 1: cluster shared memory, 2: local shared memory)
-// with `iters` reads per thread on every SM and returns the rate in entries
+// with `iters` reads per thread on every SM and stores the rate in entries
 // read per second (events around one launch after a warm-up launch).
-sphq_status sphq_study_gather16(int mode, int iters, double* entries_per_s) {
-  clear_error();
-  if (!entries_per_s || iters < 1 || mode < 0 || mode > 2)
-    return set_error(SPHQ_ERR_INVALID_ARG, "sphq_study_gather16: bad argument");
+// Returns 0 on success, 1 for a bad argument, else the CUDA error code.
+int sphq_study_gather16(int mode, int iters, double* entries_per_s) {
+  if (!entries_per_s || iters < 1 || mode < 0 || mode > 2) return 1;
   int dev = 0, sms = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  if (e != cudaSuccess) return cuda_error(e, "sphq_study_gather16: device");
+  if (e != cudaSuccess) return (int)e;
   uint4* table = nullptr;
   uint32_t* out = nullptr;
   const size_t tbytes = (size_t)kStudyEntries * kStudyEntryBytes;
   const int ctas = (sms / 4) * 4 * 2;  // two CTAs per SM, whole clusters of 4
-  if ((e = cudaMalloc(&table, tbytes)) != cudaSuccess) return cuda_error(e, "cudaMalloc(table)");
+  if ((e = cudaMalloc(&table, tbytes)) != cudaSuccess) return (int)e;
   if ((e = cudaMalloc(&out, (size_t)ctas * kStudyThreads * 4)) != cudaSuccess) {
     cudaFree(table);
-    return cuda_error(e, "cudaMalloc(out)");
+    return (int)e;
   }
   cudaMemset(table, 0x5A, tbytes);
   const uint32_t smem = kStudyEntries / 4 * kStudyEntryBytes;
@@ -150,10 +172,10 @@ sphq_status sphq_study_gather16(int mode, int iters, double* entries_per_s) {
   cudaEventDestroy(e1);
   cudaFree(table);
   cudaFree(out);
-  if (e != cudaSuccess) return cuda_error(e, "sphq_study_gather16");
+  if (e != cudaSuccess) return (int)e;
   const double threads = (double)(mode == 0 ? ctas : ctas / 2) * kStudyThreads;
   *entries_per_s = threads * iters / (ms * 1e-3);
-  return SPHQ_OK;
+  return 0;
 }
 
 }  // extern "C"

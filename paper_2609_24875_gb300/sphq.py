@@ -67,6 +67,8 @@ def load() -> ctypes.CDLL:
         L.sphq_pack.restype = i32
         L.sphq_gemv.argtypes = [vp, vp, vp, i32, vp]
         L.sphq_gemv.restype = i32
+        L.sphq_gemv_noalloc.argtypes = [vp, vp, vp, i32, vp]
+        L.sphq_gemv_noalloc.restype = i32
         L.sphq_gemm.argtypes = [vp, vp, vp, i32, vp]
         L.sphq_gemm.restype = i32
         L.sphq_check.argtypes = [vp, vp]
@@ -75,8 +77,6 @@ def load() -> ctypes.CDLL:
         L.sphq_export.restype = i32
         L.sphq_import.argtypes = [vp, sz, ctypes.POINTER(vp)]
         L.sphq_import.restype = i32
-        L.sphq_study_gather16.argtypes = [i32, i32, ctypes.POINTER(ctypes.c_double)]
-        L.sphq_study_gather16.restype = i32
         L.sphq_selftest_wait_timeout.argtypes = [vp, vp]
         L.sphq_selftest_wait_timeout.restype = i32
         L.sphq_encode.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp]
@@ -281,17 +281,17 @@ class SphqMatrix:
         """sphq_gemv_noalloc: the GEMV through the entry point that guarantees
         no allocation on any call, the first included.
         x: (batch, cols) and y: (batch, rows) fp16 CUDA tensors."""
-        L = load()
-        L.sphq_gemv_noalloc.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
-                                        ctypes.c_int, ctypes.c_void_p]
-        L.sphq_gemv_noalloc.restype = ctypes.c_int
+        import torch
         if x.dim() == 1:
             x = x.unsqueeze(0)
         B = x.shape[0]
         if (x.shape[1] != self.cols or not x.is_cuda or not y.is_cuda
                 or not x.is_contiguous() or not y.is_contiguous() or y.numel() != B * self.rows):
             raise ValueError("x must be (batch, cols) and y (batch, rows), contiguous CUDA tensors")
-        _check(L.sphq_gemv_noalloc(self._h, x.data_ptr(), y.data_ptr(), B, _stream_ptr(stream)))
+        if x.element_size() != 2 or y.dtype != torch.float16:
+            raise ValueError("x must hold 2-byte (fp16) elements and y must be float16")
+        _check(load().sphq_gemv_noalloc(self._h, x.data_ptr(), y.data_ptr(), B,
+                                        _stream_ptr(stream)))
         return y
 
     def gemv_host(self, x_host, y_host, stream=None) -> None:
@@ -344,11 +344,3 @@ class SphqMatrix:
             self.close()
         except Exception:
             pass
-
-
-def study_gather16(mode: int, iters: int = 4096) -> float:
-    """sphq_study_gather16: random 32-byte reads per second from a 512 KiB
-    table (0: L2, 1: cluster shared memory, 2: local shared memory)."""
-    rate = ctypes.c_double()
-    _check(load().sphq_study_gather16(mode, iters, ctypes.byref(rate)))
-    return rate.value
