@@ -9,10 +9,10 @@ Workload (one "step" = one pass of the hot path over one batch of input):
   2. one token through the 28-layer x 7-projection linear stack of a
      7B-class decoder at W2 and at W3 (196 distinct matrices each, batch 1).
   Each pool and each stack is captured once as a CUDA graph of back-to-back
-  launches on one stream.  Codes are seeded uniformly random codes of the
-  encoded configuration's shapes (the data path and byte count do not depend
-  on the code values; parity on encoder-produced codes is covered by the
-  tests).
+  launches on one stream.  The sweep's matrices carry encoder codes: the
+  library's GPU encoder (sphq_encode) run on seeded Gaussian weights with
+  outliers (the encoded configuration); the stacks carry seeded uniformly
+  random codes, as the decoder configurations specify.
 
 value    = algorithmic bytes of all GEMVs of a step / device time per step (GB/s)
 sweep    = per shape: us per GEMV, GB/s and fraction of HBM (CUDA events
@@ -214,6 +214,33 @@ def make_pool(bits: int, rows: int, cols: int, n: int, seed: int, dev):
     return mats, xd, codes, x
 
 
+def make_encoded_pool(bits: int, n: int, P: int, seed: int, dev):
+    """P distinct device copies of one n x n matrix whose codes come from the
+    library's GPU encoder (sphq_encode, Eqs. (3), (5)-(7)) run on seeded
+    Gaussian weights N(0, 0.02^2) with 0.1% of the scalars x20 -- the encoded
+    configuration's recipe (sphq_inputs.gaussian_weights), with the random
+    positive-unit codebook and N(0, 1) activations of sphq_inputs.
+    Returns (mats, x on the device, host x)."""
+    import torch
+
+    from paper_2609_24875_gb300 import SphqMatrix
+    cb, x = inp.encoded_inputs_rng(bits, n, seed=seed)
+    w = torch.from_numpy(inp.gaussian_weights(n, n, seed=seed).astype(np.float32)).to(dev)
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int16) if a.dtype == np.uint16 else a)).to(dev)
+    cbd = t(cb)
+    zero = torch.zeros((n, n // 128), dtype=torch.int16, device=dev)
+    m0 = SphqMatrix(n, n, bits, cbd, zero, zero)
+    sg, ix, rc, sc, of = m0.encode(w)
+    del w
+    mats = [m0]
+    for _ in range(P - 1):
+        m = SphqMatrix(n, n, bits, cbd, sc, of)
+        m.pack(sg, ix, rc)
+        mats.append(m)
+    torch.cuda.synchronize()
+    return mats, t(x).view(torch.float16), x
+
+
 def capture(mats, xd, ys, stream):
     import torch
     with torch.cuda.stream(stream):
@@ -244,7 +271,7 @@ def run_gpu(args, world, rank, local):
         P = max(2, int(np.ceil(2 * L2 / probe_bytes)) + 1)
         if args.quick:
             P = 2
-        mats, xd, codes, x = make_pool(bits, n, n, P, inp.seed_for(1, sid), dev)
+        mats, xd, x = make_encoded_pool(bits, n, P, inp.seed_for(1, sid), dev)
         ys = [torch.empty((1, n), dtype=torch.float16, device=dev) for _ in mats]
         g = capture(mats, xd, ys, stream)
         shapes.append(dict(name=f"W{bits} {n}x{n}", bits=bits, n=n, mats=mats, xd=xd, ys=ys,
@@ -832,17 +859,59 @@ def run_report(args):
         torch.cuda.empty_cache()
         return e
 
+    def entry_encoded(bits, n, seed):
+        one = (7 * bits + 4) * n * n // 64
+        P = min(512, max(2, int(np.ceil(2 * L2 / one)) + 1))
+        mats, xd, _ = make_encoded_pool(bits, n, P, seed, dev)
+        ys = [torch.empty((1, n), dtype=torch.float16, device=dev) for _ in mats]
+        b = mats[0].bytes(1)
+        us = steady_us(mats, xd, ys, 1, stream)
+        e = {"us": round(us, 3), "GB/s": round(b / us / 1e3, 1),
+             "hbm_frac": round(b / us / 1e3 / hbm_peak, 4), "bytes": b, "pool": P,
+             "codes": "GPU encoder on Gaussian weights with outliers"}
+        e["cold_us"] = round(cold_us(mats[0], xd, ys[0], 1, stream, flush), 3)
+        for m in mats:
+            m.set_pdl(False)
+        e["us_no_pdl"] = round(steady_us(mats, xd, ys, 1, stream), 3)
+        for m in mats:
+            m.close()
+        torch.cuda.empty_cache()
+        return e
+
     rep = {"steady": "median of 20 graph replays over a pool > 2x L2, back-to-back with PDL",
            "cold": "one call after writing a 2x L2 buffer, events around the call",
            "us_no_pdl": "steady state with plain stream-ordered launches (sphq_set_pdl 0)"}
     rep["cfg0_w2_1024"] = entry(2, 1024, 1024, inp.seed_for(0, 0), 1, cold=True)
-    rep["cfg1_sweep"] = {f"W{b} {n}x{n}": entry(b, n, n, inp.seed_for(1, i), 1, cold=True)
+    rep["cfg1_sweep"] = {f"W{b} {n}x{n}": entry_encoded(b, n, inp.seed_for(1, i))
                          for i, (b, n) in enumerate(inp.SQUARE_SWEEP)}
+    # the same shapes on uniformly random codes: the codebook's bank
+    # conflicts depend on the index distribution, the bytes do not
+    rep["cfg1_random_codes"] = {f"W{b} {n}x{n}": entry(b, n, n, inp.seed_for(1, i), 1)
+                                for i, (b, n) in enumerate(inp.SQUARE_SWEEP)}
     rep["cfg2_w2_proj"] = {f"{nm} {r}x{c}": entry(2, r, c, inp.seed_for(2, i), 1)
                            for i, (nm, r, c) in enumerate(inp.DECODER_PROJ) if nm not in ("v", "up")}
     rep["cfg3_w3_proj_batch"] = {f"{nm} {r}x{c} B{bt}": entry(3, r, c, inp.seed_for(3, i), bt)
                                  for i, (nm, r, c) in enumerate(inp.DECODER_PROJ)
                                  if nm in ("q", "k", "gate", "down") for bt in (1, 2, 4, 8)}
+    # Compute rooflines of the small-batch GEMV beside HBM: the mma.sync rate
+    # the kernel issues its products to (one m16n8k16 per 8 cycles per SM
+    # sub-partition, measured on this part; 8 per 256-vector unit) and the
+    # plain FP32 FMA rate (128 per SM per cycle, 2 flops each), at the SM
+    # clock sampled meanwhile.
+    mhz = sm_clock_mhz()
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    mma_peak = sms * 4 / 8 * mhz * 1e6
+    alu_peak = sms * 128 * 2 * mhz * 1e6
+    for key, e in rep["cfg3_w3_proj_batch"].items():
+        rc_ = key.split()[1].split("x")
+        r, c, bt = int(rc_[0]), int(rc_[1]), int(key.split("B")[-1])
+        mma = 8 * ((r + 15) // 16) * (c // 128)
+        e["mma_frac"] = round(mma / (e["us"] * 1e-6) / mma_peak, 4)
+        e["fp32_alu_frac"] = round(2.0 * bt * r * c / (e["us"] * 1e-6) / alu_peak, 4)
+        fr = {"hbm": e["hbm_frac"], "mma": e["mma_frac"], "fp32_alu": e["fp32_alu_frac"]}
+        e["nearest_roofline"] = max(fr, key=fr.get)
+    rep["compute_rooflines"] = {"sm_mhz": mhz, "mma_sync_per_s": mma_peak,
+                                "fp32_flops_per_s": alu_peak}
     # general bit splits: W3 with 3-bit radius codes (3.00 bits per weight) and
     # the small-codebook splits of the bit-allocation ablation (sign/index/radius)
     rep["w3v3_square"] = {f"W3V3 {n}x{n} B{bt}": entry(3, n, n, inp.seed_for(1, 10 + i), bt,
@@ -886,21 +955,63 @@ def run_report(args):
                              for k, v in rates.items()}
     rep["prefill_gemm"] = gemm_report(hbm_peak)
     rep["encode"] = encode_report()
-    # CPU oracle on the 1024^2 matrix: single thread and all cores
-    import oracle
-    codes, x = inp.random_codes(2, 1024, 1024, seed=inp.seed_for(0, 0))
-    ocpu = {}
-    for th in (1, oracle.max_threads()):
-        oracle.set_threads(th)
-        t0 = time.perf_counter()
-        n = 0
-        while time.perf_counter() - t0 < 3.0:
-            oracle.decode_gemv(codes.codebook, codes.scale, codes.offset, codes.sign, codes.idx,
-                               codes.rcode, x)
-            n += 1
-        ocpu[f"threads_{th}"] = round((time.perf_counter() - t0) / n * 1e6, 1)
-    rep["oracle_cfg0_us_per_gemv"] = ocpu
+    rep["oracle_timing"] = oracle_timing()
     print(json.dumps(rep), flush=True)
+
+
+def sm_clock_mhz() -> float:
+    """Current SM clock from nvidia-smi (the maximum if the query fails)."""
+    try:
+        out = subprocess.run(["nvidia-smi", "-i", "0", "--query-gpu=clocks.sm,clocks.max.sm",
+                              "--format=csv,noheader,nounits"], capture_output=True, text=True,
+                             timeout=10).stdout.strip().split(",")
+        cur, mx = float(out[0]), float(out[1])
+        return cur if cur > 0.5 * mx else mx
+    except (OSError, ValueError, IndexError, subprocess.TimeoutExpired):
+        return 2070.0
+
+
+def oracle_timing(budget_s: float = 0.5):
+    """The float64 CPU oracle (decode + matvec) per configuration, on one thread
+    and on all host cores: us per GEMV for configurations 0-3 (every shape and
+    batch) and us per token for configuration 4 (one decoder layer's seven
+    GEMVs, times 28 layers).  Each GEMV is timed on a sample of its rows until
+    `budget_s` elapses and scaled to the full row count (rows cost the same)."""
+    import oracle
+
+    def per_gemv(bits, rows, cols, batch, threads, seed):
+        sample = min(rows, 256)
+        codes, x = inp.random_codes(bits, sample, cols, seed=seed, B=batch)
+        oracle.set_threads(threads)
+        n, t0 = 0, time.perf_counter()
+        while True:
+            oracle.decode_gemv(codes.codebook, codes.scale, codes.offset, codes.sign,
+                               codes.idx, codes.rcode, x)
+            n += 1
+            if time.perf_counter() - t0 > budget_s:
+                break
+        return (time.perf_counter() - t0) / n * rows / sample * 1e6
+
+    allc = oracle.max_threads()
+    out = {"cores": allc, "method": f"row samples of 256 rows, timed for {budget_s} s each, "
+                                    "scaled to the full matrix; config 4 = one layer x 28"}
+    cases = [("cfg0 W2 1024x1024 B1", 2, 1024, 1024, 1, inp.seed_for(0))]
+    cases += [(f"cfg1 W{b} {n}x{n} B1", b, n, n, 1, inp.seed_for(1, i))
+              for i, (b, n) in enumerate(inp.SQUARE_SWEEP)]
+    cases += [(f"cfg2 W2 {nm} {r}x{c} B1", 2, r, c, 1, inp.seed_for(2, i))
+              for i, (nm, r, c) in enumerate(inp.DECODER_PROJ)]
+    cases += [(f"cfg3 W3 {nm} {r}x{c} B{bt}", 3, r, c, bt, inp.seed_for(3, i))
+              for i, (nm, r, c) in enumerate(inp.DECODER_PROJ) for bt in (1, 2, 4, 8)]
+    for name, b, r, c, bt, seed in cases:
+        out[name] = {"us_1_thread": round(per_gemv(b, r, c, bt, 1, seed), 1),
+                     f"us_{allc}_threads": round(per_gemv(b, r, c, bt, allc, seed), 1)}
+    for bits in (2, 3):
+        layer = {th: sum(per_gemv(bits, r, c, 1, th, inp.seed_for(4, 10 * bits + i))
+                         for i, (_, r, c) in enumerate(inp.DECODER_PROJ)) for th in (1, allc)}
+        out[f"cfg4 W{bits} stack us/token"] = {
+            "us_1_thread": round(layer[1] * inp.DECODER_LAYERS, 1),
+            f"us_{allc}_threads": round(layer[allc] * inp.DECODER_LAYERS, 1)}
+    return out
 
 
 def main():

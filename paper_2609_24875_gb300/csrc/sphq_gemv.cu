@@ -159,22 +159,26 @@ static sphq_status make_plan(sphq_handle h, int batch, int forced, int optin, Ge
           continue;
         }
         const int waves = (nclusters + ncl - 1) / ncl;
-        // Estimated time per launch (us), fitted to GB300 measurements of
-        // back-to-back launches at every cluster size on the decoder and
-        // square shapes (W2 and W3, batch 1, 2, 8): a fixed part (launch,
-        // staging, reduction, and the wait for the slowest CTA of a cluster)
-        // plus ~0.05 us per unit per CTA; one-tile strips do not share
-        // activation loads between two units and keep fewer units in flight
-        // per warp.  Batch 3-8 (full mode: activations read from global
-        // memory, eight partial sums per row through the cluster) pay more
-        // for clusters: one CTA per cluster is the measured best there except
-        // on long rows (3584 x 18944).
+        // Estimated time per launch (us), fitted (least log-regret over a grid
+        // of constants) to GB300 measurements of back-to-back launches at
+        // cluster sizes 1, 2 and 4 on the decoder and square shapes (W2 and
+        // W3, batch 1 and 8): a fixed part (launch, staging, reduction) plus
+        // ~0.02 us per unit of the most loaded CTA; one-tile strips do not
+        // share activation loads between two units.  With the prologue free
+        // of divisions and per-tile cover masks, clusters of 2 and 4 cost no
+        // more than single CTAs in the batch 1-2 modes; clusters of 8 leave
+        // SMs idle (only 15 fit) and are priced out unless nothing else runs.
+        // Batch 3-8 (full mode: activations read from global memory, eight
+        // partial sums per row through the cluster) pays more for clusters.
+        // A plan that needs a second wave of clusters (its shared memory did
+        // not fit at one wave) pays the fixed part again per wave (measured:
+        // W3 18944 x 3584 batch 8 in two waves of clusters of 4, 23.3 us
+        // against 17.6 us in one wave of single CTAs).
         const double fixed = mode == kFull
-                                 ? (csize == 1 ? 2.6 : csize == 8 ? 5.8 : 4.4)
-                                 : (csize == 1 ? 2.6 : csize == 2 ? 3.6 : csize == 4 ? 3.6 : 5.0);
-        const double shallow = 1.0 + 0.66 * (kStrip - std::min(tmax, kStrip));
-        const double cost =
-            fixed + waves * 0.05 * tmax * ((h->ng + csize - 1) / csize) * shallow;
+                                 ? (csize == 1 ? 2.0 : csize == 2 ? 2.3 : csize == 4 ? 3.0 : 5.8)
+                                 : (csize == 8 ? 5.0 : 2.0);
+        const double shallow = 1.0 + 0.33 * (kStrip - std::min(tmax, kStrip));
+        const double cost = fixed * waves + waves * 0.02 * tmax * ((h->ng + csize - 1) / csize) * shallow;
         if (best.grid == 0 || cost < best_cost - 1e-9) {
           p.grid = nclusters * csize;
           p.nclusters = nclusters;

@@ -387,6 +387,44 @@ __device__ __forceinline__ void process_pair_4d(const Unit<kFmt4D>& cur,
   }
 }
 
+// Word m of one unit (the two vectors of slot 4m+q of rows gid and gid+8)
+// against the activations xm of that slot (8-D formats).
+template <int BITS, int MODE>
+__device__ __forceinline__ void process_word(const Unit<BITS>& cur, const UnitConst<BITS>& kc,
+                                             const uint4& xm, int m, int q,
+                                             const SmemCodebook& cb, Acc<MODE>& acc) {
+  uint4 sa, sb;
+  uint32_t qp;
+  word_directions<BITS>(cur, kc, m, q, cb, sa, sb, qp);
+  const uint32_t r = radius_pair<fmt_radius_bits(BITS)>(qp, kc.d2, kc.m2);
+  if constexpr (MODE == kFull) {
+    const uint4 wa = scale_block(sa, bcast_lo(r));
+    const uint4 wb = scale_block(sb, bcast_hi(r));
+    mma16816(acc.d, wa.x, wb.x, wa.y, wb.y, xm.x, xm.y);
+    mma16816(acc.d, wa.z, wb.z, wa.w, wb.w, xm.z, xm.w);
+  } else {
+    float d[4];
+    mma16816_zero(d, sa.x, sb.x, sa.y, sb.y, xm.x, xm.y);
+    mma16816(d, sa.z, sb.z, sa.w, sb.w, xm.z, xm.w);
+    const float rA = h_lo_to_f32(r), rB = h_hi_to_f32(r);
+    acc.f[0][0] = __fmaf_rn(rA, d[0], acc.f[0][0]);
+    acc.f[0][1] = __fmaf_rn(rB, d[2], acc.f[0][1]);
+    if constexpr (MODE == kFactored2) {
+      acc.f[1][0] = __fmaf_rn(rA, d[1], acc.f[1][0]);
+      acc.f[1][1] = __fmaf_rn(rB, d[3], acc.f[1][1]);
+    }
+  }
+}
+
+// The activations of word m of a group for this lane (8-D formats).
+template <int MODE>
+__device__ __forceinline__ uint4 load_x_word(const uint8_t* xp, int m) {
+  if constexpr (MODE == kFull)
+    return ldg_x16(reinterpret_cast<const uint16_t*>(xp) + 32 * m);
+  else
+    return *reinterpret_cast<const uint4*>(xp + 64 * m);
+}
+
 // One unit (16 rows x 128 columns).
 template <int BITS, int MODE>
 __device__ __forceinline__ void process_unit(const Unit<BITS>& cur, const XFrag<BITS>& xf, int q,
@@ -504,16 +542,39 @@ __device__ __forceinline__ void run_item(Unit<BITS> (&u)[kStrip], Acc<MODE> (&ac
                                          const uint8_t* xp, const uint8_t* nb, unsigned nmask,
                                          int lane, int q, const SmemCodebook& cb) {
   constexpr int UB = Layout<BITS>::kUnitBytes;
-  XFrag<BITS> xv;
-  load_x<BITS, MODE>(xv, xp);
-#pragma unroll
-  for (int j = 0; j < kStrip; ++j) {
-    if (j < SIZE) process_unit<BITS, MODE>(u[j], xv, q, cb, acc[j]);
+  auto reload = [&](int j) {
     if (LAST) {
       if (nmask >> j & 1u) u[j] = load_unit<BITS>(nb + j * UB, lane);
     } else if (j < SIZE) {
       u[j] = load_unit<BITS>(nb + j * UB, lane);
     }
+  };
+  if constexpr (BITS == kFmt4D || SIZE == 1) {
+    XFrag<BITS> xv;
+    load_x<BITS, MODE>(xv, xp);
+#pragma unroll
+    for (int j = 0; j < kStrip; ++j) {
+      if (j < SIZE) process_unit<BITS, MODE>(u[j], xv, q, cb, acc[j]);
+      reload(j);
+    }
+  } else {
+    // Two tiles share each word's activations; words 0-1 of both units
+    // first, then unit 0's words 2-3 (its slot is refilled at once, half an
+    // item ahead of use) and unit 1's: at most two words of activations are
+    // live at a time.
+    const UnitConst<BITS> k0 = unit_const<BITS>(u[0], q), k1 = unit_const<BITS>(u[1], q);
+    const uint4 x0 = load_x_word<MODE>(xp, 0), x1 = load_x_word<MODE>(xp, 1);
+    process_word<BITS, MODE>(u[0], k0, x0, 0, q, cb, acc[0]);
+    process_word<BITS, MODE>(u[1], k1, x0, 0, q, cb, acc[1]);
+    process_word<BITS, MODE>(u[0], k0, x1, 1, q, cb, acc[0]);
+    process_word<BITS, MODE>(u[1], k1, x1, 1, q, cb, acc[1]);
+    const uint4 x2 = load_x_word<MODE>(xp, 2), x3 = load_x_word<MODE>(xp, 3);
+    process_word<BITS, MODE>(u[0], k0, x2, 2, q, cb, acc[0]);
+    process_word<BITS, MODE>(u[0], k0, x3, 3, q, cb, acc[0]);
+    reload(0);
+    process_word<BITS, MODE>(u[1], k1, x2, 2, q, cb, acc[1]);
+    process_word<BITS, MODE>(u[1], k1, x3, 3, q, cb, acc[1]);
+    reload(1);
   }
 }
 
