@@ -417,36 +417,79 @@ def codebook_angles(c) -> np.ndarray:
     return theta
 
 
+def sample_directions(w, u):
+    """Radius-weighted sampling of directions (§3.1): 8-D vector i of w is
+    drawn with probability r_i^2 / sum_j r_j^2 by inverse transform of the
+    uniforms u in [0, 1): P = cumsum(r^2) in vector order, the pick for u is
+    the first i with P_i > u * P_last (so vectors of zero radius are never
+    drawn).  r_i^2 = w_0^2 + ... + w_7^2 summed in coordinate order, r_i its
+    square root and the direction d_i = |w_i| / r_i, all in float64 from the
+    float32 weights.  Returns (directions (len(u), 8) float64, indices)."""
+    w = np.asarray(w, np.float32).astype(np.float64).reshape(-1, VEC)
+    r2 = w[:, 0] * w[:, 0]
+    for j in range(1, VEC):
+        r2 = r2 + w[:, j] * w[:, j]
+    P = np.cumsum(r2)
+    if P[-1] <= 0:
+        raise ValueError("all vectors are zero")
+    u = np.asarray(u, np.float64)
+    idx = np.searchsorted(P, u * P[-1], side="right")
+    r = np.sqrt(r2[idx])
+    return np.abs(w[idx]) / r[:, None], idx
+
+
+def kmeans_scores(D, C):
+    """d_i . c_k for every sample and centre in float64, each dot taken in
+    coordinate order (products rounded, then added left to right)."""
+    s = D[:, None, 0] * C[None, :, 0]
+    for j in range(1, VEC):
+        s = s + D[:, None, j] * C[None, :, j]
+    return s
+
+
+def kmeans_step(D, C, chunk: int = 1024):
+    """One iteration of the radius-weighted spherical k-means of §3.1 on
+    sampled unit directions D (S, 8) from centres C (K, 8), float64:
+    every sample goes to the centre of largest cosine (Eq. (5); the scores of
+    kmeans_scores, ties to the lowest index); every centre becomes the
+    normalised sum of its members (an empty cluster keeps its centre).
+    Returns (new centres, assignment z, objective = mean of the assigned
+    scores, taken before the update)."""
+    D = np.asarray(D, np.float64)
+    C = np.asarray(C, np.float64)
+    S = D.shape[0]
+    z = np.empty(S, np.int64)
+    best = np.empty(S, np.float64)
+    for s0 in range(0, S, chunk):
+        sc = kmeans_scores(D[s0:s0 + chunk], C)
+        z[s0:s0 + chunk] = np.argmax(sc, axis=1)
+        best[s0:s0 + chunk] = sc[np.arange(sc.shape[0]), z[s0:s0 + chunk]]
+    sums = np.zeros_like(C)
+    np.add.at(sums, z, D)
+    norms = np.sqrt(np.sum(sums * sums, axis=1))
+    out = C.copy()
+    keep = norms > 0
+    out[keep] = sums[keep] / norms[keep, None]
+    return out, z, float(np.mean(best))
+
+
 def kmeans_codebook(w, K: int, samples: int = 65536, iters: int = 20, seed: int = 0):
     """Radius-weighted spherical k-means initialisation of the positive
     direction codebook (§3.1, App. A step 6; 65,536 samples and 20 iterations
     in the paper's runs).
 
     The 8-D vectors of w (rows, cols) are decomposed by Eq. (3); `samples`
-    directions d_i are drawn with probability proportional to r_i^2; K of them
-    seed the centres; each iteration assigns every sample to the centre of
-    largest cosine (Eq. (5), ties to the lowest index) and replaces each centre
-    by the normalised mean of its members (an empty cluster keeps its centre).
+    directions are drawn with probability proportional to r_i^2
+    (sample_directions, uniforms from a seeded generator); K of them, chosen
+    without replacement, seed the centres; then `iters` steps of kmeans_step.
     Directions are non-negative, so the centres stay in the positive orthant.
     Returns (centres (K, 8) float64, objective per iteration: the mean of
     max_k d_i . c_k over the samples, taken before each update)."""
     rng = np.random.default_rng(seed)
-    w = np.asarray(w, np.float64)
-    _, _, r, d = decompose(w.reshape(-1, VEC))
-    p = r * r
-    if p.sum() <= 0:
-        raise ValueError("all vectors are zero")
-    pick = rng.choice(d.shape[0], size=samples, replace=True, p=p / p.sum())
-    D = d[pick]
+    D, _ = sample_directions(w, rng.random(samples))
     centres = D[rng.choice(samples, size=K, replace=False)].copy()
     history = []
     for _ in range(iters):
-        scores = D @ centres.T
-        z = np.argmax(scores, axis=1)
-        history.append(float(np.mean(scores[np.arange(samples), z])))
-        sums = np.zeros_like(centres)
-        np.add.at(sums, z, D)
-        norms = np.sqrt(np.sum(sums * sums, axis=1))
-        keep = norms > 0
-        centres[keep] = sums[keep] / norms[keep, None]
+        centres, _, obj = kmeans_step(D, centres)
+        history.append(obj)
     return centres, history
