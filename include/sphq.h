@@ -172,6 +172,81 @@ sphq_status sphq_encode(sphq_handle h, const float* w, uint8_t* sign, uint16_t* 
                         uint8_t* rcode, void* scale, void* offset, sphq_stream stream);
 
 /*
+ * Codebook construction (the quantise side, run once per layer before
+ * sphq_encode; the decode GEMV never calls these).  All pointers are device
+ * pointers; every call is asynchronous on `stream` and takes its temporary
+ * buffers from the stream-ordered allocator (cudaMallocAsync / cudaFreeAsync).
+ * Results are deterministic (fixed summation orders).
+ */
+
+/*
+ * sphq_sample_directions -- radius-weighted sampling of §3.1: 8-D vector i of
+ * w is drawn with probability r_i^2 / sum_j r_j^2 (r_i = ||w_i||_2), by
+ * inverse transform of caller-supplied uniforms.
+ *
+ *   w        nvec x 8 fp32 (the weight matrix, rows x cols with cols % 8 == 0,
+ *            read as consecutive 8-D vectors), 4-byte aligned.
+ *   u        samples uniforms in [0, 1), float64.
+ *   dirs     samples x 8 float64 out: d = |w_i| / r_i (non-negative, unit).
+ *   idx      samples int32 out (the drawn vector indices), or NULL.
+ *
+ * r_i^2 sums the squares in coordinate order in float64; prefix sums P of
+ * r^2 run block-wise; the pick for u is the first i with P_i > u * P_total
+ * (vectors of zero radius are never drawn; where u * P_total rounds up to the
+ * total, the last vector of nonzero radius).  SPHQ_ERR_INVALID_ARG for NULL
+ * pointers or non-positive sizes; all-zero weights give NaN directions.
+ */
+sphq_status sphq_sample_directions(const float* w, long long nvec, const double* u, int samples,
+                                   double* dirs, int* idx, sphq_stream stream);
+
+/*
+ * sphq_kmeans_step -- one iteration of the spherical k-means that initialises
+ * the codebook (§3.1, App. A step 6): every sample goes to the centre of
+ * largest cosine (Eq. (5); scores d . c in float64 in coordinate order, each
+ * product and sum rounded once, ties to the lowest index -- found by a
+ * single-precision pass over all centres and exact re-scoring of those within
+ * 1e-5 of the best), then every centre becomes the normalised sum of its
+ * members (an empty cluster keeps its centre).
+ *
+ *   dirs         samples x 8 float64 unit directions (sphq_sample_directions).
+ *   centres      K x 8 float64 centres of norm at most ~1 (unit in practice).
+ *   centres_out  K x 8 float64 out; may equal `centres` (in place).
+ *   assign       samples int32 out (the assignment), or NULL.
+ *   objective    one float64 out: the mean assigned score before the update,
+ *                or NULL.
+ */
+sphq_status sphq_kmeans_step(const double* dirs, int samples, const double* centres, int K,
+                             double* centres_out, int* assign, double* objective,
+                             sphq_stream stream);
+
+/*
+ * sphq_kmeans -- `iters` steps of sphq_kmeans_step in place on `centres`
+ * (K x 8 float64: the initial centres in, the final ones out; the paper runs
+ * 20 iterations on 65,536 samples, §4.1).  objective_history: `iters`
+ * float64 out (the objective of each step), or NULL.
+ */
+sphq_status sphq_kmeans(const double* dirs, int samples, double* centres, int K, int iters,
+                        double* objective_history, sphq_stream stream);
+
+/*
+ * sphq_angle_codebook -- the angle-parameterised codebook of §3.3: for entry
+ * k, Eq. (sph-angle-logits) theta_j = eps + (pi/2 - 2 eps) sigmoid(phi_kj),
+ * j = 1..7, and Eq. (sph-angle-codebook) c_1 = cos theta_1,
+ * c_i = (prod_{j<i} sin theta_j) cos theta_i (2 <= i <= 7),
+ * c_8 = prod_{j<=7} sin theta_j -- non-negative and unit by construction.
+ *
+ *   phi           K x 7 fp32 logits.
+ *   eps           in [0, pi/4).
+ *   codebook_f64  K x 8 float64 out, or NULL.
+ *   codebook_f16  K x 8 fp16 out (round to nearest even: the codebook
+ *                 sphq_create takes), or NULL; not both NULL.
+ *
+ * Computed in float64 with the device's sin, cos and exp.
+ */
+sphq_status sphq_angle_codebook(const float* phi, int K, double eps, double* codebook_f64,
+                                void* codebook_f16, sphq_stream stream);
+
+/*
  * sphq_gemv -- y = W_hat x for a batch of activation rows (§3.4, App. D).
  *
  *   x      batch x cols fp16, device pointer, 16-byte aligned.

@@ -69,6 +69,14 @@ def load() -> ctypes.CDLL:
         L.sphq_gemv.restype = i32
         L.sphq_gemv_noalloc.argtypes = [vp, vp, vp, i32, vp]
         L.sphq_gemv_noalloc.restype = i32
+        L.sphq_sample_directions.argtypes = [vp, ctypes.c_longlong, vp, i32, vp, vp, vp]
+        L.sphq_sample_directions.restype = i32
+        L.sphq_kmeans_step.argtypes = [vp, i32, vp, i32, vp, vp, vp, vp]
+        L.sphq_kmeans_step.restype = i32
+        L.sphq_kmeans.argtypes = [vp, i32, vp, i32, i32, vp, vp]
+        L.sphq_kmeans.restype = i32
+        L.sphq_angle_codebook.argtypes = [vp, i32, ctypes.c_double, vp, vp, vp]
+        L.sphq_angle_codebook.restype = i32
         L.sphq_gemm.argtypes = [vp, vp, vp, i32, vp]
         L.sphq_gemm.restype = i32
         L.sphq_check.argtypes = [vp, vp]
@@ -344,3 +352,76 @@ class SphqMatrix:
             self.close()
         except Exception:
             pass
+
+
+# ---------------------------------------------------------------------------
+# codebook construction (§3.1 sampling and spherical k-means, §3.3 angles)
+# ---------------------------------------------------------------------------
+
+def _dev_f64(t, shape, what):
+    import torch
+    if not t.is_cuda or t.dtype != torch.float64 or not t.is_contiguous() or tuple(t.shape) != shape:
+        raise ValueError(f"{what} must be a contiguous {shape} float64 CUDA tensor")
+
+
+def sample_directions(w, u, stream=None):
+    """sphq_sample_directions: directions of the 8-D vectors of w (float32
+    CUDA tensor, any shape with a multiple of 8 elements) drawn with
+    probability proportional to r^2 by inverse transform of u (float64 CUDA
+    tensor of uniforms in [0, 1)).  Returns (directions (S, 8) float64,
+    indices (S,) int32)."""
+    import torch
+    if not w.is_cuda or w.dtype != torch.float32 or not w.is_contiguous() or w.numel() % 8:
+        raise ValueError("w must be a contiguous float32 CUDA tensor of 8-D vectors")
+    S = u.numel()
+    _dev_f64(u, (S,), "u")
+    dirs = torch.empty((S, 8), dtype=torch.float64, device=w.device)
+    idx = torch.empty((S,), dtype=torch.int32, device=w.device)
+    _check(load().sphq_sample_directions(w.data_ptr(), w.numel() // 8, u.data_ptr(), S,
+                                         dirs.data_ptr(), idx.data_ptr(), _stream_ptr(stream)))
+    return dirs, idx
+
+
+def kmeans_step(dirs, centres, stream=None):
+    """sphq_kmeans_step: one spherical k-means iteration.  Returns (new
+    centres (K, 8) float64, assignment (S,) int32, objective (1,) float64),
+    all CUDA tensors."""
+    import torch
+    S, K = dirs.shape[0], centres.shape[0]
+    _dev_f64(dirs, (S, 8), "dirs")
+    _dev_f64(centres, (K, 8), "centres")
+    out = torch.empty_like(centres)
+    z = torch.empty((S,), dtype=torch.int32, device=dirs.device)
+    obj = torch.empty((1,), dtype=torch.float64, device=dirs.device)
+    _check(load().sphq_kmeans_step(dirs.data_ptr(), S, centres.data_ptr(), K, out.data_ptr(),
+                                   z.data_ptr(), obj.data_ptr(), _stream_ptr(stream)))
+    return out, z, obj
+
+
+def kmeans(dirs, centres, iters: int = 20, stream=None):
+    """sphq_kmeans: `iters` k-means steps from `centres` (copied).  Returns
+    (final centres (K, 8) float64, objective per step (iters,) float64)."""
+    import torch
+    S, K = dirs.shape[0], centres.shape[0]
+    _dev_f64(dirs, (S, 8), "dirs")
+    _dev_f64(centres, (K, 8), "centres")
+    c = centres.clone()
+    hist = torch.empty((max(1, iters),), dtype=torch.float64, device=dirs.device)
+    _check(load().sphq_kmeans(dirs.data_ptr(), S, c.data_ptr(), K, iters, hist.data_ptr(),
+                              _stream_ptr(stream)))
+    return c, hist[:iters]
+
+
+def angle_codebook(phi, eps: float = 1e-4, stream=None):
+    """sphq_angle_codebook: (K, 7) float32 CUDA logits -> (codebook (K, 8)
+    float64, codebook (K, 8) fp16) CUDA tensors."""
+    import torch
+    if not phi.is_cuda or phi.dtype != torch.float32 or not phi.is_contiguous() or \
+            phi.dim() != 2 or phi.shape[1] != 7:
+        raise ValueError("phi must be a contiguous (K, 7) float32 CUDA tensor")
+    K = phi.shape[0]
+    c64 = torch.empty((K, 8), dtype=torch.float64, device=phi.device)
+    c16 = torch.empty((K, 8), dtype=torch.float16, device=phi.device)
+    _check(load().sphq_angle_codebook(phi.data_ptr(), K, float(eps), c64.data_ptr(),
+                                      c16.data_ptr(), _stream_ptr(stream)))
+    return c64, c16
