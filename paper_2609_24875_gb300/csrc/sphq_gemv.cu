@@ -26,10 +26,10 @@ static uint32_t cb_bytes_for(int fmt) {
 
 static int mode_for(int batch) { return batch == 1 ? kFactored1 : batch == 2 ? kFactored2 : kFull; }
 
-static const void* select_kernel(int fmt, int mode) {
+static const void* select_kernel(int fmt, int mode, int strip) {
   return fmt == 2 ? kptr_mode<2>(mode)
-         : fmt == 3 ? kptr_mode<3>(mode)
-         : fmt == kFmtW3V3 ? kptr_mode<kFmtW3V3>(mode)
+         : fmt == 3 ? (strip == 4 ? kptr_mode<3, 4>(mode) : kptr_mode<3, 2>(mode))
+         : fmt == kFmtW3V3 ? (strip == 4 ? kptr_mode<kFmtW3V3, 4>(mode) : kptr_mode<kFmtW3V3, 2>(mode))
                            : split_kernel(fmt, mode);
 }
 
@@ -43,11 +43,13 @@ static sphq_status allow_max_smem(int device, int optin) {
   if (device < 0 || device >= 64) return set_error(SPHQ_ERR_DEVICE, "device index out of range");
   if (done[device]) return SPHQ_OK;
   for (int fmt = 2; fmt <= kFmt4D; ++fmt)
-    for (int mode : kModes) {
-      cudaError_t e = cudaFuncSetAttribute(select_kernel(fmt, mode),
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize, optin);
-      if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute");
-    }
+    for (int mode : kModes)
+      for (int strip : {2, 4}) {
+        if (strip == 4 && !fmt_has_strip4(fmt)) continue;
+        cudaError_t e = cudaFuncSetAttribute(select_kernel(fmt, mode, strip),
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, optin);
+        if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute");
+      }
   done[device] = true;
   return SPHQ_OK;
 }
@@ -118,7 +120,7 @@ static sphq_status make_plan(sphq_handle h, int batch, int forced, int optin, Ge
       int mode = mode_for(batch);
       if (!staged) mode = kFull;
       if (staged && mode == kFull) continue;
-      const void* k = select_kernel(h->fmt, mode);
+      const void* k = select_kernel(h->fmt, mode, 2);  // both strip sizes: same resources
       for (int csize : {1, 2, 4, 8}) {
         if (csize > h->ng) break;
         if (forced && csize != forced) continue;
@@ -177,7 +179,7 @@ static sphq_status make_plan(sphq_handle h, int batch, int forced, int optin, Ge
         const double fixed = mode == kFull
                                  ? (csize == 1 ? 2.0 : csize == 2 ? 2.3 : csize == 4 ? 3.0 : 5.8)
                                  : (csize == 8 ? 5.0 : 2.0);
-        const double shallow = 1.0 + 0.33 * (kStrip - std::min(tmax, kStrip));
+        const double shallow = 1.0 + 0.33 * (2 - std::min(tmax, 2));
         const double cost = fixed * waves + waves * 0.02 * tmax * ((h->ng + csize - 1) / csize) * shallow;
         if (best.grid == 0 || cost < best_cost - 1e-9) {
           p.grid = nclusters * csize;
@@ -189,6 +191,8 @@ static sphq_status make_plan(sphq_handle h, int batch, int forced, int optin, Ge
           p.off_zero = (uint32_t)L.zero;
           p.off_recv = (uint32_t)L.recv;
           p.off_bar = (uint32_t)L.bar;
+          // four-tile strips once a cluster holds three tiles or more (W3)
+          p.strip = fmt_has_strip4(h->fmt) && tmax >= 3 ? 4 : 2;
           best = p;
           best_cost = cost;
         }
@@ -268,7 +272,7 @@ sphq_status launch_gemv(sphq_handle h, const void* x, void* y, int batch, cudaSt
   cudaLaunchAttribute attr[2];
   cudaLaunchConfig_t cfg = launch_config(p, s, attr, h->pdl);
   void* args[] = {&a};
-  cudaError_t e = cudaLaunchKernelExC(&cfg, select_kernel(h->fmt, p.mode), args);
+  cudaError_t e = cudaLaunchKernelExC(&cfg, select_kernel(h->fmt, p.mode, p.strip), args);
   if (e != cudaSuccess) return cuda_error(e, "gemv launch");
   return SPHQ_OK;
 }

@@ -27,9 +27,10 @@
 // Work decomposition.  The row tiles (16 rows) are dealt to thread-block
 // clusters in contiguous, near-equal ranges; every CTA of a cluster takes the
 // same tiles and its own contiguous share of the radius groups (split-K
-// inside the cluster).  Inside a CTA the tiles are cut into strips of two: a
-// work item is (strip, group), i.e. the two units of one group below each
-// other, so the activations of a group are loaded once for two units.  The
+// inside the cluster).  Inside a CTA the tiles are cut into strips (of two
+// tiles for the small-codebook formats, four for W3): a work item is (strip,
+// group), i.e. the units of one group below each other, so the activations of
+// a group are loaded once for all of them.  The
 // items are dealt to the warps in contiguous ranges.  Sums are reduced on
 // chip only and in a fixed order, so results do not depend on scheduling:
 // when a warp leaves a strip it sends its quad-reduced sums of each of the
@@ -74,8 +75,11 @@
 
 namespace sphq {
 
-constexpr int kStrip = 2;  // row tiles per work item (activation reuse)
-constexpr unsigned kStripMask = (1u << kStrip) - 1u;
+// Row tiles per work item (the units that share one load of a group's
+// activations) is the kernel's template parameter S: 2, or 4 for the W3
+// formats, whose 8 warps per SM have the registers for four units in flight
+// (the launch plan takes 4 when a cluster holds at least three row tiles).
+__host__ __device__ constexpr bool fmt_has_strip4(int fmt) { return fmt == 3 || fmt == 4; }
 
 // Radius application modes.
 constexpr int kFactored1 = 1;  // batch 1
@@ -504,15 +508,22 @@ __device__ __forceinline__ void send_partial(uint32_t raddr, uint32_t rbar, Acc<
 
 // First item of warp w when the items of a CTA are dealt to WARPS warps in
 // contiguous ranges of near-equal unit counts: items are (strip, group) in
-// strip-major order, ngc per strip, two units each except in the last strip
-// when the tile count T is odd (one unit).  The unit share of warp w starts
+// strip-major order, ngc per strip, S units each except in the last strip
+// when the tile count T is not a multiple of S (T mod S units).  The unit share of warp w starts
 // at unit U*w/WARPS, rounded to an item boundary.
-template <int WARPS>
+template <int WARPS, int S>
 __device__ __forceinline__ int warp_item(int T, int ngc, int w) {
-  const int full = (T / kStrip) * ngc;    // items of two units
+  const int full = (T / S) * ngc;  // items of S units
+  const int rest = T - S * (T / S);
   const int units = T * ngc;
   const int u = (int)((unsigned)units * (unsigned)w / (unsigned)WARPS);
-  return u < 2 * full ? (u + 1) / 2 : full + (u - 2 * full);
+  if (u < S * full) return (u + S / 2) / S;
+  // the tail strip's items of `rest` (1..S-1) units, without a runtime division
+  const unsigned v = (unsigned)(u - S * full + rest / 2);
+  return full + (rest == 1 ? (int)v
+                 : rest == 2 ? (int)(v >> 1)
+                 : rest == 3 ? (int)(((unsigned long long)v * 0xAAAAAAABull) >> 33)
+                             : 0);
 }
 
 // ---------------------------------------------------------------------------
@@ -537,8 +548,8 @@ __device__ __forceinline__ int share_lo_c(int n, int i) {
 // refilled with the next item's unit j as soon as it is consumed: unit j of
 // the same strip at the next group (base nb), or, for the strip's LAST item,
 // the units in nmask of the warp's next strip.
-template <int BITS, int MODE, int SIZE, bool LAST>
-__device__ __forceinline__ void run_item(Unit<BITS> (&u)[kStrip], Acc<MODE> (&acc)[kStrip],
+template <int BITS, int MODE, int SIZE, bool LAST, int S>
+__device__ __forceinline__ void run_item(Unit<BITS> (&u)[S], Acc<MODE> (&acc)[S],
                                          const uint8_t* xp, const uint8_t* nb, unsigned nmask,
                                          int lane, int q, const SmemCodebook& cb) {
   constexpr int UB = Layout<BITS>::kUnitBytes;
@@ -553,36 +564,41 @@ __device__ __forceinline__ void run_item(Unit<BITS> (&u)[kStrip], Acc<MODE> (&ac
     XFrag<BITS> xv;
     load_x<BITS, MODE>(xv, xp);
 #pragma unroll
-    for (int j = 0; j < kStrip; ++j) {
+    for (int j = 0; j < S; ++j) {
       if (j < SIZE) process_unit<BITS, MODE>(u[j], xv, q, cb, acc[j]);
       reload(j);
     }
   } else {
-    // Two tiles share each word's activations; words 0-1 of both units
-    // first, then unit 0's words 2-3 (its slot is refilled at once, half an
-    // item ahead of use) and unit 1's: at most two words of activations are
-    // live at a time.
-    const UnitConst<BITS> k0 = unit_const<BITS>(u[0], q), k1 = unit_const<BITS>(u[1], q);
+    // The units share each word's activations: words 0-1 of every unit
+    // first, then words 2-3 unit by unit, each unit's slot refilled as soon
+    // as its last word is done; at most two words of activations are live.
+    UnitConst<BITS> kc[SIZE];
+#pragma unroll
+    for (int j = 0; j < SIZE; ++j) kc[j] = unit_const<BITS>(u[j], q);
     const uint4 x0 = load_x_word<MODE>(xp, 0), x1 = load_x_word<MODE>(xp, 1);
-    process_word<BITS, MODE>(u[0], k0, x0, 0, q, cb, acc[0]);
-    process_word<BITS, MODE>(u[1], k1, x0, 0, q, cb, acc[1]);
-    process_word<BITS, MODE>(u[0], k0, x1, 1, q, cb, acc[0]);
-    process_word<BITS, MODE>(u[1], k1, x1, 1, q, cb, acc[1]);
+#pragma unroll
+    for (int j = 0; j < SIZE; ++j) process_word<BITS, MODE>(u[j], kc[j], x0, 0, q, cb, acc[j]);
+#pragma unroll
+    for (int j = 0; j < SIZE; ++j) process_word<BITS, MODE>(u[j], kc[j], x1, 1, q, cb, acc[j]);
     const uint4 x2 = load_x_word<MODE>(xp, 2), x3 = load_x_word<MODE>(xp, 3);
-    process_word<BITS, MODE>(u[0], k0, x2, 2, q, cb, acc[0]);
-    process_word<BITS, MODE>(u[0], k0, x3, 3, q, cb, acc[0]);
-    reload(0);
-    process_word<BITS, MODE>(u[1], k1, x2, 2, q, cb, acc[1]);
-    process_word<BITS, MODE>(u[1], k1, x3, 3, q, cb, acc[1]);
-    reload(1);
+#pragma unroll
+    for (int j = 0; j < SIZE; ++j) {
+      process_word<BITS, MODE>(u[j], kc[j], x2, 2, q, cb, acc[j]);
+      process_word<BITS, MODE>(u[j], kc[j], x3, 3, q, cb, acc[j]);
+      reload(j);
+    }
+    if constexpr (LAST) {
+#pragma unroll
+      for (int j = SIZE; j < S; ++j) reload(j);
+    }
   }
 }
 
 // cnt >= 1 items of one strip of SIZE tiles at consecutive groups, starting
 // at unit base ub and activations xp; the last item loads the next strip's
 // first units (base nb, mask nmask).
-template <int BITS, int MODE, int SIZE>
-__device__ __forceinline__ void run_segment(Unit<BITS> (&u)[kStrip], Acc<MODE> (&acc)[kStrip],
+template <int BITS, int MODE, int SIZE, int S>
+__device__ __forceinline__ void run_segment(Unit<BITS> (&u)[S], Acc<MODE> (&acc)[S],
                                             int cnt, const uint8_t* ub, size_t gstride,
                                             const uint8_t* xp, int xstep, const uint8_t* nb,
                                             unsigned nmask, int lane, int q,
@@ -610,26 +626,28 @@ __device__ __forceinline__ void run_segment(Unit<BITS> (&u)[kStrip], Acc<MODE> (
       ub += 2 * gstride;
       xp += 2 * xstep;
     }
-    if (c < cnt) run_item<BITS, MODE, 1, true>(u, acc, xp, nb, 0u, lane, q, cb);
+    if (c < cnt) run_item<BITS, MODE, 1, true, S>(u, acc, xp, nb, 0u, lane, q, cb);
     return;
   }
   if (lane == 0 && cnt > 1) prefetch_l2(ub + gstride, kBytes);
   for (int c = 0; c + 1 < cnt; ++c) {
     if (lane == 0 && c + 2 < cnt) prefetch_l2(ub + 2 * gstride, kBytes);
-    run_item<BITS, MODE, SIZE, false>(u, acc, xp, ub + gstride, 0u, lane, q, cb);
+    run_item<BITS, MODE, SIZE, false, S>(u, acc, xp, ub + gstride, 0u, lane, q, cb);
     ub += gstride;
     xp += xstep;
   }
-  run_item<BITS, MODE, SIZE, true>(u, acc, xp, nb, nmask, lane, q, cb);
+  run_item<BITS, MODE, SIZE, true, S>(u, acc, xp, nb, nmask, lane, q, cb);
 }
 
-template <int BITS, int MODE, int WARPS, int MINB>
+template <int BITS, int MODE, int WARPS, int MINB, int S>
 __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
   pdl_launch_dependents();
   constexpr int NBP = MODE == kFull ? kMaxBatch : MODE;  // floats per row in a partial block
   constexpr int kBlk = kRowsPerTile * NBP;                // floats per partial block
   constexpr int UB = Layout<BITS>::kUnitBytes;
+  static_assert(S == 2 || S == 4, "strip sizes");
+  constexpr unsigned kStripMask = (1u << S) - 1u;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int gid = lane >> 2, q = lane & 3;
   const int cshift = a.cshift, csize = 1 << cshift;
@@ -668,25 +686,26 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
     int d = (int)(((unsigned long long)(unsigned)v * ngc_m) >> 32);
     return d * ngc > v ? d - 1 : d;
   };
-  const int nfull = T / kStrip;  // strips with all kStrip tiles
-  const unsigned last_mask = (1u << (T - kStrip * nfull)) - 1u;
-  const int i0 = warp_item<WARPS>(T, ngc, warp), i1 = warp_item<WARPS>(T, ngc, warp + 1);
+  const int nfull = T / S;  // strips with all S tiles
+  const int rest = T - S * nfull;
+  const unsigned last_mask = (1u << rest) - 1u;
+  const int i0 = warp_item<WARPS, S>(T, ngc, warp), i1 = warp_item<WARPS, S>(T, ngc, warp + 1);
 
-  // units (t0 + kStrip s + j, g), j < kStrip, start at strip_base(s, g) + j * UB
+  // units (t0 + S s + j, g), j < S, start at strip_base(s, g) + j * UB
   const size_t gstride = (size_t)a.nrt * UB;
   auto strip_base = [&](int s, int g) {
-    return a.units + ((size_t)g * a.nrt + t0 + kStrip * s) * UB;
+    return a.units + ((size_t)g * a.nrt + t0 + S * s) * UB;
   };
   auto strip_mask = [&](int s) { return s < nfull ? kStripMask : last_mask; };
 
   // first item's units (codes are immutable: no wait needed)
-  Unit<BITS> u[kStrip] = {};
+  Unit<BITS> u[S] = {};
   int s = i0 < i1 ? div_ngc(i0) : 0;
   int g = i0 < i1 ? g0 + (i0 - s * ngc) : g0;
   if (i0 < i1) {
     const unsigned m0 = strip_mask(s);
 #pragma unroll
-    for (int j = 0; j < kStrip; ++j)
+    for (int j = 0; j < S; ++j)
       if (m0 >> j & 1u) u[j] = load_unit<BITS>(strip_base(s, g) + j * UB, lane);
   }
 
@@ -737,9 +756,9 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
   // receive slot of (owned tile k, rank r, warp w): ((k * csize + r) * WARPS + w) * kBlk floats
   const uint32_t recv_base = smem_u32(smem + a.off_recv);
 
-  Acc<MODE> acc[kStrip];
+  Acc<MODE> acc[S];
 #pragma unroll
-  for (int j = 0; j < kStrip; ++j) acc[j].zero();
+  for (int j = 0; j < S; ++j) acc[j].zero();
 
   // Units of a strip at one group are contiguous: one bulk L2 prefetch per
   // item, two items ahead inside the strip (the next item's units are already
@@ -753,14 +772,19 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
     const uint8_t* xp = x0 + (g - g0) * xstep;
     const uint8_t* nb = strip_base(s + 1, g0);
     const unsigned nmask = left > 0 ? strip_mask(s + 1) : 0u;
-    static_assert(kStrip == 2, "strip sizes dispatched below");
     if (s < nfull)
-      run_segment<BITS, MODE, 2>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask, lane, q, cb);
-    else
-      run_segment<BITS, MODE, 1>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask, lane, q, cb);
+      run_segment<BITS, MODE, S, S>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask, lane, q, cb);
+    else if (S > 1 && rest == 1)
+      run_segment<BITS, MODE, 1, S>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask, lane, q, cb);
+    else if (S > 2 && rest == 2)
+      run_segment<BITS, MODE, (S > 2 ? 2 : 1), S>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask,
+                                                  lane, q, cb);
+    else if (S > 3)
+      run_segment<BITS, MODE, (S > 3 ? 3 : 1), S>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask,
+                                                  lane, q, cb);
 #pragma unroll
-    for (int j = 0; j < kStrip; ++j) {
-      const int tau = s * kStrip + j;
+    for (int j = 0; j < S; ++j) {
+      const int tau = s * S + j;
       if (tau < T) {
         const int owner = tau & (csize - 1);
         const uint32_t slot =
@@ -777,9 +801,9 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
   // [tau_lo, tau_hi) got its partial sums): 16 bytes per lane, 64 bytes per
   // batch row
   {
-    const int w0 = warp_item<WARPS>(T, ngc, warp), w1 = warp_item<WARPS>(T, ngc, warp + 1);
-    const int tau_lo = w0 < w1 ? div_ngc(w0) * kStrip : 0;
-    const int tau_hi = w0 < w1 ? min(T, (div_ngc(w1 - 1) + 1) * kStrip) : 0;
+    const int w0 = warp_item<WARPS, S>(T, ngc, warp), w1 = warp_item<WARPS, S>(T, ngc, warp + 1);
+    const int tau_lo = w0 < w1 ? div_ngc(w0) * S : 0;
+    const int tau_hi = w0 < w1 ? min(T, (div_ngc(w1 - 1) + 1) * S) : 0;
   for (int tau = 0; tau < T; ++tau) {
     if (tau >= tau_lo && tau < tau_hi) continue;
     const uint32_t slot =
@@ -828,15 +852,16 @@ template <> struct KernelShape<kFmtW3V3> : KernelShape<3> {};
 
 constexpr int kModes[3] = {kFactored1, kFactored2, kFull};
 
-template <int BITS, int MODE>
+template <int BITS, int MODE, int S>
 inline const void* kptr() {
   return reinterpret_cast<const void*>(
-      &gemv_kernel<BITS, MODE, KernelShape<BITS>::kWarps, KernelShape<BITS>::kMinBlocks>);
+      &gemv_kernel<BITS, MODE, KernelShape<BITS>::kWarps, KernelShape<BITS>::kMinBlocks, S>);
 }
-template <int FMT>
+template <int FMT, int S = 2>
 inline const void* kptr_mode(int mode) {
-  return mode == kFactored1 ? kptr<FMT, kFactored1>() : mode == kFactored2 ? kptr<FMT, kFactored2>()
-                                                                           : kptr<FMT, kFull>();
+  return mode == kFactored1 ? kptr<FMT, kFactored1, S>()
+         : mode == kFactored2 ? kptr<FMT, kFactored2, S>()
+                              : kptr<FMT, kFull, S>();
 }
 
 // Kernels of the Tab. 4 splits (formats 5-9), instantiated in their own
