@@ -61,8 +61,8 @@ UNIT = "GB/s"
 TRAFFIC_SOURCES = ("paper_2609_24875_gb300/csrc/sphq_gemv_kernel.cuh",
                    "paper_2609_24875_gb300/csrc/sphq_gemv.cu",
                    "paper_2609_24875_gb300/csrc/sphq_layout.cuh")
-TRAFFIC_DIGEST = "18ed32c030cb271e:2fe8301989ee48b7:fb4c31fffa30dab7"
-TRAFFIC_RATIO = {2: 21046016 / 21005312, 3: 28506624 / 28475392}
+TRAFFIC_DIGEST = "c5f6845968ddbd32:e8e9a15fd59e93f0:fb4c31fffa30dab7"
+TRAFFIC_RATIO = {2: 21040640 / 21005312, 3: 28536064 / 28475392}
 
 
 def kernel_digest() -> str:
@@ -553,25 +553,34 @@ def run_case(spec: str, pool: int, launches: int):
     """Profiling driver: `bits:n[:batch]` or `bits:RxC[:batch]` -> `pool`
     distinct packed n x n (R x C) matrices, `launches` GEMVs round robin on one
     stream, no timing (for running under ncu).  bits `3v3` selects W3 with
-    3-bit radius codes, `dDvV` the 8/D/V split (e.g. `d7v2`)."""
+    3-bit radius codes, `dDvV` the 8/D/V split (e.g. `d7v2`); a leading `e`
+    (`e3:8192`) packs the encoded configuration's codes (sphq_encode on the
+    Gaussian weights of the square sweep, batch 1) instead of random codes."""
     import torch
 
     head, size, *rest = spec.split(":")
-    bits, vbits, K = parse_split(head)
+    encoded = head.startswith("e")
+    bits, vbits, K = parse_split(head.lstrip("e"))
     rows, n = (int(v) for v in size.split("x")) if "x" in size else (int(size), int(size))
     batch = int(rest[0]) if rest else 1
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     from paper_2609_24875_gb300 import SphqMatrix
-    codes, x = inp.random_codes(bits, rows, n, seed=1, B=batch, radius_bits=vbits, K=K)
     t = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int16) if a.dtype == np.uint16 else a)).to(dev)
-    mats = []
-    for _ in range(pool):
-        m = SphqMatrix(rows, n, bits, t(codes.codebook), t(codes.scale), t(codes.offset),
-                       radius_bits=vbits, K=K)
-        m.pack(t(codes.sign), t(codes.idx), t(codes.rcode))
-        mats.append(m)
-    xd = t(x).view(torch.float16)
+    if encoded:
+        if rows != n or batch != 1 or (bits, n) not in inp.SQUARE_SWEEP:
+            raise SystemExit("--case e...: one of the square sweep's shapes, batch 1")
+        mats, xd, _ = make_encoded_pool(bits, n, pool,
+                                        inp.seed_for(1, inp.SQUARE_SWEEP.index((bits, n))), dev)
+    else:
+        codes, x = inp.random_codes(bits, rows, n, seed=1, B=batch, radius_bits=vbits, K=K)
+        mats = []
+        for _ in range(pool):
+            m = SphqMatrix(rows, n, bits, t(codes.codebook), t(codes.scale), t(codes.offset),
+                           radius_bits=vbits, K=K)
+            m.pack(t(codes.sign), t(codes.idx), t(codes.rcode))
+            mats.append(m)
+        xd = t(x).view(torch.float16)
     ys = [torch.empty((batch, rows), dtype=torch.float16, device=dev) for _ in mats]
     s = torch.cuda.current_stream()
     for i in range(launches):
