@@ -422,7 +422,8 @@ def sample_directions(w, u):
     drawn with probability r_i^2 / sum_j r_j^2 by inverse transform of the
     uniforms u in [0, 1): P = cumsum(r^2) in vector order, the pick for u is
     the first i with P_i > u * P_last (so vectors of zero radius are never
-    drawn).  r_i^2 = w_0^2 + ... + w_7^2 summed in coordinate order, r_i its
+    drawn; u = 1, whose product is P_last itself, takes the last vector of
+    nonzero radius).  r_i^2 = w_0^2 + ... + w_7^2 summed in coordinate order, r_i its
     square root and the direction d_i = |w_i| / r_i, all in float64 from the
     float32 weights.  Returns (directions (len(u), 8) float64, indices)."""
     w = np.asarray(w, np.float32).astype(np.float64).reshape(-1, VEC)
@@ -434,6 +435,9 @@ def sample_directions(w, u):
         raise ValueError("all vectors are zero")
     u = np.asarray(u, np.float64)
     idx = np.searchsorted(P, u * P[-1], side="right")
+    # fl(u * total) < total for every double u < 1; u = 1 reaches the total,
+    # which no P_i exceeds: the pick is the first i with P_i = total
+    idx = np.where(idx >= P.shape[0], np.searchsorted(P, P[-1], side="left"), idx)
     r = np.sqrt(r2[idx])
     return np.abs(w[idx]) / r[:, None], idx
 

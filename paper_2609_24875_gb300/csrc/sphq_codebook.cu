@@ -107,8 +107,11 @@ __global__ void __launch_bounds__(kCbThreads) sample_kernel(
   if (s >= S) return;
   const double total = *total_p;
   double target = __dmul_rn(u[s], total);
-  // u * total can round up to the total for u just below 1: then the pick
-  // is the last vector of nonzero radius (the first i with P_i = total)
+  // For u < 1 the rounded product stays below the total (total * 2^-53 is
+  // more than half a unit in the last place below a total that is not a
+  // power of two, and the product is exact when it is one); u = 1 reaches
+  // the total, which no P_i exceeds: the pick is then the last vector of
+  // nonzero radius (the first i with P_i = total)
   const bool top = !(target < total);
   long long lo = 0, hi = n - 1;
   while (lo < hi) {

@@ -30,7 +30,7 @@ def _weights(rows, cols, seed):
 def test_sample_directions_matches_oracle(rows, cols, S):
     w = _weights(rows, cols, seed=rows + cols)
     u = np.random.default_rng(S).random(S)
-    u[:4] = [0.0, 0.5, 1.0 - 2.0 ** -53, 0.25]
+    u[:5] = [0.0, 0.5, 1.0 - 2.0 ** -53, 0.25, 1.0]
     d_gpu, i_gpu = sphq.sample_directions(torch.from_numpy(w).to(DEV),
                                           torch.from_numpy(u).to(DEV))
     torch.cuda.synchronize()

@@ -77,6 +77,28 @@ def test_sample_directions_inverse_transform_hand_case():
     assert np.all(d >= 0)
 
 
+def test_sample_directions_top_of_range():
+    # radii^2 1, 2, 0: P = [1, 3, 3], total 3.  The largest double below 1,
+    # u = 1 - 2^-53, gives u * 3 = 3 - 3 * 2^-53, which rounds to 3 - 2^-51
+    # (spacing 2^-51 on [2, 4)): still below the total, so the pick is the
+    # first P_i above it, index 1, never the zero-radius vector 2.  u = 1
+    # itself reaches the total and takes the same last nonzero vector.
+    u_top = 1.0 - 2.0 ** -53
+    assert u_top * 3.0 == 3.0 - 2.0 ** -51
+    w = np.zeros((1, 24), np.float32)
+    w[0, 0] = 1.0
+    w[0, 8:10] = [1.0, -1.0]
+    d, idx = oracle.sample_directions(w, np.array([u_top, 1.0, 0.5, 1.0 / 3.0]))
+    # 0.5 * 3 = 1.5 lies in [P_0, P_1); (1/3) * 3 rounds to exactly 1 = P_0
+    assert list(idx) == [1, 1, 1, 1]
+    assert np.array_equal(d[0], np.array([1.0, 1.0, 0, 0, 0, 0, 0, 0]) / np.sqrt(2.0))
+    # a trailing zero-radius vector after a total that is a power of two:
+    # P = [1, 2, 2]; 2 * (1 - 2^-53) = 2 - 2^-52 is exact and below 2
+    w[0, 8:10] = [1.0, 0.0]
+    _, idx = oracle.sample_directions(w, np.array([u_top, 1.0]))
+    assert list(idx) == [1, 1]
+
+
 def test_sample_directions_frequencies_follow_squared_radius():
     rng = np.random.default_rng(11)
     w = (rng.standard_normal((1, 40)) * np.array([1, 1, 1, 1, 1, 1, 1, 1] * 5)).astype(np.float32)
