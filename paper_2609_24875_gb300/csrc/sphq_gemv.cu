@@ -164,21 +164,18 @@ static sphq_status make_plan(sphq_handle h, int batch, int forced, int optin, Ge
         // Estimated time per launch (us), fitted (least log-regret over a grid
         // of constants) to GB300 measurements of back-to-back launches at
         // cluster sizes 1, 2 and 4 on the decoder and square shapes (W2 and
-        // W3, batch 1 and 8): a fixed part (launch, staging, reduction) plus
-        // ~0.02 us per unit of the most loaded CTA; one-tile strips do not
-        // share activation loads between two units.  With the prologue free
-        // of divisions and per-tile cover masks, clusters of 2 and 4 cost no
-        // more than single CTAs in the batch 1-2 modes; clusters of 8 leave
-        // SMs idle (only 15 fit) and are priced out unless nothing else runs.
-        // Batch 3-8 (full mode: activations read from global memory, eight
-        // partial sums per row through the cluster) pays more for clusters.
-        // A plan that needs a second wave of clusters (its shared memory did
-        // not fit at one wave) pays the fixed part again per wave (measured:
-        // W3 18944 x 3584 batch 8 in two waves of clusters of 4, 23.3 us
-        // against 17.6 us in one wave of single CTAs).
-        const double fixed = mode == kFull
-                                 ? (csize == 1 ? 2.0 : csize == 2 ? 2.3 : csize == 4 ? 3.0 : 5.8)
-                                 : (csize == 8 ? 5.0 : 2.0);
+        // W3, batch 1, 2, 4 and 8): a fixed part (launch, staging, reduction)
+        // plus ~0.02 us per unit of the most loaded CTA; one-tile strips do
+        // not share activation loads between two units.  With the prologue
+        // free of divisions and per-tile cover masks, clusters of 2 and 4 cost
+        // no more than single CTAs in every mode (worst regret against the
+        // best of the three sizes: 2.3% at batch 4-8, 5.9% at batch 1-2);
+        // clusters of 8 leave SMs idle (only 15 fit) and are priced out unless
+        // nothing else runs.  A plan that needs a second wave of clusters (its
+        // shared memory did not fit at one wave) pays the fixed part again per
+        // wave (measured: W3 18944 x 3584 batch 8 in two waves of clusters of
+        // 4, 22.1 us against 15.6 us in one wave of single CTAs).
+        const double fixed = csize == 8 ? (mode == kFull ? 5.8 : 5.0) : 2.0;
         const double shallow = 1.0 + 0.33 * (2 - std::min(tmax, 2));
         const double cost = fixed * waves + waves * 0.02 * tmax * ((h->ng + csize - 1) / csize) * shallow;
         if (best.grid == 0 || cost < best_cost - 1e-9) {
