@@ -431,6 +431,10 @@ typedef struct sphq_plan_info {
   int warps_per_cta;
   int smem_bytes;        /* dynamic shared memory per CTA */
   int staged_x;          /* 1: activations copied to shared memory (batch 1-2), 0: read via L1 */
+  int ctas_per_sm;       /* CTAs per SM the kernel is built for: 2 (W2 and the small-codebook
+                            splits, at most 128 registers per thread) or 1 (W3; and W2 when
+                            the row tiles bound the cluster count, with the whole register
+                            file) */
 } sphq_plan_info;
 sphq_status sphq_get_plan(sphq_handle h, int batch, sphq_plan_info* out);
 

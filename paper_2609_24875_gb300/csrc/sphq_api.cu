@@ -312,6 +312,7 @@ sphq_status sphq_get_plan(sphq_handle h, int batch, sphq_plan_info* out) {
   out->warps_per_cta = p.warps_per_cta;
   out->smem_bytes = (int)p.smem;
   out->staged_x = p.mode != 8;
+  out->ctas_per_sm = p.ctas_per_sm;
   return SPHQ_OK;
 }
 

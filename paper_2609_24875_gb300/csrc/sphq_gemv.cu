@@ -26,8 +26,11 @@ static uint32_t cb_bytes_for(int fmt) {
 
 static int mode_for(int batch) { return batch == 1 ? kFactored1 : batch == 2 ? kFactored2 : kFull; }
 
-static const void* select_kernel(int fmt, int mode, int strip) {
-  return fmt == 2 ? kptr_mode<2>(mode)
+// formats with a one-CTA-per-SM build beside the two-CTA one
+static bool has_solo(int fmt) { return fmt == 2; }
+
+static const void* select_kernel(int fmt, int mode, int strip, bool solo = false) {
+  return fmt == 2 ? (solo ? kptr_mode_solo<2>(mode) : kptr_mode<2>(mode))
          : fmt == 3 ? (strip == 4 ? kptr_mode<3, 4>(mode) : kptr_mode<3, 2>(mode))
          : fmt == kFmtW3V3 ? (strip == 4 ? kptr_mode<kFmtW3V3, 4>(mode) : kptr_mode<kFmtW3V3, 2>(mode))
                            : split_kernel(fmt, mode);
@@ -44,12 +47,14 @@ static sphq_status allow_max_smem(int device, int optin) {
   if (done[device]) return SPHQ_OK;
   for (int fmt = 2; fmt <= kFmt4D; ++fmt)
     for (int mode : kModes)
-      for (int strip : {2, 4}) {
-        if (strip == 4 && !fmt_has_strip4(fmt)) continue;
-        cudaError_t e = cudaFuncSetAttribute(select_kernel(fmt, mode, strip),
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, optin);
-        if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute");
-      }
+      for (int strip : {2, 4})
+        for (int solo = 0; solo < 2; ++solo) {
+          if (strip == 4 && !fmt_has_strip4(fmt)) continue;
+          if (solo && !has_solo(fmt)) continue;
+          cudaError_t e = cudaFuncSetAttribute(select_kernel(fmt, mode, strip, solo),
+                                               cudaFuncAttributeMaxDynamicSharedMemorySize, optin);
+          if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute");
+        }
   done[device] = true;
   return SPHQ_OK;
 }
@@ -120,78 +125,89 @@ static sphq_status make_plan(sphq_handle h, int batch, int forced, int optin, Ge
       int mode = mode_for(batch);
       if (!staged) mode = kFull;
       if (staged && mode == kFull) continue;
-      const void* k = select_kernel(h->fmt, mode, 2);  // both strip sizes: same resources
-      for (int csize : {1, 2, 4, 8}) {
-        if (csize > h->ng) break;
-        if (forced && csize != forced) continue;
-        // clusters: as many as fit at once, at most one per row tile; the
-        // tile range of a cluster is limited by its shared memory
-        GemvPlan p;
-        p.mode = mode;
-        p.warps_per_cta = warps;
-        p.csize = csize;
-        p.grid = csize;
-        p.smem = smem_layout(h, mode, warps, csize, 1).total;
-        if (p.smem > (size_t)optin) continue;
-        cudaLaunchAttribute attr[2];
-        cudaLaunchConfig_t cfg = launch_config(p, nullptr, attr);
-        int ncl = 0;
-        e = cudaOccupancyMaxActiveClusters(&ncl, k, &cfg);
-        if (e != cudaSuccess) {
-          (void)cudaGetLastError();
-          continue;
-        }
-        if (ncl < 1) continue;
-        int nclusters = std::min(ncl, h->nrt);
-        int tmax = (h->nrt + nclusters - 1) / nclusters;
-        SmemLayout L = smem_layout(h, mode, warps, csize, tmax);
-        // grow the cluster count (extra waves) until a cluster's tiles fit
-        while (L.total > (size_t)optin && tmax > 1) {
-          nclusters = std::min(h->nrt, nclusters * 2);
-          tmax = (h->nrt + nclusters - 1) / nclusters;
-          L = smem_layout(h, mode, warps, csize, tmax);
-        }
-        if (L.total > (size_t)optin) continue;
-        // with the final shared-memory size the resident count may be lower
-        p.smem = L.total;
-        cfg = launch_config(p, nullptr, attr);
-        e = cudaOccupancyMaxActiveClusters(&ncl, k, &cfg);
-        if (e != cudaSuccess || ncl < 1) {
-          (void)cudaGetLastError();
-          continue;
-        }
-        const int waves = (nclusters + ncl - 1) / ncl;
-        // Estimated time per launch (us), fitted (least log-regret over a grid
-        // of constants) to GB300 measurements of back-to-back launches at
-        // cluster sizes 1, 2 and 4 on the decoder and square shapes (W2 and
-        // W3, batch 1, 2, 4 and 8): a fixed part (launch, staging, reduction)
-        // plus ~0.02 us per unit of the most loaded CTA; one-tile strips do
-        // not share activation loads between two units.  With the prologue
-        // free of divisions and per-tile cover masks, clusters of 2 and 4 cost
-        // no more than single CTAs in every mode (worst regret against the
-        // best of the three sizes: 2.3% at batch 4-8, 5.9% at batch 1-2);
-        // clusters of 8 leave SMs idle (only 15 fit) and are priced out unless
-        // nothing else runs.  A plan that needs a second wave of clusters (its
-        // shared memory did not fit at one wave) pays the fixed part again per
-        // wave (measured: W3 18944 x 3584 batch 8 in two waves of clusters of
-        // 4, 22.1 us against 15.6 us in one wave of single CTAs).
-        const double fixed = csize == 8 ? (mode == kFull ? 5.8 : 5.0) : 2.0;
-        const double shallow = 1.0 + 0.33 * (2 - std::min(tmax, 2));
-        const double cost = fixed * waves + waves * 0.02 * tmax * ((h->ng + csize - 1) / csize) * shallow;
-        if (best.grid == 0 || cost < best_cost - 1e-9) {
-          p.grid = nclusters * csize;
-          p.nclusters = nclusters;
-          p.tmax = tmax;
-          p.cb_bytes = cb_bytes_for(h->fmt);
-          p.x_pitch = L.x_pitch;
-          p.off_x = (uint32_t)L.x;
-          p.off_zero = (uint32_t)L.zero;
-          p.off_recv = (uint32_t)L.recv;
-          p.off_bar = (uint32_t)L.bar;
-          // four-tile strips once a cluster holds three tiles or more (W3)
-          p.strip = fmt_has_strip4(h->fmt) && tmax >= 3 ? 4 : 2;
-          best = p;
-          best_cost = cost;
+      for (int solo = 0; solo < (has_solo(h->fmt) ? 2 : 1); ++solo) {
+        // both strip sizes: same resources
+        const void* k = select_kernel(h->fmt, mode, 2, solo);
+        for (int csize : {1, 2, 4, 8}) {
+          if (csize > h->ng) break;
+          if (forced && csize != forced) continue;
+          // clusters: as many as fit at once, at most one per row tile; the
+          // tile range of a cluster is limited by its shared memory
+          GemvPlan p;
+          p.mode = mode;
+          p.warps_per_cta = warps;
+          p.csize = csize;
+          p.grid = csize;
+          p.smem = smem_layout(h, mode, warps, csize, 1).total;
+          if (p.smem > (size_t)optin) continue;
+          cudaLaunchAttribute attr[2];
+          cudaLaunchConfig_t cfg = launch_config(p, nullptr, attr);
+          int ncl = 0;
+          e = cudaOccupancyMaxActiveClusters(&ncl, k, &cfg);
+          if (e != cudaSuccess) {
+            (void)cudaGetLastError();
+            continue;
+          }
+          if (ncl < 1) continue;
+          int nclusters = std::min(ncl, h->nrt);
+          int tmax = (h->nrt + nclusters - 1) / nclusters;
+          SmemLayout L = smem_layout(h, mode, warps, csize, tmax);
+          // grow the cluster count (extra waves) until a cluster's tiles fit
+          while (L.total > (size_t)optin && tmax > 1) {
+            nclusters = std::min(h->nrt, nclusters * 2);
+            tmax = (h->nrt + nclusters - 1) / nclusters;
+            L = smem_layout(h, mode, warps, csize, tmax);
+          }
+          if (L.total > (size_t)optin) continue;
+          // with the final shared-memory size the resident count may be lower
+          p.smem = L.total;
+          cfg = launch_config(p, nullptr, attr);
+          e = cudaOccupancyMaxActiveClusters(&ncl, k, &cfg);
+          if (e != cudaSuccess || ncl < 1) {
+            (void)cudaGetLastError();
+            continue;
+          }
+          const int waves = (nclusters + ncl - 1) / ncl;
+          // Estimated time per launch (us), fitted (least log-regret over a grid
+          // of constants) to GB300 measurements of back-to-back launches at
+          // cluster sizes 1, 2 and 4 on the decoder and square shapes (W2 and
+          // W3, batch 1, 2, 4 and 8): a fixed part (launch, staging, reduction)
+          // plus ~0.02 us per unit of the most loaded CTA; one-tile strips do
+          // not share activation loads between two units.  With the prologue
+          // free of divisions and per-tile cover masks, clusters of 2 and 4 cost
+          // no more than single CTAs in every mode (worst regret against the
+          // best of the three sizes: 2.3% at batch 4-8, 5.9% at batch 1-2);
+          // clusters of 8 leave SMs idle (only 15 fit) and are priced out unless
+          // nothing else runs.  A plan that needs a second wave of clusters (its
+          // shared memory did not fit at one wave) pays the fixed part again per
+          // wave (measured: W3 18944 x 3584 batch 8 in two waves of clusters of
+          // 4, 22.1 us against 15.6 us in one wave of single CTAs).
+          const double fixed = csize == 8 ? (mode == kFull ? 5.8 : 5.0) : 2.0;
+          const double shallow = 1.0 + 0.33 * (2 - std::min(tmax, 2));
+          const double cost = fixed * waves + waves * 0.02 * tmax * ((h->ng + csize - 1) / csize) * shallow;
+          // The one-CTA-per-SM build wins ties: at equal load the row tiles
+          // bound the cluster count, and no second CTA would share an SM.
+          const bool better = best.grid == 0 || cost < best_cost - 1e-9 ||
+                              (solo && !best.solo && cost <= best_cost + 1e-9);
+          if (better) {
+            p.grid = nclusters * csize;
+            p.nclusters = nclusters;
+            p.tmax = tmax;
+            p.cb_bytes = cb_bytes_for(h->fmt);
+            p.x_pitch = L.x_pitch;
+            p.off_x = (uint32_t)L.x;
+            p.off_zero = (uint32_t)L.zero;
+            p.off_recv = (uint32_t)L.recv;
+            p.off_bar = (uint32_t)L.bar;
+            // four-tile strips once a cluster holds three tiles or more (W3)
+            p.strip = fmt_has_strip4(h->fmt) && tmax >= 3 ? 4 : 2;
+            p.solo = solo != 0;
+          p.ctas_per_sm = solo ? 1
+                          : fmt_small(h->fmt) || h->fmt == kFmt4D ? KernelShape<2>::kMinBlocks
+                                                                   : KernelShape<3>::kMinBlocks;
+            best = p;
+            best_cost = cost;
+          }
         }
       }
       if (best.grid > 0) break;  // staged activations fit: keep that mode
@@ -269,7 +285,7 @@ sphq_status launch_gemv(sphq_handle h, const void* x, void* y, int batch, cudaSt
   cudaLaunchAttribute attr[2];
   cudaLaunchConfig_t cfg = launch_config(p, s, attr, h->pdl);
   void* args[] = {&a};
-  cudaError_t e = cudaLaunchKernelExC(&cfg, select_kernel(h->fmt, p.mode, p.strip), args);
+  cudaError_t e = cudaLaunchKernelExC(&cfg, select_kernel(h->fmt, p.mode, p.strip, p.solo), args);
   if (e != cudaSuccess) return cuda_error(e, "gemv launch");
   return SPHQ_OK;
 }

@@ -20,6 +20,8 @@ struct GemvPlan {
   size_t smem = 0;         // dynamic shared memory per CTA
   int mode = 0;            // radius application: 1, 2 (factored) or 8 (full)
   int strip = 2;           // row tiles per work item (2, or 4 for W3 with >= 3 tiles per cluster)
+  bool solo = false;       // W2: the kernel built for one CTA per SM (whole register file)
+  int ctas_per_sm = 0;     // CTAs per SM the kernel is built for (its register budget)
   uint32_t cb_bytes = 0;   // staged codebook image
   uint32_t x_pitch = 0;    // bytes between staged activation rows
   uint32_t off_x = 0, off_zero = 0, off_recv = 0, off_bar = 0;

@@ -35,7 +35,7 @@ class PlanInfo(ctypes.Structure):
     _fields_ = [("grid", ctypes.c_int), ("cluster_size", ctypes.c_int),
                 ("clusters", ctypes.c_int), ("tiles_per_cluster", ctypes.c_int),
                 ("warps_per_cta", ctypes.c_int), ("smem_bytes", ctypes.c_int),
-                ("staged_x", ctypes.c_int)]
+                ("staged_x", ctypes.c_int), ("ctas_per_sm", ctypes.c_int)]
 
 
 class GemmInfo(ctypes.Structure):

@@ -88,3 +88,19 @@ def test_extreme_shapes(bits, rows, cols, batch):
     assert np.all(np.isfinite(got[:, sel]))
     assert np.all(err <= oracle.gemv_tolerance(absdot)), float(np.max(err / oracle.gemv_tolerance(absdot)))
     m.close()
+
+
+# W2 has two builds of the kernel: two CTAs per SM (at most 128 registers per
+# thread) and one CTA per SM with the whole register file, which the plan
+# takes when the row tiles bound the cluster count (no second CTA would share
+# an SM).  W3 always runs one CTA per SM.  Every row, every batch mode.
+@pytest.mark.parametrize("bits,rows,cols,ctas", [(2, 512, 3584, 1), (2, 4096, 1024, 2),
+                                                 (2, 509, 3584, 1), (3, 512, 3584, 1)])
+def test_kernel_build_per_plan(bits, rows, cols, ctas):
+    codes, x = inp.random_codes(bits, rows, cols, seed=8800 + rows + bits, B=5)
+    m = G.make_matrix(codes)
+    for batch in (1, 2, 5):
+        p = m.plan(batch)
+        assert p["ctas_per_sm"] == ctas, (batch, p)
+        _check(m, codes, x[:batch], batch)
+    m.close()
