@@ -603,11 +603,15 @@ def parse_split(head: str):
 
 
 def run_gemm_case(spec: str, launches: int):
-    """Profiling driver of the prefill GEMM: `bits:rows:cols:batch` ->
-    `launches` sphq_gemm calls on one matrix, no timing (for ncu)."""
+    """Profiling driver of the prefill GEMM: `bits:rows:cols:batch[:ws]` ->
+    `launches` sphq_gemm calls on one matrix (with `:ws`, sphq_gemm_ws calls:
+    the decode pass and the dense pass), no timing (for ncu)."""
     import torch
 
     head, *rest = spec.split(":")
+    two_pass = rest[-1] == "ws"
+    if two_pass:
+        rest = rest[:-1]
     bits, vbits, K = parse_split(head)
     rows, cols, batch = (int(v) for v in rest)
     dev = torch.device("cuda", 0)
@@ -621,10 +625,15 @@ def run_gemm_case(spec: str, launches: int):
     xd = t(x).view(torch.float16)
     y = torch.empty((batch, rows), dtype=torch.float16, device=dev)
     s = torch.cuda.current_stream()
+    ws = torch.empty(rows * cols, dtype=torch.float16, device=dev) if two_pass else None
     for _ in range(launches):
-        m.gemm_ptr(xd.data_ptr(), y.data_ptr(), batch, s.cuda_stream)
+        if two_pass:
+            m.gemm_ws(xd, ws, y=y)
+        else:
+            m.gemm_ptr(xd.data_ptr(), y.data_ptr(), batch, s.cuda_stream)
     m.check()
-    print(f"gemm case W{bits} V={vbits} K={K} {rows}x{cols} batch {batch}: {launches} launches done")
+    print(f"gemm case W{bits} V={vbits} K={K} {rows}x{cols} batch {batch}"
+          f"{' two-pass' if two_pass else ''}: {launches} launches done")
 
 
 def run_encode_case(spec: str, launches: int):
@@ -743,13 +752,24 @@ def gemm_report(hbm_peak):
             y = torch.empty(batch, rows, device=dev, dtype=torch.half)
             us = timed(lambda: m.gemm_ptr(x.data_ptr(), y.data_ptr(), batch, stream.cuda_stream))
             m.check(stream)
+            # the two-pass form (W_hat decoded into a workspace, then the dense
+            # tensor-core pass), whichever the library would choose
+            ws = torch.empty(rows * cols, dtype=torch.float16, device=dev)
+            us_2 = timed(lambda: m.gemm_ws(x, ws, y=y, stream=stream))
+            m.check(stream)
+            advice = m.gemm_workspace(batch)
+            del ws
             wd = m.decode()
             torch.cuda.synchronize()
             us_d = timed(lambda: torch.matmul(x, wd.t()))
             fl = 2.0 * batch * rows * cols
+            best = min(us, us_2)
             out[f"{name} {rows}x{cols} B{batch}"] = {
                 "us": round(us, 2), "TF/s": round(fl / us / 1e6, 1),
                 "tensor_frac": round(fl / us / 1e6 / tf_peak, 4),
+                "two_pass_us": round(us_2, 2), "two_pass_TF/s": round(fl / us_2 / 1e6, 1),
+                "library_choice": "two-pass" if advice else "fused",
+                "best_tensor_frac": round(fl / best / 1e6 / tf_peak, 4),
                 "dense_fp16_cublas_us": round(us_d, 2)}
             m.close()
             del wd, x, y

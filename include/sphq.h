@@ -343,6 +343,34 @@ sphq_status sphq_gemv_noalloc(sphq_handle h, const void* x, void* y, int batch,
 sphq_status sphq_gemm(sphq_handle h, const void* x, void* y, int batch, sphq_stream stream);
 
 /*
+ * sphq_gemm_workspace / sphq_gemm_ws -- the same product in two passes, for
+ * large batches of the formats whose fused kernel is bound by its codebook
+ * gathers (§3.4 with W_hat from Eq. (7) and Eq. (4), computed in a different
+ * order: decode once, then multiply).
+ *
+ * Pass 1 decodes W_hat (rows x cols fp16, exactly sphq_decode's output) into
+ * a caller-provided device workspace; pass 2 is a dense tensor-core product
+ * that loads W_hat and X tiles with TMA.  The decode then costs one write and
+ * one read of 2 bytes per weight per call instead of a shared-memory gather
+ * per weight and activation tile.  Products, accumulation order and rounding
+ * are those of sphq_gemm: Y is equal to sphq_gemm's bit for bit.
+ *
+ * sphq_gemm_workspace sets *bytes to rows x cols x 2 when the two-pass form is
+ * estimated faster than the fused kernel for this batch, else to 0.
+ *
+ * sphq_gemm_ws takes the arguments of sphq_gemm plus the workspace:
+ *   workspace        device pointer, 16-byte aligned, at least rows x cols x 2
+ *                    bytes (SPHQ_ERR_INVALID_ARG otherwise), owned by the
+ *                    caller, overwritten; NULL runs the fused kernel
+ *                    (= sphq_gemm).
+ * Asynchronous on `stream` (two launches), no allocation.  A workspace must not
+ * be shared by calls that overlap on the GPU.
+ */
+sphq_status sphq_gemm_workspace(sphq_handle h, int batch, size_t* bytes);
+sphq_status sphq_gemm_ws(sphq_handle h, const void* x, void* y, int batch, void* workspace,
+                         size_t workspace_bytes, sphq_stream stream);
+
+/*
  * sphq_gemm_info / sphq_get_gemm_shape -- the launch shape sphq_gemm uses for
  * `batch`: activation tiles of 128 rows per CTA (1 or 2), weight rows per CTA
  * (128 or 256), columns per pipeline stage (64 or 32), ring stages, grid and

@@ -664,6 +664,33 @@ sphq_status sphq_gemm(sphq_handle h, const void* x, void* y, int batch, sphq_str
   return launch_gemm(h, x, y, batch, reinterpret_cast<cudaStream_t>(stream));
 }
 
+sphq_status sphq_gemm_workspace(sphq_handle h, int batch, size_t* bytes) {
+  g_last_error.clear();
+  if (!h || !bytes) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemm_workspace: NULL argument");
+  *bytes = 0;
+  if (batch < 1 || batch > SPHQ_GEMM_MAX_BATCH)
+    return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm_workspace: batch out of range");
+  if (h->dim != 8) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm_workspace: 8-D vectors only");
+  return gemm_workspace_bytes(h, batch, bytes);
+}
+
+sphq_status sphq_gemm_ws(sphq_handle h, const void* x, void* y, int batch, void* workspace,
+                         size_t workspace_bytes, sphq_stream stream) {
+  g_last_error.clear();
+  if (!h) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemm_ws: NULL handle");
+  if (batch < 1 || batch > SPHQ_GEMM_MAX_BATCH)
+    return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm_ws: batch must be 1..SPHQ_GEMM_MAX_BATCH");
+  if (!x || reinterpret_cast<uintptr_t>(x) % 16)
+    return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemm_ws: x must be a 16-byte aligned pointer");
+  if (!y || reinterpret_cast<uintptr_t>(y) % 2)
+    return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemm_ws: y must be a 2-byte aligned pointer");
+  if (!h->packed) return set_error(SPHQ_ERR_NOT_PACKED, "sphq_gemm_ws: handle not packed");
+  if (h->dim != 8) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm_ws: 8-D vectors only");
+  if (!workspace) return launch_gemm(h, x, y, batch, reinterpret_cast<cudaStream_t>(stream));
+  return launch_gemm_two_pass(h, x, y, batch, workspace, workspace_bytes,
+                              reinterpret_cast<cudaStream_t>(stream));
+}
+
 sphq_status sphq_get_gemm_shape(sphq_handle h, int batch, sphq_gemm_info* out) {
   g_last_error.clear();
   if (!h || !out) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_get_gemm_shape: NULL argument");

@@ -37,6 +37,7 @@
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cstdio>
 #include <mutex>
 
@@ -46,6 +47,10 @@
 namespace sphq {
 
 constexpr int kGemmBM = 128;                    // activation rows per tile (MMA M)
+// Pseudo format of the two-pass product: the B operand is a decoded W_hat
+// (rows x cols fp16 in global memory, written by decode_units_kernel) that
+// the TMA warp loads beside the activations; no codebook, no decode warps.
+constexpr int kFmtDense = 0;
 // One decode warp per 16-row tile of the weight tile (16 or 8), then the MMA
 // warp and the TMA warp.
 constexpr int gemm_threads(int bn) { return (bn / kRowsPerTile + 2) * 32; }
@@ -129,7 +134,9 @@ __device__ __forceinline__ void decode_word(const Unit<FMT>& u, const UnitConst<
 // or 32 (64-byte swizzle, half the ring memory, for the 128 KiB W3 codebook).
 template <int FMT, int MT, int BK, int BN>
 __global__ void __launch_bounds__(gemm_threads(BN), 1)
-    gemm_kernel(const GemmArgs a, const __grid_constant__ CUtensorMap tmap) {
+    gemm_kernel(const GemmArgs a, const __grid_constant__ CUtensorMap tmap,
+                const __grid_constant__ CUtensorMap tmap_w) {
+  constexpr bool kDense = FMT == kFmtDense;   // B tiles by TMA from a decoded W_hat
   constexpr int kTilesN = BN / kRowsPerTile;  // row tiles per weight tile
   constexpr int kDecodeWarps = kTilesN;       // one row tile each
   constexpr int kMmaWarp = kDecodeWarps, kTmaWarp = kDecodeWarps + 1;
@@ -155,15 +162,17 @@ __global__ void __launch_bounds__(gemm_threads(BN), 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
-      mbar_init(full0 + 8u * s, kDecodeWarps + 1);
+      mbar_init(full0 + 8u * s, kDense ? 1 : kDecodeWarps + 1);
       mbar_init(empty0 + 8u * s, 1);
     }
     mbar_init(acc_bar, 1);
     mbar_init(cb_bar, 1);
     fence_mbar_init();
-    mbar_arrive_expect_tx(cb_bar, a.cb_bytes);
-    for (uint32_t o = 0; o < a.cb_bytes; o += 32768u)
-      bulk_g2s(sbase + a.off_cb + o, a.cbimage + o, min(32768u, a.cb_bytes - o), cb_bar);
+    if constexpr (!kDense) {
+      mbar_arrive_expect_tx(cb_bar, a.cb_bytes);
+      for (uint32_t o = 0; o < a.cb_bytes; o += 32768u)
+        bulk_g2s(sbase + a.off_cb + o, a.cbimage + o, min(32768u, a.cb_bytes - o), cb_bar);
+    }
   }
   if (warp == kMmaWarp) {
     umma::tmem_alloc(smem_u32(tslot), kCols);
@@ -177,10 +186,14 @@ __global__ void __launch_bounds__(gemm_threads(BN), 1)
   if (warp == kTmaWarp) {
     if (lane == 0) {
       umma::prefetch_tmap(&tmap);
+      if constexpr (kDense) umma::prefetch_tmap(&tmap_w);
       for (int i = 0, s = 0, r = 0; i < nk; ++i) {
         if (r > 0 && !mbar_wait(empty0 + 8u * s, (r - 1) & 1)) atomicOr(a.flag, 2);
-        mbar_arrive_expect_tx(full0 + 8u * s, kStageA);
+        mbar_arrive_expect_tx(full0 + 8u * s, kStageA + (kDense ? kTileB : 0u));
         umma::tma_load_2d(sbase + s * kStageA, &tmap, i * BK, tok0, full0 + 8u * s);
+        if constexpr (kDense)  // the W_hat tile: BN weight rows x BK columns
+          umma::tma_load_2d(sbase + a.off_b + s * kTileB, &tmap_w, i * BK, rt0 * kRowsPerTile,
+                            full0 + 8u * s);
         if (++s == S) s = 0, ++r;
       }
     }
@@ -209,6 +222,7 @@ __global__ void __launch_bounds__(gemm_threads(BN), 1)
     }
     __syncwarp();
   } else {
+    if constexpr (!kDense) {
     // ---- decode warps: W_hat slices into the B tiles ----
     const int q = lane & 3, gid = lane >> 2;
     constexpr int UB = Layout<FMT>::kUnitBytes;
@@ -257,6 +271,7 @@ __global__ void __launch_bounds__(gemm_threads(BN), 1)
       if (lane == 0) mbar_arrive(full0 + 8u * s);
       if (++s == S) s = 0, ++r;
     }
+    }  // decode warps (the two-pass form has none in the main loop)
 
     // ---- epilogue: accumulators -> fp16 Y ----
     if (!mbar_wait(acc_bar, 0) && lane == 0) atomicOr(a.flag, 2);
@@ -308,6 +323,64 @@ __global__ void __launch_bounds__(gemm_threads(BN), 1)
   }
 }
 
+// First pass of the two-pass product: W_hat (rows x cols fp16, row-major)
+// from the packed units, exactly as Eq. (7) and Eq. (4) define it (the
+// GEMV's batch 3-8 decode, bit for bit the output of sphq_decode).  CTAs are
+// persistent (a grid of the resident count) and stage the codebook image once;
+// each of the 16 warps takes whole units, with the next unit's load in flight
+// while it decodes the current one; a lane rebuilds its eight vectors and
+// stores each as 16 bytes (a row's four lanes write 64 contiguous bytes per
+// word).
+constexpr int kDecodeUnitsWarps = 16;
+template <int FMT>
+__global__ void __launch_bounds__(kDecodeUnitsWarps * 32) decode_units_kernel(const uint8_t* __restrict__ units,
+                                                           const uint8_t* __restrict__ cbimage,
+                                                           uint32_t cb_bytes, uint16_t* __restrict__ w,
+                                                           int rows, int cols, int nrt, int ng,
+                                                           int* flag) {
+  extern __shared__ __align__(128) uint8_t smem[];
+  __shared__ __align__(8) uint64_t bar;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int q = lane & 3, gid = lane >> 2;
+  const uint32_t b = smem_u32(&bar);
+  if (threadIdx.x == 0) {
+    mbar_init(b, 1);
+    fence_mbar_init();
+    mbar_arrive_expect_tx(b, cb_bytes);
+    for (uint32_t o = 0; o < cb_bytes; o += 32768u)
+      bulk_g2s(smem_u32(smem) + o, cbimage + o, min(32768u, cb_bytes - o), b);
+  }
+  __syncthreads();
+  if (!mbar_wait(b, 0) && lane == 0) atomicOr(flag, 2);
+  SmemCodebook cb;
+  cb.base = smem;
+  cb.copyoff = fmt_small(FMT) ? (uint32_t)(lane & 7) * 16u : 0u;
+  constexpr int UB = Layout<FMT>::kUnitBytes;
+  const int total = nrt * ng;
+  const int nwarps = (int)gridDim.x * kDecodeUnitsWarps;
+  int u = (int)blockIdx.x * kDecodeUnitsWarps + warp;
+  Unit<FMT> nxt = {};
+  if (u < total) nxt = load_unit<FMT>(units + (size_t)u * UB, lane);
+  for (; u < total; u += nwarps) {
+    const int g = u / nrt, rt = u - g * nrt;  // unit (rt, g) is number g * nrt + rt
+    const Unit<FMT> un = nxt;
+    if (u + nwarps < total) nxt = load_unit<FMT>(units + (size_t)(u + nwarps) * UB, lane);
+    const UnitConst<FMT> kc = unit_const<FMT>(un, q);
+    const int rA = rt * kRowsPerTile + gid, rB = rA + 8;
+    uint16_t* pa = w + (size_t)rA * cols + (size_t)g * kGroupCols + 8 * q;
+    uint16_t* pb = pa + (size_t)8 * cols;
+#pragma unroll
+    for (int m = 0; m < 4; ++m) {
+      uint4 sa, sb;
+      uint32_t qp;
+      word_directions<FMT>(un, kc, m, q, cb, sa, sb, qp);
+      const uint32_t r = radius_pair<fmt_radius_bits(FMT)>(qp, kc.d2, kc.m2);
+      if (rA < rows) *reinterpret_cast<uint4*>(pa + 32 * m) = scale_block(sa, bcast_lo(r));
+      if (rB < rows) *reinterpret_cast<uint4*>(pb + 32 * m) = scale_block(sb, bcast_hi(r));
+    }
+  }
+}
+
 // ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
@@ -353,6 +426,12 @@ static const void* gemm_ptr(int mt, int bk, int bn) {
 }
 
 static const void* gemm_kernel_ptr(int fmt, int mt, int bk, int bn) {
+  if (fmt == kFmtDense) {
+    if (bk != 64) return nullptr;
+    if (bn == 256) return mt == 2 ? (const void*)&gemm_kernel<kFmtDense, 2, 64, 256>
+                                  : (const void*)&gemm_kernel<kFmtDense, 1, 64, 256>;
+    return bn == 128 && mt == 1 ? (const void*)&gemm_kernel<kFmtDense, 1, 64, 128> : nullptr;
+  }
   switch (fmt) {
 #define SPHQ_GEMM_PTR(F) \
   case F:                \
@@ -380,9 +459,10 @@ struct GemmSmem {
   size_t total = 0;
 };
 
-static GemmSmem gemm_smem(const sphq_handle_s* h, int optin, int mt, int bk, int bn) {
+static GemmSmem gemm_smem(const sphq_handle_s* h, int optin, int mt, int bk, int bn,
+                          bool dense = false) {
   GemmSmem L;
-  L.cb_bytes = fmt_small(h->fmt) ? (uint32_t)h->K * 8u * 16u : (uint32_t)h->K * 16u;
+  L.cb_bytes = dense ? 0u : fmt_small(h->fmt) ? (uint32_t)h->K * 8u * 16u : (uint32_t)h->K * 16u;
   for (int S = 4; S >= 2; --S) {
     const size_t off_b = (size_t)S * mt * tile_a_bytes(bk);
     const size_t off_cb = off_b + (size_t)S * tile_b_bytes(bk, bn);
@@ -411,7 +491,8 @@ struct GemmShape {
 // 0.64, one of 128 rows: 0.5), unless sphq_set_gemm_shape fixed MT / BN; a
 // candidate needs a ring of two stages next to the codebook, with 64-column
 // stages if they fit, else 32-column ones (W3 with two activation tiles).
-static GemmShape select_gemm_shape(const sphq_handle_s* h, int batch, int optin) {
+static GemmShape select_gemm_shape(const sphq_handle_s* h, int batch, int optin,
+                                   bool dense = false) {
   const int sms = h->sm_count > 0 ? h->sm_count : 1;
   static const int kShapes[3][2] = {{2, 256}, {1, 256}, {1, 128}};
   static const double kEff[3] = {1.0, 0.64, 0.5};
@@ -422,8 +503,8 @@ static GemmShape select_gemm_shape(const sphq_handle_s* h, int batch, int optin)
     if (h->gemm_mt ? m != h->gemm_mt : (m == 2 && batch <= kGemmBM)) continue;
     if (h->gemm_bn && n != h->gemm_bn) continue;
     for (int k : {64, 32}) {
-      if (!gemm_kernel_ptr(h->fmt, m, k, n)) continue;
-      const GemmSmem T = gemm_smem(h, optin, m, k, n);
+      if (!gemm_kernel_ptr(dense ? kFmtDense : h->fmt, m, k, n)) continue;
+      const GemmSmem T = gemm_smem(h, optin, m, k, n, dense);
       if (T.stages < 2) continue;
       const long long ctas = (long long)((h->nrt + n / kRowsPerTile - 1) / (n / kRowsPerTile)) *
                              ((batch + kGemmBM * m - 1) / (kGemmBM * m));
@@ -460,23 +541,29 @@ sphq_status gemm_shape_info(sphq_handle h, int batch, sphq_gemm_info* out) {
   return SPHQ_OK;
 }
 
-sphq_status launch_gemm(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s) {
+// One launch of the product kernel: the fused form (w_hat == nullptr), or the
+// second pass of the two-pass form reading the decoded w_hat.
+static sphq_status launch_gemm_kernel(sphq_handle h, const void* x, void* y, int batch,
+                                      cudaStream_t s, const void* w_hat) {
+  const bool dense = w_hat != nullptr;
   EncodeTiledFn enc = encode_fn();
   if (!enc) return set_error(SPHQ_ERR_CUDA, "sphq_gemm: cuTensorMapEncodeTiled unavailable");
   int optin = 0;
   sphq_status st = device_smem_optin(h, &optin);
   if (st != SPHQ_OK) return st;
-  const GemmShape g = select_gemm_shape(h, batch, optin);
+  const GemmShape g = select_gemm_shape(h, batch, optin, dense);
   if (!g.mt) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm: no shape fits this device");
   const int mt = g.mt, bk = g.bk, bn = g.bn;
   const GemmSmem& L = g.L;
   if (log_enabled())
     std::fprintf(stderr,
-                 "sphq: gemm %d x %d, batch %d: %d activation tile(s) x %d weight rows, "
+                 "sphq: gemm %d x %d, batch %d%s: %d activation tile(s) x %d weight rows, "
                  "%d-column stages x %d, %zu B shared\n",
-                 h->rows, h->cols, batch, mt, bn, bk, L.stages, L.total);
+                 h->rows, h->cols, batch, dense ? " (two-pass, decoded W_hat)" : "", mt, bn, bk,
+                 L.stages, L.total);
   cudaError_t e;
-  const void* kfn = gemm_kernel_ptr(h->fmt, mt, bk, bn);
+  const int kfmt = dense ? kFmtDense : h->fmt;
+  const void* kfn = gemm_kernel_ptr(kfmt, mt, bk, bn);
   {
     // the attribute belongs to the kernel on the current device: once per
     // (device, kernel)
@@ -484,7 +571,7 @@ sphq_status launch_gemm(sphq_handle h, const void* x, void* y, int batch, cudaSt
     static bool done[64][16][3][2][2] = {};
     std::lock_guard<std::mutex> lock(mu);
     if (h->device < 0 || h->device >= 64) return set_error(SPHQ_ERR_DEVICE, "device index out of range");
-    bool& d = done[h->device][h->fmt][mt][bk == 64][bn == 256];
+    bool& d = done[h->device][kfmt][mt][bk == 64][bn == 256];
     if (!d) {
       e = cudaFuncSetAttribute(kfn, cudaFuncAttributeMaxDynamicSharedMemorySize, optin);
       if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(gemm)");
@@ -503,9 +590,22 @@ sphq_status launch_gemm(sphq_handle h, const void* x, void* y, int batch, cudaSt
                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (cr != CUDA_SUCCESS)
     return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemm: cuTensorMapEncodeTiled rejected x");
+  // decoded weights (two-pass form): rows x cols fp16, boxes of BN rows x 64
+  // columns in the 128-byte swizzle, the layout the decode warps write
+  CUtensorMap tmap_w = tmap;
+  if (dense) {
+    const cuuint64_t wdim[2] = {(cuuint64_t)h->cols, (cuuint64_t)h->rows};
+    const cuuint64_t wstride[1] = {(cuuint64_t)h->cols * 2};
+    const cuuint32_t wbox[2] = {(cuuint32_t)bk, (cuuint32_t)bn};
+    cr = enc(&tmap_w, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(w_hat), wdim, wstride,
+             wbox, estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (cr != CUDA_SUCCESS)
+      return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemm_ws: cuTensorMapEncodeTiled rejected the workspace");
+  }
   GemmArgs a;
-  a.units = (const uint8_t*)h->units;
-  a.cbimage = (const uint8_t*)(fmt_small(h->fmt) ? h->cbimage : h->codebook);
+  a.units = dense ? nullptr : (const uint8_t*)h->units;
+  a.cbimage = dense ? nullptr : (const uint8_t*)(fmt_small(h->fmt) ? h->cbimage : h->codebook);
   a.y = (uint16_t*)y;
   a.flag = h->flag + 1;
   a.rows = h->rows;
@@ -519,10 +619,93 @@ sphq_status launch_gemm(sphq_handle h, const void* x, void* y, int batch, cudaSt
   a.off_bar = L.off_bar;
   const dim3 grid((unsigned)((h->nrt + bn / kRowsPerTile - 1) / (bn / kRowsPerTile)),
                   (unsigned)((batch + kGemmBM * mt - 1) / (kGemmBM * mt)));
-  void* args[] = {&a, &tmap};
+  void* args[] = {&a, &tmap, &tmap_w};
   e = cudaLaunchKernel(kfn, grid, dim3(gemm_threads(bn)), args, L.total, s);
   if (e != cudaSuccess) return cuda_error(e, "gemm launch");
   return SPHQ_OK;
+}
+
+sphq_status launch_gemm(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s) {
+  return launch_gemm_kernel(h, x, y, batch, s, nullptr);
+}
+
+static const void* decode_units_ptr(int fmt) {
+  switch (fmt) {
+#define SPHQ_DECODE_UNITS_PTR(F) \
+  case F:                        \
+    return (const void*)&decode_units_kernel<F>;
+    SPHQ_DECODE_UNITS_PTR(2)
+    SPHQ_DECODE_UNITS_PTR(3)
+    SPHQ_DECODE_UNITS_PTR(4)
+    SPHQ_DECODE_UNITS_PTR(5)
+    SPHQ_DECODE_UNITS_PTR(6)
+    SPHQ_DECODE_UNITS_PTR(7)
+    SPHQ_DECODE_UNITS_PTR(8)
+    SPHQ_DECODE_UNITS_PTR(9)
+#undef SPHQ_DECODE_UNITS_PTR
+    default:
+      return nullptr;
+  }
+}
+
+// Estimated times (us) of the two forms on this GB300: the fused kernel at its
+// measured rate per format family at large shapes (small codebooks ~1.3
+// PFLOP/s, the 8192-entry tables ~0.8, bound by their shared-memory
+// codebook gathers), the two-pass form as the decode pass (bytes written and
+// read at ~5 TB/s) plus the dense product at ~1.45 PFLOP/s.
+static void gemm_form_times(const sphq_handle_s* h, int batch, double* fused, double* two_pass) {
+  const double flops = 2.0 * batch * (double)h->rows * h->cols;
+  const double fused_rate = fmt_small(h->fmt) ? 1.30e15 : 0.80e15;
+  *fused = flops / fused_rate * 1e6;
+  const double wbytes = 2.0 * (double)h->rows * h->cols + (double)h->unit_bytes * h->nrt * h->ng;
+  *two_pass = wbytes / 5.0e12 * 1e6 + flops / 1.45e15 * 1e6;
+}
+
+sphq_status gemm_workspace_bytes(sphq_handle h, int batch, size_t* bytes) {
+  double tf = 0, tt = 0;
+  gemm_form_times(h, batch, &tf, &tt);
+  *bytes = tt < tf ? (size_t)h->rows * h->cols * 2 : 0;
+  return SPHQ_OK;
+}
+
+sphq_status launch_gemm_two_pass(sphq_handle h, const void* x, void* y, int batch, void* ws,
+                                 size_t ws_bytes, cudaStream_t s) {
+  const size_t need = (size_t)h->rows * h->cols * 2;
+  if (ws_bytes < need)
+    return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemm_ws: workspace smaller than rows x cols x 2 bytes");
+  if (reinterpret_cast<uintptr_t>(ws) % 16)
+    return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemm_ws: workspace must be 16-byte aligned");
+  const void* kfn = decode_units_ptr(h->fmt);
+  if (!kfn) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm_ws: unknown format");
+  const uint32_t cb_bytes = fmt_small(h->fmt) ? (uint32_t)h->K * 8u * 16u : (uint32_t)h->K * 16u;
+  cudaError_t e;
+  {
+    static std::mutex mu;
+    static bool done[64][16] = {};
+    std::lock_guard<std::mutex> lock(mu);
+    if (h->device < 0 || h->device >= 64) return set_error(SPHQ_ERR_DEVICE, "device index out of range");
+    if (!done[h->device][h->fmt]) {
+      e = cudaFuncSetAttribute(kfn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cb_bytes);
+      if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(decode_units)");
+      done[h->device][h->fmt] = true;
+    }
+  }
+  int per_sm = 0;
+  const int threads = kDecodeUnitsWarps * 32;
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kfn, threads, cb_bytes);
+  if (e != cudaSuccess || per_sm < 1) return cuda_error(e, "decode_units occupancy");
+  const long long units = (long long)h->nrt * h->ng;
+  const long long want = (units + kDecodeUnitsWarps - 1) / kDecodeUnitsWarps;
+  const int grid = (int)std::min<long long>(want, (long long)h->sm_count * per_sm);
+  const uint8_t* cb = (const uint8_t*)(fmt_small(h->fmt) ? h->cbimage : h->codebook);
+  const uint8_t* un = (const uint8_t*)h->units;
+  uint16_t* w = (uint16_t*)ws;
+  int rows = h->rows, cols = h->cols, nrt = h->nrt, ng = h->ng;
+  int* flag = h->flag + 1;
+  void* args[] = {&un, &cb, const_cast<uint32_t*>(&cb_bytes), &w, &rows, &cols, &nrt, &ng, &flag};
+  e = cudaLaunchKernel(kfn, dim3(grid), dim3(threads), args, cb_bytes, s);
+  if (e != cudaSuccess) return cuda_error(e, "decode_units launch");
+  return launch_gemm_kernel(h, x, y, batch, s, ws);
 }
 
 }  // namespace sphq

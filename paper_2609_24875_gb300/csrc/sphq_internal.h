@@ -78,6 +78,13 @@ sphq_status launch_encode(sphq_handle h, const float* w, uint8_t* sign, uint16_t
 sphq_status gemm_shape_info(sphq_handle h, int batch, sphq_gemm_info* out);
 // Enqueues the tensor-core product for any batch (validated arguments).
 sphq_status launch_gemm(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s);
+// Workspace bytes of the two-pass product for `batch` when it is estimated
+// faster than the fused kernel, else 0.
+sphq_status gemm_workspace_bytes(sphq_handle h, int batch, size_t* bytes);
+// Enqueues the two-pass product: W_hat decoded into `ws`, then the dense
+// tensor-core product reading it (validated x, y, batch).
+sphq_status launch_gemm_two_pass(sphq_handle h, const void* x, void* y, int batch, void* ws,
+                                 size_t ws_bytes, cudaStream_t s);
 // Enqueues the GEMV with caller-provided split-K scratch: `ws` holds at least
 // h->ws_floats floats and `tickets` h->nrt zeroed counters.
 sphq_status launch_gemv_scratch(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s,

@@ -79,6 +79,10 @@ def load() -> ctypes.CDLL:
         L.sphq_angle_codebook.restype = i32
         L.sphq_gemm.argtypes = [vp, vp, vp, i32, vp]
         L.sphq_gemm.restype = i32
+        L.sphq_gemm_workspace.argtypes = [vp, i32, ctypes.POINTER(sz)]
+        L.sphq_gemm_workspace.restype = i32
+        L.sphq_gemm_ws.argtypes = [vp, vp, vp, i32, vp, sz, vp]
+        L.sphq_gemm_ws.restype = i32
         L.sphq_check.argtypes = [vp, vp]
         L.sphq_check.restype = i32
         L.sphq_export.argtypes = [vp, vp, sz, ctypes.POINTER(sz)]
@@ -259,6 +263,38 @@ class SphqMatrix:
         if y is None:
             y = torch.empty((B, self.rows), dtype=torch.float16, device=x.device)
         _check(load().sphq_gemm(self._h, x.data_ptr(), y.data_ptr(), B, _stream_ptr(stream)))
+        return y
+
+    def gemm_workspace(self, batch: int) -> int:
+        """Workspace bytes for sphq_gemm_ws at `batch` when the two-pass form
+        is estimated faster, else 0 (sphq_gemm_workspace)."""
+        n = ctypes.c_size_t(0)
+        _check(load().sphq_gemm_workspace(self._h, batch, ctypes.byref(n)))
+        return n.value
+
+    def gemm_ws(self, x, workspace, y=None, stream=None):
+        """sphq_gemm_ws: the product with a caller-provided device workspace
+        (W_hat decoded into it, then a dense tensor-core pass); workspace None
+        runs the fused kernel.  x: (batch, cols) fp16; returns (batch, rows)."""
+        import torch
+        if x.dim() == 1:
+            x = x.unsqueeze(0)
+        B = x.shape[0]
+        if x.shape[1] != self.cols or x.element_size() != 2 or not x.is_cuda:
+            raise ValueError("x must be a (batch, cols) 2-byte CUDA tensor")
+        x = x.contiguous()
+        if y is None:
+            y = torch.empty((B, self.rows), dtype=torch.float16, device=x.device)
+        elif y.dtype != torch.float16 or y.numel() < B * self.rows or not y.is_contiguous():
+            raise ValueError("y must be a contiguous fp16 tensor of batch x rows elements")
+        if workspace is None:
+            wp, wn = None, 0
+        else:
+            if not workspace.is_cuda or not workspace.is_contiguous():
+                raise ValueError("workspace must be a contiguous CUDA tensor")
+            wp, wn = workspace.data_ptr(), workspace.numel() * workspace.element_size()
+        _check(load().sphq_gemm_ws(self._h, x.data_ptr(), y.data_ptr(), B, wp, wn,
+                                   _stream_ptr(stream)))
         return y
 
     def gemm_ptr(self, x_ptr: int, y_ptr: int, batch: int, stream_ptr: int) -> None:
