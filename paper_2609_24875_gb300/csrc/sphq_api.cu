@@ -727,8 +727,14 @@ sphq_status sphq_check(sphq_handle h, sphq_stream stream) {
 }
 
 // Copies n16 16-byte words from host memory (a mapped pinned buffer read over
-// the CPU-GPU link) into a device buffer.
+// the CPU-GPU link) into a device buffer.  Launched as a programmatic
+// dependent: it lets the GEMV that follows launch at once (its prologue only
+// reads the immutable codes and codebook), and waits for the previous kernel
+// before it reads x (which that kernel may have written) or overwrites the
+// staging buffer (which a previous GEMV of this handle may still read).
 __global__ void stage_x_kernel(const uint4* __restrict__ src, uint4* __restrict__ dst, int n16) {
+  asm volatile("griddepcontrol.launch_dependents;");
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i < n16) dst[i] = src[i];
 }
@@ -765,10 +771,19 @@ sphq_status sphq_gemv_host(sphq_handle h, const void* x_host, void* y_host, int 
   void* yd = const_cast<void*>(mapped_device_pointer(y_host));
   if (xd && yd && reinterpret_cast<uintptr_t>(xd) % 16 == 0 &&
       reinterpret_cast<uintptr_t>(yd) % 4 == 0) {
-    const int n16 = batch * h->cols * 2 / 16;
-    stage_x_kernel<<<(n16 + 255) / 256, 256, 0, s>>>(static_cast<const uint4*>(xd),
-                                                    static_cast<uint4*>(h->xstage), n16);
-    SPHQ_CUDA(cudaGetLastError(), "stage x");
+    int n16 = batch * h->cols * 2 / 16;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)((n16 + 255) / 256));
+    cfg.blockDim = dim3(256);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = h->pdl ? 1 : 0;
+    const uint4* src = static_cast<const uint4*>(xd);
+    uint4* dst = static_cast<uint4*>(h->xstage);
+    SPHQ_CUDA(cudaLaunchKernelEx(&cfg, stage_x_kernel, src, dst, n16), "stage x");
     return launch_gemv(h, h->xstage, yd, batch, s);
   }
   SPHQ_CUDA(cudaMemcpyAsync(h->xstage, x_host, (size_t)batch * h->cols * 2,

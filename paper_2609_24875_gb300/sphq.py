@@ -342,15 +342,15 @@ class SphqMatrix:
         """Host-buffer GEMV: x_host (batch, cols) and y_host (batch, rows) are
         2-byte CPU tensors (pinned for asynchrony); the copies and the GEMV are
         enqueued on the stream, so synchronise it before reading y_host."""
-        if x_host.is_cuda or y_host.is_cuda:
-            raise ValueError("gemv_host takes host tensors")
-        if x_host.dim() == 1:
-            x_host = x_host.unsqueeze(0)
-        B = x_host.shape[0]
-        if (x_host.shape[1] != self.cols or tuple(y_host.shape[-1:]) != (self.rows,)
-                or not x_host.is_contiguous() or not y_host.is_contiguous()
+        xs, ys = x_host.shape, y_host.shape
+        if len(xs) == 1:
+            xs = (1, xs[0])
+        B = xs[0]
+        if (xs[1] != self.cols or len(ys) == 0 or ys[-1] != self.rows or x_host.is_cuda
+                or y_host.is_cuda or not x_host.is_contiguous() or not y_host.is_contiguous()
                 or y_host.numel() != B * self.rows):
-            raise ValueError("x_host must be (batch, cols) and y_host (batch, rows), contiguous")
+            raise ValueError("gemv_host takes contiguous host tensors x_host (batch, cols) and "
+                             "y_host (batch, rows)")
         _check(load().sphq_gemv_host(self._h, x_host.data_ptr(), y_host.data_ptr(), B,
                                      _stream_ptr(stream)))
 
