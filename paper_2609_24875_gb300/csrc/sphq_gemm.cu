@@ -679,21 +679,26 @@ sphq_status launch_gemm_two_pass(sphq_handle h, const void* x, void* y, int batc
   if (!kfn) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm_ws: unknown format");
   const uint32_t cb_bytes = fmt_small(h->fmt) ? (uint32_t)h->K * 8u * 16u : (uint32_t)h->K * 16u;
   cudaError_t e;
+  const int threads = kDecodeUnitsWarps * 32;
+  int per_sm = 0;
   {
+    // the kernel's shared-memory attribute and its resident count, once per
+    // (device, format), so that later calls (and stream captures) only launch
     static std::mutex mu;
-    static bool done[64][16] = {};
+    static int resident[64][16] = {};
     std::lock_guard<std::mutex> lock(mu);
     if (h->device < 0 || h->device >= 64) return set_error(SPHQ_ERR_DEVICE, "device index out of range");
-    if (!done[h->device][h->fmt]) {
+    if (!resident[h->device][h->fmt]) {
       e = cudaFuncSetAttribute(kfn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)cb_bytes);
       if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(decode_units)");
-      done[h->device][h->fmt] = true;
+      int n = 0;
+      e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kfn, threads, cb_bytes);
+      if (e != cudaSuccess) return cuda_error(e, "decode_units occupancy");
+      if (n < 1) return set_error(SPHQ_ERR_CUDA, "decode_units: no resident block");
+      resident[h->device][h->fmt] = n;
     }
+    per_sm = resident[h->device][h->fmt];
   }
-  int per_sm = 0;
-  const int threads = kDecodeUnitsWarps * 32;
-  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kfn, threads, cb_bytes);
-  if (e != cudaSuccess || per_sm < 1) return cuda_error(e, "decode_units occupancy");
   const long long units = (long long)h->nrt * h->ng;
   const long long want = (units + kDecodeUnitsWarps - 1) / kDecodeUnitsWarps;
   const int grid = (int)std::min<long long>(want, (long long)h->sm_count * per_sm);
