@@ -334,9 +334,10 @@ sphq_status sphq_gemv_noalloc(sphq_handle h, const void* x, void* y, int batch,
  *   y      batch x rows fp16, device pointer, 2-byte aligned; written in full.
  *   batch  1..SPHQ_GEMM_MAX_BATCH; efficient from a few dozen rows up (tiles
  *          of 128 activation rows); sphq_gemv is the fast path for batch <= 8.
- *          Batches of 9..16 run as two GEMV launches of 3..8 rows (full mode:
- *          exact w_hat, fp32 accumulation of exact products) when y is 4-byte
- *          aligned and no shape is fixed with sphq_set_gemm_shape.
+ *          Batches of 9..64 run as GEMV launches of 3..8 rows (full mode:
+ *          exact w_hat, fp32 accumulation of exact products) when that is
+ *          estimated faster than the tensor-core kernel, y is 4-byte aligned
+ *          and no shape is fixed with sphq_set_gemm_shape.
  *
  * Asynchronous on `stream`, no allocation (graph-capturable).  Numerics: each
  * weight is the exact fp16 W_hat of sphq_decode, products are exact in fp32,

@@ -662,20 +662,27 @@ sphq_status sphq_gemm(sphq_handle h, const void* x, void* y, int batch, sphq_str
   if (!h->packed) return set_error(SPHQ_ERR_NOT_PACKED, "sphq_gemm: handle not packed");
   if (h->dim != 8) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm: 8-D vectors only");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  // 9..16 rows: two GEMV launches of 3..8 rows each (their full mode forms
-  // every w_hat exactly and accumulates the exact products in fp32, like the
-  // tensor-core kernel), which stream the weights twice but keep every SM
-  // busy, where the tensor-core kernel would have only rows / 128 CTAs
-  // (measured 2-2.5x faster on the 7B-class projections and 8192^2).  The
-  // first part is 6 or 8 rows so that the second part's y stays 4-byte
-  // aligned; a y that is not 4-byte aligned takes the tensor-core kernel.
-  if (batch > SPHQ_MAX_BATCH && batch <= 2 * SPHQ_MAX_BATCH && h->gemm_mt == 0 &&
-      h->gemm_bn == 0 && reinterpret_cast<uintptr_t>(y) % 4 == 0) {
-    const int b0 = batch <= 12 ? 6 : 8;
-    sphq_status st = launch_gemv(h, x, y, b0, s);
-    if (st != SPHQ_OK) return st;
-    return launch_gemv(h, static_cast<const uint16_t*>(x) + (size_t)b0 * h->cols,
-                       static_cast<uint16_t*>(y) + (size_t)b0 * h->rows, batch - b0, s);
+  // 9..64 rows, when estimated faster: GEMV launches of 3..8 rows (their full
+  // mode forms every w_hat exactly and accumulates the exact products in
+  // fp32, like the tensor-core kernel), which stream the weights once per
+  // launch but keep every SM busy, where the tensor-core kernel has only
+  // rows / BN CTAs per 128 rows.  Parts are 8 rows, or 6 before a last part of
+  // 3 or 4, so every part starts at an even row and its y stays 4-byte
+  // aligned; a y that is not 4-byte aligned, or a shape fixed with
+  // sphq_set_gemm_shape, takes the tensor-core kernel.
+  if (h->gemm_mt == 0 && h->gemm_bn == 0 && reinterpret_cast<uintptr_t>(y) % 4 == 0 &&
+      gemm_prefers_gemv(h, batch)) {
+    const uint16_t* xs = static_cast<const uint16_t*>(x);
+    uint16_t* ys = static_cast<uint16_t*>(y);
+    for (int done = 0; done < batch;) {
+      const int left = batch - done;
+      const int part = left > 10 ? 8 : left > 8 ? 6 : left;
+      sphq_status st = launch_gemv(h, xs + (size_t)done * h->cols, ys + (size_t)done * h->rows,
+                                   part, s);
+      if (st != SPHQ_OK) return st;
+      done += part;
+    }
+    return SPHQ_OK;
   }
   return launch_gemm(h, x, y, batch, s);
 }

@@ -78,6 +78,9 @@ sphq_status launch_encode(sphq_handle h, const float* w, uint8_t* sign, uint16_t
 sphq_status gemm_shape_info(sphq_handle h, int batch, sphq_gemm_info* out);
 // Enqueues the tensor-core product for any batch (validated arguments).
 sphq_status launch_gemm(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s);
+// Whether a batch of 9..64 rows is estimated faster as GEMV launches of 3..8
+// rows than on the tensor-core kernel.
+bool gemm_prefers_gemv(sphq_handle h, int batch);
 // Workspace bytes of the two-pass product for `batch` when it is estimated
 // faster than the fused kernel, else 0.
 sphq_status gemm_workspace_bytes(sphq_handle h, int batch, size_t* bytes);

@@ -173,10 +173,11 @@ def test_report_sizes_sampled(fmt, rows, cols, batch):
     torch.cuda.empty_cache()
 
 
-@pytest.mark.parametrize("batch", [9, 12, 13, 16])
-def test_batches_9_to_16(batch):
-    # two GEMV launches (6 + rest or 8 + rest rows) with an odd row count, and
-    # the tensor-core kernel when the shape is fixed: both against the oracle
+@pytest.mark.parametrize("batch", [9, 12, 13, 16, 19, 34, 64])
+def test_batches_9_to_64(batch):
+    # GEMV launches of 8 (or 6 before a last part of 3-4) rows where they are
+    # estimated faster, with an odd row count, and the tensor-core kernel when
+    # the shape is fixed: both against the oracle
     bits, v, K = 3, 4, 8192
     codes, x = inp.random_codes(bits, 1001, 768, seed=2100 + batch, B=batch, radius_bits=v, K=K)
     m = G.make_matrix(codes)
