@@ -173,13 +173,15 @@ def test_report_sizes_sampled(fmt, rows, cols, batch):
     torch.cuda.empty_cache()
 
 
+@pytest.mark.parametrize("fmt", FORMATS[:4], ids=FIDS[:4])
 @pytest.mark.parametrize("batch", [9, 12, 13, 16, 19, 34, 64])
-def test_batches_9_to_64(batch):
+def test_batches_9_to_64(fmt, batch):
     # GEMV launches of 8 (or 6 before a last part of 3-4) rows where they are
     # estimated faster, with an odd row count, and the tensor-core kernel when
     # the shape is fixed: both against the oracle
-    bits, v, K = 3, 4, 8192
-    codes, x = inp.random_codes(bits, 1001, 768, seed=2100 + batch, B=batch, radius_bits=v, K=K)
+    bits, v, K = fmt
+    codes, x = inp.random_codes(bits, 1001, 768, seed=2100 + batch + v, B=batch, radius_bits=v,
+                                K=K)
     m = G.make_matrix(codes)
     check_gemm(m, codes, x)
     m.set_gemm_shape(1, 256)
