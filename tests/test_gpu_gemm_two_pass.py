@@ -160,3 +160,24 @@ def test_graph_capture_and_side_stream():
         assert torch.equal(_bits(y12), _bits(y12_ref))
     m.check()
     m.close()
+
+
+@pytest.mark.parametrize("rows,cols,batch", [(1, 128, 1), (1, 128, 129), (17, 256, 200),
+                                             (300, 128, 64)])
+def test_tiny_and_ragged_shapes(rows, cols, batch):
+    # one row, one radius group, a batch of one: the W_hat and X tiles read
+    # zeros past the matrix and the batch; equal to the fused kernel and
+    # within the oracle's tolerance
+    codes, x = inp.random_codes(3, rows, cols, seed=1970 + rows + batch, B=batch)
+    m = G.make_matrix(codes)
+    m.set_gemm_shape(1, 128)  # the tensor-core kernel for every batch size
+    xd = G.x_dev(x)
+    y_fused = m.gemm(xd)
+    y_two = m.gemm_ws(xd, _ws(m))
+    torch.cuda.synchronize()
+    assert torch.equal(_bits(y_fused), _bits(y_two))
+    y = y_two.float().cpu().numpy().astype(np.float64)
+    y_ref, absdot = oracle.gemv(G.oracle_decode(codes, np.arange(rows)), x)
+    assert np.all(np.abs(y - y_ref) <= oracle.gemv_tolerance(absdot))
+    m.check()
+    m.close()
