@@ -19,7 +19,7 @@
  *
  * Supported settings (§3.1 bit budget, App. B): bits = 2 (W2: K = 64 entries,
  * 8 sign + 6 index + 4 radius bits = 2.25 bits/weight) and bits = 3
- * (W3: K = 8192 entries, 8 + 13 + 4 = 3.125 bits/weight); batch 1..8.
+ * (W3: K = 8192 entries, 8 + 13 + 4 = 3.125 bits/weight); batch 1..16.
  *
  * Conventions
  *   - All fp16 data are IEEE binary16 bit patterns (uint16_t storage).
@@ -64,7 +64,7 @@ typedef enum sphq_status {
   SPHQ_ERR_TIMEOUT = 7        /* a kernel gave up an on-chip wait (sphq_check) */
 } sphq_status;
 
-#define SPHQ_MAX_BATCH 8
+#define SPHQ_MAX_BATCH 16
 #define SPHQ_GEMM_MAX_BATCH (1 << 22)
 #define SPHQ_GROUP_COLS 128   /* scalars per radius group (§3.1)   */
 #define SPHQ_VECTOR_DIM 8     /* 8-D vectors (§3.1)                */
@@ -251,7 +251,11 @@ sphq_status sphq_angle_codebook(const float* phi, int K, double eps, double* cod
  *
  *   x      batch x cols fp16, device pointer, 16-byte aligned.
  *   y      batch x rows fp16, device pointer, 4-byte aligned; written in full.
- *   batch  1..SPHQ_MAX_BATCH.
+ *   batch  1..SPHQ_MAX_BATCH (16).  Each decoded weight serves every row of
+ *          the batch: 1-2 rows with the radius factored out of the dot
+ *          products, 3-8 rows as the N dimension of the tensor-core products,
+ *          9-16 rows as two such halves per decoded block (8-D vectors; 4-D
+ *          handles run 9-16 rows as two launches).
  *
  * Asynchronous on `stream`: no host synchronisation and no allocation, so it
  * may be captured in a CUDA graph.  One handle should not run two gemv calls
@@ -333,8 +337,8 @@ sphq_status sphq_gemv_noalloc(sphq_handle h, const void* x, void* y, int batch,
  *   x      batch x cols fp16, device pointer, 16-byte aligned.
  *   y      batch x rows fp16, device pointer, 2-byte aligned; written in full.
  *   batch  1..SPHQ_GEMM_MAX_BATCH; efficient from a few dozen rows up (tiles
- *          of 128 activation rows); sphq_gemv is the fast path for batch <= 8.
- *          Batches of 9..64 run as GEMV launches of 3..8 rows (full mode:
+ *          of 128 activation rows); sphq_gemv is the fast path for batch <= 16.
+ *          Batches of 9..64 run as GEMV launches of 3..16 rows (full modes:
  *          exact w_hat, fp32 accumulation of exact products) when that is
  *          estimated faster than the tensor-core kernel, y is 4-byte aligned
  *          and no shape is fixed with sphq_set_gemm_shape.
@@ -443,7 +447,7 @@ sphq_status sphq_decode(sphq_handle h, void* w, sphq_stream stream);
  * chosen with sphq_create_v) +
  * group parameters (4 bytes per 128 weights)
  * + codebook (K*16 bytes, once) + activations (2*batch*cols) + outputs
- * (2*batch*rows).  Returns 0 for a NULL handle or a batch outside 1..8.
+ * (2*batch*rows).  Returns 0 for a NULL handle or a batch outside 1..16.
  */
 size_t sphq_bytes(sphq_handle h, int batch);
 
@@ -453,7 +457,8 @@ size_t sphq_bytes(sphq_handle h, int batch);
  * work split.)  Row tiles of 16 rows go to thread-block clusters in contiguous
  * ranges; the CTAs of a cluster split the 128-column groups and reduce their
  * partial sums through distributed shared memory.  Fills *out; returns
- * SPHQ_ERR_INVALID_ARG for a NULL handle or out, or a batch outside 1..8.
+ * SPHQ_ERR_INVALID_ARG for a NULL handle or out, or a batch outside 1..16
+ * (4-D handles have no 16-row plan: grid 0 for batches above 8).
  */
 typedef struct sphq_plan_info {
   int grid;              /* CTAs launched */

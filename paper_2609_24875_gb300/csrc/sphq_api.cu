@@ -303,7 +303,7 @@ sphq_status sphq_get_plan(sphq_handle h, int batch, sphq_plan_info* out) {
   g_last_error.clear();
   if (!h || !out) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_get_plan: NULL handle or out");
   if (batch < 1 || batch > SPHQ_MAX_BATCH)
-    return set_error(SPHQ_ERR_INVALID_ARG, "sphq_get_plan: batch must be 1..8");
+    return set_error(SPHQ_ERR_INVALID_ARG, "sphq_get_plan: batch must be 1..16");
   const GemvPlan& p = h->plan[batch];
   out->grid = p.grid;
   out->cluster_size = p.csize;
@@ -311,7 +311,7 @@ sphq_status sphq_get_plan(sphq_handle h, int batch, sphq_plan_info* out) {
   out->tiles_per_cluster = p.tmax;
   out->warps_per_cta = p.warps_per_cta;
   out->smem_bytes = (int)p.smem;
-  out->staged_x = p.mode != 8;
+  out->staged_x = p.grid > 0 && p.mode <= 2;  // factored modes (1-2 rows) stage x
   out->ctas_per_sm = p.ctas_per_sm;
   return SPHQ_OK;
 }
@@ -320,7 +320,7 @@ sphq_status sphq_set_cluster_size(sphq_handle h, int batch, int cluster_size) {
   g_last_error.clear();
   if (!h) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_set_cluster_size: NULL handle");
   if (batch < 1 || batch > SPHQ_MAX_BATCH)
-    return set_error(SPHQ_ERR_INVALID_ARG, "sphq_set_cluster_size: batch must be 1..8");
+    return set_error(SPHQ_ERR_INVALID_ARG, "sphq_set_cluster_size: batch must be 1..16");
   if (cluster_size != 0 && cluster_size != 1 && cluster_size != 2 && cluster_size != 4 &&
       cluster_size != 8)
     return set_error(SPHQ_ERR_INVALID_ARG, "sphq_set_cluster_size: size must be 0, 1, 2, 4 or 8");
@@ -641,7 +641,7 @@ sphq_status sphq_gemv(sphq_handle h, const void* x, void* y, int batch, sphq_str
   g_last_error.clear();
   if (!h) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemv: NULL handle");
   if (batch < 1 || batch > SPHQ_MAX_BATCH)
-    return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemv: batch must be 1..8");
+    return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemv: batch must be 1..16");
   if (!x || reinterpret_cast<uintptr_t>(x) % 16)
     return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemv: x must be a 16-byte aligned pointer");
   if (!y || reinterpret_cast<uintptr_t>(y) % 4)
@@ -662,12 +662,12 @@ sphq_status sphq_gemm(sphq_handle h, const void* x, void* y, int batch, sphq_str
   if (!h->packed) return set_error(SPHQ_ERR_NOT_PACKED, "sphq_gemm: handle not packed");
   if (h->dim != 8) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm: 8-D vectors only");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  // 9..64 rows, when estimated faster: GEMV launches of 3..8 rows (their full
-  // mode forms every w_hat exactly and accumulates the exact products in
+  // 9..64 rows, when estimated faster: GEMV launches of 3..16 rows (their full
+  // modes form every w_hat exactly and accumulate the exact products in
   // fp32, like the tensor-core kernel), which stream the weights once per
   // launch but keep every SM busy, where the tensor-core kernel has only
-  // rows / BN CTAs per 128 rows.  Parts are 8 rows, or 6 before a last part of
-  // 3 or 4, so every part starts at an even row and its y stays 4-byte
+  // rows / BN CTAs per 128 rows.  Parts are 16 rows, or 14 before a last part
+  // of 3 or 4, so every part starts at an even row and its y stays 4-byte
   // aligned; a y that is not 4-byte aligned, or a shape fixed with
   // sphq_set_gemm_shape, takes the tensor-core kernel.
   if (h->gemm_mt == 0 && h->gemm_bn == 0 && reinterpret_cast<uintptr_t>(y) % 4 == 0 &&
@@ -676,7 +676,7 @@ sphq_status sphq_gemm(sphq_handle h, const void* x, void* y, int batch, sphq_str
     uint16_t* ys = static_cast<uint16_t*>(y);
     for (int done = 0; done < batch;) {
       const int left = batch - done;
-      const int part = left > 10 ? 8 : left > 8 ? 6 : left;
+      const int part = left > 18 ? 16 : left > 16 ? 14 : left;
       sphq_status st = launch_gemv(h, xs + (size_t)done * h->cols, ys + (size_t)done * h->rows,
                                    part, s);
       if (st != SPHQ_OK) return st;
@@ -781,7 +781,7 @@ sphq_status sphq_gemv_host(sphq_handle h, const void* x_host, void* y_host, int 
   g_last_error.clear();
   if (!h) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemv_host: NULL handle");
   if (batch < 1 || batch > SPHQ_MAX_BATCH)
-    return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemv_host: batch must be 1..8");
+    return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemv_host: batch must be 1..16");
   if (!x_host || !y_host) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemv_host: NULL buffer");
   if (!h->packed) return set_error(SPHQ_ERR_NOT_PACKED, "sphq_gemv_host: handle not packed");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);

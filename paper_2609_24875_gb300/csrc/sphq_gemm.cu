@@ -663,15 +663,15 @@ static void gemm_form_times(const sphq_handle_s* h, int batch, double* fused, do
   *two_pass = wbytes / 5.0e12 * 1e6 + flops / 1.45e15 * 1e6;
 }
 
-// Batches of 9..64 rows: whether ceil(batch / 8) GEMV launches (each
+// Batches of 9..64 rows: whether ceil(batch / 16) GEMV launches (each
 // streaming the weights once with every SM busy) are estimated faster than
 // the tensor-core kernel, whose CTAs each run the whole K and number only
 // rows / BN per 128 activation rows.  Per-CTA time of that kernel measured on
 // this GB300: ~5.2e-5 us per (column x weight row) for the small codebooks,
-// ~7.3e-5 for the 8192-entry tables; a GEMV of 3-8 rows ~2 us plus its bytes
-// at 28% of the HBM rate.
+// ~7.3e-5 for the 8192-entry tables; a GEMV of up to 16 rows ~2 us plus its
+// bytes at 25% of the HBM rate.
 bool gemm_prefers_gemv(sphq_handle h, int batch) {
-  if (batch <= SPHQ_MAX_BATCH || batch > 8 * SPHQ_MAX_BATCH) return false;
+  if (batch <= 8 || batch > 64) return false;
   int optin = 0;
   if (device_smem_optin(h, &optin) != SPHQ_OK) return false;
   const GemmShape g = select_gemm_shape(h, batch, optin);
@@ -681,9 +681,9 @@ bool gemm_prefers_gemv(sphq_handle h, int batch) {
                          ((batch + kGemmBM * g.mt - 1) / (kGemmBM * g.mt));
   const double waves = (double)((ctas + sms - 1) / sms);
   const double per_cta = (double)h->cols * g.bn * g.mt * (fmt_small(h->fmt) ? 5.2e-5 : 7.3e-5);
-  const double bytes8 = (double)h->unit_bytes * h->nrt * h->ng + 16.0 * (h->rows + h->cols);
+  const double bytes8 = (double)h->unit_bytes * h->nrt * h->ng + 32.0 * (h->rows + h->cols);
   const double t_gemv = (double)((batch + SPHQ_MAX_BATCH - 1) / SPHQ_MAX_BATCH) *
-                        (2.0 + bytes8 / (0.28 * 6794e9) * 1e6);
+                        (2.0 + bytes8 / (0.25 * 6794e9) * 1e6);
   return t_gemv < waves * per_cta;
 }
 

@@ -24,12 +24,17 @@ static uint32_t cb_bytes_for(int fmt) {
                                          : KernelShape<3>::kCbBytes;
 }
 
-static int mode_for(int batch) { return batch == 1 ? kFactored1 : batch == 2 ? kFactored2 : kFull; }
+static int mode_for(int batch) {
+  return batch == 1 ? kFactored1 : batch == 2 ? kFactored2 : batch <= kMaxBatch ? kFull : kFull16;
+}
 
 // formats with a one-CTA-per-SM build beside the two-CTA one
 static bool has_solo(int fmt) { return fmt == 2; }
 
 static const void* select_kernel(int fmt, int mode, int strip, bool solo = false) {
+  if (mode == kFull16)  // one build per format (strips of two, one CTA per SM)
+    return fmt == 2 ? kptr_full16<2>() : fmt == 3 ? kptr_full16<3>()
+           : fmt == kFmtW3V3 ? kptr_full16<kFmtW3V3>() : split_kernel(fmt, mode);
   return fmt == 2 ? (solo ? kptr_mode_solo<2>(mode) : kptr_mode<2>(mode))
          : fmt == 3 ? (strip == 4 ? kptr_mode<3, 4>(mode) : kptr_mode<3, 2>(mode))
          : fmt == kFmtW3V3 ? (strip == 4 ? kptr_mode<kFmtW3V3, 4>(mode) : kptr_mode<kFmtW3V3, 2>(mode))
@@ -51,8 +56,9 @@ static sphq_status allow_max_smem(int device, int optin) {
         for (int solo = 0; solo < 2; ++solo) {
           if (strip == 4 && !fmt_has_strip4(fmt)) continue;
           if (solo && !has_solo(fmt)) continue;
-          cudaError_t e = cudaFuncSetAttribute(select_kernel(fmt, mode, strip, solo),
-                                               cudaFuncAttributeMaxDynamicSharedMemorySize, optin);
+          const void* k = select_kernel(fmt, mode, strip, solo);
+          if (!k) continue;  // no 16-row build for 4-D vectors
+          cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, optin);
           if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute");
         }
   done[device] = true;
@@ -69,7 +75,7 @@ struct SmemLayout {
 
 static SmemLayout smem_layout(const sphq_handle_s* h, int mode, int warps, int csize, int tmax) {
   SmemLayout L{};
-  const int nbp = mode == kFull ? kMaxBatch : mode;
+  const int nbp = mode;  // batch rows of a partial block
   const size_t blk = (size_t)kRowsPerTile * nbp * 4;
   const int ngc_max = (h->ng + csize - 1) / csize;
   const int nown_max = (tmax + csize - 1) / csize;  // tiles one CTA owns
@@ -81,7 +87,7 @@ static SmemLayout smem_layout(const sphq_handle_s* h, int mode, int warps, int c
   L.zero = o;
   L.x = o + 320;
   L.x_pitch = (uint32_t)((size_t)ngc_max * kGroupCols * 2 + 64);
-  if (mode != kFull) o = L.x + (size_t)L.x_pitch * mode;
+  if (!mode_full(mode)) o = L.x + (size_t)L.x_pitch * mode;
   // receive slots: one block per (owned tile, rank, warp)
   o = align_up(o, 16);
   L.recv = o;
@@ -123,11 +129,13 @@ static sphq_status make_plan(sphq_handle h, int batch, int forced, int optin, Ge
     const int warps = warps_for(h->fmt);
     for (int staged = 1; staged >= 0; --staged) {
       int mode = mode_for(batch);
-      if (!staged) mode = kFull;
-      if (staged && mode == kFull) continue;
-      for (int solo = 0; solo < (has_solo(h->fmt) ? 2 : 1); ++solo) {
+      if (!staged && !mode_full(mode)) mode = kFull;
+      if (staged && mode_full(mode)) continue;
+      const int nsolo = mode == kFull16 ? 1 : has_solo(h->fmt) ? 2 : 1;
+      for (int solo = 0; solo < nsolo; ++solo) {
         // both strip sizes: same resources
         const void* k = select_kernel(h->fmt, mode, 2, solo);
+        if (!k) continue;
         for (int csize : {1, 2, 4, 8}) {
           if (csize > h->ng) break;
           if (forced && csize != forced) continue;
@@ -182,7 +190,7 @@ static sphq_status make_plan(sphq_handle h, int batch, int forced, int optin, Ge
           // shared memory did not fit at one wave) pays the fixed part again per
           // wave (measured: W3 18944 x 3584 batch 8 in two waves of clusters of
           // 4, 22.1 us against 15.6 us in one wave of single CTAs).
-          const double fixed = csize == 8 ? (mode == kFull ? 5.8 : 5.0) : 2.0;
+          const double fixed = csize == 8 ? (mode_full(mode) ? 5.8 : 5.0) : 2.0;
           const double shallow = 1.0 + 0.33 * (2 - std::min(tmax, 2));
           const double cost = fixed * waves + waves * 0.02 * tmax * ((h->ng + csize - 1) / csize) * shallow;
           // The one-CTA-per-SM build wins ties: at equal load the row tiles
@@ -200,9 +208,9 @@ static sphq_status make_plan(sphq_handle h, int batch, int forced, int optin, Ge
             p.off_recv = (uint32_t)L.recv;
             p.off_bar = (uint32_t)L.bar;
             // four-tile strips once a cluster holds three tiles or more (W3)
-            p.strip = fmt_has_strip4(h->fmt) && tmax >= 3 ? 4 : 2;
-            p.solo = solo != 0;
-          p.ctas_per_sm = solo ? 1
+            p.strip = mode != kFull16 && fmt_has_strip4(h->fmt) && tmax >= 3 ? 4 : 2;
+            p.solo = solo != 0 || mode == kFull16;
+          p.ctas_per_sm = p.solo ? 1
                           : fmt_small(h->fmt) || h->fmt == kFmt4D ? KernelShape<2>::kMinBlocks
                                                                    : KernelShape<3>::kMinBlocks;
             best = p;
@@ -232,6 +240,10 @@ sphq_status make_gemv_plans(sphq_handle h) {
   sphq_status st = device_optin(h, &optin);
   if (st != SPHQ_OK) return st;
   for (int batch = 1; batch <= SPHQ_MAX_BATCH; ++batch) {
+    if (batch > kMaxBatch && h->fmt == kFmt4D) {
+      h->plan[batch] = GemvPlan{};  // 4-D: two launches of at most 8 rows
+      continue;
+    }
     st = make_plan(h, batch, 0, optin, h->plan[batch]);
     if (st != SPHQ_OK) return st;
   }
@@ -251,6 +263,14 @@ sphq_status set_gemv_cluster_size(sphq_handle h, int batch, int csize) {
 }
 
 sphq_status launch_gemv(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s) {
+  if (batch > kMaxBatch && h->plan[batch].grid == 0) {
+    // no 16-row build (4-D vectors): 8 rows, then the rest
+    sphq_status st = launch_gemv(h, x, y, kMaxBatch, s);
+    if (st != SPHQ_OK) return st;
+    return launch_gemv(h, static_cast<const uint16_t*>(x) + (size_t)kMaxBatch * h->cols,
+                       static_cast<uint16_t*>(y) + (size_t)kMaxBatch * h->rows, batch - kMaxBatch,
+                       s);
+  }
   const GemvPlan& p = h->plan[batch];
   GemvArgs a;
   a.units = (const uint8_t*)h->units;

@@ -85,6 +85,9 @@ __host__ __device__ constexpr bool fmt_has_strip4(int fmt) { return fmt == 3 || 
 constexpr int kFactored1 = 1;  // batch 1
 constexpr int kFactored2 = 2;  // batch 2
 constexpr int kFull = 8;       // batch 3..8
+constexpr int kFull16 = 16;    // batch 9..16: two batch halves of 8 rows per decoded block
+// Modes that form w_hat exactly and put the batch in the MMA's N dimension.
+__host__ __device__ constexpr bool mode_full(int m) { return m == kFull || m == kFull16; }
 
 struct GemvArgs {
   const uint8_t* units;
@@ -319,20 +322,26 @@ __device__ __forceinline__ void word_directions(const Unit<BITS>& u, const UnitC
 // Accumulators of one warp for one row tile.
 template <int MODE>
 struct Acc {
-  static constexpr int NB = MODE == kFull ? 1 : MODE;
+  static constexpr int NB = mode_full(MODE) ? 1 : MODE;
   float f[NB][2];  // factored: [batch row][row gid / gid+8]
-  float d[4];      // full: MMA accumulator fragment
+  float d[4];      // full: MMA accumulator fragment (batch rows 0-7)
+  float e[MODE == kFull16 ? 4 : 1];  // batch rows 8-15 (kFull16)
   __device__ __forceinline__ void zero() {
 #pragma unroll
     for (int i = 0; i < NB; ++i) f[i][0] = f[i][1] = 0.f;
 #pragma unroll
     for (int i = 0; i < 4; ++i) d[i] = 0.f;
+    if constexpr (MODE == kFull16) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) e[i] = 0.f;
+    }
   }
 };
 
 // The lane's B-fragment data of one group: 8-D, v[m] = its activation row
-// at slot 4m+q (16 bytes); 4-D, v[s] = at vector 4s+q (8 bytes); or zeros.
-template <int BITS> struct XFrag { uint4 v[4]; };
+// at slot 4m+q (16 bytes), v2[m] the same for the second batch half (kFull16);
+// 4-D, v[s] = at vector 4s+q (8 bytes); or zeros.
+template <int BITS> struct XFrag { uint4 v[4]; uint4 v2[4]; };
 template <> struct XFrag<kFmt4D> { uint2 v[8]; };
 
 // 8-byte activation load kept in L1 (batch 3-8, 4-D vectors)
@@ -343,9 +352,10 @@ __device__ __forceinline__ uint2 ldg_x8(const uint8_t* p) {
 }
 
 // xp: this lane's first activation bytes of the group (8-D: slot q at 16 q,
-// words 64 bytes apart; 4-D: vector q at 8 q, pairs 32 bytes apart).
+// words 64 bytes apart; 4-D: vector q at 8 q, pairs 32 bytes apart); x2off:
+// bytes from its row to its second-half row (kFull16).
 template <int BITS, int MODE>
-__device__ __forceinline__ void load_x(XFrag<BITS>& xv, const uint8_t* xp) {
+__device__ __forceinline__ void load_x(XFrag<BITS>& xv, const uint8_t* xp, int x2off = 0) {
   if constexpr (BITS == kFmt4D) {
 #pragma unroll
     for (int s = 0; s < 8; ++s) {
@@ -357,12 +367,15 @@ __device__ __forceinline__ void load_x(XFrag<BITS>& xv, const uint8_t* xp) {
   } else {
 #pragma unroll
     for (int m = 0; m < 4; ++m) {
-      if constexpr (MODE == kFull)
+      if constexpr (mode_full(MODE))
         xv.v[m] = ldg_x16(reinterpret_cast<const uint16_t*>(xp) + 32 * m);
       else
         xv.v[m] = *reinterpret_cast<const uint4*>(xp + 64 * m);
+      if constexpr (MODE == kFull16)
+        xv.v2[m] = ldg_x16(reinterpret_cast<const uint16_t*>(xp + x2off) + 32 * m);
     }
   }
+  (void)x2off;
 }
 
 // One pair s of a 4-D unit: one MMA for the two 4-D vectors of the lane.
@@ -371,6 +384,7 @@ __device__ __forceinline__ void process_pair_4d(const Unit<kFmt4D>& cur,
                                                 const UnitConst<kFmt4D>& kc,
                                                 const XFrag<kFmt4D>& xv, const SmemCodebook& cb,
                                                 Acc<MODE>& acc) {
+  static_assert(MODE != kFull16, "4-D vectors take batches of at most 8 rows per launch");
   uint2 sa, sb;
   directions_4d<S>(cur.w, cur.s1, cb, cb.copyoff, true, sa, sb);
   const uint32_t r = radius_pair<4>(qpair_4d<S>(cur.w), kc.d2, kc.m2);
@@ -392,20 +406,26 @@ __device__ __forceinline__ void process_pair_4d(const Unit<kFmt4D>& cur,
 }
 
 // Word m of one unit (the two vectors of slot 4m+q of rows gid and gid+8)
-// against the activations xm of that slot (8-D formats).
+// against the activations xm of that slot (8-D formats); xm2: the second
+// batch half's (kFull16).
 template <int BITS, int MODE>
 __device__ __forceinline__ void process_word(const Unit<BITS>& cur, const UnitConst<BITS>& kc,
                                              const uint4& xm, int m, int q,
-                                             const SmemCodebook& cb, Acc<MODE>& acc) {
+                                             const SmemCodebook& cb, Acc<MODE>& acc,
+                                             const uint4& xm2 = uint4{}) {
   uint4 sa, sb;
   uint32_t qp;
   word_directions<BITS>(cur, kc, m, q, cb, sa, sb, qp);
   const uint32_t r = radius_pair<fmt_radius_bits(BITS)>(qp, kc.d2, kc.m2);
-  if constexpr (MODE == kFull) {
+  if constexpr (mode_full(MODE)) {
     const uint4 wa = scale_block(sa, bcast_lo(r));
     const uint4 wb = scale_block(sb, bcast_hi(r));
     mma16816(acc.d, wa.x, wb.x, wa.y, wb.y, xm.x, xm.y);
     mma16816(acc.d, wa.z, wb.z, wa.w, wb.w, xm.z, xm.w);
+    if constexpr (MODE == kFull16) {
+      mma16816(acc.e, wa.x, wb.x, wa.y, wb.y, xm2.x, xm2.y);
+      mma16816(acc.e, wa.z, wb.z, wa.w, wb.w, xm2.z, xm2.w);
+    }
   } else {
     float d[4];
     mma16816_zero(d, sa.x, sb.x, sa.y, sb.y, xm.x, xm.y);
@@ -423,7 +443,7 @@ __device__ __forceinline__ void process_word(const Unit<BITS>& cur, const UnitCo
 // The activations of word m of a group for this lane (8-D formats).
 template <int MODE>
 __device__ __forceinline__ uint4 load_x_word(const uint8_t* xp, int m) {
-  if constexpr (MODE == kFull)
+  if constexpr (mode_full(MODE))
     return ldg_x16(reinterpret_cast<const uint16_t*>(xp) + 32 * m);
   else
     return *reinterpret_cast<const uint4*>(xp + 64 * m);
@@ -452,11 +472,15 @@ __device__ __forceinline__ void process_unit(const Unit<BITS>& cur, const XFrag<
     uint32_t qp;
     word_directions<BITS>(cur, kc, m, q, cb, sa, sb, qp);
     const uint32_t r = radius_pair<fmt_radius_bits(BITS)>(qp, kc.d2, kc.m2);
-    if constexpr (MODE == kFull) {
+    if constexpr (mode_full(MODE)) {
       const uint4 wa = scale_block(sa, bcast_lo(r));
       const uint4 wb = scale_block(sb, bcast_hi(r));
       mma16816(acc.d, wa.x, wb.x, wa.y, wb.y, xv[m].x, xv[m].y);
       mma16816(acc.d, wa.z, wb.z, wa.w, wb.w, xv[m].z, xv[m].w);
+      if constexpr (MODE == kFull16) {
+        mma16816(acc.e, wa.x, wb.x, wa.y, wb.y, xf.v2[m].x, xf.v2[m].y);
+        mma16816(acc.e, wa.z, wb.z, wa.w, wb.w, xf.v2[m].z, xf.v2[m].w);
+      }
     } else {
       float d[4];
       mma16816_zero(d, sa.x, sb.x, sa.y, sb.y, xv[m].x, xv[m].y);
@@ -481,7 +505,7 @@ template <int MODE>
 __device__ __forceinline__ void send_partial(uint32_t raddr, uint32_t rbar, Acc<MODE>& acc,
                                              int lane, int batch) {
   const int gid = lane >> 2, q = lane & 3;
-  if constexpr (MODE == kFull) {
+  if constexpr (mode_full(MODE)) {
     // d[0..3] = D[gid][2q], D[gid][2q+1], D[gid+8][2q], D[gid+8][2q+1]
     if (2 * q < batch) {
       st_async4(raddr + 4u * ((2 * q) * kRowsPerTile + gid), acc.d[0], rbar);
@@ -490,6 +514,16 @@ __device__ __forceinline__ void send_partial(uint32_t raddr, uint32_t rbar, Acc<
     if (2 * q + 1 < batch) {
       st_async4(raddr + 4u * ((2 * q + 1) * kRowsPerTile + gid), acc.d[1], rbar);
       st_async4(raddr + 4u * ((2 * q + 1) * kRowsPerTile + gid + 8), acc.d[3], rbar);
+    }
+    if constexpr (MODE == kFull16) {  // e: batch rows 8 + 2q, 8 + 2q + 1
+      if (8 + 2 * q < batch) {
+        st_async4(raddr + 4u * ((8 + 2 * q) * kRowsPerTile + gid), acc.e[0], rbar);
+        st_async4(raddr + 4u * ((8 + 2 * q) * kRowsPerTile + gid + 8), acc.e[2], rbar);
+      }
+      if (9 + 2 * q < batch) {
+        st_async4(raddr + 4u * ((9 + 2 * q) * kRowsPerTile + gid), acc.e[1], rbar);
+        st_async4(raddr + 4u * ((9 + 2 * q) * kRowsPerTile + gid + 8), acc.e[3], rbar);
+      }
     }
   } else {
     // sum the lane's slots, then the quad's four lanes (slots q = 0..3)
@@ -551,7 +585,7 @@ __device__ __forceinline__ int share_lo_c(int n, int i) {
 template <int BITS, int MODE, int SIZE, bool LAST, int S>
 __device__ __forceinline__ void run_item(Unit<BITS> (&u)[S], Acc<MODE> (&acc)[S],
                                          const uint8_t* xp, const uint8_t* nb, unsigned nmask,
-                                         int lane, int q, const SmemCodebook& cb) {
+                                         int lane, int q, const SmemCodebook& cb, int x2off) {
   constexpr int UB = Layout<BITS>::kUnitBytes;
   auto reload = [&](int j) {
     if (LAST) {
@@ -562,7 +596,7 @@ __device__ __forceinline__ void run_item(Unit<BITS> (&u)[S], Acc<MODE> (&acc)[S]
   };
   if constexpr (BITS == kFmt4D || SIZE == 1) {
     XFrag<BITS> xv;
-    load_x<BITS, MODE>(xv, xp);
+    load_x<BITS, MODE>(xv, xp, x2off);
 #pragma unroll
     for (int j = 0; j < S; ++j) {
       if (j < SIZE) process_unit<BITS, MODE>(u[j], xv, q, cb, acc[j]);
@@ -576,15 +610,18 @@ __device__ __forceinline__ void run_item(Unit<BITS> (&u)[S], Acc<MODE> (&acc)[S]
 #pragma unroll
     for (int j = 0; j < SIZE; ++j) kc[j] = unit_const<BITS>(u[j], q);
     const uint4 x0 = load_x_word<MODE>(xp, 0), x1 = load_x_word<MODE>(xp, 1);
+    uint4 y0{}, y1{}, y2{}, y3{};  // the second batch half's words (kFull16)
+    if constexpr (MODE == kFull16) y0 = load_x_word<MODE>(xp + x2off, 0), y1 = load_x_word<MODE>(xp + x2off, 1);
 #pragma unroll
-    for (int j = 0; j < SIZE; ++j) process_word<BITS, MODE>(u[j], kc[j], x0, 0, q, cb, acc[j]);
+    for (int j = 0; j < SIZE; ++j) process_word<BITS, MODE>(u[j], kc[j], x0, 0, q, cb, acc[j], y0);
 #pragma unroll
-    for (int j = 0; j < SIZE; ++j) process_word<BITS, MODE>(u[j], kc[j], x1, 1, q, cb, acc[j]);
+    for (int j = 0; j < SIZE; ++j) process_word<BITS, MODE>(u[j], kc[j], x1, 1, q, cb, acc[j], y1);
     const uint4 x2 = load_x_word<MODE>(xp, 2), x3 = load_x_word<MODE>(xp, 3);
+    if constexpr (MODE == kFull16) y2 = load_x_word<MODE>(xp + x2off, 2), y3 = load_x_word<MODE>(xp + x2off, 3);
 #pragma unroll
     for (int j = 0; j < SIZE; ++j) {
-      process_word<BITS, MODE>(u[j], kc[j], x2, 2, q, cb, acc[j]);
-      process_word<BITS, MODE>(u[j], kc[j], x3, 3, q, cb, acc[j]);
+      process_word<BITS, MODE>(u[j], kc[j], x2, 2, q, cb, acc[j], y2);
+      process_word<BITS, MODE>(u[j], kc[j], x3, 3, q, cb, acc[j], y3);
       reload(j);
     }
     if constexpr (LAST) {
@@ -602,7 +639,7 @@ __device__ __forceinline__ void run_segment(Unit<BITS> (&u)[S], Acc<MODE> (&acc)
                                             int cnt, const uint8_t* ub, size_t gstride,
                                             const uint8_t* xp, int xstep, const uint8_t* nb,
                                             unsigned nmask, int lane, int q,
-                                            const SmemCodebook& cb) {
+                                            const SmemCodebook& cb, int x2off) {
   constexpr uint32_t kBytes = SIZE * Layout<BITS>::kUnitBytes;
   if constexpr (SIZE == 1) {
     // One-tile strips use the two register slots as a two-item ring (slot
@@ -617,33 +654,33 @@ __device__ __forceinline__ void run_segment(Unit<BITS> (&u)[S], Acc<MODE> (&acc)
       if (lane == 0 && c + 4 < cnt) prefetch_l2(ub + 4 * gstride, kBytes);
       if (lane == 0 && c + 5 < cnt) prefetch_l2(ub + 5 * gstride, kBytes);
       XFrag<BITS> xv;
-      load_x<BITS, MODE>(xv, xp);
+      load_x<BITS, MODE>(xv, xp, x2off);
       process_unit<BITS, MODE>(u[0], xv, q, cb, acc[0]);
       if (c + 2 < cnt) u[0] = load_unit<BITS>(ub + 2 * gstride, lane);
-      load_x<BITS, MODE>(xv, xp + xstep);
+      load_x<BITS, MODE>(xv, xp + xstep, x2off);
       process_unit<BITS, MODE>(u[1], xv, q, cb, acc[0]);
       if (c + 3 < cnt) u[1] = load_unit<BITS>(ub + 3 * gstride, lane);
       ub += 2 * gstride;
       xp += 2 * xstep;
     }
-    if (c < cnt) run_item<BITS, MODE, 1, true, S>(u, acc, xp, nb, 0u, lane, q, cb);
+    if (c < cnt) run_item<BITS, MODE, 1, true, S>(u, acc, xp, nb, 0u, lane, q, cb, x2off);
     return;
   }
   if (lane == 0 && cnt > 1) prefetch_l2(ub + gstride, kBytes);
   for (int c = 0; c + 1 < cnt; ++c) {
     if (lane == 0 && c + 2 < cnt) prefetch_l2(ub + 2 * gstride, kBytes);
-    run_item<BITS, MODE, SIZE, false, S>(u, acc, xp, ub + gstride, 0u, lane, q, cb);
+    run_item<BITS, MODE, SIZE, false, S>(u, acc, xp, ub + gstride, 0u, lane, q, cb, x2off);
     ub += gstride;
     xp += xstep;
   }
-  run_item<BITS, MODE, SIZE, true, S>(u, acc, xp, nb, nmask, lane, q, cb);
+  run_item<BITS, MODE, SIZE, true, S>(u, acc, xp, nb, nmask, lane, q, cb, x2off);
 }
 
 template <int BITS, int MODE, int WARPS, int MINB, int S>
 __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
   pdl_launch_dependents();
-  constexpr int NBP = MODE == kFull ? kMaxBatch : MODE;  // floats per row in a partial block
+  constexpr int NBP = MODE;  // floats per row in a partial block (batch rows of the mode)
   constexpr int kBlk = kRowsPerTile * NBP;                // floats per partial block
   constexpr int UB = Layout<BITS>::kUnitBytes;
   static_assert(S == 2 || S == 4, "strip sizes");
@@ -709,13 +746,13 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
       if (m0 >> j & 1u) u[j] = load_unit<BITS>(strip_base(s, g) + j * UB, lane);
   }
 
-  if (MODE != kFull && threadIdx.x < 16)  // zero block read by lanes that supply no activations
+  if (!mode_full(MODE) && threadIdx.x < 16)  // zero block read by lanes that supply no activations
     reinterpret_cast<uint4*>(smem + a.off_zero)[threadIdx.x] = make_uint4(0, 0, 0, 0);
   __syncthreads();                  // mbarrier initialisation visible to the CTA
   if (csize > 1) cluster_arrive_relaxed();  // ... and to the cluster (waited on below)
 
   pdl_wait();  // the previous kernel's outputs (our activations) are complete
-  if (MODE != kFull && threadIdx.x == 0) {
+  if (!mode_full(MODE) && threadIdx.x == 0) {
     const uint32_t row_bytes = (uint32_t)ngc * kGroupCols * 2;
     mbar_arrive_expect_tx(bar_x, row_bytes * MODE);
     for (int b = 0; b < MODE; ++b)
@@ -724,7 +761,7 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
   }
   if (csize > 1) cluster_wait();  // every CTA's receive mbarrier is initialised
   bool ok = mbar_wait_poll(bar_cb, 0);
-  if (MODE != kFull) ok &= mbar_wait_poll(bar_x, 0);
+  if (!mode_full(MODE)) ok &= mbar_wait_poll(bar_x, 0);
   if (!ok && lane == 0) atomicOr(a.flag, 2);
 
   SmemCodebook cb;
@@ -737,7 +774,7 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
   // read a zero block (stride 0), so the loop has no lane-dependent branch.
   int xb;
   bool provider;
-  if (MODE == kFull) {
+  if (mode_full(MODE)) {
     xb = gid;
     provider = gid < a.batch;
   } else {
@@ -745,13 +782,17 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
     provider = xb >= 0 && xb < MODE;
   }
   const uint8_t* x0;  // this lane's activation bytes of group g0
-  if (MODE == kFull)
+  if (mode_full(MODE))
     x0 = provider ? reinterpret_cast<const uint8_t*>(a.x + (size_t)xb * a.cols + (size_t)g0 * kGroupCols)
                   : reinterpret_cast<const uint8_t*>(a.zeros);
   else
     x0 = provider ? smem + a.off_x + xb * a.x_pitch : smem + a.off_zero;
   x0 += q * (BITS == kFmt4D ? 8 : 16);
   const int xstep = provider ? kGroupCols * 2 : 0;
+  // kFull16: bytes from this lane's activation row to its second-half row
+  // (batch row gid + 8), or 0 where that row is past the batch (the lane then
+  // reads its own row again; those product columns are never sent)
+  const int x2off = MODE == kFull16 && gid + 8 < a.batch ? 16 * a.cols : 0;
 
   // receive slot of (owned tile k, rank r, warp w): ((k * csize + r) * WARPS + w) * kBlk floats
   const uint32_t recv_base = smem_u32(smem + a.off_recv);
@@ -773,15 +814,15 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
     const uint8_t* nb = strip_base(s + 1, g0);
     const unsigned nmask = left > 0 ? strip_mask(s + 1) : 0u;
     if (s < nfull)
-      run_segment<BITS, MODE, S, S>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask, lane, q, cb);
+      run_segment<BITS, MODE, S, S>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask, lane, q, cb, x2off);
     else if (S > 1 && rest == 1)
-      run_segment<BITS, MODE, 1, S>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask, lane, q, cb);
+      run_segment<BITS, MODE, 1, S>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask, lane, q, cb, x2off);
     else if (S > 2 && rest == 2)
       run_segment<BITS, MODE, (S > 2 ? 2 : 1), S>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask,
-                                                  lane, q, cb);
+                                                  lane, q, cb, x2off);
     else if (S > 3)
       run_segment<BITS, MODE, (S > 3 ? 3 : 1), S>(u, acc, cnt, ub, gstride, xp, xstep, nb, nmask,
-                                                  lane, q, cb);
+                                                  lane, q, cb, x2off);
 #pragma unroll
     for (int j = 0; j < S; ++j) {
       const int tau = s * S + j;
@@ -809,9 +850,14 @@ __global__ void __launch_bounds__(WARPS * 32, MINB) gemv_kernel(const GemvArgs a
     const uint32_t slot =
         recv_base + 4u * (uint32_t)(((((tau >> cshift) << cshift) + crank) * WARPS + warp) * kBlk);
     const uint32_t owner = (uint32_t)(tau & (csize - 1));
-    if (lane < 4 * a.batch)
+    if constexpr (MODE == kFull16) {
+      for (int i = lane; i < 4 * a.batch; i += 32)  // 64 bytes per batch row
+        st_async16(mapa(slot, owner) + 16u * (uint32_t)i, make_float4(-0.f, -0.f, -0.f, -0.f),
+                   mapa(bar_recv, owner));
+    } else if (lane < 4 * a.batch) {
       st_async16(mapa(slot, owner) + 16u * (uint32_t)lane, make_float4(-0.f, -0.f, -0.f, -0.f),
                  mapa(bar_recv, owner));
+    }
   }
   }
   // Owned tiles (tau = crank + k * csize): wait for every warp of the
@@ -850,7 +896,19 @@ template <> struct KernelShape<3> {
 };
 template <> struct KernelShape<kFmtW3V3> : KernelShape<3> {};
 
-constexpr int kModes[3] = {kFactored1, kFactored2, kFull};
+constexpr int kModes[4] = {kFactored1, kFactored2, kFull, kFull16};
+
+// Batches of 9-16 rows (8-D formats): one build per format with the whole
+// register file (one CTA per SM) and strips of two tiles, which hold the
+// second batch half's accumulators and activations; none for 4-D vectors.
+template <int FMT>
+inline const void* kptr_full16() {
+  if constexpr (FMT == kFmt4D)
+    return nullptr;
+  else
+    return reinterpret_cast<const void*>(
+        &gemv_kernel<FMT, kFull16, KernelShape<FMT>::kWarps, 1, 2>);
+}
 
 template <int BITS, int MODE, int S>
 inline const void* kptr() {
@@ -861,7 +919,8 @@ template <int FMT, int S = 2>
 inline const void* kptr_mode(int mode) {
   return mode == kFactored1 ? kptr<FMT, kFactored1, S>()
          : mode == kFactored2 ? kptr<FMT, kFactored2, S>()
-                              : kptr<FMT, kFull, S>();
+         : mode == kFull      ? kptr<FMT, kFull, S>()
+                              : kptr_full16<FMT>();
 }
 
 // W2 built for one CTA per SM, with the whole register file instead of the
@@ -873,7 +932,8 @@ inline const void* kptr_mode_solo(int mode) {
   constexpr int W = KernelShape<FMT>::kWarps;
   return mode == kFactored1   ? reinterpret_cast<const void*>(&gemv_kernel<FMT, kFactored1, W, 1, S>)
          : mode == kFactored2 ? reinterpret_cast<const void*>(&gemv_kernel<FMT, kFactored2, W, 1, S>)
-                              : reinterpret_cast<const void*>(&gemv_kernel<FMT, kFull, W, 1, S>);
+         : mode == kFull      ? reinterpret_cast<const void*>(&gemv_kernel<FMT, kFull, W, 1, S>)
+                              : kptr_full16<FMT>();
 }
 
 // Kernels of the Tab. 4 splits (formats 5-9), instantiated in their own

@@ -50,7 +50,7 @@ extern "C" sphq_status sphq_gemv_noalloc(sphq_handle h, const void* x, void* y, 
   set_error(SPHQ_OK, "");
   if (!h) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemv_noalloc: NULL handle");
   if (batch < 1 || batch > SPHQ_MAX_BATCH)
-    return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemv_noalloc: batch must be 1..8");
+    return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemv_noalloc: batch must be 1..16");
   if (!x || reinterpret_cast<uintptr_t>(x) % 16)
     return set_error(SPHQ_ERR_INVALID_ARG,
                      "sphq_gemv_noalloc: x must be a 16-byte aligned pointer");

@@ -19,7 +19,7 @@ SPHQ_OK = 0
 STATUS = {0: "SPHQ_OK", 1: "SPHQ_ERR_INVALID_ARG", 2: "SPHQ_ERR_UNSUPPORTED",
           3: "SPHQ_ERR_NOT_PACKED", 4: "SPHQ_ERR_CUDA", 5: "SPHQ_ERR_OOM",
           6: "SPHQ_ERR_DEVICE", 7: "SPHQ_ERR_TIMEOUT"}
-MAX_BATCH = 8
+MAX_BATCH = 16
 
 _lib = None
 

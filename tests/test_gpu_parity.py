@@ -122,7 +122,7 @@ def test_invalid_codes_rejected_and_unpacked_handle_refuses():
     with pytest.raises(SphqError):
         m.gemv_ptr(xb.data_ptr() + 2, xb.data_ptr(), 1, 0)
     with pytest.raises(SphqError):
-        m.gemv(G.x_dev(np.zeros((9, 256), np.uint16)))
+        m.gemv(G.x_dev(np.zeros((17, 256), np.uint16)))
     m.close()
 
 
