@@ -921,10 +921,11 @@ def run_report(args):
                            for i, (nm, r, c) in enumerate(inp.DECODER_PROJ) if nm not in ("v", "up")}
     rep["cfg3_w3_proj_batch"] = {f"{nm} {r}x{c} B{bt}": entry(3, r, c, inp.seed_for(3, i), bt)
                                  for i, (nm, r, c) in enumerate(inp.DECODER_PROJ)
-                                 if nm in ("q", "k", "gate", "down") for bt in (1, 2, 4, 8)}
+                                 if nm in ("q", "k", "gate", "down") for bt in (1, 2, 4, 8, 16)}
     # Compute rooflines of the small-batch GEMV beside HBM: the mma.sync rate
     # the kernel issues its products to (one m16n8k16 per 8 cycles per SM
-    # sub-partition, measured on this part; 8 per 256-vector unit) and the
+    # sub-partition, measured on this part; 8 per 256-vector unit, 16 for
+    # 9-16 rows, whose two batch halves each take the decoded block) and the
     # plain FP32 FMA rate (128 per SM per cycle, 2 flops each), at the SM
     # clock sampled meanwhile.
     mhz = sm_clock_mhz()
@@ -934,7 +935,7 @@ def run_report(args):
     for key, e in rep["cfg3_w3_proj_batch"].items():
         rc_ = key.split()[1].split("x")
         r, c, bt = int(rc_[0]), int(rc_[1]), int(key.split("B")[-1])
-        mma = 8 * ((r + 15) // 16) * (c // 128)
+        mma = (16 if bt > 8 else 8) * ((r + 15) // 16) * (c // 128)
         e["mma_frac"] = round(mma / (e["us"] * 1e-6) / mma_peak, 4)
         e["fp32_alu_frac"] = round(2.0 * bt * r * c / (e["us"] * 1e-6) / alu_peak, 4)
         fr = {"hbm": e["hbm_frac"], "mma": e["mma_frac"], "fp32_alu": e["fp32_alu_frac"]}
