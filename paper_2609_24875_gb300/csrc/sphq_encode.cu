@@ -29,12 +29,13 @@
 //     zero vectors) the thread re-scores all K entries the same way.
 // So the result equals a single-precision CPU encoder bit for bit.
 //
-// Kernel 1 (persistent, one CTA per SM): 4 vector warps (one vector per
-// thread, 128 per tile) decompose, write the split directions as the A
-// operand and scan the scores; one MMA warp issues one MMA per chunk of 256
-// entries into a double-buffered 2 x 256-column tensor-memory ring.  Kernel 2
-// quantises the radii per group.  Every mbarrier wait is bounded (2 s; error
-// word bit 1).
+// Kernel 1 (persistent, one CTA per SM): 4 primary vector warps (one vector
+// per thread, 128 per tile) decompose, write the split directions as the A
+// operand and take the final choice; they and 4 partner warps (one per
+// tensor-memory lane quarter) scan the scores, each warp half of every chunk;
+// one MMA warp issues one MMA per chunk of 256 entries into a double-buffered
+// 2 x 256-column tensor-memory ring.  Kernel 2 quantises the radii per group.
+// Every mbarrier wait is bounded (2 s; error word bit 1).
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 
@@ -46,9 +47,10 @@
 
 namespace sphq {
 
-constexpr int kEncVecWarps = 4;                 // 128 vectors per tile = MMA M
+constexpr int kEncPrimWarps = 4;                // 128 vectors per tile = MMA M
+constexpr int kEncVecWarps = 2 * kEncPrimWarps;  // + a partner per lane quarter for the scan
 constexpr int kEncThreads = (kEncVecWarps + 1) * 32;
-constexpr int kEncTile = 32 * kEncVecWarps;
+constexpr int kEncTile = 32 * kEncPrimWarps;
 constexpr int kEncChunk = 256;                  // entries per MMA (N), at most
 constexpr int kCand = 4;                        // candidates kept per vector
 constexpr float kDelta = 1e-5f;                 // candidate window (relative to max(1, |best|))
@@ -107,7 +109,7 @@ __global__ void __launch_bounds__(kEncThreads, 1) encode_vectors_kernel(const En
 
   if (threadIdx.x == 0) {
     mbar_init(cb_bar, 1);
-    mbar_init(a_full, kEncVecWarps);
+    mbar_init(a_full, kEncPrimWarps);
     for (int b = 0; b < 2; ++b) {
       mbar_init(t_full0 + 8u * b, 1);
       mbar_init(t_free0 + 8u * b, kEncVecWarps);
@@ -152,52 +154,69 @@ __global__ void __launch_bounds__(kEncThreads, 1) encode_vectors_kernel(const En
     __syncwarp();
   } else {
     // ---- vector warps ----
+    // Warps w and w + 4 read the same tensor-memory lanes (the same 32
+    // vectors): the first ("primary") decomposes its vectors, writes the A
+    // operand and takes the final choice; both scan the coarse scores, the
+    // primary the first half of every chunk of entries and its partner the
+    // second half, and they exchange their maxima and candidates through
+    // shared memory at a barrier of the pair.
+    __shared__ float x_max[kEncPrimWarps][32];
+    __shared__ int x_nc[kEncPrimWarps][32];
+    __shared__ int x_ck[kEncPrimWarps][kCand][32];
+    const bool prim = warp < kEncPrimWarps;
+    const int quarter = warp & (kEncPrimWarps - 1);
+    const int half = prim ? 0 : 1;
+    const int hcols = a.chunk / 2;  // columns of a chunk one warp scans
+    const int pair_bar = 1 + quarter;
+    auto pair_sync = [&]() { asm volatile("bar.sync %0, 64;" ::"r"(pair_bar) : "memory"); };
     long long u = 0;
     for (long long tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
-      const long long v = tile * kEncTile + threadIdx.x;
+      const long long v = tile * kEncTile + quarter * 32 + lane;
       const bool valid = v < a.nvec;
       float p[8], d[8];
       uint32_t sbits = 0;
-      {
-        float x[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-        if (valid) {
-          const float4 x0 = reinterpret_cast<const float4*>(a.w + v * 8)[0];
-          const float4 x1 = reinterpret_cast<const float4*>(a.w + v * 8)[1];
-          x[0] = x0.x, x[1] = x0.y, x[2] = x0.z, x[3] = x0.w;
-          x[4] = x1.x, x[5] = x1.y, x[6] = x1.z, x[7] = x1.w;
-        }
-        float acc = 0.f;
+      if (prim) {
+        {
+          float x[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+          if (valid) {
+            const float4 x0 = reinterpret_cast<const float4*>(a.w + v * 8)[0];
+            const float4 x1 = reinterpret_cast<const float4*>(a.w + v * 8)[1];
+            x[0] = x0.x, x[1] = x0.y, x[2] = x0.z, x[3] = x0.w;
+            x[4] = x1.x, x[5] = x1.y, x[6] = x1.z, x[7] = x1.w;
+          }
+          float acc = 0.f;
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          p[j] = fabsf(x[j]);
-          if (x[j] < 0.f) sbits |= 1u << j;
-          acc = fmaf(p[j], p[j], acc);
-        }
-        const float r = __fsqrt_rn(acc);
-        const float den = r > 1e-12f ? r : 1e-12f;
+          for (int j = 0; j < 8; ++j) {
+            p[j] = fabsf(x[j]);
+            if (x[j] < 0.f) sbits |= 1u << j;
+            acc = fmaf(p[j], p[j], acc);
+          }
+          const float r = __fsqrt_rn(acc);
+          const float den = r > 1e-12f ? r : 1e-12f;
 #pragma unroll
-        for (int j = 0; j < 8; ++j) d[j] = __fdiv_rn(p[j], den);
+          for (int j = 0; j < 8; ++j) d[j] = __fdiv_rn(p[j], den);
+        }
+        // A operand: d_hi and d_lo planes, row = vector of the tile
+        {
+          uint32_t hi[4], lo[4];
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const __half h0 = __float2half_rn(d[2 * j]), h1 = __float2half_rn(d[2 * j + 1]);
+            const __half l0 = __float2half_rn(__fsub_rn(d[2 * j], __half2float(h0)));
+            const __half l1 = __float2half_rn(__fsub_rn(d[2 * j + 1], __half2float(h1)));
+            hi[j] = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
+            lo[j] = (uint32_t)__half_as_ushort(l0) | ((uint32_t)__half_as_ushort(l1) << 16);
+          }
+          const int t = quarter * 32 + lane;
+          const uint32_t off = (uint32_t)((t & 7) * 16 + (t >> 3) * 128);
+          *reinterpret_cast<uint4*>(smem + a.off_a + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+          *reinterpret_cast<uint4*>(smem + a.off_a + kEncPlane + off) =
+              make_uint4(lo[0], lo[1], lo[2], lo[3]);
+        }
+        umma::fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) enc_arrive(a_full);
       }
-      // A operand: d_hi and d_lo planes, row = thread
-      {
-        uint32_t hi[4], lo[4];
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const __half h0 = __float2half_rn(d[2 * j]), h1 = __float2half_rn(d[2 * j + 1]);
-          const __half l0 = __float2half_rn(__fsub_rn(d[2 * j], __half2float(h0)));
-          const __half l1 = __float2half_rn(__fsub_rn(d[2 * j + 1], __half2float(h1)));
-          hi[j] = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
-          lo[j] = (uint32_t)__half_as_ushort(l0) | ((uint32_t)__half_as_ushort(l1) << 16);
-        }
-        const int t = threadIdx.x;
-        const uint32_t off = (uint32_t)((t & 7) * 16 + (t >> 3) * 128);
-        *reinterpret_cast<uint4*>(smem + a.off_a + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-        *reinterpret_cast<uint4*>(smem + a.off_a + kEncPlane + off) =
-            make_uint4(lo[0], lo[1], lo[2], lo[3]);
-      }
-      umma::fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) enc_arrive(a_full);
 
       // Two passes over the coarse scores (the MMAs are repeated, which is
       // cheap): the first takes the maximum, the second collects, in
@@ -211,16 +230,22 @@ __global__ void __launch_bounds__(kEncThreads, 1) encode_vectors_kernel(const En
       bool overflow = false;
       for (int c = 0; c < 2 * nchunks; ++c, ++u) {
         const bool collect = c >= nchunks;
-        if (c == nchunks) thr = cmax - kDelta * fmaxf(1.f, fabsf(cmax));
+        if (c == nchunks) {  // the pair's maximum, then the window
+          x_max[quarter][lane] = cmax;
+          pair_sync();
+          cmax = fmaxf(cmax, x_max[quarter][lane]);
+          pair_sync();  // both read before either writes again
+          thr = cmax - kDelta * fmaxf(1.f, fabsf(cmax));
+        }
         const int b = (int)(u & 1);
         if (!mbar_wait(t_full0 + 8u * b, (uint32_t)((u / 2) & 1)) && lane == 0)
           atomicOr(a.flag, 2);
         umma::fence_after_sync();
-        const int kc = (collect ? c - nchunks : c) * a.chunk;
-        for (int cc = 0; cc < a.chunk / 32; ++cc) {
+        const int kc = (collect ? c - nchunks : c) * a.chunk + half * hcols;
+        for (int cc = 0; cc < hcols / 32; ++cc) {
           uint32_t sv[32];
-          umma::ld_32x32b_x32(taddr + ((uint32_t)(32 * warp) << 16) +
-                                  (uint32_t)(b * kEncChunk + 32 * cc),
+          umma::ld_32x32b_x32(taddr + ((uint32_t)(32 * quarter) << 16) +
+                                  (uint32_t)(b * kEncChunk + half * hcols + 32 * cc),
                               sv);
           umma::wait_ld();
           float m8[8];
@@ -249,27 +274,49 @@ __global__ void __launch_bounds__(kEncThreads, 1) encode_vectors_kernel(const En
         if (lane == 0) enc_arrive(t_free0 + 8u * b);
       }
 
-      // exact choice among the candidates (all entries after an overflow)
-      int z = 0;
-      float zs = 0.f;
-      if (overflow) {
-        for (int k = 0; k < a.K; ++k) {
-          const float s = dot8(d, smem, k);
-          if (k == 0 || s > zs) zs = s, z = k;
-        }
-      } else {
+      // the partner's candidates (the second halves of the chunks) to the
+      // primary; more than kCand in all is an overflow
+      if (!prim) {
+        x_nc[quarter][lane] = overflow ? -1 : nc;
 #pragma unroll
-        for (int i = 0; i < kCand; ++i)
-          if (i < nc) {
-            const float s = dot8(d, smem, ck[i]);
-            if (i == 0 || s > zs) zs = s, z = ck[i];
+        for (int i = 0; i < kCand; ++i) x_ck[quarter][i][lane] = i < nc ? ck[i] : 0;
+      }
+      pair_sync();
+      if (prim) {
+        const int nq = x_nc[quarter][lane];
+        int cq[kCand];
+#pragma unroll
+        for (int i = 0; i < kCand; ++i) cq[i] = x_ck[quarter][i][lane];
+        if (nq < 0 || nc + nq > kCand) overflow = true;
+        // exact choice among the candidates of both halves (all entries after
+        // an overflow): the largest single-precision score, lowest k on ties
+        int z = 0;
+        float zs = 0.f;
+        if (overflow) {
+          for (int k = 0; k < a.K; ++k) {
+            const float s2 = dot8(d, smem, k);
+            if (k == 0 || s2 > zs) zs = s2, z = k;
           }
+        } else {
+          bool any = false;
+#pragma unroll
+          for (int i = 0; i < 2 * kCand; ++i) {
+            const bool have = i < kCand ? i < nc : i - kCand < nq;
+            if (have) {
+              const int k = i < kCand ? ck[i] : cq[i - kCand];
+              const float s2 = dot8(d, smem, k);
+              if (!any || s2 > zs || (s2 == zs && k < z)) zs = s2, z = k;
+              any = true;
+            }
+          }
+        }
+        if (valid) {
+          a.sign[v] = (uint8_t)sbits;
+          a.idx[v] = (uint16_t)z;
+          a.rtilde[v] = dot8(p, smem, z);
+        }
       }
-      if (valid) {
-        a.sign[v] = (uint8_t)sbits;
-        a.idx[v] = (uint16_t)z;
-        a.rtilde[v] = dot8(p, smem, z);
-      }
+      pair_sync();  // the partner's lists are read before it writes the next tile's
     }
   }
   umma::fence_before_sync();
@@ -331,7 +378,13 @@ sphq_status launch_encode(sphq_handle h, const float* w, uint8_t* sign, uint16_t
   // columns) runs per SM
   const size_t need = 1024 + (size_t)a.off_bar + 64;
   const size_t smem = std::max(need, (size_t)120 * 1024);
-  if (smem > (size_t)optin) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_encode: shared memory");
+  // the kernel's static shared memory (the scan partners' exchange) counts
+  // against the same per-block limit as the dynamic part
+  cudaFuncAttributes fa;
+  e = cudaFuncGetAttributes(&fa, encode_vectors_kernel);
+  if (e != cudaSuccess) return cuda_error(e, "cudaFuncGetAttributes(encode)");
+  const size_t dyn_max = (size_t)optin > fa.sharedSizeBytes ? (size_t)optin - fa.sharedSizeBytes : 0;
+  if (smem > dyn_max) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_encode: shared memory");
   {
     // once per device (the attribute belongs to the kernel on the current device)
     static std::mutex mu;
@@ -340,7 +393,7 @@ sphq_status launch_encode(sphq_handle h, const float* w, uint8_t* sign, uint16_t
     if (h->device < 0 || h->device >= 64) return set_error(SPHQ_ERR_DEVICE, "device index out of range");
     if (!done[h->device]) {
       e = cudaFuncSetAttribute(encode_vectors_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               optin);
+                               (int)dyn_max);
       if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(encode)");
       done[h->device] = true;
     }
