@@ -34,7 +34,8 @@ def test_ragged_shapes(fmt, batch):
     m.close()
 
 
-@pytest.mark.parametrize("bits,rows,cols", [(2, 80, 1024), (3, 1000, 1024), (3, 112, 2048)])
+@pytest.mark.parametrize("bits,rows,cols", [(2, 80, 1024), (3, 1000, 1024), (3, 112, 2048),
+                                            (2, 1, 1024), (3, 17, 1024)])
 @pytest.mark.parametrize("batch", [10, 16])
 def test_every_cluster_size(bits, rows, cols, batch):
     codes, x = inp.random_codes(bits, rows, cols, seed=2300 + rows + bits + batch, B=batch)
@@ -99,5 +100,15 @@ def test_dim4_two_launches(batch):
                           codes.rcode)
     ref, absdot = oracle.gemv(w, x)
     assert np.all(np.abs(got - ref) <= oracle.gemv_tolerance(absdot))
+    m.check()
+    m.close()
+
+
+@pytest.mark.parametrize("bits", [2, 3])
+@pytest.mark.parametrize("batch", [9, 16])
+def test_one_row_one_group(bits, batch):
+    codes, x = inp.random_codes(bits, 1, 128, seed=2700 + bits + batch, B=batch)
+    m = G.make_matrix(codes)
+    G.check_gemv(m, codes, x)
     m.check()
     m.close()

@@ -33,7 +33,8 @@ def _bits16(t):
 
 @pytest.mark.parametrize("bits,rows,cols,batch,wrapper",
                          [(2, 3584, 3584, 1, False), (3, 512, 3584, 4, False),
-                          (2, 1000, 1024, 2, True), (3, 96, 18944, 8, False)])
+                          (2, 1000, 1024, 2, True), (3, 96, 18944, 8, False),
+                          (3, 300, 1024, 16, False)])
 def test_noalloc_matches_gemv_on_two_calls(bits, rows, cols, batch, wrapper):
     codes, x = inp.random_codes(bits, rows, cols, seed=4242 + rows + bits, B=batch)
     m = G.make_matrix(codes)
