@@ -1,6 +1,6 @@
 // Fused spherical dequantize-GEMV kernel for decode (SPHQuant §3.4, App. D), sm_103a.
 //
-// y[n][r] = sum_j w_hat[r][j] x[n][j] for a batch of n <= 8 activation rows.
+// y[n][r] = sum_j w_hat[r][j] x[n][j] for a batch of n <= 16 activation rows.
 //
 // Decode stays on the CUDA cores: each thread rebuilds whole 8-D blocks in
 // registers (codebook entry from shared memory, coordinate signs, radius of
@@ -22,7 +22,9 @@
 //    result differs from the exact W_hat x by at most one fp16 rounding of
 //    each product r_hat * c (2^-11 relative), inside the stated tolerance.
 //  * batch 3-8 ("full"): the lane forms w_hat = RN16(r_hat * (s (.) c_z))
-//    exactly as Eq. (4) defines it and the MMA's N dimension is the batch.
+//    exactly as Eq. (4) defines it and the MMA's N dimension is the batch;
+//    batch 9-16 feeds each such block to a second pair of MMAs for batch
+//    rows 8-15.
 //
 // Work decomposition.  The row tiles (16 rows) are dealt to thread-block
 // clusters in contiguous, near-equal ranges; every CTA of a cluster takes the
