@@ -35,7 +35,8 @@ static const void* select_kernel(int fmt, int mode, int strip, bool solo = false
   if (mode == kFull16)  // one build per format (strips of two, one CTA per SM)
     return fmt == 2 ? kptr_full16<2>() : fmt == 3 ? kptr_full16<3>()
            : fmt == kFmtW3V3 ? kptr_full16<kFmtW3V3>() : split_kernel(fmt, mode);
-  return fmt == 2 ? (solo ? kptr_mode_solo<2>(mode) : kptr_mode<2>(mode))
+  return fmt == 2 ? (solo ? (strip == 4 ? kptr_mode_solo<2, 4>(mode) : kptr_mode_solo<2>(mode))
+                           : kptr_mode<2>(mode))
          : fmt == 3 ? (strip == 4 ? kptr_mode<3, 4>(mode) : kptr_mode<3, 2>(mode))
          : fmt == kFmtW3V3 ? (strip == 4 ? kptr_mode<kFmtW3V3, 4>(mode) : kptr_mode<kFmtW3V3, 2>(mode))
                            : split_kernel(fmt, mode);
@@ -54,7 +55,7 @@ static sphq_status allow_max_smem(int device, int optin) {
     for (int mode : kModes)
       for (int strip : {2, 4})
         for (int solo = 0; solo < 2; ++solo) {
-          if (strip == 4 && !fmt_has_strip4(fmt)) continue;
+          if (strip == 4 && !fmt_has_strip4(fmt) && !(solo && has_solo(fmt))) continue;
           if (solo && !has_solo(fmt)) continue;
           const void* k = select_kernel(fmt, mode, strip, solo);
           if (!k) continue;  // no 16-row build for 4-D vectors
@@ -126,6 +127,10 @@ static sphq_status make_plan(sphq_handle h, int batch, int forced, int optin, Ge
   {
     GemvPlan best{};
     double best_cost = 0;
+    // W2: the one-CTA-per-SM build with four-tile strips, kept aside and
+    // compared below by the work of the busiest SM
+    GemvPlan packed{};
+    double packed_load = 0;
     const int warps = warps_for(h->fmt);
     for (int staged = 1; staged >= 0; --staged) {
       int mode = mode_for(batch);
@@ -197,7 +202,12 @@ static sphq_status make_plan(sphq_handle h, int batch, int forced, int optin, Ge
           // bound the cluster count, and no second CTA would share an SM.
           const bool better = best.grid == 0 || cost < best_cost - 1e-9 ||
                               (solo && !best.solo && cost <= best_cost + 1e-9);
-          if (better) {
+          const bool strip4_ok =
+              mode != kFull16 && (fmt_has_strip4(h->fmt) || (solo && has_solo(h->fmt)));
+          const double load = (double)tmax * ((h->ng + csize - 1) / csize) * waves;
+          const bool packed_candidate = solo && has_solo(h->fmt) && mode != kFull16 && tmax >= 3 &&
+                                        (packed.grid == 0 || load < packed_load);
+          if (better || packed_candidate) {
             p.grid = nclusters * csize;
             p.nclusters = nclusters;
             p.tmax = tmax;
@@ -208,17 +218,40 @@ static sphq_status make_plan(sphq_handle h, int batch, int forced, int optin, Ge
             p.off_recv = (uint32_t)L.recv;
             p.off_bar = (uint32_t)L.bar;
             // four-tile strips once a cluster holds three tiles or more (W3)
-            p.strip = mode != kFull16 && fmt_has_strip4(h->fmt) && tmax >= 3 ? 4 : 2;
+            p.strip = strip4_ok && tmax >= 3 ? 4 : 2;
             p.solo = solo != 0 || mode == kFull16;
           p.ctas_per_sm = p.solo ? 1
                           : fmt_small(h->fmt) || h->fmt == kFmt4D ? KernelShape<2>::kMinBlocks
                                                                    : KernelShape<3>::kMinBlocks;
-            best = p;
-            best_cost = cost;
+            if (packed_candidate) {
+              packed = p;
+              packed_load = load;
+            }
+            if (better) {
+              best = p;
+              best_cost = cost;
+            }
           }
         }
       }
       if (best.grid > 0) break;  // staged activations fit: keep that mode
+    }
+    // When more CTAs of the two-per-SM build are launched than there are SMs,
+    // some SMs run two of them: their work is twice a CTA's.  The one-CTA
+    // build with four-tile strips takes the same tiles in fewer, longer CTAs
+    // (and shares each activation load among up to four units); take it when
+    // its busiest SM has clearly less work, counting its 8 warps per SM as 7%
+    // slower per unit than 16, and its CTAs have long rows of work (32 groups
+    // or more: with fewer, the items dealt to 8 warps are too coarse to gain).
+    // Measured: W2 3584 x 18944 at batch 1-8 13-14% faster; 3584^2 (14
+    // groups per CTA) 2% slower, hence the row condition; 8192^2 and
+    // 18944 x 3584 unchanged.
+    if (packed.grid > 0 && best.grid > 0 && !best.solo && !forced &&
+        (h->ng + packed.csize - 1) / packed.csize >= 32) {
+      const int sms = h->sm_count > 0 ? h->sm_count : 1;
+      const int per_sm = std::min(best.ctas_per_sm, (best.grid + sms - 1) / sms);
+      const double best_load = (double)best.tmax * ((h->ng + best.csize - 1) / best.csize) * per_sm;
+      if (packed_load * 1.07 < 0.95 * best_load) best = packed;
     }
     if (best.grid == 0)
       return set_error(forced ? SPHQ_ERR_UNSUPPORTED : SPHQ_ERR_CUDA,

@@ -112,3 +112,17 @@ def test_one_row_one_group(bits, batch):
     G.check_gemv(m, codes, x)
     m.check()
     m.close()
+
+
+@pytest.mark.parametrize("batch", [1, 2, 4, 8])
+def test_w2_long_rows_one_cta_four_tile_strips(batch):
+    # 3584 x 18944 (the down projection): more two-per-SM CTAs than SMs would
+    # put two on some SMs, so the plan takes the one-CTA build with four-tile
+    # strips; every row checked against the oracle
+    codes, x = inp.random_codes(2, 3584, 18944, seed=2800 + batch, B=batch)
+    m = G.make_matrix(codes)
+    p = m.plan(batch)
+    assert p["ctas_per_sm"] == 1 and p["tiles_per_cluster"] >= 3
+    G.check_gemv(m, codes, x)
+    m.check()
+    m.close()
