@@ -144,6 +144,14 @@ static sphq_status make_plan(sphq_handle h, int batch, int forced, int optin, Ge
         for (int csize : {1, 2, 4, 8}) {
           if (csize > h->ng) break;
           if (forced && csize != forced) continue;
+          // 9-16 rows: partial blocks of 16 batch rows make the reduction in a
+          // cluster twice as heavy, and strips of two tiles leave one-tile
+          // strips in odd tile ranges; single CTAs measured best (8192^2 W3
+          // 20.7 against 23.3 us in clusters of 2, W2 3584 x 18944 16.1 against
+          // 22.3) unless the row tiles cannot fill half the SMs (512 x 3584:
+          // clusters of 4, 3.5 against 4.5 us)
+          if (!forced && mode == kFull16 && csize > 1 && 2 * h->nrt >= std::max(h->sm_count, 1))
+            continue;
           // clusters: as many as fit at once, at most one per row tile; the
           // tile range of a cluster is limited by its shared memory
           GemvPlan p;
