@@ -248,18 +248,21 @@ static sphq_status make_plan(sphq_handle h, int batch, int forced, int optin, Ge
     // some SMs run two of them: their work is twice a CTA's.  The one-CTA
     // build with four-tile strips takes the same tiles in fewer, longer CTAs
     // (and shares each activation load among up to four units); take it when
-    // its busiest SM has clearly less work, counting its 8 warps per SM as 7%
-    // slower per unit than 16, and its CTAs have long rows of work (32 groups
-    // or more: with fewer, the items dealt to 8 warps are too coarse to gain).
-    // Measured: W2 3584 x 18944 at batch 1-8 13-14% faster; 3584^2 (14
-    // groups per CTA) 2% slower, hence the row condition; 8192^2 and
-    // 18944 x 3584 unchanged.
+    // its busiest SM has clearly less work and its CTAs have long rows of work
+    // (32 groups or more: with fewer, the items dealt to 8 warps are too
+    // coarse to gain).  Per unit its 8 warps per SM count 7% slower than 16
+    // at 1-2 rows, and 7% faster at 3-8 rows, where each strip of four shares
+    // one read of the activations through L1.  Measured: W2 3584 x 18944 at
+    // batch 1-8 13-14% faster, W2 8192^2 at 4-8 rows 8-11% faster; 3584^2 (14
+    // groups per CTA) 2% slower, hence the row condition; 18944 x 3584
+    // unchanged.
     if (packed.grid > 0 && best.grid > 0 && !best.solo && !forced &&
         (h->ng + packed.csize - 1) / packed.csize >= 32) {
       const int sms = h->sm_count > 0 ? h->sm_count : 1;
       const int per_sm = std::min(best.ctas_per_sm, (best.grid + sms - 1) / sms);
       const double best_load = (double)best.tmax * ((h->ng + best.csize - 1) / best.csize) * per_sm;
-      if (packed_load * 1.07 < 0.95 * best_load) best = packed;
+      const double per_unit = packed.mode == kFull ? 0.93 : 1.07;
+      if (packed_load * per_unit < 0.95 * best_load) best = packed;
     }
     if (best.grid == 0)
       return set_error(forced ? SPHQ_ERR_UNSUPPORTED : SPHQ_ERR_CUDA,

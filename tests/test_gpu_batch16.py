@@ -126,3 +126,16 @@ def test_w2_long_rows_one_cta_four_tile_strips(batch):
     G.check_gemv(m, codes, x)
     m.check()
     m.close()
+
+
+@pytest.mark.parametrize("batch", [4, 8])
+def test_w2_square_one_cta_four_tile_strips_at_3_to_8_rows(batch):
+    # 8192 x 8192 at 3-8 rows: the strips of four share each activation read,
+    # so the plan takes the one-CTA build; sampled rows against the oracle
+    codes, x = inp.random_codes(2, 8192, 8192, seed=2900 + batch, B=batch)
+    m = G.make_matrix(codes)
+    p = m.plan(batch)
+    assert p["ctas_per_sm"] == 1 and p["tiles_per_cluster"] >= 3
+    G.check_gemv(m, codes, x, G.sample_rows(8192, 256, seed=batch))
+    m.check()
+    m.close()
