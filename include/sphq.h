@@ -381,15 +381,21 @@ sphq_status sphq_gemm_ws(sphq_handle h, const void* x, void* y, int batch, void*
 /*
  * sphq_gemm_info / sphq_get_gemm_shape -- the launch shape sphq_gemm uses for
  * `batch`: activation tiles of 128 rows per CTA (1 or 2), weight rows per CTA
- * (128 or 256), columns per pipeline stage (64 or 32), ring stages, grid and
- * dynamic shared memory.  (No counterpart in the paper.)
+ * (128 or 256), columns per pipeline stage (64 or 32), ring stages, output
+ * tiles (grid_x weight tiles x grid_y activation tiles of act_tiles x 128
+ * rows), dynamic shared memory, and split_ctas: with two activation tiles,
+ * the CTAs of one activation tile that take a final partial wave of output
+ * tiles (two per output tile; 0 when the wave is not split).  (No counterpart
+ * in the paper.)
  * sphq_set_gemm_shape -- fix act_tiles (1, 2; 0 = automatic) and weight_rows
  * (128, 256; 0 = automatic) for later sphq_gemm calls on the handle; 128 rows
- * go with one activation tile only.  Invalid values give SPHQ_ERR_INVALID_ARG.
+ * go with one activation tile only; a fixed act_tiles also keeps the final
+ * wave whole.  Invalid values give SPHQ_ERR_INVALID_ARG.
  */
 typedef struct sphq_gemm_info {
   int act_tiles, weight_rows, stage_cols, stages, grid_x, grid_y;
   long long smem_bytes;
+  int split_ctas;
 } sphq_gemm_info;
 sphq_status sphq_get_gemm_shape(sphq_handle h, int batch, sphq_gemm_info* out);
 sphq_status sphq_set_gemm_shape(sphq_handle h, int act_tiles, int weight_rows);

@@ -15,8 +15,14 @@
 // the columns in steps of 64 (128-byte swizzled operand rows) or 32 (64-byte
 // swizzle).  Two activation tiles per decoded weight tile halve the decode
 // and shared-memory traffic per flop; they are used when the batch exceeds
-// 128.  Next to the 128 KiB W3 codebook only 32-column steps leave room for a
-// ring of three stages with two activation tiles.  Per step:
+// 128.  With two, a final partial wave of CTAs (e.g. 512 output tiles on 152
+// SMs: three full waves and 56 tiles, which would take as long as a fourth
+// full wave) can be split: each of its output tiles goes to two CTAs of one
+// activation tile, so it spreads over twice the SMs (8192^2 x 4096: the
+// two-pass product 3.6-3.8% faster, the fused one 1.6% (W2) to 3.8% (W3)).
+// Next to the 128 KiB W3 codebook only
+// 32-column steps leave room for a ring of three stages with two activation
+// tiles.  Per step:
 //  * one TMA warp loads the 128 (256) x BK activation tile (A operand,
 //    K-major, swizzled; rows past the batch read zeros);
 //  * one decode warp per 16-row tile (16 or 8 warps) rebuilds its 16 x BK
@@ -66,6 +72,8 @@ struct GemmArgs {
   uint16_t* y;             // batch x rows fp16
   int* flag;               // device error word: bit 1 = an mbarrier wait gave up
   int rows, cols, nrt, batch;
+  int nwt;                 // weight tiles (of BN rows) across the rows
+  int n_big;               // CTAs with MT activation tiles; the rest take one
   int stages;              // ring depth
   uint32_t cb_bytes;
   uint32_t off_b, off_cb, off_bar;  // from the 1024-byte aligned base; A tiles at 0
@@ -159,8 +167,25 @@ __global__ void __launch_bounds__(gemm_threads(BN), 1)
   const uint32_t acc_bar = empty0 + 8u * S;
   const uint32_t cb_bar = acc_bar + 8u;
   uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + a.off_bar + 16u * S + 16u);
-  const int rt0 = blockIdx.x * kTilesN;
-  const int tok0 = blockIdx.y * kGemmBM * MT;
+  // This CTA's output tile.  The first n_big CTAs take MT activation tiles
+  // (weight tile fastest); the rest split the remaining MT-tile outputs into
+  // one activation tile each (two CTAs per output tile, a final wave that
+  // spreads over twice the SMs).
+  int wt, tok0, mt;
+  if ((int)blockIdx.x < a.n_big) {
+    wt = (int)blockIdx.x % a.nwt;
+    tok0 = (int)blockIdx.x / a.nwt * (kGemmBM * MT);
+    mt = MT;
+  } else {
+    const int j = (int)blockIdx.x - a.n_big, L = a.n_big + (j >> 1);
+    wt = L % a.nwt;
+    tok0 = L / a.nwt * (kGemmBM * MT) + (j & 1) * kGemmBM;
+    mt = 1;
+  }
+  if (tok0 >= a.batch) return;  // a half tile wholly past the batch: no work
+  // activation tiles wholly past the batch are neither loaded nor multiplied
+  mt = min(mt, (a.batch - tok0 + kGemmBM - 1) / kGemmBM);
+  const int rt0 = wt * kTilesN;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -191,8 +216,12 @@ __global__ void __launch_bounds__(gemm_threads(BN), 1)
       if constexpr (kDense) umma::prefetch_tmap(&tmap_w);
       for (int i = 0, s = 0, r = 0; i < nk; ++i) {
         if (r > 0 && !mbar_wait_poll(empty0 + 8u * s, (r - 1) & 1)) atomicOr(a.flag, 2);
-        mbar_arrive_expect_tx(full0 + 8u * s, kStageA + (kDense ? kTileB : 0u));
-        umma::tma_load_2d(sbase + s * kStageA, &tmap, i * BK, tok0, full0 + 8u * s);
+        mbar_arrive_expect_tx(full0 + 8u * s, (uint32_t)mt * kTileA + (kDense ? kTileB : 0u));
+#pragma unroll
+        for (int t = 0; t < MT; ++t)
+          if (t < mt)
+            umma::tma_load_2d(sbase + s * kStageA + t * kTileA, &tmap, i * BK, tok0 + t * kGemmBM,
+                              full0 + 8u * s);
         if constexpr (kDense)  // the W_hat tile: BN weight rows x BK columns
           umma::tma_load_2d(sbase + a.off_b + s * kTileB, &tmap_w, i * BK, rt0 * kRowsPerTile,
                             full0 + 8u * s);
@@ -208,7 +237,8 @@ __global__ void __launch_bounds__(gemm_threads(BN), 1)
         umma::fence_after_sync();
         const uint32_t at = sbase + s * kStageA, bt = sbase + a.off_b + s * kTileB;
 #pragma unroll
-        for (int t = 0; t < MT; ++t)
+        for (int t = 0; t < MT; ++t) {
+          if (t >= mt) break;
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk) {
             const uint32_t ad = at + t * kTileA + 32u * kk, bd = bt + 32u * kk;
@@ -217,6 +247,7 @@ __global__ void __launch_bounds__(gemm_threads(BN), 1)
                           BK == 64 ? umma::smem_desc_sw128(bd) : umma::smem_desc_sw64(bd), idesc,
                           (i | kk) != 0);
           }
+        }
         umma::commit(empty0 + 8u * s);
         if (++s == S) s = 0, ++r;
       }
@@ -288,7 +319,7 @@ __global__ void __launch_bounds__(gemm_threads(BN), 1)
     const int acc = start / BN;
     const int token = tok0 + kGemmBM * acc + 32 * quarter + lane;
 #pragma unroll 1
-    for (int cc = 0; cc < kColsPerWarp / 32; ++cc) {
+    for (int cc = 0; cc < (acc < mt ? kColsPerWarp / 32 : 0); ++cc) {
       const int col = start % BN + 32 * cc;  // within the accumulator
       const uint32_t tcol = (uint32_t)(acc * BN + col);
       uint32_t v[32];
@@ -487,6 +518,39 @@ struct GemmShape {
   GemmSmem L;
 };
 
+// The grid of a launch shape: nwt x ntok output tiles of BN weight rows x MT
+// activation tiles, in whole waves of SMs plus a final partial wave.  With
+// MT = 2 (and MT automatic), a final wave of r tiles that fit twice over on
+// the SMs goes to 2r CTAs of one activation tile each when that is estimated
+// faster: a wave of one-tile CTAs takes c of a wave of two-tile CTAs
+// (measured on this GB300 at 8192^2 x 4096, 56 output tiles in the final
+// wave: the dense pass 0.8, the fused kernel 0.85 (W3) to 0.94 (W2)).
+// `waves` is the estimated time in two-tile CTA times.
+struct GemmGrid {
+  int nwt = 0, ntok = 0, n_big = 0, n_small = 0;
+  double waves = 0;
+};
+
+static GemmGrid gemm_grid(const sphq_handle_s* h, int batch, int mt, int bn, bool dense) {
+  GemmGrid G;
+  const long long sms = h->sm_count > 0 ? h->sm_count : 1;
+  G.nwt = (h->nrt + bn / kRowsPerTile - 1) / (bn / kRowsPerTile);
+  G.ntok = (batch + kGemmBM * mt - 1) / (kGemmBM * mt);
+  const long long n = (long long)G.nwt * G.ntok;
+  G.n_big = (int)n;
+  G.waves = (double)((n + sms - 1) / sms);
+  if (mt == 2 && !h->gemm_mt) {
+    const long long full = n / sms, r = n - full * sms;
+    const double c = dense ? 0.8 : 0.9;
+    if (full >= 1 && r > 0 && 2 * r <= sms && full + c < G.waves - 1e-9) {
+      G.n_big = (int)(full * sms);
+      G.n_small = (int)(2 * r);
+      G.waves = (double)full + c;
+    }
+  }
+  return G;
+}
+
 // Shape (MT activation tiles, BN weight rows per CTA): the least estimated
 // time = waves of CTAs x time per CTA, the latter relative to the work of one
 // CTA (MT x BN) over its measured efficiency (two tiles of 256 rows: 1, one:
@@ -508,9 +572,7 @@ static GemmShape select_gemm_shape(const sphq_handle_s* h, int batch, int optin,
       if (!gemm_kernel_ptr(dense ? kFmtDense : h->fmt, m, k, n)) continue;
       const GemmSmem T = gemm_smem(h, optin, m, k, n, dense);
       if (T.stages < 2) continue;
-      const long long ctas = (long long)((h->nrt + n / kRowsPerTile - 1) / (n / kRowsPerTile)) *
-                             ((batch + kGemmBM * m - 1) / (kGemmBM * m));
-      const double t = (double)((ctas + sms - 1) / sms) * (m * n) / kEff[c];
+      const double t = gemm_grid(h, batch, m, n, dense).waves * (m * n) / kEff[c];
       if (!best.mt || t < best_t - 1e-9) {
         best.mt = m, best.bk = k, best.bn = n, best.L = T;
         best_t = t;
@@ -537,9 +599,11 @@ sphq_status gemm_shape_info(sphq_handle h, int batch, sphq_gemm_info* out) {
   out->weight_rows = g.bn;
   out->stage_cols = g.bk;
   out->stages = g.L.stages;
-  out->grid_x = (h->nrt + g.bn / kRowsPerTile - 1) / (g.bn / kRowsPerTile);
-  out->grid_y = (batch + kGemmBM * g.mt - 1) / (kGemmBM * g.mt);
+  const GemmGrid G = gemm_grid(h, batch, g.mt, g.bn, false);
+  out->grid_x = G.nwt;
+  out->grid_y = G.ntok;
   out->smem_bytes = (long long)g.L.total;
+  out->split_ctas = G.n_small;
   return SPHQ_OK;
 }
 
@@ -557,12 +621,13 @@ static sphq_status launch_gemm_kernel(sphq_handle h, const void* x, void* y, int
   if (!g.mt) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm: no shape fits this device");
   const int mt = g.mt, bk = g.bk, bn = g.bn;
   const GemmSmem& L = g.L;
+  const GemmGrid G = gemm_grid(h, batch, mt, bn, dense);
   if (log_enabled())
     std::fprintf(stderr,
                  "sphq: gemm %d x %d, batch %d%s: %d activation tile(s) x %d weight rows, "
-                 "%d-column stages x %d, %zu B shared\n",
+                 "%d-column stages x %d, %zu B shared, %d + %d split CTAs\n",
                  h->rows, h->cols, batch, dense ? " (two-pass, decoded W_hat)" : "", mt, bn, bk,
-                 L.stages, L.total);
+                 L.stages, L.total, G.n_big, G.n_small);
   cudaError_t e;
   const int kfmt = dense ? kFmtDense : h->fmt;
   const void* kfn = gemm_kernel_ptr(kfmt, mt, bk, bn);
@@ -580,11 +645,12 @@ static sphq_status launch_gemm_kernel(sphq_handle h, const void* x, void* y, int
       d = true;
     }
   }
-  // activations: a batch x cols fp16 tensor, boxes of 128 rows x 64 columns
+  // activations: a batch x cols fp16 tensor, boxes of 128 rows x BK columns
+  // (one per activation tile)
   CUtensorMap tmap;
   const cuuint64_t gdim[2] = {(cuuint64_t)h->cols, (cuuint64_t)batch};
   const cuuint64_t gstride[1] = {(cuuint64_t)h->cols * 2};
-  const cuuint32_t box[2] = {(cuuint32_t)bk, (cuuint32_t)(kGemmBM * mt)};
+  const cuuint32_t box[2] = {(cuuint32_t)bk, (cuuint32_t)kGemmBM};
   const cuuint32_t estride[2] = {1, 1};
   CUresult cr = enc(&tmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(x), gdim, gstride,
                     box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
@@ -614,13 +680,14 @@ static sphq_status launch_gemm_kernel(sphq_handle h, const void* x, void* y, int
   a.cols = h->cols;
   a.nrt = h->nrt;
   a.batch = batch;
+  a.nwt = G.nwt;
+  a.n_big = G.n_big;
   a.stages = L.stages;
   a.cb_bytes = L.cb_bytes;
   a.off_b = L.off_b;
   a.off_cb = L.off_cb;
   a.off_bar = L.off_bar;
-  const dim3 grid((unsigned)((h->nrt + bn / kRowsPerTile - 1) / (bn / kRowsPerTile)),
-                  (unsigned)((batch + kGemmBM * mt - 1) / (kGemmBM * mt)));
+  const dim3 grid((unsigned)(G.n_big + G.n_small));
   void* args[] = {&a, &tmap, &tmap_w};
   e = cudaLaunchKernel(kfn, grid, dim3(gemm_threads(bn)), args, L.total, s);
   if (e != cudaSuccess) return cuda_error(e, "gemm launch");

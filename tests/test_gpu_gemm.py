@@ -76,6 +76,41 @@ def test_every_launch_shape(fmt, shape):
     m.close()
 
 
+@pytest.mark.parametrize("fmt", FORMATS[:4], ids=FIDS[:4])
+@pytest.mark.parametrize("batch,ntok,split", [(1250, 5, 16), (2600, 11, 96)])
+def test_split_final_wave(fmt, batch, ntok, split):
+    # 8000 rows (32 weight tiles, the last of 4 row tiles) x ntok tiles of 256
+    # activation rows on 152 SMs: whole waves, and the output tiles of the
+    # final partial wave split into two CTAs of one activation tile each (at
+    # batch 2600 the second half of the last row of tiles is wholly past the
+    # batch and does no work).  The split plan equals the whole-wave plan bit
+    # for bit (the same products in the same order), the two-pass form equals
+    # both, all against the oracle.
+    bits, v, K = fmt
+    rows, cols = 8000, 512
+    codes, x = inp.random_codes(bits, rows, cols, seed=3100 + batch + v + bits, B=batch,
+                                radius_bits=v, K=K)
+    m = G.make_matrix(codes)
+    info = m.gemm_shape(batch)
+    assert (info["act_tiles"], info["grid_x"], info["grid_y"]) == (2, 32, ntok)
+    if torch.cuda.get_device_properties(0).multi_processor_count == 152:
+        assert info["split_ctas"] == split
+    xd = G.x_dev(x)
+    y_split = m.gemm(xd)
+    ws = torch.empty(rows * cols, dtype=torch.float16, device="cuda")
+    y_two = m.gemm_ws(xd, ws)
+    m.set_gemm_shape(2, 256)
+    assert m.gemm_shape(batch)["split_ctas"] == 0
+    y_whole = m.gemm(xd)
+    torch.cuda.synchronize()
+    assert torch.equal(y_split.view(torch.int16), y_whole.view(torch.int16))
+    assert torch.equal(y_two.view(torch.int16), y_whole.view(torch.int16))
+    m.set_gemm_shape(0, 0)
+    check_gemm(m, codes, x, G.sample_rows(rows, 400, seed=batch))
+    m.check()
+    m.close()
+
+
 def test_shape_choice_and_invalid_shapes():
     codes, _ = inp.random_codes(2, 8192, 1024, seed=6)
     m = G.make_matrix(codes)
