@@ -983,6 +983,34 @@ def run_report(args):
     rep["gather16_study"] = {k: {"G_entries/s": round(v / 1e9, 1),
                                  "max_hbm_frac_16d": round(min(1.0, v / need), 3)}
                              for k, v in rates.items()}
+    # 16-D vectors: the GEMV gathers one 32-byte codebook entry per vector
+    # through L1/L2, so beside HBM its roofline is the L2 gather rate above
+    rep["dim16"] = {}
+    for i, (r, c) in enumerate(((4096, 4096), (8192, 8192), (3584, 18944))):
+        for bt in (1, 8):
+            codes, x = inp.random_codes_dim(16, 2, r, c, seed=inp.seed_for(1, 40 + i), B=bt)
+            one = r * c * 19 // 64
+            P = min(512, max(2, int(np.ceil(2 * L2 / one)) + 1))
+            cb, sc, of = t(codes.codebook), t(codes.scale), t(codes.offset)
+            sg, ix, rc = t(codes.sign), t(codes.idx), t(codes.rcode)
+            mats = []
+            for _ in range(P):
+                m = SphqMatrix(r, c, 2, cb, sc, of, radius_bits=4, K=1 << 14, dim=16)
+                m.pack(sg, ix, rc)
+                mats.append(m)
+            xd = t(x).view(torch.float16)
+            ys = [torch.empty((bt, r), dtype=torch.float16, device=dev) for _ in mats]
+            b = mats[0].bytes(bt)
+            us = steady_us(mats, xd, ys, bt, stream)
+            ents = r * c // 16 / us / 1e3  # G entries gathered per second
+            rep["dim16"][f"16-D {r}x{c} B{bt}"] = {
+                "us": round(us, 3), "GB/s": round(b / us / 1e3, 1),
+                "hbm_frac": round(b / us / 1e3 / hbm_peak, 4), "G_entries/s": round(ents, 1),
+                "l2_gather_frac": round(ents / (rates["l2"] / 1e9), 4), "bytes": b, "pool": P,
+                "cluster_size": mats[0].plan(bt)["cluster_size"]}
+            for m in mats:
+                m.close()
+            torch.cuda.empty_cache()
     rep["prefill_gemm"] = gemm_report(hbm_peak)
     rep["encode"] = encode_report()
     rep["oracle_timing"] = oracle_timing()

@@ -124,8 +124,17 @@ sphq_status sphq_create_v(int rows, int cols, int bits, int radius_bits, int K,
  *           rejected) and rows x cols/4 codes.  sphq_gemv, sphq_gemv_host,
  *           sphq_decode, sphq_export support it; sphq_gemm and sphq_encode
  *           do not (SPHQ_ERR_UNSUPPORTED).
- *   dim 16  SPHQ_ERR_UNSUPPORTED: the W2 codebook (2^14 entries x 32 B =
- *           512 KiB) exceeds an SM's shared memory.
+ *   dim 16  bits = 2, K = 16384 (15B - 16 = 14 index bits), radius_bits = 4:
+ *           16 sign bits + 14 + 4 = 34 bits per 16 weights (2.125 bits per
+ *           weight); codebook K x 16 fp16 (512 KiB, beyond an SM's shared
+ *           memory: the GEMV gathers its entries from global memory, so it
+ *           is bound by random L2 reads, ~14% of the HBM rate on GB300);
+ *           radius groups of 128 scalars (8 vectors); sphq_pack takes the
+ *           sign argument as rows x cols/16 uint16 (bit j = coordinate j,
+ *           2-byte aligned) and rows x cols/16 codes.  sphq_gemv (batch
+ *           1..16; 9..16 as launches of 8 rows and the rest),
+ *           sphq_gemv_host, sphq_gemv_noalloc, sphq_decode, sphq_export /
+ *           sphq_import support it; sphq_gemm and sphq_encode do not.
  */
 sphq_status sphq_create_dim(int rows, int cols, int dim, int bits, int radius_bits, int K,
                             const void* codebook, const void* scale, const void* offset,
@@ -137,7 +146,8 @@ sphq_status sphq_create_dim(int rows, int cols, int dim, int bits, int radius_bi
  *
  *   sign   rows x (cols/8) uint8, bit j set <=> coordinate j of the vector is
  *          negative (§3.1, Eq. (3)); vector t of a row covers columns 8t..8t+7
- *          (4-D handles: rows x (cols/4), columns 4t..4t+3, bits 0-3).
+ *          (4-D handles: rows x (cols/4), columns 4t..4t+3, bits 0-3; 16-D
+ *          handles: rows x (cols/16) uint16, columns 16t..16t+15).
  *   idx    rows x (cols/8) uint16, direction index z < K (Eq. (5)).
  *   rcode  rows x (cols/8) uint8, radius code q < 2^V (Eq. (7); V = 4, or
  *          the handle's radius_bits).

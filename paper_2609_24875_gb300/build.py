@@ -17,7 +17,8 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libsphq.so")
 SOURCES = ["sphq_api.cu", "sphq_gemv.cu", "sphq_gemv_splits.cu", "sphq_gemm.cu",
-           "sphq_encode.cu", "sphq_io.cu", "sphq_noalloc.cu", "sphq_codebook.cu"]
+           "sphq_encode.cu", "sphq_io.cu", "sphq_noalloc.cu", "sphq_codebook.cu",
+           "sphq_dim16.cu"]
 STUDY_SRC = os.path.join(CSRC, "study", "gather16.cu")
 STUDY_LIB = os.path.join(HERE, "libsphq_study.so")
 HEADERS = ["sphq_layout.cuh", "sphq_gemv_kernel.cuh", "sphq_umma.cuh", "sphq_internal.h"]

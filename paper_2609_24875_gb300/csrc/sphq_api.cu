@@ -385,6 +385,12 @@ static sphq_status create_impl(int rows, int cols, int dim, int bits, int radius
       return set_error(SPHQ_ERR_UNSUPPORTED,
                        "sphq_create_dim: 4-D vectors take bits = 2, K = 4, radius_bits = 4");
     fmt = kFmt4D;
+  } else if (dim == 16) {
+    // Tab. 7, W2 allocation: 15 B - 16 = 14 index bits (K = 16384), V = 4
+    if (bits != 2 || K != 16384 || radius_bits != 4)
+      return set_error(SPHQ_ERR_UNSUPPORTED,
+                       "sphq_create_dim: 16-D vectors take bits = 2, K = 16384, radius_bits = 4");
+    fmt = kFmt16D;
   } else if (dim == 8) {
     // direction index bits D = log2 K: 13 for W3; 6 (the §3.1 rule), 7 or 8 (Tab. 4) for W2
     const bool k_ok = bits == 3 ? dbits == 13 : (dbits >= 6 && dbits <= 8);
@@ -397,10 +403,7 @@ static sphq_status create_impl(int rows, int cols, int dim, int bits, int radius
                        "sphq_create: unsupported split; sign/index/radius bits must be one of "
                        "8/6/4, 8/6/3, 8/6/2, 8/7/3, 8/7/2, 8/8/2, 8/13/4, 8/13/3");
   } else {
-    return set_error(SPHQ_ERR_UNSUPPORTED,
-                     dim == 16 ? "sphq_create_dim: 16-D vectors are not supported (their W2 "
-                                 "codebook is 512 KiB, beyond shared memory)"
-                               : "sphq_create_dim: dim must be 4 or 8");
+    return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_create_dim: dim must be 4, 8 or 16");
   }
   const size_t cb_bytes = (size_t)K * dim * 2;
   if (!codebook || !scale || !offset)
@@ -468,6 +471,10 @@ static sphq_status create_impl(int rows, int cols, int dim, int bits, int radius
                             (size_t)K, cudaMemcpyDeviceToDevice)) != cudaSuccess)
         return fail(cuda_error(e, "codebook image"));
   }
+  if (fmt == kFmt16D) {
+    sphq_status st = build_cbimage16(h);
+    if (st != SPHQ_OK) return fail(st);
+  }
   if (fmt_small(fmt)) {
     // shared-memory image of the small-codebook GEMV: entry k, copy c at 128 k + 16 c
     if ((e = cudaMalloc(&h->cbimage, (size_t)K * 8 * 16)) != cudaSuccess)
@@ -528,7 +535,12 @@ static sphq_status pack_codes(sphq_handle h, const uint8_t* sign, const uint16_t
   const long long threads = (long long)h->nrt * h->ng * 32;
   const int block = 256;
   const unsigned grid = (unsigned)((threads + block - 1) / block);
-  if (h->fmt == kFmt4D) {
+  if (h->fmt == kFmt16D) {
+    if (reinterpret_cast<uintptr_t>(sign) % 2)
+      return set_error(SPHQ_ERR_INVALID_ARG, "sphq_pack: 16-D signs must be 2-byte aligned");
+    sphq_status st = pack16(h, reinterpret_cast<const uint16_t*>(sign), idx, rcode, scale, offset, s);
+    if (st != SPHQ_OK) return st;
+  } else if (h->fmt == kFmt4D) {
     pack4_kernel<<<grid, block, 0, s>>>(sign, idx, rcode, scale, offset, (uint8_t*)h->units,
                                         h->rows, h->ng, h->nrt, h->flag);
   } else switch (h->fmt) {
@@ -616,7 +628,10 @@ sphq_status sphq_decode(sphq_handle h, void* w, sphq_stream stream) {
   const long long n = (long long)h->rows * (h->cols / kVec);
   const int block = 256;
   const unsigned grid = (unsigned)((n + block - 1) / block);
-  if (h->fmt == kFmt4D) {
+  if (h->fmt == kFmt16D) {
+    sphq_status st = decode16(h, w, s);
+    if (st != SPHQ_OK) return st;
+  } else if (h->fmt == kFmt4D) {
     const long long nv4 = (long long)h->rows * (h->cols / 4);
     decode4_kernel<<<(unsigned)((nv4 + 255) / 256), 256, 0, s>>>(
         (const uint8_t*)h->units, (const uint8_t*)h->codebook, (uint16_t*)w, h->rows, h->cols,

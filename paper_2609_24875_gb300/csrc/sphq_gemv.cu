@@ -280,6 +280,17 @@ static sphq_status device_optin(sphq_handle h, int* optin) {
 }
 
 sphq_status make_gemv_plans(sphq_handle h) {
+  if (h->fmt == kFmt16D) {  // batches 9-16: launches of 8 rows and the rest
+    for (int batch = 1; batch <= SPHQ_MAX_BATCH; ++batch) {
+      h->plan[batch] = GemvPlan{};
+      if (batch <= kMaxBatch) {
+        sphq_status st = make_gemv16_plan(h, batch, 0, h->plan[batch]);
+        if (st != SPHQ_OK) return st;
+      }
+    }
+    h->ws_floats = 0;
+    return SPHQ_OK;
+  }
   int optin = 0;
   sphq_status st = device_optin(h, &optin);
   if (st != SPHQ_OK) return st;
@@ -296,6 +307,12 @@ sphq_status make_gemv_plans(sphq_handle h) {
 }
 
 sphq_status set_gemv_cluster_size(sphq_handle h, int batch, int csize) {
+  if (h->fmt == kFmt16D) {
+    if (batch > kMaxBatch)
+      return set_error(SPHQ_ERR_UNSUPPORTED,
+                       "sphq_set_cluster_size: 16-D batches above 8 run as launches of 8 and the rest");
+    return make_gemv16_plan(h, batch, csize, h->plan[batch]);
+  }
   int optin = 0;
   sphq_status st = device_optin(h, &optin);
   if (st != SPHQ_OK) return st;
@@ -308,13 +325,14 @@ sphq_status set_gemv_cluster_size(sphq_handle h, int batch, int csize) {
 
 sphq_status launch_gemv(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s) {
   if (batch > kMaxBatch && h->plan[batch].grid == 0) {
-    // no 16-row build (4-D vectors): 8 rows, then the rest
+    // no 16-row build (4-D and 16-D vectors): 8 rows, then the rest
     sphq_status st = launch_gemv(h, x, y, kMaxBatch, s);
     if (st != SPHQ_OK) return st;
     return launch_gemv(h, static_cast<const uint16_t*>(x) + (size_t)kMaxBatch * h->cols,
                        static_cast<uint16_t*>(y) + (size_t)kMaxBatch * h->rows, batch - kMaxBatch,
                        s);
   }
+  if (h->fmt == kFmt16D) return launch_gemv16(h, x, y, batch, s);
   const GemvPlan& p = h->plan[batch];
   GemvArgs a;
   a.units = (const uint8_t*)h->units;

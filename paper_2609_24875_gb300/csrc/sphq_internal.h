@@ -33,7 +33,7 @@ struct sphq_handle_s {
   int rows = 0, cols = 0, bits = 0, K = 0;
   int vbits = 4;           // radius code bits V
   int dbits = 6;           // direction index bits D = log2 K
-  int dim = 8;             // vector dimension (8, or 4)
+  int dim = 8;             // vector dimension (8, 4 or 16)
   int fmt = 0;             // device format id (sphq_layout.cuh), one per bit split
   int nrt = 0;             // row tiles of 16 rows
   int ng = 0;              // radius groups per row (cols / 128)
@@ -42,7 +42,7 @@ struct sphq_handle_s {
   size_t unit_bytes = 0;
   void* units = nullptr;       // packed units, nrt * ng * unit_bytes
   void* codebook = nullptr;    // K * 8 fp16
-  void* cbimage = nullptr;     // W2: eight interleaved codebook copies (8 KiB)
+  void* cbimage = nullptr;     // W2: eight interleaved codebook copies (8 KiB); 16-D: lane-ordered entries
   uint32_t* params = nullptr;  // rows * ng words: Delta | r_min << 16
   float* ws = nullptr;         // split-K partial sums of plans that need them (none today)
   size_t ws_floats = 0;
@@ -88,6 +88,15 @@ sphq_status gemm_workspace_bytes(sphq_handle h, int batch, size_t* bytes);
 // tensor-core product reading it (validated x, y, batch).
 sphq_status launch_gemm_two_pass(sphq_handle h, const void* x, void* y, int batch, void* ws,
                                  size_t ws_bytes, cudaStream_t s);
+// 16-D vectors (sphq_dim16.cu): the lane-ordered codebook image (synchronous),
+// pack and decode launches, the GEMV plan of one batch size (csize 0:
+// automatic) and its launch (batch 1..8).
+sphq_status build_cbimage16(sphq_handle h);
+sphq_status pack16(sphq_handle h, const uint16_t* sign, const uint16_t* idx, const uint8_t* rcode,
+                   const uint16_t* scale, const uint16_t* offset, cudaStream_t s);
+sphq_status decode16(sphq_handle h, void* w, cudaStream_t s);
+sphq_status make_gemv16_plan(sphq_handle h, int batch, int csize, GemvPlan& out);
+sphq_status launch_gemv16(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s);
 // Enqueues the GEMV with caller-provided split-K scratch: `ws` holds at least
 // h->ws_floats floats and `tickets` h->nrt zeroed counters.
 sphq_status launch_gemv_scratch(sphq_handle h, const void* x, void* y, int batch, cudaStream_t s,

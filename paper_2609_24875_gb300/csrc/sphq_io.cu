@@ -97,7 +97,8 @@ sphq_status sphq_import(const void* buf, size_t size, sphq_handle* out) {
     return set_error(SPHQ_ERR_INVALID_ARG, "sphq_import: bad shape in header");
   const uint8_t* p = static_cast<const uint8_t*>(buf) + sizeof(BlobHeader);
   const int dim = hd.dim == 0 ? 8 : hd.dim;
-  if (dim != 4 && dim != 8) return set_error(SPHQ_ERR_INVALID_ARG, "sphq_import: bad dimension");
+  if (dim != 4 && dim != 8 && dim != 16)
+    return set_error(SPHQ_ERR_INVALID_ARG, "sphq_import: bad dimension");
   const size_t np = (size_t)hd.rows * (hd.cols / 128);
   const size_t cbb = (size_t)hd.K * dim * 2;
   const size_t fixed = sizeof(BlobHeader) + cbb + 2 * np * 2;

@@ -110,14 +110,22 @@ constexpr int kFmt862 = 5, kFmt863 = 6, kFmt872 = 7, kFmt873 = 8, kFmt882 = 9;
 // 4-D vectors at the W2 allocation (Tab. 7): 4 sign bits, a 2-bit index into
 // K = 4 directions, a 4-bit radius code (2.5 bits per weight).
 constexpr int kFmt4D = 10;
+// 16-D vectors at the W2 allocation (Tab. 7): 16 sign bits, a 14-bit index
+// into K = 16384 directions (a 512 KiB codebook, gathered from global memory),
+// a 4-bit radius code (2.125 bits per weight); kernels in sphq_dim16.cu.
+constexpr int kFmt16D = 11;
 __host__ __device__ constexpr int fmt_dir_bits(int fmt) {
-  return fmt == 3 || fmt == 4 ? 13 : fmt == 7 || fmt == 8 ? 7 : fmt == 9 ? 8 : fmt == kFmt4D ? 2 : 6;
+  return fmt == 3 || fmt == 4 ? 13 : fmt == 7 || fmt == 8 ? 7 : fmt == 9 ? 8 : fmt == kFmt4D ? 2
+         : fmt == kFmt16D ? 14 : 6;
 }
 __host__ __device__ constexpr int fmt_radius_bits(int fmt) {
-  return fmt == 2 || fmt == 3 || fmt == kFmt4D ? 4 : fmt == 4 || fmt == 6 || fmt == 8 ? 3 : 2;
+  return fmt == 2 || fmt == 3 || fmt == kFmt4D || fmt == kFmt16D ? 4
+         : fmt == 4 || fmt == 6 || fmt == 8 ? 3 : 2;
 }
 // vector dimension of a format
-__host__ __device__ constexpr int fmt_dim(int fmt) { return fmt == kFmt4D ? 4 : 8; }
+__host__ __device__ constexpr int fmt_dim(int fmt) {
+  return fmt == kFmt4D ? 4 : fmt == kFmt16D ? 16 : 8;
+}
 // formats whose codebook (K <= 256) is kept as eight interleaved copies
 __host__ __device__ constexpr bool fmt_small(int fmt) { return fmt == 2 || (fmt >= 5 && fmt <= 9); }
 // format id of a split, or -1
@@ -157,6 +165,14 @@ template <> struct Layout<kFmt4D> {
   static constexpr int kS1Off = 512;
   static constexpr int kParamOff = 640;
 };
+// 16-D unit (16 rows x 128 columns = 128 vectors): 608 B = 128 words of 32
+// bits + 8 radius words + 8 parameter pairs; see sphq_dim16.cu.
+template <> struct Layout<kFmt16D> {
+  static constexpr int K = 16384;
+  static constexpr int kUnitBytes = 608;
+  static constexpr int kHiOff = 512;
+  static constexpr int kParamOff = 544;
+};
 template <> struct Layout<3> {
   static constexpr int K = 8192;
   static constexpr int kUnitBytes = 864;
@@ -170,6 +186,7 @@ __host__ __device__ constexpr int fmt_unit_bytes(int fmt) {
   return fmt == 3 ? Layout<3>::kUnitBytes
          : fmt == kFmtW3V3 ? Layout<kFmtW3V3>::kUnitBytes
          : fmt == kFmt4D ? Layout<kFmt4D>::kUnitBytes
+         : fmt == kFmt16D ? Layout<kFmt16D>::kUnitBytes
          : fmt_dir_bits(fmt) + fmt_radius_bits(fmt) == 10 ? 640
          : fmt_dir_bits(fmt) + fmt_radius_bits(fmt) == 9 ? 608
                                                           : 576;

@@ -149,7 +149,8 @@ class SphqMatrix:
                  radius_bits: int = 4, K: int | None = None, dim: int = 8):
         """bits 2 or 3; K defaults to 2^((dim-1)*bits - dim) (64 / 8192 for 8-D);
         the Tab. 4 splits take K = 128 or 256 at bits = 2 and radius_bits 2 or 3
-        (sphq_create_v); dim = 4 takes bits 2, K 4 (sphq_create_dim)."""
+        (sphq_create_v); dim = 4 takes bits 2, K 4 and dim = 16 bits 2, K 16384
+        (sphq_create_dim)."""
         import torch
         L = load()
         if K is None:
@@ -174,13 +175,16 @@ class SphqMatrix:
         return self._h.value
 
     def pack(self, sign, idx, rcode, stream=None) -> None:
-        """sign/idx/rcode: (rows, cols/dim) uint8 / uint16(int16) / uint8 device tensors."""
+        """sign/idx/rcode: (rows, cols/dim) uint8 (16-D: 2-byte) / uint16(int16) / uint8
+        device tensors."""
         nv = self.cols // self.dim
         for t in (sign, idx, rcode):
             if tuple(t.shape) != (self.rows, nv) or not t.is_cuda or not t.is_contiguous():
                 raise ValueError("codes must be contiguous CUDA tensors of shape (rows, cols/8)")
-        if sign.element_size() != 1 or rcode.element_size() != 1 or idx.element_size() != 2:
-            raise ValueError("sign/rcode must be 1-byte and idx 2-byte tensors")
+        if (sign.element_size() != (2 if self.dim == 16 else 1) or rcode.element_size() != 1
+                or idx.element_size() != 2):
+            raise ValueError("sign (2 bytes for 16-D vectors, else 1) / rcode 1-byte and idx "
+                             "2-byte tensors expected")
         _check(load().sphq_pack(self._h, sign.data_ptr(), idx.data_ptr(), rcode.data_ptr(),
                                 _stream_ptr(stream)))
 

@@ -118,11 +118,6 @@ def test_code_validation_and_unsupported_entry_points():
         m.gemm(G.x_dev(np.zeros((16, 256), np.uint16)))
     assert e.value.status == 2
     m.close()
-    cb16 = inp.to_f16_bits(np.full((1 << 14, 16), 0.25))
-    sc = inp.to_f16_bits(np.ones((16, 1)))
-    with pytest.raises(SphqError) as e:
-        SphqMatrix(16, 128, 2, G.to_dev(cb16), G.to_dev(sc), G.to_dev(sc), K=1 << 14, dim=16)
-    assert e.value.status == 2
 
 
 def test_8192_square_sampled_rows():
