@@ -168,8 +168,10 @@ __device__ __forceinline__ void cluster_arrive_release() {
 // through shared memory, then the cluster's CTAs in rank order through
 // distributed shared memory into rank 0, which rounds to fp16 and writes y.
 // The two cluster barriers are hardware barriers that every thread of every
-// CTA of the cluster reaches (no early exit before them).
-__global__ void __launch_bounds__(kWarps16 * 32, 2) gemv16_kernel(const Gemv16Args a) {
+// CTA of the cluster reaches (no early exit before them).  MINB: CTAs per SM
+// the build's registers allow (2: 115 registers, 4: 64, neither spills).
+template <int MINB>
+__global__ void __launch_bounds__(kWarps16 * 32, MINB) gemv16_kernel(const Gemv16Args a) {
   __shared__ float red[kWarps16][kRowsPerTile][8];
   __shared__ float recv[8][kRowsPerTile][8];
   pdl_launch_dependents();
@@ -307,7 +309,10 @@ sphq_status decode16(sphq_handle h, void* w, cudaStream_t s) {
 // batch 1 and 8): a CTA per SM beats more CTAs -- 4096^2 7.7 / 10.2 / 13.1 us
 // at clusters of 1 / 2 / 4, 8192^2 25.9 / 31.1 / 34.1 -- while 512 x 3584
 // (32 row tiles) needs clusters of 8 to fill the SMs (3.0 us against 4.9 for
-// single CTAs).
+// single CTAs).  Grids of three CTAs per SM or more take the 4-per-SM build
+// (more warps hide the L2 gathers: 8192^2 26.0 -> 24.7 us, 18944 x 3584
+// 26.0 -> 23.8); smaller grids the 2-per-SM one (the 4-per-SM build put
+// 4096^2's 256 CTAs on fewer SMs: 7.8 -> 12.9 us).
 sphq_status make_gemv16_plan(sphq_handle h, int batch, int csize, GemvPlan& out) {
   (void)batch;
   int cs = csize;
@@ -325,7 +330,7 @@ sphq_status make_gemv16_plan(sphq_handle h, int batch, int csize, GemvPlan& out)
   p.smem = 0;
   p.mode = kFull;
   p.strip = 1;
-  p.ctas_per_sm = 2;
+  p.ctas_per_sm = (long long)p.grid >= 3LL * std::max(h->sm_count, 1) ? 4 : 2;
   out = p;
   return SPHQ_OK;
 }
@@ -361,7 +366,8 @@ sphq_status launch_gemv16(sphq_handle h, const void* x, void* y, int batch, cuda
   cfg.attrs = attr;
   cfg.numAttrs = h->pdl ? 2 : 1;
   void* args[] = {&a};
-  cudaError_t e = cudaLaunchKernelExC(&cfg, (const void*)gemv16_kernel, args);
+  const void* k = p.ctas_per_sm == 4 ? (const void*)gemv16_kernel<4> : (const void*)gemv16_kernel<2>;
+  cudaError_t e = cudaLaunchKernelExC(&cfg, k, args);
   if (e != cudaSuccess) return cuda_error(e, "gemv16 launch");
   return SPHQ_OK;
 }
