@@ -132,7 +132,18 @@ static sphq_status make_plan(sphq_handle h, int batch, int forced, int optin, Ge
     GemvPlan packed{};
     double packed_load = 0;
     const int warps = warps_for(h->fmt);
-    for (int staged = 1; staged >= 0; --staged) {
+    // Batch 2 reads its activations through L1 (the full mode: exact w_hat,
+    // no staged copy) for the 8192-entry tables and for small matrices:
+    // measured against the staged factored mode, W3 3584^2 5.57 -> 5.17 us,
+    // 4096^2 6.07 -> 5.75, 8192^2 16.13 -> 15.26, 512 x 3584 2.50 -> 2.37
+    // (18944 x 3584 15.28 / 15.37: equal); W2 512 x 3584 2.06 -> 1.89,
+    // 3584^2 4.30 -> 4.15, 4096^2 4.48 -> 4.32, while from 32768 units up the
+    // staged mode stays faster (8192^2 10.61 against 11.19).  Batch 1 keeps
+    // the staged mode (the full mode within -2% to +4% of it).
+    const bool full2 = batch == 2 && (!fmt_small(h->fmt) && h->fmt != kFmt4D
+                                          ? true
+                                          : (long long)h->nrt * h->ng <= 16384);
+    for (int staged = full2 ? 0 : 1; staged >= 0; --staged) {
       int mode = mode_for(batch);
       if (!staged && !mode_full(mode)) mode = kFull;
       if (staged && mode_full(mode)) continue;

@@ -104,3 +104,19 @@ def test_kernel_build_per_plan(bits, rows, cols, ctas):
         assert p["ctas_per_sm"] == ctas, (batch, p)
         _check(m, codes, x[:batch], batch)
     m.close()
+
+
+# Batch 2 reads its activations through L1 (the full mode) for the 8192-entry
+# tables and for matrices of up to 16384 units; larger small-codebook
+# matrices stage them in shared memory (the factored mode).
+@pytest.mark.parametrize("bits,rows,cols,staged", [(3, 512, 3584, False), (3, 18944, 3584, False),
+                                                   (2, 512, 3584, False), (2, 3584, 18944, True)])
+def test_batch2_mode_choice(bits, rows, cols, staged):
+    codes, x = inp.random_codes(bits, rows, cols, seed=4200 + rows + bits, B=2)
+    m = G.make_matrix(codes)
+    assert bool(m.plan(2)["staged_x"]) == staged
+    assert bool(m.plan(1)["staged_x"])  # batch 1 always stages
+    G.check_gemv(m, codes, x, G.sample_rows(rows, 160, seed=rows))
+    G.check_gemv(m, codes, x[:1], G.sample_rows(rows, 160, seed=rows + 1))
+    m.check()
+    m.close()
