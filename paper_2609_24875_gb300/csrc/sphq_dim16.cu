@@ -321,6 +321,8 @@ sphq_status make_gemv16_plan(sphq_handle h, int batch, int csize, GemvPlan& out)
     cs = 1;
     while (cs < 8 && 2 * cs <= h->ng && (long long)h->nrt * cs < sms) cs *= 2;
   }
+  if ((long long)h->nrt * cs > 0x7FFFFFFFLL)
+    return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemv: too many row tiles for one 16-D launch");
   GemvPlan p;
   p.warps_per_cta = kWarps16;
   p.csize = cs;
