@@ -361,28 +361,42 @@ sphq_status sphq_gemv_noalloc(sphq_handle h, const void* x, void* y, int batch,
 sphq_status sphq_gemm(sphq_handle h, const void* x, void* y, int batch, sphq_stream stream);
 
 /*
- * sphq_gemm_workspace / sphq_gemm_ws -- the same product in two passes, for
- * large batches of the formats whose fused kernel is bound by its codebook
- * gathers (§3.4 with W_hat from Eq. (7) and Eq. (4), computed in a different
- * order: decode once, then multiply).
+ * sphq_gemm_workspace / sphq_gemm_ws -- the same product with a caller
+ * workspace, in one of two forms (§3.4 with W_hat from Eq. (7) and Eq. (4)).
  *
- * Pass 1 decodes W_hat (rows x cols fp16, exactly sphq_decode's output) into
- * a caller-provided device workspace; pass 2 is a dense tensor-core product
- * that loads W_hat and X tiles with TMA.  The decode then costs one write and
- * one read of 2 bytes per weight per call instead of a shared-memory gather
- * per weight and activation tile.  Products, accumulation order and rounding
- * are those of sphq_gemm: Y is equal to sphq_gemm's bit for bit.
+ * Two-pass form, for large batches of the formats whose fused kernel is bound
+ * by its codebook gathers: pass 1 decodes W_hat (rows x cols fp16, exactly
+ * sphq_decode's output) into the workspace; pass 2 is a dense tensor-core
+ * product that loads W_hat and X tiles with TMA.  The decode then costs one
+ * write and one read of 2 bytes per weight per call instead of a
+ * shared-memory gather per weight and activation tile.  Products,
+ * accumulation order and rounding are those of sphq_gemm: Y is equal to
+ * sphq_gemm's bit for bit.
  *
- * sphq_gemm_workspace sets *bytes to rows x cols x 2 when the two-pass form is
- * estimated faster than the fused kernel for this batch, else to 0.
+ * Split-K form, for batches of 41..256 (shape automatic) when the output
+ * tiles are too few to fill the GPU and each tile's columns can be shared by
+ * several CTAs of at least 16 radius groups each: every CTA multiplies its
+ * share, writes an fp32 partial tile into the workspace, and the tile's last
+ * CTA adds the partials in share order (a fixed order: repeatable bit for
+ * bit; not equal to sphq_gemm's bits, within the same tolerance).  The
+ * workspace holds the partial tiles and one counter per tile, which a memset
+ * clears on the stream before the launch.  sphq_get_gemm_shape reports the
+ * shares (ksplit).
+ *
+ * sphq_gemm_workspace sets *bytes to the split-K form's size where it
+ * applies, else to rows x cols x 2 when the two-pass form is estimated
+ * faster than the fused kernel for this batch, else to 0.
  *
  * sphq_gemm_ws takes the arguments of sphq_gemm plus the workspace:
- *   workspace        device pointer, 16-byte aligned, at least rows x cols x 2
- *                    bytes (SPHQ_ERR_INVALID_ARG otherwise), owned by the
- *                    caller, overwritten; NULL runs the fused kernel
- *                    (= sphq_gemm).
- * Asynchronous on `stream` (two launches), no allocation.  A workspace must not
- * be shared by calls that overlap on the GPU.
+ *   workspace        device pointer, 16-byte aligned, owned by the caller,
+ *                    overwritten; NULL runs sphq_gemm.
+ *   workspace_bytes  the split-K form runs where it applies and the
+ *                    workspace holds its size; otherwise the two-pass form,
+ *                    which needs rows x cols x 2 bytes (SPHQ_ERR_INVALID_ARG
+ *                    otherwise).
+ * Asynchronous on `stream` (two launches: the decode and the product, or the
+ * counter memset and the product), no allocation.  A workspace must not be
+ * shared by calls that overlap on the GPU.
  */
 sphq_status sphq_gemm_workspace(sphq_handle h, int batch, size_t* bytes);
 sphq_status sphq_gemm_ws(sphq_handle h, const void* x, void* y, int batch, void* workspace,
@@ -395,8 +409,9 @@ sphq_status sphq_gemm_ws(sphq_handle h, const void* x, void* y, int batch, void*
  * tiles (grid_x weight tiles x grid_y activation tiles of act_tiles x 128
  * rows), dynamic shared memory, and split_ctas: with two activation tiles,
  * the CTAs of one activation tile that take a final partial wave of output
- * tiles (two per output tile; 0 when the wave is not split).  (No counterpart
- * in the paper.)
+ * tiles (two per output tile; 0 when the wave is not split), and ksplit: the
+ * CTAs that share each output tile's columns in sphq_gemm_ws's split-K form
+ * (1 where that form does not apply).  (No counterpart in the paper.)
  * sphq_set_gemm_shape -- fix act_tiles (1, 2; 0 = automatic) and weight_rows
  * (128, 256; 0 = automatic) for later sphq_gemm calls on the handle; 128 rows
  * go with one activation tile only; a fixed act_tiles also keeps the final
@@ -405,7 +420,7 @@ sphq_status sphq_gemm_ws(sphq_handle h, const void* x, void* y, int batch, void*
 typedef struct sphq_gemm_info {
   int act_tiles, weight_rows, stage_cols, stages, grid_x, grid_y;
   long long smem_bytes;
-  int split_ctas;
+  int split_ctas, ksplit;
 } sphq_gemm_info;
 sphq_status sphq_get_gemm_shape(sphq_handle h, int batch, sphq_gemm_info* out);
 sphq_status sphq_set_gemm_shape(sphq_handle h, int act_tiles, int weight_rows);

@@ -725,8 +725,8 @@ sphq_status sphq_gemm_ws(sphq_handle h, const void* x, void* y, int batch, void*
   if (!h->packed) return set_error(SPHQ_ERR_NOT_PACKED, "sphq_gemm_ws: handle not packed");
   if (h->dim != 8) return set_error(SPHQ_ERR_UNSUPPORTED, "sphq_gemm_ws: 8-D vectors only");
   if (!workspace) return launch_gemm(h, x, y, batch, reinterpret_cast<cudaStream_t>(stream));
-  return launch_gemm_two_pass(h, x, y, batch, workspace, workspace_bytes,
-                              reinterpret_cast<cudaStream_t>(stream));
+  return launch_gemm_ws(h, x, y, batch, workspace, workspace_bytes,
+                        reinterpret_cast<cudaStream_t>(stream));
 }
 
 sphq_status sphq_get_gemm_shape(sphq_handle h, int batch, sphq_gemm_info* out) {

@@ -59,6 +59,8 @@ constexpr int kGemmBM = 128;                    // activation rows per tile (MMA
 // (rows x cols fp16 in global memory, written by decode_units_kernel) that
 // the TMA warp loads beside the activations; no codebook, no decode warps.
 constexpr int kFmtDense = 0;
+// Batches taking the split-K form (with a workspace, the shape automatic).
+constexpr int kSplitMinBatch = 41, kSplitMaxBatch = 256, kSplitMinGroups = 16;
 // One decode warp per 16-row tile of the weight tile (16 or 8), then the MMA
 // warp and the TMA warp.
 constexpr int gemm_threads(int bn) { return (bn / kRowsPerTile + 2) * 32; }
@@ -74,6 +76,9 @@ struct GemmArgs {
   int rows, cols, nrt, batch;
   int nwt;                 // weight tiles (of BN rows) across the rows
   int n_big;               // CTAs with MT activation tiles; the rest take one
+  int ksplit;              // CTAs per output tile, each a share of the radius groups (split-K)
+  float* part;             // split-K: fp32 partial tiles, [tile][ksplit][MT x 128][BN]
+  unsigned* tickets;       // split-K: per output tile, CTAs done (zeroed before the launch)
   int stages;              // ring depth
   uint32_t cb_bytes;
   uint32_t off_b, off_cb, off_bar;  // from the 1024-byte aligned base; A tiles at 0
@@ -90,6 +95,20 @@ __device__ __forceinline__ void sts16(uint32_t addr, uint4 v) {
 
 __device__ __forceinline__ uint4 sel4(bool p, uint4 a, uint4 b) {
   return make_uint4(p ? a.x : b.x, p ? a.y : b.y, p ? a.z : b.z, p ? a.w : b.w);
+}
+
+// Element (activation row t, weight row n) of a split-K partial tile sits at
+// t * BN + n; a thread stores / sums 32 consecutive weight rows of one
+// activation row (one tcgen05.ld of 32 columns).
+__device__ __forceinline__ void store_part32(float* p, const uint32_t (&v)[32]) {
+#pragma unroll
+  for (int t = 0; t < 8; ++t)
+    reinterpret_cast<float4*>(p)[t] =
+        make_float4(__uint_as_float(v[4 * t]), __uint_as_float(v[4 * t + 1]),
+                    __uint_as_float(v[4 * t + 2]), __uint_as_float(v[4 * t + 3]));
+}
+__device__ __forceinline__ void named_sync(int id, int threads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
 }
 
 // Decodes words M and M+1 (the stage's 64 columns) of the lane's unit and
@@ -160,24 +179,34 @@ __global__ void __launch_bounds__(gemm_threads(BN), 1)
   const uint32_t sbase = smem_u32(smem);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int S = a.stages;
-  const int nk = a.cols / BK;
   const int ng = a.cols / kGroupCols;
   const uint32_t full0 = sbase + a.off_bar;  // full[S], empty[S], acc, cb, tmem slot
   const uint32_t empty0 = full0 + 8u * S;
   const uint32_t acc_bar = empty0 + 8u * S;
   const uint32_t cb_bar = acc_bar + 8u;
   uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + a.off_bar + 16u * S + 16u);
+  // Split-K: the ksplit consecutive CTAs of an output tile take consecutive
+  // shares of the radius groups (columns) and sum their fp32 partials through
+  // global memory in share order.
+  int bid = (int)blockIdx.x, kidx = 0;
+  if (a.ksplit > 1) {
+    kidx = bid % a.ksplit;
+    bid /= a.ksplit;
+  }
+  const int g_lo = kidx * (ng / a.ksplit) + min(kidx, ng % a.ksplit);
+  const int g_hi = g_lo + ng / a.ksplit + (kidx < ng % a.ksplit ? 1 : 0);
+  const int i_lo = g_lo * kStepsPerGroup, i_hi = g_hi * kStepsPerGroup;
   // This CTA's output tile.  The first n_big CTAs take MT activation tiles
   // (weight tile fastest); the rest split the remaining MT-tile outputs into
   // one activation tile each (two CTAs per output tile, a final wave that
   // spreads over twice the SMs).
   int wt, tok0, mt;
-  if ((int)blockIdx.x < a.n_big) {
-    wt = (int)blockIdx.x % a.nwt;
-    tok0 = (int)blockIdx.x / a.nwt * (kGemmBM * MT);
+  if (bid < a.n_big) {
+    wt = bid % a.nwt;
+    tok0 = bid / a.nwt * (kGemmBM * MT);
     mt = MT;
   } else {
-    const int j = (int)blockIdx.x - a.n_big, L = a.n_big + (j >> 1);
+    const int j = bid - a.n_big, L = a.n_big + (j >> 1);
     wt = L % a.nwt;
     tok0 = L / a.nwt * (kGemmBM * MT) + (j & 1) * kGemmBM;
     mt = 1;
@@ -214,7 +243,7 @@ __global__ void __launch_bounds__(gemm_threads(BN), 1)
     if (lane == 0) {
       umma::prefetch_tmap(&tmap);
       if constexpr (kDense) umma::prefetch_tmap(&tmap_w);
-      for (int i = 0, s = 0, r = 0; i < nk; ++i) {
+      for (int i = i_lo, s = 0, r = 0; i < i_hi; ++i) {
         if (r > 0 && !mbar_wait_poll(empty0 + 8u * s, (r - 1) & 1)) atomicOr(a.flag, 2);
         mbar_arrive_expect_tx(full0 + 8u * s, (uint32_t)mt * kTileA + (kDense ? kTileB : 0u));
 #pragma unroll
@@ -232,7 +261,7 @@ __global__ void __launch_bounds__(gemm_threads(BN), 1)
   } else if (warp == kMmaWarp) {
     if (lane == 0) {
       constexpr uint32_t idesc = umma::idesc_f16_f32(kGemmBM, BN);
-      for (int i = 0, s = 0, r = 0; i < nk; ++i) {
+      for (int i = i_lo, s = 0, r = 0; i < i_hi; ++i) {
         if (!mbar_wait_poll(full0 + 8u * s, r & 1)) atomicOr(a.flag, 2);
         umma::fence_after_sync();
         const uint32_t at = sbase + s * kStageA, bt = sbase + a.off_b + s * kTileB;
@@ -245,7 +274,7 @@ __global__ void __launch_bounds__(gemm_threads(BN), 1)
             umma::mma_f16(taddr + t * BN,
                           BK == 64 ? umma::smem_desc_sw128(ad) : umma::smem_desc_sw64(ad),
                           BK == 64 ? umma::smem_desc_sw128(bd) : umma::smem_desc_sw64(bd), idesc,
-                          (i | kk) != 0);
+                          (i != i_lo || kk != 0));
           }
         }
         umma::commit(empty0 + 8u * s);
@@ -267,14 +296,14 @@ __global__ void __launch_bounds__(gemm_threads(BN), 1)
     const uint8_t* ub0 = a.units + (size_t)(rt0 + jt) * UB;  // group 0; + g * nrt * UB
     const size_t gstride = (size_t)a.nrt * UB;
     Unit<FMT> cur = {}, nxt = {};
-    if (ok) nxt = load_unit<FMT>(ub0, lane);
+    if (ok) nxt = load_unit<FMT>(ub0 + (size_t)g_lo * gstride, lane);
     if (!mbar_wait(cb_bar, 0) && lane == 0) atomicOr(a.flag, 2);
-    for (int i = 0, s = 0, r = 0; i < nk; ++i) {
+    for (int i = i_lo, s = 0, r = 0; i < i_hi; ++i) {
       const int g = i / kStepsPerGroup;
       const int step = i % kStepsPerGroup;
       if (step == 0) {
         cur = nxt;
-        if (ok && g + 1 < ng) nxt = load_unit<FMT>(ub0 + (size_t)(g + 1) * gstride, lane);
+        if (ok && g + 1 < g_hi) nxt = load_unit<FMT>(ub0 + (size_t)(g + 1) * gstride, lane);
       }
       // one lane polls the stage's release (the MMAs that read it are
       // complete); the warp's stores follow it through __syncwarp
@@ -318,32 +347,78 @@ __global__ void __launch_bounds__(gemm_threads(BN), 1)
     const int start = part * kColsPerWarp;
     const int acc = start / BN;
     const int token = tok0 + kGemmBM * acc + 32 * quarter + lane;
+    const int ncc = acc < mt ? kColsPerWarp / 32 : 0;
+    // 32 results of this thread's activation row, weight rows row0.. -> fp16 Y
+    auto store_y = [&](int row0, const uint32_t (&v)[32]) {
+      if (token >= a.batch || row0 >= a.rows) return;
+      uint16_t* dst = a.y + (size_t)token * a.rows + row0;
+      if (row0 + 32 <= a.rows && (reinterpret_cast<uintptr_t>(dst) & 15u) == 0) {
+        uint32_t hv[16];
+#pragma unroll
+        for (int t = 0; t < 16; ++t) {
+          const __half2 p = __floats2half2_rn(__uint_as_float(v[2 * t]),
+                                              __uint_as_float(v[2 * t + 1]));
+          hv[t] = *reinterpret_cast<const uint32_t*>(&p);
+        }
+#pragma unroll
+        for (int t = 0; t < 4; ++t)
+          reinterpret_cast<uint4*>(dst)[t] =
+              make_uint4(hv[4 * t], hv[4 * t + 1], hv[4 * t + 2], hv[4 * t + 3]);
+      } else {
+#pragma unroll
+        for (int t = 0; t < 32; ++t)
+          if (row0 + t < a.rows) dst[t] = f32_to_h_rn(__uint_as_float(v[t]));
+      }
+    };
+    // split-K partial rows of this thread: activation row (token - tok0)
+    constexpr size_t kPartFloats = (size_t)kGemmBM * MT * BN;
+    const size_t prow = (size_t)(kGemmBM * acc + 32 * quarter + lane) * BN;
 #pragma unroll 1
-    for (int cc = 0; cc < (acc < mt ? kColsPerWarp / 32 : 0); ++cc) {
+    for (int cc = 0; cc < ncc; ++cc) {
       const int col = start % BN + 32 * cc;  // within the accumulator
       const uint32_t tcol = (uint32_t)(acc * BN + col);
       uint32_t v[32];
       umma::ld_32x32b_x32(taddr + ((uint32_t)(32 * quarter) << 16) + tcol, v);
       umma::wait_ld();
-      const int row0 = rt0 * kRowsPerTile + col;
-      if (token < a.batch && row0 < a.rows) {
-        uint16_t* dst = a.y + (size_t)token * a.rows + row0;
-        if (row0 + 32 <= a.rows && (reinterpret_cast<uintptr_t>(dst) & 15u) == 0) {
-          uint32_t hv[16];
+      if (a.ksplit > 1)
+        store_part32(a.part + ((size_t)bid * a.ksplit + kidx) * kPartFloats + prow + col, v);
+      else
+        store_y(rt0 * kRowsPerTile + col, v);
+    }
+    if (a.ksplit > 1) {
+      // The last of the tile's CTAs to finish sums the partials in share
+      // order (a fixed order: deterministic) and writes Y.  No CTA waits for
+      // another: the others just leave.
+      int* last = reinterpret_cast<int*>(tslot + 1);
+      __threadfence();
+      named_sync(1, kDecodeWarps * 32);
+      if (warp == 0 && lane == 0)
+        *last = atomicAdd(a.tickets + bid, 1u) == (unsigned)(a.ksplit - 1);
+      named_sync(1, kDecodeWarps * 32);
+      if (*last) {
+        __threadfence();
+#pragma unroll 1
+        for (int cc = 0; cc < ncc; ++cc) {
+          const int col = start % BN + 32 * cc;
+          float sum[32];
 #pragma unroll
-          for (int t = 0; t < 16; ++t) {
-            const __half2 p = __floats2half2_rn(__uint_as_float(v[2 * t]),
-                                                __uint_as_float(v[2 * t + 1]));
-            hv[t] = *reinterpret_cast<const uint32_t*>(&p);
+          for (int t = 0; t < 32; ++t) sum[t] = 0.f;
+          for (int k = 0; k < a.ksplit; ++k) {  // shares in order
+            const float4* pp = reinterpret_cast<const float4*>(
+                a.part + ((size_t)bid * a.ksplit + k) * kPartFloats + prow + col);
+#pragma unroll
+            for (int t = 0; t < 8; ++t) {
+              const float4 q4 = __ldcg(pp + t);
+              sum[4 * t] += q4.x;
+              sum[4 * t + 1] += q4.y;
+              sum[4 * t + 2] += q4.z;
+              sum[4 * t + 3] += q4.w;
+            }
           }
+          uint32_t v[32];
 #pragma unroll
-          for (int t = 0; t < 4; ++t)
-            reinterpret_cast<uint4*>(dst)[t] =
-                make_uint4(hv[4 * t], hv[4 * t + 1], hv[4 * t + 2], hv[4 * t + 3]);
-        } else {
-#pragma unroll
-          for (int t = 0; t < 32; ++t)
-            if (row0 + t < a.rows) dst[t] = f32_to_h_rn(__uint_as_float(v[t]));
+          for (int t = 0; t < 32; ++t) v[t] = __float_as_uint(sum[t]);
+          store_y(rt0 * kRowsPerTile + col, v);
         }
       }
     }
@@ -518,6 +593,15 @@ struct GemmShape {
   GemmSmem L;
 };
 
+// Split-K plan of sphq_gemm_ws (gemm_splitk_plan below): CTAs per output
+// tile, workspace bytes (partials, then one counter per tile).
+struct SplitK {
+  int ksplit = 1;
+  size_t part_bytes = 0, bytes = 0;
+  long long tiles = 0;
+};
+static SplitK gemm_splitk_plan(const sphq_handle_s* h, int batch);
+
 // The grid of a launch shape: nwt x ntok output tiles of BN weight rows x MT
 // activation tiles, in whole waves of SMs plus a final partial wave.  With
 // MT = 2 (and MT automatic), a final wave of r tiles that fit twice over on
@@ -604,13 +688,15 @@ sphq_status gemm_shape_info(sphq_handle h, int batch, sphq_gemm_info* out) {
   out->grid_y = G.ntok;
   out->smem_bytes = (long long)g.L.total;
   out->split_ctas = G.n_small;
+  out->ksplit = gemm_splitk_plan(h, batch).ksplit;
   return SPHQ_OK;
 }
 
 // One launch of the product kernel: the fused form (w_hat == nullptr), or the
 // second pass of the two-pass form reading the decoded w_hat.
 static sphq_status launch_gemm_kernel(sphq_handle h, const void* x, void* y, int batch,
-                                      cudaStream_t s, const void* w_hat) {
+                                      cudaStream_t s, const void* w_hat, int ksplit = 1,
+                                      float* part = nullptr, unsigned* tickets = nullptr) {
   const bool dense = w_hat != nullptr;
   EncodeTiledFn enc = encode_fn();
   if (!enc) return set_error(SPHQ_ERR_CUDA, "sphq_gemm: cuTensorMapEncodeTiled unavailable");
@@ -682,12 +768,15 @@ static sphq_status launch_gemm_kernel(sphq_handle h, const void* x, void* y, int
   a.batch = batch;
   a.nwt = G.nwt;
   a.n_big = G.n_big;
+  a.ksplit = ksplit;
+  a.part = part;
+  a.tickets = tickets;
   a.stages = L.stages;
   a.cb_bytes = L.cb_bytes;
   a.off_b = L.off_b;
   a.off_cb = L.off_cb;
   a.off_bar = L.off_bar;
-  const dim3 grid((unsigned)(G.n_big + G.n_small));
+  const dim3 grid((unsigned)((G.n_big + G.n_small) * ksplit));
   void* args[] = {&a, &tmap, &tmap_w};
   e = cudaLaunchKernel(kfn, grid, dim3(gemm_threads(bn)), args, L.total, s);
   if (e != cudaSuccess) return cuda_error(e, "gemm launch");
@@ -754,11 +843,69 @@ bool gemm_prefers_gemv(sphq_handle h, int batch) {
   return t_gemv < waves * per_cta;
 }
 
+// Split-K form of the fused kernel for mid-size batches: with the shape
+// automatic and fewer output tiles than half the SMs, each tile's columns
+// (whole radius groups) are shared by ksplit CTAs, as many as fill the SMs
+// in one wave with at least two groups each, and their fp32 partials are
+// summed in share order by the tile's last CTA.  Workspace: the partial
+// tiles, then one counter per tile.
+static SplitK gemm_splitk_plan(const sphq_handle_s* h, int batch) {
+  SplitK r;
+  if (h->gemm_mt || h->gemm_bn || h->dim != 8 || batch < kSplitMinBatch || batch > kSplitMaxBatch)
+    return r;
+  int optin = 0;
+  if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, h->device) !=
+      cudaSuccess) {
+    (void)cudaGetLastError();
+    return r;
+  }
+  const GemmShape g = select_gemm_shape(h, batch, optin);
+  if (!g.mt) return r;
+  const GemmGrid G = gemm_grid(h, batch, g.mt, g.bn, false);
+  const long long sms = h->sm_count > 0 ? h->sm_count : 1;
+  const long long tiles = G.n_big;
+  if (G.n_small || 2 * tiles > sms) return r;
+  // at least kSplitMinGroups radius groups per CTA: below that the shares'
+  // partial tiles cost more to write and sum than their columns save
+  // (measured: 3584^2 in 5 shares of 5-6 groups 28-31 us against 16-33 for
+  // the unsplit kernel or GEMV launches; 8192^2 in 2 shares of 32 groups 45
+  // against 62-65 at batch 48-128)
+  const int ks = (int)std::min<long long>(std::min<long long>(sms / tiles, h->ng / kSplitMinGroups), 64);
+  if (ks < 2) return r;
+  r.ksplit = ks;
+  r.tiles = tiles;
+  r.part_bytes = align_to((size_t)tiles * ks * kGemmBM * g.mt * g.bn * sizeof(float), 256);
+  r.bytes = r.part_bytes + align_to((size_t)tiles * sizeof(unsigned), 256);
+  return r;
+}
+
 sphq_status gemm_workspace_bytes(sphq_handle h, int batch, size_t* bytes) {
+  const SplitK sk = gemm_splitk_plan(h, batch);
+  if (sk.ksplit > 1) {
+    *bytes = sk.bytes;
+    return SPHQ_OK;
+  }
   double tf = 0, tt = 0;
   gemm_form_times(h, batch, &tf, &tt);
   *bytes = tt < tf ? (size_t)h->rows * h->cols * 2 : 0;
   return SPHQ_OK;
+}
+
+// sphq_gemm_ws with a workspace: the split-K form where it applies and the
+// workspace holds its partials, else the two-pass form (validated x, y, batch).
+sphq_status launch_gemm_ws(sphq_handle h, const void* x, void* y, int batch, void* ws,
+                           size_t ws_bytes, cudaStream_t s) {
+  const SplitK sk = gemm_splitk_plan(h, batch);
+  if (sk.ksplit > 1 && ws_bytes >= sk.bytes) {
+    if (reinterpret_cast<uintptr_t>(ws) % 16)
+      return set_error(SPHQ_ERR_INVALID_ARG, "sphq_gemm_ws: workspace must be 16-byte aligned");
+    float* part = static_cast<float*>(ws);
+    unsigned* tickets = reinterpret_cast<unsigned*>(static_cast<uint8_t*>(ws) + sk.part_bytes);
+    cudaError_t e = cudaMemsetAsync(tickets, 0, (size_t)sk.tiles * sizeof(unsigned), s);
+    if (e != cudaSuccess) return cuda_error(e, "sphq_gemm_ws: clear split-K counters");
+    return launch_gemm_kernel(h, x, y, batch, s, nullptr, sk.ksplit, part, tickets);
+  }
+  return launch_gemm_two_pass(h, x, y, batch, ws, ws_bytes, s);
 }
 
 sphq_status launch_gemm_two_pass(sphq_handle h, const void* x, void* y, int batch, void* ws,

@@ -88,6 +88,10 @@ sphq_status gemm_workspace_bytes(sphq_handle h, int batch, size_t* bytes);
 // tensor-core product reading it (validated x, y, batch).
 sphq_status launch_gemm_two_pass(sphq_handle h, const void* x, void* y, int batch, void* ws,
                                  size_t ws_bytes, cudaStream_t s);
+// sphq_gemm_ws with a workspace: the split-K form of the fused kernel where it
+// applies (mid-size batches, few output tiles), else the two-pass form.
+sphq_status launch_gemm_ws(sphq_handle h, const void* x, void* y, int batch, void* ws,
+                           size_t ws_bytes, cudaStream_t s);
 // 16-D vectors (sphq_dim16.cu): the lane-ordered codebook image (synchronous),
 // pack and decode launches, the GEMV plan of one batch size (csize 0:
 // automatic) and its launch (batch 1..8).

@@ -43,7 +43,8 @@ class GemmInfo(ctypes.Structure):
     _fields_ = [("act_tiles", ctypes.c_int), ("weight_rows", ctypes.c_int),
                 ("stage_cols", ctypes.c_int), ("stages", ctypes.c_int),
                 ("grid_x", ctypes.c_int), ("grid_y", ctypes.c_int),
-                ("smem_bytes", ctypes.c_longlong), ("split_ctas", ctypes.c_int)]
+                ("smem_bytes", ctypes.c_longlong), ("split_ctas", ctypes.c_int),
+                ("ksplit", ctypes.c_int)]
 
 
 def load() -> ctypes.CDLL:

@@ -103,7 +103,8 @@ def test_workspace_advice_and_errors():
     m = G.make_matrix(codes)
     need = m.rows * m.cols * 2
     for batch in (1, 8, 200, 4096):
-        assert m.gemm_workspace(batch) in (0, need)
+        # W_hat for the two-pass form, the partials of the split-K form, or none
+        assert m.gemm_workspace(batch) in (0, need) or m.gemm_shape(batch)["ksplit"] > 1
     big = G.make_matrix(inp.random_codes(3, 8192, 8192, seed=1951, B=1)[0])
     assert big.gemm_workspace(4096) == 8192 * 8192 * 2  # the 8192-entry table at prefill size
     big.close()
@@ -179,5 +180,45 @@ def test_tiny_and_ragged_shapes(rows, cols, batch):
     y = y_two.float().cpu().numpy().astype(np.float64)
     y_ref, absdot = oracle.gemv(G.oracle_decode(codes, np.arange(rows)), x)
     assert np.all(np.abs(y - y_ref) <= oracle.gemv_tolerance(absdot))
+    m.check()
+    m.close()
+
+
+@pytest.mark.parametrize("fmt", FORMATS, ids=FIDS)
+@pytest.mark.parametrize("rows,cols,batch", [(8000, 4096, 48), (1000, 8192, 200), (300, 4096, 41),
+                                             (3584, 18944, 256)])
+def test_split_k(fmt, rows, cols, batch):
+    # batches of 41-256 with a workspace and at least 16 radius groups per
+    # share: the output tiles' columns are shared by several CTAs whose fp32
+    # partials the tile's last CTA sums in share order (ragged rows, ragged
+    # batch); against the oracle and repeatable bit for bit
+    bits, v, K = fmt
+    codes, x = inp.random_codes(bits, rows, cols, seed=2000 + rows + batch + v + bits, B=batch,
+                                radius_bits=v, K=K)
+    m = G.make_matrix(codes)
+    info = m.gemm_shape(batch)
+    assert info["ksplit"] >= 2
+    need = m.gemm_workspace(batch)  # the split-K partials and counters
+    assert need > 0
+    ws = torch.empty(need, dtype=torch.uint8, device="cuda")
+    xd = G.x_dev(x)
+    y1 = m.gemm_ws(xd, ws)
+    y2 = m.gemm_ws(xd, ws)
+    torch.cuda.synchronize()
+    assert torch.equal(_bits(y1), _bits(y2))
+    sel = np.arange(rows) if rows <= 1000 else G.sample_rows(rows, 300, seed=batch)
+    y = y1.float().cpu().numpy().astype(np.float64)
+    y_ref, absdot = oracle.gemv(G.oracle_decode(codes, sel), x)
+    err = np.abs(y[:, sel] - y_ref)
+    tol = oracle.gemv_tolerance(absdot)
+    assert np.all(np.isfinite(y[:, sel]))
+    assert np.all(err <= tol), f"max err/tol = {float(np.max(err / tol)):.3g}"
+    # a workspace too small for the partials (and for W_hat) is refused
+    with pytest.raises(SphqError):
+        m.gemm_ws(xd, ws[: need // 2])
+    # a fixed shape turns the split off
+    m.set_gemm_shape(1, 128)
+    assert m.gemm_shape(batch)["ksplit"] == 1
+    m.set_gemm_shape(0, 0)
     m.check()
     m.close()
