@@ -782,6 +782,64 @@ def gemm_report(hbm_peak):
     return out
 
 
+def midbatch_report():
+    """Batches of 16-256 rows: sphq_gemm (GEMV launches of up to 16 rows or the
+    tensor-core kernel, whichever the library picks) against sphq_gemm_ws with
+    the workspace sphq_gemm_workspace advises (the split-K form where it
+    applies); one call after writing a 256 MiB buffer (an L2 flush), CUDA
+    events around the call, median of 15."""
+    import torch
+
+    from paper_2609_24875_gb300 import SphqMatrix
+    dev = torch.device("cuda", 0)
+    stream = torch.cuda.Stream(device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int16) if a.dtype == np.uint16 else a)).to(dev)
+
+    def timed(fn, reps=15):
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                fn()
+        stream.synchronize()
+        times = []
+        for _ in range(reps):
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            with torch.cuda.stream(stream):
+                flush.zero_()
+                e0.record(stream)
+                fn()
+                e1.record(stream)
+            stream.synchronize()
+            times.append(e0.elapsed_time(e1) * 1e3)
+        return statistics.median(times)
+
+    out = {}
+    for bits in (2, 3):
+        for rows, cols in ((8192, 8192), (3584, 18944)):
+            codes, _ = inp.random_codes(bits, rows, cols, seed=inp.seed_for(6, rows % 97))
+            m = SphqMatrix(rows, cols, bits, t(codes.codebook), t(codes.scale), t(codes.offset))
+            m.pack(t(codes.sign), t(codes.idx), t(codes.rcode))
+            for batch in (16, 32, 64, 128, 256):
+                x = torch.randn(batch, cols, device=dev).half()
+                y = torch.empty(batch, rows, device=dev, dtype=torch.half)
+                us = timed(lambda: m.gemm_ptr(x.data_ptr(), y.data_ptr(), batch, stream.cuda_stream))
+                e = {"gemm_us": round(us, 2), "ksplit": m.gemm_shape(batch)["ksplit"]}
+                need = m.gemm_workspace(batch)
+                if need:
+                    ws = torch.empty(need, dtype=torch.uint8, device=dev)
+                    e["ws_us"] = round(timed(lambda: m.gemm_ws(x, ws, y=y, stream=stream)), 2)
+                    e["ws_bytes"] = need
+                    del ws
+                m.check(stream)
+                out[f"W{bits} {rows}x{cols} B{batch}"] = e
+            m.close()
+            torch.cuda.empty_cache()
+    del flush
+    torch.cuda.empty_cache()
+    return out
+
+
 def study_gather16(mode: int, iters: int = 4096) -> float:
     """Random 32-byte reads per second from a 512 KiB table (0: L2, 1: cluster
     shared memory, 2: local shared memory), from the profiling library
@@ -1017,6 +1075,7 @@ def run_report(args):
                 m.close()
             torch.cuda.empty_cache()
     rep["prefill_gemm"] = gemm_report(hbm_peak)
+    rep["mid_batch_gemm"] = midbatch_report()
     rep["encode"] = encode_report()
     rep["oracle_timing"] = oracle_timing()
     print(json.dumps(rep), flush=True)
