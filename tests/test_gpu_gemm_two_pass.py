@@ -222,3 +222,28 @@ def test_split_k(fmt, rows, cols, batch):
     m.set_gemm_shape(0, 0)
     m.check()
     m.close()
+
+
+def test_split_k_graph_capture():
+    # the counter memset and the split-K launch captured in a CUDA graph on a
+    # side stream: replays equal the eager call bit for bit
+    codes, x = inp.random_codes(3, 300, 4096, seed=2050, B=64)
+    m = G.make_matrix(codes)
+    assert m.gemm_shape(64)["ksplit"] >= 2
+    ws = torch.empty(m.gemm_workspace(64), dtype=torch.uint8, device="cuda")
+    xd = G.x_dev(x)
+    y_ref = m.gemm_ws(xd, ws)
+    torch.cuda.synchronize()
+    s = torch.cuda.Stream()
+    y = torch.empty_like(y_ref)
+    s.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        m.gemm_ws(xd, ws, y=y, stream=s)
+    for _ in range(3):
+        y.zero_()
+        g.replay()
+        torch.cuda.synchronize()
+        assert torch.equal(_bits(y), _bits(y_ref))
+    m.check()
+    m.close()
