@@ -553,16 +553,16 @@ def run_case(spec: str, pool: int, launches: int):
     """Profiling driver: `bits:n[:batch]` or `bits:RxC[:batch]` -> `pool`
     distinct packed n x n (R x C) matrices, `launches` GEMVs round robin on one
     stream, no timing (for running under ncu).  bits `3v3` selects W3 with
-    3-bit radius codes, `dDvV` the 8/D/V split (e.g. `d7v2`), `v16` 16-D
-    vectors (Tab. 7, W2 allocation); a leading `e` (`e3:8192`) packs the
+    3-bit radius codes, `dDvV` the 8/D/V split (e.g. `d7v2`), `v4` / `v16` 4-D
+    / 16-D vectors (Tab. 7, W2 allocation); a leading `e` (`e3:8192`) packs the
     encoded configuration's codes (sphq_encode on the Gaussian weights of the
     square sweep, batch 1) instead of random codes."""
     import torch
 
     head, size, *rest = spec.split(":")
     encoded = head.startswith("e")
-    dim16 = head == "v16"
-    bits, vbits, K = (2, 4, 1 << 14) if dim16 else parse_split(head.lstrip("e"))
+    vdim = {"v4": 4, "v16": 16}.get(head, 8)
+    bits, vbits, K = (2, 4, 1 << (2 * (vdim - 1) - vdim)) if vdim != 8 else parse_split(head.lstrip("e"))
     rows, n = (int(v) for v in size.split("x")) if "x" in size else (int(size), int(size))
     batch = int(rest[0]) if rest else 1
     dev = torch.device("cuda", 0)
@@ -575,15 +575,16 @@ def run_case(spec: str, pool: int, launches: int):
         mats, xd, _ = make_encoded_pool(bits, n, pool,
                                         inp.seed_for(1, inp.SQUARE_SWEEP.index((bits, n))), dev)
     else:
-        if dim16:
-            codes, x = inp.random_codes_dim(16, 2, rows, n, seed=1, B=batch)
+        if vdim != 8:
+            codes, x = inp.random_codes_dim(vdim, 2, rows, n, seed=1, B=batch)
         else:
             codes, x = inp.random_codes(bits, rows, n, seed=1, B=batch, radius_bits=vbits, K=K)
         mats = []
         for _ in range(pool):
             m = SphqMatrix(rows, n, bits, t(codes.codebook), t(codes.scale), t(codes.offset),
-                           radius_bits=vbits, K=K, dim=16 if dim16 else 8)
-            m.pack(t(codes.sign), t(codes.idx), t(codes.rcode))
+                           radius_bits=vbits, K=K, dim=vdim)
+            m.pack(t(codes.sign.astype(np.uint8) if vdim == 4 else codes.sign), t(codes.idx),
+                   t(codes.rcode))
             mats.append(m)
         xd = t(x).view(torch.float16)
     ys = [torch.empty((batch, rows), dtype=torch.float16, device=dev) for _ in mats]
