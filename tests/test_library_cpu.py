@@ -55,3 +55,25 @@ def test_invalid_arguments_rejected_on_host(lib):
     assert lib.sphq_set_cluster_size(None, 1, 2) == 1
     assert lib.sphq_destroy(None) == 0
     assert lib.sphq_last_error() == b""
+
+
+def test_vector_dimension_and_workspace_arguments_rejected_on_host(lib):
+    h = ctypes.c_void_p()
+    buf = ctypes.create_string_buffer(1 << 16)
+    p = ctypes.cast(buf, ctypes.c_void_p)
+    # 16-D vectors take the W2 allocation only: bits 2, K = 2^14, 4 radius bits
+    assert lib.sphq_create_dim(32, 128, 16, 2, 4, 1 << 13, p, p, p, ctypes.byref(h)) == 2
+    assert lib.sphq_create_dim(32, 128, 16, 3, 4, 1 << 14, p, p, p, ctypes.byref(h)) == 2
+    assert lib.sphq_create_dim(32, 128, 16, 2, 3, 1 << 14, p, p, p, ctypes.byref(h)) == 2
+    assert b"16-D" in lib.sphq_last_error()
+    # 4-D likewise (bits 2, K 4, 4 radius bits); other dimensions are unsupported
+    assert lib.sphq_create_dim(32, 128, 4, 2, 4, 8, p, p, p, ctypes.byref(h)) == 2
+    assert lib.sphq_create_dim(32, 128, 12, 2, 4, 64, p, p, p, ctypes.byref(h)) == 2
+    assert h.value is None
+    # the workspace entry points and shape queries with a NULL handle
+    n = ctypes.c_size_t(7)
+    assert lib.sphq_gemm_workspace(None, 64, ctypes.byref(n)) == 1
+    assert lib.sphq_gemm_ws(None, p, p, 64, p, 1 << 16, None) == 1
+    info = sphq.GemmInfo()
+    assert lib.sphq_get_gemm_shape(None, 64, ctypes.byref(info)) == 1
+    assert lib.sphq_set_gemm_shape(None, 1, 128) == 1
