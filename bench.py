@@ -61,7 +61,7 @@ UNIT = "GB/s"
 TRAFFIC_SOURCES = ("paper_2609_24875_gb300/csrc/sphq_gemv_kernel.cuh",
                    "paper_2609_24875_gb300/csrc/sphq_gemv.cu",
                    "paper_2609_24875_gb300/csrc/sphq_layout.cuh")
-TRAFFIC_DIGEST = "4def4c1a9071d23c:aee7ee8072d8a4f1:4e816d7cd02affb6"
+TRAFFIC_DIGEST = "0db785fb6516774e:aee7ee8072d8a4f1:4e816d7cd02affb6"
 TRAFFIC_RATIO = {2: 21040640 / 21005312, 3: 28536064 / 28475392}
 
 

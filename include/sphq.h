@@ -262,10 +262,11 @@ sphq_status sphq_angle_codebook(const float* phi, int K, double eps, double* cod
  *   x      batch x cols fp16, device pointer, 16-byte aligned.
  *   y      batch x rows fp16, device pointer, 4-byte aligned; written in full.
  *   batch  1..SPHQ_MAX_BATCH (16).  Each decoded weight serves every row of
- *          the batch: 1-2 rows with the radius factored out of the dot
- *          products, 3-8 rows as the N dimension of the tensor-core products,
- *          9-16 rows as two such halves per decoded block (8-D vectors; 4-D
- *          handles run 9-16 rows as two launches).
+ *          the batch: 1 row (and 2 rows on large small-codebook matrices)
+ *          with the radius factored out of the dot products, 2-8 rows
+ *          otherwise as the N dimension of the tensor-core products, 9-16
+ *          rows as two such halves per decoded block (8-D vectors; 4-D and
+ *          16-D handles run 9-16 rows as two launches).
  *
  * Asynchronous on `stream`: no host synchronisation and no allocation, so it
  * may be captured in a CUDA graph.  One handle should not run two gemv calls
@@ -498,7 +499,8 @@ typedef struct sphq_plan_info {
   int tiles_per_cluster; /* most row tiles of one cluster */
   int warps_per_cta;
   int smem_bytes;        /* dynamic shared memory per CTA */
-  int staged_x;          /* 1: activations copied to shared memory (batch 1-2), 0: read via L1 */
+  int staged_x;          /* 1: activations copied to shared memory (the factored mode of batch
+                            1, and of batch 2 on large small-codebook matrices), 0: read via L1 */
   int ctas_per_sm;       /* CTAs per SM the kernel is built for: 2 (W2 and the small-codebook
                             splits, at most 128 registers per thread) or 1 (W3; and W2 when
                             the row tiles bound the cluster count, with the whole register

@@ -13,7 +13,9 @@
 // fp16 values are exact in fp32.
 //
 // Two ways of applying the radius, chosen by batch size:
-//  * batch 1-2 ("factored"): the A fragment holds the signed unit direction
+//  * batch 1-2 ("factored"; the planner takes it for batch 1, and for batch
+//    2 on small-codebook matrices of more than 16384 units): the A fragment
+//    holds the signed unit direction
 //    s (.) c_z and the B fragment is block diagonal -- column 2c + b carries
 //    batch row b of slot c only -- so every MMA pair returns, in the lane
 //    that decoded them, the per-vector dots d = (s (.) c_z) . x_b.  The lane
